@@ -40,7 +40,9 @@ def denoise(velocity, x0, budgets, n_exec=None, tr=True, gac=True, gac_mask=None
       final         [H, D]  actions as handed to the controller: released actions for early
                             tokens, x_{N*} (+ GAC) for the rest
       released      [H, D]  a^i for early tokens (NaN elsewhere)
-      ghost         [H, D]  reconciled end states: x'_{N*} for early tokens, x_{N*} elsewhere
+      ghost         [H, D]  reconciled end states: x'_{N*} for early tokens, x_{N*} elsewhere;
+                            without TR there is no reconciled state (ghosts exist through
+                            TR, Sec. 4.3), so early rows hold the frozen action fed back
       release_step  [H]     N_i for early tokens, N* for the others (when they are available)
       E             [D]     Eq. 8 estimate (zeros when GAC does not run)
       evals         int     evaluations of the velocity network (N*)
@@ -85,7 +87,7 @@ def denoise(velocity, x0, budgets, n_exec=None, tr=True, gac=True, gac_mask=None
                 release_step[i] = k
     final = x.copy()
     ghost = x.copy()
-    ghost[early] = g[early]
+    ghost[early] = g[early] if tr else released[early]
     E = np.zeros(D)
     tail = []
     if gac and not chunk_relative and early:

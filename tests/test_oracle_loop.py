@@ -226,6 +226,7 @@ def test_tr_off_freezes_released_inputs():
     assert [float(t[0]) for _, t in seen] == [0.0, 1.0, 1.0]
     assert [float(u[0, 0]) for u, _ in seen] == [0.0, 1.0, 1.0]
     assert out["released"][0, 0] == 1.0
+    assert out["ghost"][0, 0] == 1.0          # no reconciled state: the frozen action
     with pytest.raises(ValueError):
         denoise(vel, x0, [1, 3, 3], tr=False, gac=True)
 
