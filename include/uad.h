@@ -1,0 +1,184 @@
+/*
+ * uad.h -- C ABI of the Urgency-Aware Denoising (UAD) library for GB300 (sm_103a).
+ *
+ * The library runs the denoising loop of a flow-matching action expert on one GPU:
+ * per-action Euler steps with per-action flow times (Sec. 3, Eqs. 1-2; Sec. 4.2, Eqs. 4-5),
+ * Urgency-Aware Early Release of actions whose budget ends before N* (Sec. 4.2),
+ * Trajectory Reconciliation of released actions with zero extra evaluations (Sec. 4.3,
+ * Eqs. 6-7), ghost actions, and Ghost Action Correction of the executable tail (Sec. 4.4,
+ * Eqs. 8-9). Releases are handed to the host while the tail keeps refining on the GPU
+ * (App. C.1, "Asynchronous Execution").
+ *
+ * Conventions
+ *   - Every call returns an int: UAD_OK (0) or a negative code below. uad_last_error()
+ *     gives a message for the last failure on a context.
+ *   - Pointers marked "host or device" may point to either; the library inspects them.
+ *   - The caller owns every buffer it passes and may reuse it as soon as the call returns
+ *     (the library copies what it keeps). The library owns its weights, state, scratch and
+ *     the pinned release buffer, all freed by uad_destroy.
+ *   - All arguments are validated on the host before anything is launched.
+ *   - No call waits on the GPU without a deadline; no call traps the GPU.
+ *   - A context is used by one host thread at a time.
+ */
+#ifndef UAD_H
+#define UAD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define UAD_OK 0
+#define UAD_EINVAL (-22)     /* invalid argument or configuration */
+#define UAD_ESTATE (-1)      /* call out of order (e.g. finish without denoise) */
+#define UAD_ENOMEM (-12)     /* device or pinned allocation failed */
+#define UAD_ECUDA (-5)       /* a CUDA runtime call failed; see uad_last_error */
+#define UAD_ETIMEDOUT (-110) /* the deadline passed before the GPU finished */
+#define UAD_ENONFINITE (-33) /* a velocity was NaN or Inf; outputs are still written */
+
+#define UAD_KIND_ADARMS 0    /* joint attention over prefix KV + chunk, adaptive RMSNorm */
+#define UAD_KIND_DIT 1       /* chunk self-attention + cross-attention, adaLN-zero */
+
+#define UAD_DTYPE_F32 0
+#define UAD_DTYPE_BF16 1
+
+#define UAD_MAX_STEPS 64     /* largest step budget N_i */
+
+/* Shape of the action expert F_theta (Sec. 3, Eq. 1). */
+typedef struct uad_arch {
+  int32_t kind;          /* UAD_KIND_ADARMS or UAD_KIND_DIT */
+  int32_t dtype;         /* UAD_DTYPE_F32: fp32 everywhere; UAD_DTYPE_BF16: bf16 weights and
+                            GEMM/attention operands, fp32 accumulation, state and velocities */
+  int32_t n_layers;
+  int32_t width;         /* W */
+  int32_t n_heads;       /* query heads */
+  int32_t n_kv_heads;    /* key/value heads (divides n_heads; DiT: == n_heads) */
+  int32_t head_dim;
+  int32_t mlp_dim;
+  int32_t action_dim;    /* D */
+  int32_t chunk_len;     /* H, actions per chunk (Sec. 3) */
+  int32_t prefix_len;    /* P, observation prefix tokens */
+  int32_t prefix_width;  /* DiT: width of the prefix tokens (cross-attention input) */
+  int32_t rope;          /* ADARMS: RoPE on chunk queries/keys at positions P + i */
+  int32_t max_batch;     /* robots per call, >= 1 */
+} uad_arch;
+
+/* The urgency schedule of one call (Sec. 4.2, Eq. 4, generalised to per-action budgets). */
+typedef struct uad_schedule {
+  const int32_t* budgets;  /* host, [batch][chunk_len], N_i >= 1; N* = max over a robot's row */
+  int32_t batch;           /* robots in this call, 1..max_batch */
+  int32_t n_exec;          /* S, actions executed before replanning; 0 means chunk_len */
+  int32_t tr;              /* Trajectory Reconciliation on (1) or off (0, UAER-only ablation:
+                              released actions are fed back frozen at flow time 1) */
+  int32_t gac;             /* Ghost Action Correction on/off; needs tr unless chunk_relative */
+  int32_t chunk_relative;  /* actions relative to the chunk start: GAC is skipped (Sec. 4.4) */
+  const uint8_t* gac_mask; /* host [action_dim], 1 = additive dimension corrected by Eq. 9,
+                              0 = left unchanged (rotation / gripper); NULL = all additive */
+} uad_schedule;
+
+typedef struct uad_stats {
+  int32_t evals;           /* velocity-network evaluations of the chunk (= N*; TR adds none) */
+  int32_t n_star;          /* max step budget of the call */
+  int32_t nonfinite;       /* count of non-finite velocity entries */
+  int32_t tr_extra_evals;  /* evaluations spent on reconciliation: always 0 */
+} uad_stats;
+
+typedef struct uad_ctx uad_ctx;
+
+/* Create a context on the current CUDA device.
+ * weights: host or device fp32 blob of n_floats values, tensors in this order (linear
+ *   weights [in][out], y = x W + b):
+ *     t_w1[W][W] t_b1[W] t_w2[W][W] t_b2[W] in_w[D][W] in_b[W]
+ *     per layer, ADARMS: mod1_w[W][3W] mod1_b[3W] wq[W][Hq*dh] wk[W][Hkv*dh] wv[W][Hkv*dh]
+ *                        wo[Hq*dh][W] mod2_w[W][3W] mod2_b[3W] wg[W][F] wu[W][F] wd[F][W]
+ *                DiT:    mod_w[W][6W] mod_b[6W] wq wk wv[W][Hq*dh] wo[Hq*dh][W]
+ *                        wqc[W][Hq*dh] wkc wvc[Pw][Hq*dh] woc[Hq*dh][W]
+ *                        w1[W][F] b1[F] w2[F][W] b2[W]
+ *     modf_w[W][2W] modf_b[2W] out_w[W][D] out_b[D]
+ *   Modulation vectors are (scale, shift, gate) for ADARMS and (shift1, scale1, gate1,
+ *   shift2, scale2, gate2) for DiT; the final one is (scale, shift) / (shift, scale).
+ *   For bf16 architectures every weight is rounded to bf16 (nearest, ties to even).
+ * The weights are copied into the library's own layout; the blob may be freed afterwards.
+ * Errors: UAD_EINVAL (shape, n_floats), UAD_ENOMEM, UAD_ECUDA. */
+int uad_init(const uad_arch* arch, const float* weights, size_t n_floats, uad_ctx** out);
+
+/* Bind robot `robot`'s observation context (the cached vision-language prefix, Sec. 3).
+ * ADARMS: k, v = per-layer prefix keys and values [L][P][Hkv][dh] (keys already carry
+ *         their own position encoding).
+ * DiT:    k = prefix tokens [P][prefix_width], v = NULL; the per-layer cross-attention K/V
+ *         are projected here, once per observation.
+ * dtype: UAD_DTYPE_F32 or UAD_DTYPE_BF16 element type of the given buffers (host or device);
+ * they are copied (converted to the arch dtype). prefix_len must equal arch.prefix_len.
+ * Errors: UAD_EINVAL, UAD_ESTATE (a chunk is in flight), UAD_ECUDA. Synchronous. */
+int uad_set_prefix_kv(uad_ctx* ctx, int32_t robot, const void* k, const void* v,
+                      int32_t prefix_len, int32_t dtype);
+
+/* Precompute the per-action time conditioning for every flow time j/n, 1 <= n <= max_budget,
+ * plus 1 (App. C.1). Optional: uad_denoise computes missing times itself. Synchronous. */
+int uad_prepare_times(uad_ctx* ctx, int32_t max_budget);
+
+/* Start denoising one chunk for sched->batch robots (robots 0..batch-1) on `stream`
+ * (a cudaStream_t; NULL = legacy default stream). Asynchronous: returns once the work is
+ * enqueued. noise: host or device fp32 [batch][H][D], the initial state x_0 (Sec. 3).
+ * n_star: 0, or the largest budget of the call (checked). Every robot must have a prefix.
+ * Early actions are released into pinned host memory after their last step (UAER); the
+ * tail continues on the stream. Errors: UAD_EINVAL, UAD_ESTATE (previous chunk not
+ * finished), UAD_ECUDA. */
+int uad_denoise(uad_ctx* ctx, const float* noise, const uad_schedule* sched, int32_t n_star,
+                void* stream);
+
+/* Host-side hand-off of released actions (App. C.1: urgent actions go to the execution
+ * queue while the tail refines). Waits until at least `min_ready` of robot `robot`'s
+ * actions are available, or until timeout_us passes (0: do not wait).
+ * out [H][D] (host): rows of ready actions are written (others untouched);
+ * ready [H] (host, may be NULL): 1 if available; release_step [H] (may be NULL): the step
+ * after which the action became available (N_i for early actions, N* for the tail, whose
+ * rows already include GAC). Released actions never change afterwards (Sec. 4.4).
+ * Returns the number of ready actions (>= min_ready), UAD_ETIMEDOUT, or an error. */
+int uad_poll_released(uad_ctx* ctx, int32_t robot, int32_t min_ready, int64_t timeout_us,
+                      float* out, int32_t* ready, int32_t* release_step);
+
+/* Wait (at most timeout_us; < 0 = no limit) for the chunk to complete and read it back.
+ * final [batch][H][D]: released actions for early actions, x_{N*} plus GAC (Eq. 9) for the
+ *   executable tail, x_{N*} for the rest;
+ * ghost [batch][H][D]: reconciled end states x'_{N*} (ghost actions, Sec. 4.3) for early
+ *   actions, x_{N*} (before GAC) for the others;
+ * gac_error [batch][D]: E of Eq. 8 (zeros where GAC did not run).
+ * Any output may be NULL; each may be host or device memory.
+ * Returns UAD_OK, UAD_ENONFINITE (outputs written), UAD_ETIMEDOUT (the chunk stays in
+ * flight; call again), UAD_ESTATE, UAD_ECUDA. */
+int uad_finish(uad_ctx* ctx, float* final_actions, float* ghost, float* gac_error,
+               uad_stats* stats, int64_t timeout_us);
+
+/* Device timestamps of the last finished chunk: ms[k-1] = time from the chunk's first
+ * kernel to the end of step k (k = 1..n_star), from the GPU's global timer. Returns the
+ * number of entries written. */
+int uad_step_times(const uad_ctx* ctx, double* ms, int32_t max_entries);
+
+/* Kernel launches the library enqueues per uad_denoise of the given batch and N*
+ * (excluding one-time time-conditioning fills). */
+int uad_launches_per_chunk(const uad_ctx* ctx, int32_t batch, int32_t n_star);
+
+void uad_destroy(uad_ctx* ctx);
+const char* uad_last_error(const uad_ctx* ctx);
+
+/* ---- Host-only helpers (no GPU needed) ------------------------------------------------ */
+
+/* Plan of step k (1-based) for one robot with budgets[H] (Sec. 4.2, Eqs. 4-5; Sec. 4.3, Eq. 7):
+ * flags[i] bit 0 = active (k <= N_i: own Euler step 1/N_i), bit 1 = ghost input (early action
+ * past its release, fed its reconciled state), bit 2 = released after this step, bit 3 =
+ * early (N_i < N*: a TR running sum is kept), bit 4 = frozen input (TR off);
+ * tau = tau_num[i] / tau_den[i] (reduced fraction), the flow time fed to the network.
+ * Returns N* or UAD_EINVAL. */
+int uad_plan_step(const int32_t* budgets, int32_t H, int32_t k, int32_t tr, int32_t* flags,
+                  int32_t* tau_num, int32_t* tau_den);
+
+/* Library version string. */
+const char* uad_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* UAD_H */

@@ -1,0 +1,314 @@
+// Tensor-core projection GEMM for sm_103a: out[m][n] = epi(sum_k X[m][k] * Wt[n][k]).
+//
+// Swap-AB tiling for few tokens: 128 weight rows form the MMA's M side, 64 tokens its N
+// side, so one CTA computes a 128 x 64 fp32 tile in tensor memory (TMEM). Weights are
+// pre-tiled at init into 128 x 64 bf16 blocks already in the 128-byte-swizzled K-major
+// shared-memory layout, so each block arrives with one 16 KB bulk copy (cp.async.bulk);
+// activation tiles come through a 2-D TMA tensor map (cp.async.bulk.tensor) with the same
+// swizzle and zero fill past the last row. One thread issues tcgen05.mma, one thread feeds
+// the TMA ring, four warps drain TMEM with tcgen05.ld.
+//
+// Split-K: CTAs sharing an output tile each own a K range; they add their partial tile into
+// an fp32 accumulator in L2 (red.global.add) and the last one to arrive (per-tile counter)
+// applies the epilogue, then clears the accumulator and counter for the next launch.
+// Every wait is bounded: on timeout the kernel records an error code and winds down.
+#include <cuda.h>
+#include "uad_internal.cuh"
+
+namespace uad {
+
+namespace {
+
+constexpr int kBM = 128, kBN = 64, kBK = 64;
+constexpr int kStageA = kBM * kBK * 2;  // 16 KB
+constexpr int kStageB = kBN * kBK * 2;  // 8 KB
+constexpr unsigned long long kWaitNs = 2000000000ull;  // 2 s bound on any wait
+
+__device__ __forceinline__ uint32_t su32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ unsigned long long gtime() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void mbar_init(uint64_t* b, uint32_t n) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(b)), "r"(n));
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* b, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(b)), "r"(bytes) : "memory");
+}
+// Wait for the phase with the given parity to complete; false (and *err set) after kWaitNs.
+__device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity, int* err, int code) {
+  unsigned long long t0 = 0;
+  for (uint32_t it = 0;; ++it) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok) : "r"(su32(b)), "r"(parity) : "memory");
+    if (ok) return true;
+    if ((it & 255) == 0) {
+      const unsigned long long t = gtime();
+      if (t0 == 0) t0 = t;
+      else if (t - t0 > kWaitNs) {
+        atomicCAS(err, 0, code);
+        return false;
+      }
+    }
+  }
+}
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar, uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;"
+      ::"r"(su32(dst)), "l"(src), "r"(bytes), "r"(su32(bar)), "l"(pol) : "memory");
+}
+__device__ __forceinline__ void tma_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+      ::"r"(su32(dst)), "l"(map), "r"(x), "r"(y), "r"(su32(bar)) : "memory");
+}
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row core groups 1024 B apart.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
+         ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+// Instruction descriptor, kind::f16: bf16 x bf16 -> fp32, both K-major, M = 128, N = 64.
+constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kBN >> 3) << 17) |
+                            ((uint32_t)(kBM >> 4) << 24);
+
+__device__ __forceinline__ void mma_bf16(uint32_t d, uint64_t a, uint64_t b, uint32_t accum) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n"
+      ::"r"(d), "l"(a), "l"(b), "r"(kIdesc), "r"(accum));
+}
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(su32(bar)) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ float gelu_tanh_f(float x) {
+  const float k0 = 0.7978845608028654f;
+  return 0.5f * x * (1.f + tanhf(k0 * (x + 0.044715f * x * x * x)));
+}
+
+__device__ __forceinline__ void store_out(void* out, long long i, float v, int dt) {
+  if (dt == BF16) static_cast<__nv_bfloat16*>(out)[i] = __float2bfloat16_rn(v);
+  else static_cast<float*>(out)[i] = v;
+}
+
+// Apply the epilogue to one value of row n (this thread) and token m.
+__device__ __forceinline__ void epi_one(const TcGemmArgs& p, int m, int n, float acc, bool lane_even,
+                                        float partner) {
+  switch (p.epi) {
+    case EPI_GEGLU:
+      if (lane_even) store_out(p.out, (long long)m * p.ldo + n / 2, gelu_tanh_f(acc) * partner, p.out_dtype);
+      break;
+    case EPI_RESID_GATE: {
+      const float r = acc + (p.bias ? p.bias[n] : 0.f);
+      const float gt = p.gate_tab ? p.gate_tab[(long long)p.tau_row[m] * p.gate_stride + n] : 1.f;
+      float* dst = p.resid + (long long)m * p.ldr + n;
+      *dst = fmaf(gt, r, *dst);
+      break;
+    }
+    case EPI_BIAS_GELU:
+      store_out(p.out, (long long)m * p.ldo + n, gelu_tanh_f(acc + (p.bias ? p.bias[n] : 0.f)), p.out_dtype);
+      break;
+    default:
+      store_out(p.out, (long long)m * p.ldo + n, acc + (p.bias ? p.bias[n] : 0.f), p.out_dtype);
+      break;
+  }
+}
+
+__global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__ CUtensorMap tmx, TcGemmArgs p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  const int t = blockIdx.x, mt = blockIdx.y, s = blockIdx.z;
+  const int KC = p.K / kBK;
+  const int c0 = s * KC / p.splits, c1 = (s + 1) * KC / p.splits, nch = c1 - c0;
+  const int stages = nch < kTcMaxStages ? nch : kTcMaxStages;
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + (size_t)stages * kStageA;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sB + (size_t)stages * kStageB);
+  uint64_t* empty = full + kTcMaxStages;
+  uint64_t* done = empty + kTcMaxStages;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  int* last_flag = reinterpret_cast<int*>(tmem_slot + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < stages; ++i) {
+      mbar_init(full + i, 1);
+      mbar_init(empty + i, 1);
+    }
+    mbar_init(done, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(tmem_slot)), "r"(kBN));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (threadIdx.x == 0) {
+    // ---- producer: weight block (bulk copy) + activation tile (tensor map) per K chunk ----
+    const uint64_t pol = policy_evict_first();
+    const uint8_t* wt = static_cast<const uint8_t*>(p.w_tiled) + ((size_t)t * KC + c0) * kStageA;
+    int issued = 0;
+    for (int i = 0; i < nch; ++i) {
+      const int st = i % stages, round = i / stages;
+      if (round > 0 && !mbar_wait(empty + st, (round - 1) & 1, p.err, 11)) break;
+      mbar_expect_tx(full + st, kStageA + kStageB);
+      bulk_g2s(sA + (size_t)st * kStageA, wt + (size_t)i * kStageA, kStageA, full + st, pol);
+      tma_2d(sB + (size_t)st * kStageB, &tmx, (c0 + i) * kBK, mt * kBN, full + st);
+      ++issued;
+    }
+    // do not leave copies in flight into shared memory of an exiting CTA
+    for (int i = issued - stages > 0 ? issued - stages : 0; i < issued; ++i)
+      mbar_wait(full + i % stages, (i / stages) & 1, p.err, 12);
+  } else if (threadIdx.x == 32) {
+    // ---- MMA issuer ----
+    bool ok = true;
+    for (int i = 0; i < nch && ok; ++i) {
+      const int st = i % stages, round = i / stages;
+      ok = mbar_wait(full + st, round & 1, p.err, 13);
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t a0 = su32(sA + (size_t)st * kStageA), b0 = su32(sB + (size_t)st * kStageB);
+#pragma unroll
+      for (int k = 0; k < kBK / 16; ++k)
+        mma_bf16(tmem, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), (i > 0 || k > 0) ? 1u : 0u);
+      mma_commit(empty + st);
+    }
+    mma_commit(done);
+  }
+  __syncwarp();
+
+  // ---- epilogue: TMEM -> registers, one weight row (output feature) per thread ----
+  const bool ok = mbar_wait(done, 0, p.err, 14);
+  tc_fence_after();
+  const int row = warp * 32 + lane;
+  const int n = t * kBM + row;
+  const int m0 = mt * kBN;
+  const int mcount = p.M - m0 < kBN ? p.M - m0 : kBN;
+  float v[kBN];
+  __syncwarp();
+#pragma unroll
+  for (int c = 0; c < kBN; c += 16) tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + c, v + c);
+  const bool even = (lane & 1) == 0;
+  if (ok && nch > 0) {
+    if (p.splits == 1) {
+#pragma unroll
+      for (int j = 0; j < kBN; ++j) {
+        if (j < mcount) {
+          const float partner = __shfl_xor_sync(0xffffffffu, v[j], 1);
+          epi_one(p, m0 + j, n, v[j], even, partner);
+        }
+      }
+    } else {
+      float* acc = p.acc + (size_t)m0 * p.N + n;
+#pragma unroll
+      for (int j = 0; j < kBN; ++j)
+        if (j < mcount)
+          asm volatile("red.global.add.f32 [%0], %1;" ::"l"(acc + (size_t)j * p.N), "f"(v[j]) : "memory");
+      __threadfence();
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        const int tile = mt * gridDim.x + t;
+        const int prev = atomicAdd(p.counters + tile, 1);
+        *last_flag = prev == p.splits - 1;
+      }
+      __syncthreads();
+      if (*last_flag) {
+        __threadfence();
+        for (int j = 0; j < mcount; ++j) {
+          float* a = acc + (size_t)j * p.N;
+          const float sum = __ldcg(a);
+          __stcg(a, 0.f);
+          const float partner = __shfl_xor_sync(0xffffffffu, sum, 1);
+          epi_one(p, m0 + j, n, sum, even, partner);
+        }
+        if (threadIdx.x == 0) p.counters[mt * gridDim.x + t] = 0;
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kBN));
+}
+
+// ---- weight re-layout into 128 x 64 swizzled blocks --------------------------------------
+__global__ void relayout_tiled_kernel(const float* src, int K, int N, __nv_bfloat16* dst, int mult, long long off) {
+  __shared__ float tt[32][33];
+  const int k0 = blockIdx.y * 32, n0 = blockIdx.x * 32;
+  for (int r = threadIdx.y; r < 32; r += blockDim.y) {
+    const int k = k0 + r, n = n0 + threadIdx.x;
+    tt[r][threadIdx.x] = (k < K && n < N) ? src[(long long)k * N + n] : 0.f;
+  }
+  __syncthreads();
+  const int KC = K / kBK;
+  for (int r = threadIdx.y; r < 32; r += blockDim.y) {
+    const int n = n0 + r, k = k0 + threadIdx.x;
+    if (n >= N || k >= K) continue;
+    const long long row = (long long)n * mult + off;
+    const long long tile = (row / kBM) * KC + k / kBK;
+    const int rr = (int)(row % kBM), kk = k % kBK;
+    const int gran = (kk >> 3) ^ (rr & 7);
+    dst[tile * (kBM * kBK) + rr * kBK + gran * 8 + (kk & 7)] = __float2bfloat16_rn(tt[threadIdx.x][r]);
+  }
+}
+
+}  // namespace
+
+size_t gemm_tc_smem_bytes(int stages) {
+  return 1024 + (size_t)stages * (kStageA + kStageB) + (2 * kTcMaxStages + 1) * 8 + 16;
+}
+
+void gemm_tc_prepare() {
+  cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       (int)gemm_tc_smem_bytes(kTcMaxStages));
+}
+
+int gemm_tc_splits(int M, int N, int K, int sms) {
+  const int tiles = (N / kBM) * ((M + kBN - 1) / kBN);
+  const int KC = K / kBK;
+  int s = (sms + tiles / 2) / tiles;
+  if (s < 1) s = 1;
+  if (s > KC) s = KC;
+  return s;
+}
+
+void launch_gemm_tc(const CUtensorMap* tmx, const TcGemmArgs& a, cudaStream_t s) {
+  const int KC = a.K / kBK;
+  const int per = (KC + a.splits - 1) / a.splits;
+  const int stages = per < kTcMaxStages ? per : kTcMaxStages;
+  dim3 grid(a.N / kBM, (a.M + kBN - 1) / kBN, a.splits);
+  gemm_tc_kernel<<<grid, 128, gemm_tc_smem_bytes(stages), s>>>(*tmx, a);
+}
+
+void launch_relayout_tiled(const float* src, int K, int N, void* dst, int mult, long long off, cudaStream_t s) {
+  dim3 grid((N + 31) / 32, (K + 31) / 32);
+  relayout_tiled_kernel<<<grid, dim3(32, 8), 0, s>>>(src, K, N, static_cast<__nv_bfloat16*>(dst), mult, off);
+}
+
+}  // namespace uad

@@ -1,0 +1,122 @@
+// Internal declarations shared by the library's translation units.
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+namespace uad {
+
+constexpr int kMaxSteps = 64;              // = UAD_MAX_STEPS
+constexpr int kFlagStride = kMaxSteps + 1;  // host flag slots per robot (steps 1..64)
+
+enum DType { F32 = 0, BF16 = 1 };
+
+// GEMM epilogues (out[m][n] from acc = sum_k A[m][k] * Wt[n][k]).
+enum Epi {
+  EPI_STORE = 0,       // out = acc (+ bias) (+ add_rows[m % add_mod][n])
+  EPI_BIAS_SILU = 1,   // out = silu(acc + bias)
+  EPI_RESID_GATE = 2,  // resid[m][n] += gate(m, n) * (acc + bias); gate = 1 when gate_tab is null
+  EPI_GEGLU = 3,       // rows interleaved (2j = gate, 2j+1 = up): out[m][j] = gelu_tanh(g) * u
+  EPI_BIAS_GELU = 4,   // out = gelu_tanh(acc + bias)
+};
+
+struct GemmArgs {
+  const void* A = nullptr; int lda = 0; int a_dtype = F32;  // activations [M][K]
+  const void* W = nullptr; int w_dtype = F32;               // weights [N][K], K contiguous
+  int M = 0, N = 0, K = 0;
+  int epi = EPI_STORE;
+  void* out = nullptr; int ldo = 0; int out_dtype = F32;
+  const float* bias = nullptr;                     // [N]
+  const float* add_rows = nullptr; int add_mod = 1; // EPI_STORE: + add_rows[(m % add_mod) * N + n]
+  float* resid = nullptr; int ldr = 0;             // EPI_RESID_GATE target, fp32
+  const float* gate_tab = nullptr; int gate_stride = 0;  // gate(m, n) = gate_tab[tau_row[m] * gate_stride + n]
+  const int* tau_row = nullptr;
+};
+
+struct NormArgs {
+  const float* h = nullptr; int ldh = 0;   // fp32 [M][W]
+  int M = 0, W = 0;
+  int layer_norm = 0;                      // 0: RMSNorm, 1: LayerNorm (no affine)
+  const float* tab = nullptr; int stride = 0; int scale_off = 0, shift_off = 0;  // modulation
+  const int* tau_row = nullptr;
+  void* out = nullptr; int ldo = 0; int out_dtype = F32;
+};
+
+struct AttnArgs {
+  int n_heads = 0, n_kv_heads = 0, head_dim = 0, H = 0, B = 0;
+  const void* q = nullptr; int q_ld = 0;                 // q[(b*H + i) * q_ld + hq*dh + d]
+  const void* kp = nullptr; const void* vp = nullptr;    // prefix segment
+  int P = 0; long long kp_bstride = 0; int kp_ld = 0;    //   kp[b*kp_bstride + p*kp_ld + g*dh + d]
+  const void* kc = nullptr; const void* vc = nullptr;    // chunk segment (may be null)
+  int kc_ld = 0;                                         //   kc[(b*H + i) * kc_ld + g*dh + d]
+  const float* rope_cs = nullptr;                        // [H][dh/2][2] (cos, sin) at positions P+i
+  void* out = nullptr; int out_ld = 0;                   // out[(b*H + i) * out_ld + hq*dh + d]
+  int dtype = F32;
+  float scale = 1.f;
+};
+
+// Per-step, per-token plan entry (built on the host).
+enum PlanFlag { PF_ACTIVE = 1, PF_GHOST = 2, PF_RELEASE = 4, PF_EARLY = 8, PF_FROZEN = 16,
+                PF_NEXT_X = 32, PF_NEXT_G = 64, PF_NEXT_REL = 128, PF_LAST = 256 };
+
+struct PlanTok {
+  int flags;
+  float dx;       // 1/N_i (fp32) when active
+};
+
+struct EulerArgs {
+  int B = 0, H = 0, D = 0, k = 0;
+  const PlanTok* plan = nullptr;     // this step's [B][H]
+  const float* gstep = nullptr;      // [B] fp32(1/N*_b)
+  const int* last_step = nullptr;    // [B] N*_b
+  const int* tail_count = nullptr;   // [B] executable tail size (0: no GAC)
+  const unsigned char* gac_mask = nullptr;  // [D]
+  const int* tail_flag = nullptr;    // [B][H] 1 if corrected by GAC
+  const float* v = nullptr;          // [B*H][D]
+  float* x = nullptr; float* g = nullptr; float* u = nullptr; float* rel = nullptr;
+  float* final_out = nullptr; float* ghost_out = nullptr; float* E_out = nullptr;  // device
+  float* host_rel = nullptr;         // mapped pinned [B][H][D]
+  int* host_flags = nullptr;         // mapped pinned [B][UAD_MAX_STEPS + 1]
+  const int* epoch = nullptr;        // device scalar
+  int* nonfinite = nullptr;
+  int* evals = nullptr;                  // velocity evaluations consumed this chunk
+  unsigned long long* stamps = nullptr;  // [UAD_MAX_STEPS + 1], [0] = start
+};
+
+// kernels_simt.cu
+void launch_gemm_simt(const GemmArgs& a, cudaStream_t s);
+void launch_norm(const NormArgs& a, cudaStream_t s);
+void launch_attention(const AttnArgs& a, cudaStream_t s);
+void launch_euler(const EulerArgs& a, cudaStream_t s);
+void launch_begin(const float* noise, float* x, float* g, float* u, int n, int* nonfinite, int* evals,
+                  unsigned long long* stamps, cudaStream_t s);
+// dst[(n * mult + off) * K + k] = src[k * N + n]: transpose [K][N] -> rows of K, convert dtype
+void launch_relayout(const float* src, int K, int N, void* dst, int dtype, int mult, long long off,
+                     cudaStream_t s);
+size_t attention_smem_bytes(int dh);
+void launch_attention_prepare(int dh);  // opt in to > 48 KB dynamic shared memory (call once)
+void launch_convert(const void* src, int src_dtype, void* dst, int dst_dtype, long long n, cudaStream_t s);
+
+// gemm_tc.cu: tcgen05 projection GEMM (bf16 operands, fp32 accumulation in TMEM)
+constexpr int kTcMaxStages = 8;
+struct TcGemmArgs {
+  const void* w_tiled = nullptr;   // [N/128][K/64] blocks of 128 x 64 bf16, 128B-swizzled K-major
+  int M = 0, N = 0, K = 0, splits = 1;
+  int epi = EPI_STORE;
+  void* out = nullptr; int ldo = 0; int out_dtype = BF16;
+  const float* bias = nullptr;
+  float* resid = nullptr; int ldr = 0;
+  const float* gate_tab = nullptr; int gate_stride = 0; const int* tau_row = nullptr;
+  float* acc = nullptr;            // split-K accumulator [M][N] fp32, zero between launches
+  int* counters = nullptr;         // split-K arrival counters per output tile, zero between launches
+  int* err = nullptr;              // set to a nonzero code if a bounded wait gave up
+};
+size_t gemm_tc_smem_bytes(int stages);
+void gemm_tc_prepare();
+int gemm_tc_splits(int M, int N, int K, int sms);
+void launch_gemm_tc(const CUtensorMap* tmx, const TcGemmArgs& a, cudaStream_t s);
+// element (k, n) of src [K][N] -> row n * mult + off, column k of the tiled bf16 layout (K cols)
+void launch_relayout_tiled(const float* src, int K, int N, void* dst, int mult, long long off, cudaStream_t s);
+
+}  // namespace uad

@@ -1,0 +1,294 @@
+"""GPU parity: the CUDA path through the C ABI against the fp64 oracle on the same seeded
+inputs. Tolerance (stated in the spec of the path): max |a_gpu - a_oracle| / max |a_oracle|
+over each output set <= 1e-4 in fp32 mode and <= 2e-2 in bf16 mode; release steps and the
+evaluation count are compared exactly."""
+import itertools
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2609_37772_gb300 as uad
+from oracle.model import build_model
+from oracle.uad import denoise
+from uad_inputs import (ARCHS, draw_sweep_schedules, group_budgets, make_noise, make_prefix_kv,
+                        make_prefix_tokens, make_weights)
+
+pytestmark = pytest.mark.gpu
+TOL = {"f32": 1e-4, "bf16": 2e-2}
+TIMEOUT = 120_000_000
+
+
+def rel_err(got, ref):
+    return float(np.abs(np.asarray(got, np.float64) - ref).max() / max(1e-6, np.abs(ref).max()))
+
+
+def prefixes(a, B, seed=0):
+    if a.kind == "dit":
+        return [make_prefix_tokens(a, robot=b, seed=seed) for b in range(B)]
+    return [make_prefix_kv(a, robot=b, seed=seed) for b in range(B)]
+
+
+class Case:
+    def __init__(self, arch, B=1, seed=0, blob=None):
+        self.a, self.B = arch, B
+        self.blob = make_weights(arch, seed=seed) if blob is None else blob
+        self.pre = prefixes(arch, B, seed)
+        self.ex = uad.Expert(arch, self.blob, max_batch=B)
+        for b, p in enumerate(self.pre):
+            if arch.kind == "dit":
+                self.ex.set_prefix(b, p)
+            else:
+                self.ex.set_prefix(b, *p)
+        self._models = None
+
+    def models(self):
+        if self._models is None:
+            self._models = [build_model(self.a, self.blob, p) for p in self.pre]
+        return self._models
+
+    def gpu(self, noise, budgets, poll=True, **kw):
+        budgets = np.asarray(budgets, np.int32).reshape(self.B, -1)
+        self.ex.denoise(noise, budgets, **kw)
+        polled = []
+        if poll:
+            for b in range(self.B):
+                rc, out, ready, step = self.ex.poll(b, min_ready=self.a.chunk_len, timeout_us=TIMEOUT)
+                assert rc == self.a.chunk_len, rc
+                polled.append((out.copy(), step.copy()))
+        res = self.ex.finish(timeout_us=TIMEOUT)
+        res["polled"] = polled
+        return res
+
+    def oracle(self, noise, budgets, **kw):
+        budgets = np.asarray(budgets, np.int32).reshape(self.B, -1)
+        kw = {("n_exec" if k == "n_exec" else k): v for k, v in kw.items()}
+        if kw.get("n_exec", 0) == 0:
+            kw.pop("n_exec", None)
+        return [denoise(m.velocity, noise[b], budgets[b], **kw) for b, m in enumerate(self.models())]
+
+    def close(self):
+        self.ex.close()
+
+
+def check(case, res, refs, budgets, tol):
+    budgets = np.asarray(budgets).reshape(case.B, -1)
+    for b, ref in enumerate(refs):
+        assert rel_err(res["final"][b], ref["final"]) <= tol, ("final", b, rel_err(res["final"][b], ref["final"]))
+        assert rel_err(res["ghost"][b], ref["ghost"]) <= tol, ("ghost", b, rel_err(res["ghost"][b], ref["ghost"]))
+        if np.abs(ref["E"]).max() > 0:
+            assert np.abs(res["E"][b] - ref["E"]).max() <= tol * max(1e-6, np.abs(ref["final"]).max()) * 4
+        else:
+            assert np.all(res["E"][b] == 0)
+        if res["polled"]:
+            out, step = res["polled"][b]
+            assert np.array_equal(step, ref["release_step"].astype(np.int32))
+            # what the controller received is exactly what finish reports
+            assert np.array_equal(out, res["final"][b])
+    assert res["evals"] == max(r["evals"] for r in refs) and res["tr_extra_evals"] == 0
+
+
+# ---------------------------------------------------------------------------------------------
+@pytest.fixture(scope="module")
+def tiny():
+    c = Case(ARCHS["tiny"])
+    yield c
+    c.close()
+
+
+def test_tiny_fp32_urgent4_at5(tiny):
+    a = tiny.a
+    noise = make_noise(a)
+    bud = group_budgets(a.chunk_len, [(0, 3, 5), (4, a.chunk_len - 1, 10)])
+    res = tiny.gpu(noise, bud)
+    check(tiny, res, tiny.oracle(noise, bud), bud, TOL["f32"])
+
+
+@pytest.mark.parametrize("kw", [dict(tr=False, gac=False), dict(gac=False), dict(chunk_relative=True),
+                                dict(n_exec=10), dict(gac_mask=[1, 1, 1, 0, 0, 0, 0])])
+def test_tiny_variants(tiny, kw):
+    a = tiny.a
+    noise = make_noise(a, seed=3)
+    bud = group_budgets(a.chunk_len, [(0, 1, 2), (2, 5, 6), (6, a.chunk_len - 1, 8)])
+    res = tiny.gpu(noise, bud, **kw)
+    check(tiny, res, tiny.oracle(noise, bud, **kw), bud, TOL["f32"])
+
+
+def test_k1_exact_recovery_bitwise(tiny):
+    """Sec. 4.3: with K = 1, tail and ghost actions equal vanilla inference exactly."""
+    a = tiny.a
+    noise = make_noise(a, seed=5)
+    van = tiny.gpu(noise, np.full(a.chunk_len, 10), poll=False)
+    uadr = tiny.gpu(noise, group_budgets(a.chunk_len, [(0, 4, 1), (5, a.chunk_len - 1, 10)]), gac=False, poll=False)
+    assert np.array_equal(uadr["ghost"], van["final"])
+    assert np.array_equal(uadr["final"][:, 5:], van["final"][:, 5:])
+
+
+def test_uniform_schedule_is_vanilla(tiny):
+    a = tiny.a
+    noise = make_noise(a, seed=6)
+    bud = np.full(a.chunk_len, 7)
+    res = tiny.gpu(noise, bud)
+    assert np.array_equal(res["final"], res["ghost"]) and np.all(res["E"] == 0)
+    check(tiny, res, tiny.oracle(noise, bud), bud, TOL["f32"])
+
+
+def test_deterministic(tiny):
+    a = tiny.a
+    noise = make_noise(a, seed=8)
+    bud = group_budgets(a.chunk_len, [(0, 3, 3), (4, a.chunk_len - 1, 9)])
+    r1 = tiny.gpu(noise, bud, poll=False)
+    r2 = tiny.gpu(noise, bud, poll=False)
+    for k in ("final", "ghost", "E"):
+        assert np.array_equal(r1[k], r2[k])
+
+
+def test_released_actions_never_change(tiny):
+    """Poll the urgent group as soon as it is released, then compare with finish."""
+    a = tiny.a
+    noise = make_noise(a, seed=9)
+    bud = group_budgets(a.chunk_len, [(0, 3, 2), (4, a.chunk_len - 1, 10)])
+    tiny.ex.denoise(noise, bud[None])
+    rc, out, ready, step = tiny.ex.poll(0, min_ready=4, timeout_us=TIMEOUT)
+    assert rc >= 4 and ready[:4].all() and (step[:4] == 2).all()
+    snap = out[:4].copy()
+    res = tiny.ex.finish(timeout_us=TIMEOUT)
+    assert np.array_equal(res["final"][0, :4], snap)
+    rc2, out2, ready2, _ = tiny.ex.poll(0, min_ready=a.chunk_len, timeout_us=TIMEOUT)
+    assert rc2 == a.chunk_len and np.array_equal(out2[:4], snap)
+
+
+def test_device_buffers(tiny):
+    a = tiny.a
+    noise = make_noise(a, seed=10)
+    bud = group_budgets(a.chunk_len, [(0, 3, 5), (4, a.chunk_len - 1, 10)])
+    host = tiny.gpu(noise, bud, poll=False)
+    dn = torch.from_numpy(noise).cuda()
+    tiny.ex.denoise(dn, bud[None], stream=torch.cuda.current_stream())
+    f = torch.zeros_like(dn)
+    g = torch.zeros_like(dn)
+    e = torch.zeros(1, a.action_dim, device="cuda")
+    tiny.ex.finish(timeout_us=TIMEOUT, final=f, ghost=g, gac_error=e)
+    assert np.array_equal(f.cpu().numpy(), host["final"]) and np.array_equal(g.cpu().numpy(), host["ghost"])
+
+
+def test_errors_are_reported(tiny):
+    a = tiny.a
+    noise = make_noise(a)
+    with pytest.raises(uad.UADError) as ei:
+        tiny.ex.finish()
+    assert ei.value.code == uad.UAD_ESTATE
+    with pytest.raises(uad.UADError) as ei:
+        tiny.ex.denoise(noise, np.zeros(a.chunk_len))
+    assert ei.value.code == uad.UAD_EINVAL
+    with pytest.raises(uad.UADError) as ei:
+        tiny.ex.denoise(noise, np.full(a.chunk_len, 3), tr=False, gac=True)
+    assert ei.value.code == uad.UAD_EINVAL
+    with pytest.raises(uad.UADError):
+        tiny.ex.denoise(noise, np.full(a.chunk_len, 3), n_star=4)
+    tiny.ex.denoise(noise, np.full(a.chunk_len, 3)[None])
+    with pytest.raises(uad.UADError) as ei:
+        tiny.ex.denoise(noise, np.full(a.chunk_len, 3)[None])
+    assert ei.value.code == uad.UAD_ESTATE
+    tiny.ex.finish(timeout_us=TIMEOUT)
+
+
+def test_nonfinite_is_reported(tiny):
+    a = tiny.a
+    noise = make_noise(a)
+    noise[0, 2, 1] = np.nan
+    tiny.ex.denoise(noise, np.full(a.chunk_len, 2)[None])
+    res = tiny.ex.finish(timeout_us=TIMEOUT, check=False)
+    assert res["rc"] == uad.UAD_ENONFINITE and res["nonfinite"] > 0
+
+
+def test_brute_force_small_chunks():
+    """All 4^3 budget assignments on a 3-action chunk with 2-dim actions (fp32)."""
+    a = ARCHS["tiny"].replace(chunk_len=3, action_dim=2, n_layers=1)
+    c = Case(a, seed=4)
+    noise = make_noise(a, seed=4)
+    try:
+        for bud in itertools.product(range(1, 5), repeat=3):
+            res = c.gpu(noise, bud)
+            check(c, res, c.oracle(noise, bud), bud, TOL["f32"])
+    finally:
+        c.close()
+
+
+def test_fp32_rope_gqa_arch():
+    a = ARCHS["tiny_f32_rope"]
+    c = Case(a, seed=2)
+    try:
+        noise = make_noise(a, seed=2)
+        bud = group_budgets(a.chunk_len, [(0, 3, 4), (4, 9, 7), (10, a.chunk_len - 1, 10)])
+        check(c, c.gpu(noise, bud), c.oracle(noise, bud), bud, TOL["f32"])
+    finally:
+        c.close()
+
+
+@pytest.mark.parametrize("name", ["pi0_small", "dit_small"])
+def test_bf16_small_archs(name):
+    a = ARCHS[name]
+    c = Case(a, seed=1)
+    try:
+        noise = make_noise(a, seed=1)
+        H = a.chunk_len
+        bud = group_budgets(H, [(0, 3, 4), (4, H // 2, 7), (H // 2 + 1, H - 1, 10)])
+        check(c, c.gpu(noise, bud), c.oracle(noise, bud), bud, TOL["bf16"])
+    finally:
+        c.close()
+
+
+def test_batched_robots_own_schedules():
+    a = ARCHS["pi0_small"]
+    B = 4
+    c = Case(a, B=B, seed=7)
+    try:
+        noise = make_noise(a, batch=B, seed=7)
+        bud = draw_sweep_schedules(a.chunk_len, B, seed=7)
+        check(c, c.gpu(noise, bud), c.oracle(noise, bud), bud, TOL["bf16"])
+    finally:
+        c.close()
+
+
+# ---- full-size workloads -----------------------------------------------------------------------
+def test_pi0_full_three_groups():
+    """pi0-like bf16 expert, B = 1, groups 0-9 @ 4, 10-24 @ 7, 25-49 @ 10 (all outputs)."""
+    a = ARCHS["pi0"]
+    c = Case(a)
+    try:
+        noise = make_noise(a)
+        bud = group_budgets(50, [(0, 9, 4), (10, 24, 7), (25, 49, 10)])
+        check(c, c.gpu(noise, bud), c.oracle(noise, bud), bud, TOL["bf16"])
+    finally:
+        c.close()
+
+
+@pytest.mark.parametrize("ns", [4, 16])
+def test_dit_full(ns):
+    a = ARCHS["dit"]
+    c = Case(a)
+    try:
+        noise = make_noise(a)
+        bud = group_budgets(16, [(0, 3, ns // 2), (4, 15, ns)])
+        check(c, c.gpu(noise, bud), c.oracle(noise, bud), bud, TOL["bf16"])
+    finally:
+        c.close()
+
+
+def test_tensor_core_gemm_matches_cuda_core_gemm(monkeypatch):
+    """The tcgen05 projection path against the CUDA-core GEMM on the same bf16 operands."""
+    a = ARCHS["pi0_small"]
+    blob = make_weights(a, seed=11)
+    noise = make_noise(a, seed=11)
+    bud = group_budgets(a.chunk_len, [(0, 9, 3), (10, a.chunk_len - 1, 6)])
+    outs = []
+    for mode in ("simt", "tc"):
+        monkeypatch.setenv("UAD_GEMM", mode)
+        c = Case(a, seed=11, blob=blob)
+        try:
+            outs.append(c.gpu(noise, bud, poll=False))
+        finally:
+            c.close()
+    for k in ("final", "ghost"):
+        assert rel_err(outs[1][k], outs[0][k].astype(np.float64)) <= 5e-3, k

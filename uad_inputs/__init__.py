@@ -8,7 +8,8 @@ prefix tokens, initial noise and urgency schedules.
 Recipe (stands in for the paper's pretrained SmolVLA / pi0.5 checkpoints and the
 LIBERO / Meta-World observations, which are not available):
 
-* weights and biases ~ N(0, 0.02), drawn in blob order from one numpy PCG64 stream;
+* weights and biases ~ N(0, 0.02), drawn in blob order in blocks of 4 Mi values, each
+  block from its own numpy PCG64 stream keyed (seed, 1, block);
   for bf16 architectures every value is rounded to the nearest bf16 (ties to even), so
   the fp32 blob holds exactly representable bf16 values;
 * prefix K/V (attention-prefix architectures) ~ N(0, 1) per layer, [L, P, Hkv, dh],
@@ -117,15 +118,31 @@ def _rng(seed: int, *key: int) -> np.random.Generator:
     return np.random.Generator(np.random.PCG64(np.random.SeedSequence([seed, *key])))
 
 
+_BLOCK = 1 << 22
+
+
+def _normal_blocks(n: int, seed: int, tag: int, std: float, bf16: bool) -> np.ndarray:
+    """n values ~ N(0, std^2), drawn in blocks of 4 Mi values, block j from its own PCG64
+    stream keyed (seed, tag, j): the result does not depend on how many threads fill it."""
+    import concurrent.futures as cf
+    import os
+    out = np.empty(n, dtype=np.float32)
+
+    def fill(j):
+        lo, hi = j * _BLOCK, min(n, (j + 1) * _BLOCK)
+        blk = _rng(seed, tag, j).standard_normal(hi - lo, dtype=np.float32)
+        blk *= np.float32(std)
+        out[lo:hi] = round_to_bf16(blk) if bf16 else blk
+
+    nblk = (n + _BLOCK - 1) // _BLOCK
+    with cf.ThreadPoolExecutor(max_workers=min(16, os.cpu_count() or 1)) as ex:
+        list(ex.map(fill, range(nblk)))
+    return out
+
+
 def make_weights(a: Arch, seed: int = 0, std: float = 0.02) -> np.ndarray:
     """Flat fp32 weight blob in weight_specs order, N(0, std), bf16-exact for bf16 archs."""
-    g = _rng(seed, 1)
-    n = weight_count(a)
-    blob = g.standard_normal(n, dtype=np.float32)
-    blob *= np.float32(std)
-    if a.dtype == "bf16":
-        blob = round_to_bf16(blob)
-    return blob
+    return _normal_blocks(weight_count(a), seed, 1, std, a.dtype == "bf16")
 
 
 def blob_from_weights(a: Arch, weights: dict) -> np.ndarray:
