@@ -1,0 +1,371 @@
+#!/usr/bin/env python
+"""Benchmark of the UAD hot path on GB300: one "step" = one action chunk denoised end to end
+(N* velocity-network evaluations with per-action Euler steps, early release, Trajectory
+Reconciliation and Ghost Action Correction) for the configured robots.
+
+Default workload: the pi0-like bf16 action expert at batch 1 (18 layers, width 1024, GeGLU 4096,
+8 query / 1 KV heads of 256, 816 prefix tokens, H = 50, D = 32) with three release groups
+(actions 0-9 after 4 steps, 10-24 after 7, 25-49 after 10). Inputs are seeded synthetic data.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload NAME]
+
+Prints one JSON line (rank 0). Multi-GPU runs are independent replicas (one robot batch per
+rank, no collective on the data path); value = all ranks' action tokens / max-over-ranks time.
+"""
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from uad_inputs import (ARCHS, draw_sweep_schedules, group_budgets, make_noise, make_prefix_kv,  # noqa: E402
+                        make_prefix_tokens, make_weights)
+
+WORKLOADS = {
+    "pi0-b1": dict(arch="pi0", batch=1, groups=[(0, 9, 4), (10, 24, 7), (25, 49, 10)], t_act_ms=10.0,
+                   desc="pi0-like bf16 expert, B=1, groups 0-9@4 10-24@7 25-49@10, TR+GAC, S=H=50"),
+    "pi0-vanilla": dict(arch="pi0", batch=1, groups=[(0, 49, 10)], t_act_ms=10.0,
+                        desc="pi0-like bf16 expert, B=1, vanilla N=10 (uniform schedule)"),
+    "dit-k4": dict(arch="dit", batch=1, groups=[(0, 3, 2), (4, 15, 4)], t_act_ms=10.0,
+                   desc="DiT bf16 head, B=1, first 4 actions after 2 of 4 steps"),
+    "dit-k16": dict(arch="dit", batch=1, groups=[(0, 3, 8), (4, 15, 16)], t_act_ms=10.0,
+                    desc="DiT bf16 head, B=1, first 4 actions after 8 of 16 steps"),
+    "tiny": dict(arch="tiny", batch=1, groups=[(0, 3, 5), (4, 15, 10)], t_act_ms=10.0,
+                 desc="tiny fp32 expert, B=1, first 4 actions after 5 of 10 steps"),
+}
+for _b in (4, 16, 64):
+    WORKLOADS[f"pi0-b{_b}"] = dict(arch="pi0", batch=_b, groups=None, t_act_ms=10.0,
+                                   desc=f"pi0-like bf16 expert, B={_b} robots, schedules drawn from the sweep grid")
+
+# ncu DRAM traffic per launch of the dominant kernel class, with the sha1 of the source file it
+# was measured on (reported as null once that source changes). Filled from profiles/.
+TRAFFIC = {}
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d["hbm_gbs"], d["bf16_tflops"], d.get("bf16_tflops_sustained"), "measured"
+    return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def budgets_for(wl, a, rank=0):
+    B = wl["batch"]
+    if wl["groups"] is None:
+        return draw_sweep_schedules(a.chunk_len, B, seed=1000 + rank)
+    return np.tile(group_budgets(a.chunk_len, wl["groups"]), (B, 1)).astype(np.int32)
+
+
+def aal_ms(ready_ms, t_act, n_exec):
+    """Average action availability latency under the control clock (Sec. 5.1, App. C.3)."""
+    waits, request, start = [], 0.0, 0.0
+    for i, r in enumerate(ready_ms[:n_exec]):
+        if i > 0:
+            request = start + t_act
+        start = max(request, r)
+        waits.append(max(0.0, r - request))
+    return sum(waits) / n_exec
+
+
+class Clocks:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index, self.p = index, None
+
+    def __enter__(self):
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                                       "--format=csv,noheader,nounits", "-lms", "200"],
+                                      stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.p = None
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.p:
+            self.p.terminate()
+            try:
+                self.out, _ = self.p.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.p.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in (self.out or "").splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = max(mx, float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx or None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = os.environ.get("UAD_BENCH_BACKEND", "nccl")
+        dist.init_process_group(backend)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x, world, device="cpu"):
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# -------------------------------------------------------------------------------------------
+def oracle_chunks(wl, seconds, max_chunks=None):
+    """Time the CPU oracle, as it stands, on whole chunks of robot 0 of this workload."""
+    from oracle.model import build_model
+    from oracle.uad import denoise
+    a = ARCHS[wl["arch"]]
+    blob = make_weights(a)
+    pre = make_prefix_tokens(a) if a.kind == "dit" else make_prefix_kv(a)
+    model = build_model(a, blob, pre)
+    bud = budgets_for(wl, a)[0]
+    x0 = make_noise(a, 1)[0]
+    times = []
+    t_end = time.perf_counter() + seconds
+    while True:
+        t0 = time.perf_counter()
+        denoise(model.velocity, x0, bud)
+        times.append(time.perf_counter() - t0)
+        if time.perf_counter() >= t_end or (max_chunks and len(times) >= max_chunks):
+            break
+    return a, times
+
+
+def run_reference(args, wl, world, rank):
+    if rank != 0:
+        return 0
+    a, times = oracle_chunks(wl, float("inf"), max_chunks=args.warmup + args.steps)
+    timed = times[args.warmup:] if len(times) > args.warmup else times
+    per = statistics.mean(timed)
+    value = a.chunk_len / per
+    cores = os.cpu_count()
+    line = {
+        "impl": "reference", "metric": "action-tokens/s", "value": value, "unit": "tokens/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": per * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded random-init weights, N(0,1) prefix and noise)",
+        "config": {"workload": wl["desc"], "global_batch": 1, "seq_len": a.chunk_len, "parallelism": "none"},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                         "sample": "one full chunk of robot 0 per step (fp64 numpy oracle)"},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# -------------------------------------------------------------------------------------------
+def run_ours(args, wl, world, rank, local):
+    import torch
+    import paper_2609_37772_gb300 as uad
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    a = ARCHS[wl["arch"]]
+    B, H, D = wl["batch"], a.chunk_len, a.action_dim
+    blob = make_weights(a)
+    ex = uad.Expert(a, blob, max_batch=B)
+    for b in range(B):
+        robot = rank * B + b
+        if a.kind == "dit":
+            ex.set_prefix(b, make_prefix_tokens(a, robot=robot))
+        else:
+            ex.set_prefix(b, *make_prefix_kv(a, robot=robot))
+    bud = budgets_for(wl, a, rank)
+    n_star = int(bud.max())
+    ex.prepare_times(max(n_star, 10))            # model load: conditioning for every j/n
+    noise_np = make_noise(a, B, seed=rank)
+    noise = torch.from_numpy(noise_np).to(dev)
+    fin = torch.empty(B, H, D, device=dev)
+    gho = torch.empty(B, H, D, device=dev)
+    err = torch.empty(B, D, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        ex.denoise(noise, bud, stream=stream)
+        return ex.finish(timeout_us=60_000_000, final=fin, ghost=gho, gac_error=err)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    step_times = []
+    with Clocks(local) as clk:
+        barrier(world)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(args.steps):
+            step()
+            step_times.append(ex.step_times())
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier(world)
+    ms_total = e0.elapsed_time(e1)
+    ms_total_max = max_over_ranks(ms_total, world, dev if world > 1 and os.environ.get("UAD_BENCH_BACKEND", "nccl") == "nccl" else "cpu")
+    ms_per_step = ms_total_max / args.steps
+    value = world * B * H * args.steps / (ms_total_max / 1e3)
+
+    # device-side release times of robot 0 (global timer, relative to the chunk's first kernel)
+    st = np.array(step_times)                      # [K][N*]
+    ready = [[float(st[c][int(bud[0][i]) - 1]) for i in range(H)] for c in range(len(st))]
+    aal = statistics.mean(aal_ms(r, wl["t_act_ms"], H) for r in ready)
+    first = statistics.mean(r[0] for r in ready)
+    ms_per_eval = statistics.mean(float(s[-1]) / n_star for s in st)
+
+    # ---- end to end through the C ABI with host buffers (pinned), host clock ----
+    noise_h = torch.from_numpy(noise_np).pin_memory()
+    fin_h = torch.empty(B, H, D).pin_memory()
+    gho_h = torch.empty(B, H, D).pin_memory()
+    err_h = torch.empty(B, D).pin_memory()
+    order = sorted(set(int(x) for x in bud[0]))
+    counts = [int((bud[0] <= g).sum()) for g in order]
+    host_ready = []
+    for _ in range(args.warmup):
+        ex.denoise(noise_h, bud)
+        ex.finish(timeout_us=60_000_000, final=fin_h, ghost=gho_h, gac_error=err_h)
+    torch.cuda.synchronize()
+    barrier(world)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        ts = time.perf_counter()
+        ex.denoise(noise_h, bud)
+        marks = []
+        for cnt in counts:                        # controller thread: wait for each release group
+            ex.poll(0, min_ready=cnt, timeout_us=60_000_000)
+            marks.append((time.perf_counter() - ts) * 1e3)
+        ex.finish(timeout_us=60_000_000, final=fin_h, ghost=gho_h, gac_error=err_h)
+        host_ready.append([marks[order.index(int(n))] for n in bud[0]])
+    t_e2e = time.perf_counter() - t0
+    barrier(world)
+    t_e2e = max_over_ranks(t_e2e, world)
+    e2e_value = world * B * H * args.steps / t_e2e
+    aal_host = statistics.mean(aal_ms(r, wl["t_act_ms"], H) for r in host_ready)
+    al = lambda x: (x + 15) & ~15                 # the library's plan block, uploaded per chunk
+    o = al(n_star * B * H * 8)
+    o = al(o + n_star * B * H * 4)
+    for extra in (B * 4, B * 4, B * 4, B * H * 4, D, 4):
+        o = al(o + extra)
+    plan_bytes = o
+    h2d = noise_np.nbytes + plan_bytes
+    d2h = fin_h.numel() * 4 + gho_h.numel() * 4 + err_h.numel() * 4
+
+    # ---- per-kernel CUDA-event profile of one chunk (eager replay on the worker stream) ----
+    prof = ex.profile(noise, bud)
+    hbm, bf16, bf16_sus, src = peaks()
+    dom = max(prof, key=lambda r: r["total_ms"])
+    achieved = dom["bytes"] / (dom["total_ms"] / 1e3) / 1e9
+    eval_bytes = sum(r["bytes"] for r in prof) / n_star
+    eval_flops = sum(r["flops"] for r in prof) / n_star
+    tkey = f"{dom['name']}@{args.workload}"
+    traffic = None
+    if tkey in TRAFFIC:
+        per_launch, path, sha = TRAFFIC[tkey]
+        cur = hashlib.sha1(open(os.path.join(ROOT, path), "rb").read()).hexdigest()
+        traffic = per_launch if cur == sha else None
+    roofline = {"bound": "hbm", "kernel": dom["name"], "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                "frac": achieved / hbm, "traffic": traffic,
+                "peak_source": f"{src} hbm_gbs (MEASURED_PEAKS.json)" if src == "measured" else "fallback",
+                "bytes_per_launch": dom["bytes"] / dom["launches"],
+                "avg_launch_us": dom["total_ms"] * 1e3 / dom["launches"],
+                "step": {"algorithmic_bytes_per_eval": eval_bytes, "flops_per_eval": eval_flops,
+                         "ms_per_eval": ms_per_eval,
+                         "achieved_gbs": eval_bytes / (ms_per_eval / 1e3) / 1e9,
+                         "frac": eval_bytes / (ms_per_eval / 1e3) / 1e9 / hbm}}
+    kernels = sorted(({"name": r["name"], "launches": r["launches"], "ms": round(r["total_ms"], 4),
+                       "gbs": round(r["bytes"] / max(r["total_ms"], 1e-9) / 1e6, 1)} for r in prof),
+                     key=lambda r: -r["ms"])
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        _, times = oracle_chunks(wl, args.cpu_seconds)
+        cpu = {"value": H / statistics.mean(times), "unit": "tokens/s", "cores": os.cpu_count(),
+               "kind": "oracle", "sample": f"{len(times)} full chunk(s) of robot 0 (fp64 numpy oracle), "
+                                           f"{sum(times):.1f} s"}
+
+    launches = ex.launches_per_chunk(B, n_star) * args.steps
+    ex.close()
+    if rank != 0:
+        return 0
+    line = {
+        "metric": "action-tokens/s", "value": value, "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if a.dtype == "bf16" else "f32",
+        "data": "synthetic (seeded random-init weights ~N(0,0.02), prefix KV and noise ~N(0,1))",
+        "config": {"workload": wl["desc"], "model": a.name, "global_batch": B * world, "seq_len": H,
+                   "parallelism": f"replicas x{world}" if world > 1 else "none",
+                   "l2": "no flush: every evaluation streams the full weight set, larger than L2"},
+        "aal_ms": aal, "first_action_ms": first, "ms_per_eval": ms_per_eval,
+        "aal_definition": "device release times, T_act = %g ms, S = H" % wl["t_act_ms"],
+        "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
+                "d2h_bytes_per_step": int(d2h), "aal_ms_host": aal_host,
+                "first_action_ms_host": statistics.mean(r[0] for r in host_ready)},
+        "roofline": roofline, "kernels": kernels, "gpu_launches": launches,
+        "clocks": clk.summary(), "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="pi0-b1", choices=sorted(WORKLOADS))
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    wl = WORKLOADS[args.workload]
+    world, rank, local = dist_setup()
+    try:
+        if args.impl == "reference":
+            return run_reference(args, wl, world, rank)
+        return run_ours(args, wl, world, rank, local)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    sys.exit(main())

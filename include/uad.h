@@ -161,6 +161,22 @@ int uad_step_times(const uad_ctx* ctx, double* ms, int32_t max_entries);
  * (excluding one-time time-conditioning fills). */
 int uad_launches_per_chunk(const uad_ctx* ctx, int32_t batch, int32_t n_star);
 
+/* Per-kernel profile of one chunk (measurement support, not part of the method). */
+typedef struct uad_kernel_stat {
+  char name[32];          /* kernel class, e.g. "gate_up_proj", "attention", "euler_tr_gac" */
+  int32_t launches;       /* launches of this class in the chunk */
+  int32_t pad;
+  double total_ms;        /* sum of CUDA-event durations of those launches */
+  double bytes;           /* algorithmic HBM bytes of those launches (operands read once) */
+  double flops;           /* algorithmic flops of those launches */
+} uad_kernel_stat;
+
+/* Run one chunk like uad_denoise + uad_finish, but launched eagerly (no graph) on the
+ * library's worker stream with a CUDA event pair around every kernel, and return per-class
+ * totals in out[0..n). Returns n, or an error. Synchronous; results are discarded. */
+int uad_profile_chunk(uad_ctx* ctx, const float* noise, const uad_schedule* sched,
+                      uad_kernel_stat* out, int32_t max_stats, int64_t timeout_us);
+
 void uad_destroy(uad_ctx* ctx);
 const char* uad_last_error(const uad_ctx* ctx);
 

@@ -40,6 +40,11 @@ class uad_stats(C.Structure):
     _fields_ = [("evals", _I32), ("n_star", _I32), ("nonfinite", _I32), ("tr_extra_evals", _I32)]
 
 
+class uad_kernel_stat(C.Structure):
+    _fields_ = [("name", C.c_char * 32), ("launches", _I32), ("pad", _I32), ("total_ms", C.c_double),
+                ("bytes", C.c_double), ("flops", C.c_double)]
+
+
 def _fn(name, res, *args):
     f = getattr(_lib, name)
     f.restype = res
@@ -59,10 +64,11 @@ uad_step_times = _fn("uad_step_times", C.c_int, _P, _P, _I32)
 uad_launches_per_chunk = _fn("uad_launches_per_chunk", C.c_int, _P, _I32, _I32)
 uad_destroy = _fn("uad_destroy", None, _P)
 uad_plan_step = _fn("uad_plan_step", C.c_int, _P, _I32, _I32, _I32, _P, _P, _P)
+uad_profile_chunk = _fn("uad_profile_chunk", C.c_int, _P, _P, C.POINTER(uad_schedule), _P, _I32, C.c_int64)
 
 EXPORTS = ["uad_version", "uad_last_error", "uad_init", "uad_set_prefix_kv", "uad_prepare_times",
            "uad_denoise", "uad_poll_released", "uad_finish", "uad_step_times",
-           "uad_launches_per_chunk", "uad_destroy", "uad_plan_step"]
+           "uad_launches_per_chunk", "uad_destroy", "uad_plan_step", "uad_profile_chunk"]
 
 
 class UADError(RuntimeError):
@@ -141,19 +147,35 @@ class Expert:
     def prepare_times(self, max_budget):
         return self._check(uad_prepare_times(self.h, max_budget), "prepare_times")
 
-    def denoise(self, noise, budgets, n_exec=0, tr=True, gac=True, chunk_relative=False,
-                gac_mask=None, n_star=0, stream=None):
+    def _schedule(self, budgets, n_exec, tr, gac, chunk_relative, gac_mask):
         b = np.ascontiguousarray(budgets, dtype=np.int32).reshape(-1, self.H)
         m = None if gac_mask is None else np.ascontiguousarray(gac_mask, dtype=np.uint8)
         sc = uad_schedule(budgets=b.ctypes.data_as(C.POINTER(_I32)), batch=b.shape[0], n_exec=n_exec,
                           tr=int(tr), gac=int(gac), chunk_relative=int(chunk_relative),
                           gac_mask=None if m is None else m.ctypes.data_as(C.POINTER(C.c_uint8)))
+        return sc, (b, m)
+
+    def denoise(self, noise, budgets, n_exec=0, tr=True, gac=True, chunk_relative=False,
+                gac_mask=None, n_star=0, stream=None):
+        sc, keep = self._schedule(budgets, n_exec, tr, gac, chunk_relative, gac_mask)
         if isinstance(noise, np.ndarray):
             noise = np.ascontiguousarray(noise, dtype=np.float32)
         self._keep = noise
-        self._B = b.shape[0]
+        self._B = keep[0].shape[0]
         return self._check(uad_denoise(self.h, _ptr(noise), C.byref(sc), n_star, _stream_handle(stream)),
                            "denoise")
+
+    def profile(self, noise, budgets, n_exec=0, tr=True, gac=True, chunk_relative=False, gac_mask=None,
+                timeout_us=120_000_000):
+        """Per-kernel-class CUDA-event times of one eagerly launched chunk."""
+        sc, keep = self._schedule(budgets, n_exec, tr, gac, chunk_relative, gac_mask)
+        if isinstance(noise, np.ndarray):
+            noise = np.ascontiguousarray(noise, dtype=np.float32)
+        self._B = keep[0].shape[0]
+        stats = (uad_kernel_stat * 64)()
+        n = self._check(uad_profile_chunk(self.h, _ptr(noise), C.byref(sc), stats, 64, int(timeout_us)), "profile")
+        return [dict(name=st.name.decode(), launches=st.launches, total_ms=st.total_ms, bytes=st.bytes,
+                     flops=st.flops) for st in stats[:n]]
 
     def poll(self, robot, min_ready=1, timeout_us=0, out=None):
         out = np.zeros((self.H, self.D), np.float32) if out is None else out

@@ -109,6 +109,13 @@ struct uad_ctx {
   float* host_rel = nullptr; float* host_rel_dev = nullptr;
   int* host_flags = nullptr; int* host_flags_dev = nullptr;
 
+  // per-kernel profiling (uad_profile_chunk): events around every launch of one eager chunk
+  struct ProfRec { const char* name; double bytes, flops; int ev0, ev1; };
+  bool prof_on = false;
+  std::vector<ProfRec> prof;
+  std::vector<cudaEvent_t> prof_ev;
+  int prof_next = 0;
+
   cudaStream_t worker = nullptr;
   cudaEvent_t ev_in = nullptr, ev_done = nullptr;
   std::map<std::pair<int, int>, cudaGraphExec_t> graphs;
@@ -303,6 +310,36 @@ void plan_token(int k, int n_i, int ns, bool tr, int* flags, std::pair<int, int>
   *flags = f;
 }
 
+// Brackets one kernel launch with timing events when profiling is on.
+struct Mark {
+  uad_ctx* c;
+  cudaStream_t s;
+  Mark(uad_ctx* c_, cudaStream_t s_, const char* name, double bytes, double flops) : c(c_), s(s_) {
+    if (!c->prof_on) return;
+    while ((int)c->prof_ev.size() < c->prof_next + 2) {
+      cudaEvent_t e;
+      cudaEventCreate(&e);
+      c->prof_ev.push_back(e);
+    }
+    c->prof.push_back({name, bytes, flops, c->prof_next, c->prof_next + 1});
+    cudaEventRecord(c->prof_ev[c->prof_next], s);
+    c->prof_next += 2;
+  }
+  ~Mark() {
+    if (c->prof_on) cudaEventRecord(c->prof_ev[c->prof.back().ev1], s);
+  }
+};
+
+// Algorithmic HBM bytes of one projection: weights + activations in + output (+ residual r/w).
+double gemm_bytes(const GemmArgs& g, int wes) {
+  const double aes = g.a_dtype == BF16 ? 2 : 4, oes = g.out_dtype == BF16 ? 2 : 4;
+  double b = (double)g.N * g.K * wes + (double)g.M * g.K * aes;
+  if (g.epi == EPI_RESID_GATE) b += 8.0 * g.M * g.N;
+  else if (g.epi == EPI_GEGLU) b += oes * g.M * (g.N / 2);
+  else b += oes * (double)g.M * g.N;
+  return b;
+}
+
 // out = epi(A Wt^T): tensor cores when the weight is tiled, CUDA cores otherwise.
 void gemm(uad_ctx* c, const Lin& w, GemmArgs g, cudaStream_t s) {
   g.W = w.w;
@@ -366,14 +403,14 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
   const int W6 = 6 * W;
   const bool dit = a.kind == UAD_KIND_DIT;
 
-  launch_begin(c->noise, c->x, c->g, c->u, M * D, c->nonfinite, c->evals, c->stamps, s);
+  { Mark mk(c, s, "begin", 12.0 * M * D, 0); launch_begin(c->noise, c->x, c->g, c->u, M * D, c->nonfinite, c->evals, c->stamps, s); }
   for (int k = 1; k <= n_steps; ++k) {
     const int* tr = tau + (size_t)(k - 1) * M;
     GemmArgs gi;
     gi.A = c->u; gi.lda = D; gi.a_dtype = F32; gi.w_dtype = dt;
     gi.M = M; gi.N = W; gi.K = D; gi.epi = EPI_STORE; gi.out = c->h; gi.ldo = W; gi.bias = c->b_in;
     if (dit) { gi.add_rows = c->pos_code; gi.add_mod = H; }
-    gemm(c, c->w_in, gi, s);
+    { Mark mk(c, s, "in_proj", gemm_bytes(gi, c->es), 2.0 * M * W * D); gemm(c, c->w_in, gi, s); }
     for (int l = 0; l < a.n_layers; ++l) {
       const LayerW& w = c->L[l];
       const int base = l * W6;
@@ -382,11 +419,11 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
       na.stride = c->rowlen; na.tau_row = tr; na.out = c->y; na.ldo = W; na.out_dtype = dt;
       na.scale_off = dit ? base + W : base;
       na.shift_off = dit ? base : base + W;
-      launch_norm(na, s);
+      { Mark mk(c, s, "norm", (4.0 + c->es) * M * W, 0); launch_norm(na, s); }
       GemmArgs gq;
       gq.A = c->y; gq.lda = W; gq.a_dtype = dt; gq.w_dtype = dt;
       gq.M = M; gq.N = c->qkvd; gq.K = W; gq.out = c->qkv; gq.ldo = c->qkvd; gq.out_dtype = dt;
-      gemm(c, w.wqkv, gq, s);
+      { Mark mk(c, s, "qkv_proj", gemm_bytes(gq, c->es), 2.0 * M * gq.N * W); gemm(c, w.wqkv, gq, s); }
       AttnArgs at;
       at.n_heads = a.n_heads; at.n_kv_heads = a.n_kv_heads; at.head_dim = a.head_dim; at.H = H; at.B = B;
       at.q = c->qkv; at.q_ld = c->qkvd;
@@ -400,20 +437,25 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
         at.P = a.prefix_len; at.kp_bstride = (long long)a.n_layers * a.prefix_len * c->kvd;
         at.kp_ld = c->kvd; at.rope_cs = a.rope ? c->rope_cs : nullptr;
       }
-      launch_attention(at, s);
+      {
+        const double keys = (double)(at.P + H);
+        const double by = c->es * ((double)B * at.P * c->kvd * 2 + (double)M * (2 * c->qd + 2 * c->kvd));
+        Mark mk(c, s, dit ? "self_attn" : "attention", by, 4.0 * M * a.n_heads * keys * a.head_dim);
+        launch_attention(at, s);
+      }
       GemmArgs go;
       go.A = c->o; go.lda = c->qd; go.a_dtype = dt; go.w_dtype = dt;
       go.M = M; go.N = W; go.K = c->qd; go.epi = EPI_RESID_GATE; go.resid = c->h; go.ldr = W;
       go.gate_tab = c->tab + base + 2 * W; go.gate_stride = c->rowlen; go.tau_row = tr;
-      gemm(c, w.wo, go, s);
+      { Mark mk(c, s, "o_proj", gemm_bytes(go, c->es), 2.0 * M * W * c->qd); gemm(c, w.wo, go, s); }
       if (dit) {
         NormArgs nc = na;
         nc.tab = nullptr;
-        launch_norm(nc, s);
+        { Mark mk(c, s, "norm", (4.0 + c->es) * M * W, 0); launch_norm(nc, s); }
         GemmArgs gc;
         gc.A = c->y; gc.lda = W; gc.a_dtype = dt; gc.w_dtype = dt;
         gc.M = M; gc.N = c->qd; gc.K = W; gc.out = c->qc; gc.ldo = c->qd; gc.out_dtype = dt;
-        gemm(c, w.wqc, gc, s);
+        { Mark mk(c, s, "q_cross_proj", gemm_bytes(gc, c->es), 2.0 * M * c->qd * W); gemm(c, w.wqc, gc, s); }
         AttnArgs ac;
         ac.n_heads = a.n_heads; ac.n_kv_heads = a.n_heads; ac.head_dim = a.head_dim; ac.H = H; ac.B = B;
         ac.q = c->qc; ac.q_ld = c->qd;
@@ -421,39 +463,43 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
         ac.vp = static_cast<const char*>(c->vpre) + (size_t)l * a.prefix_len * c->qd * c->es;
         ac.P = a.prefix_len; ac.kp_bstride = (long long)a.n_layers * a.prefix_len * c->qd; ac.kp_ld = c->qd;
         ac.out = c->o; ac.out_ld = c->qd; ac.dtype = dt; ac.scale = at.scale;
-        launch_attention(ac, s);
+        {
+          const double by = c->es * ((double)B * ac.P * c->qd * 2 + 2.0 * M * c->qd);
+          Mark mk(c, s, "cross_attn", by, 4.0 * M * a.n_heads * (double)ac.P * a.head_dim);
+          launch_attention(ac, s);
+        }
         GemmArgs gco;
         gco.A = c->o; gco.lda = c->qd; gco.a_dtype = dt; gco.w_dtype = dt;
         gco.M = M; gco.N = W; gco.K = c->qd; gco.epi = EPI_RESID_GATE; gco.resid = c->h; gco.ldr = W;
-        gemm(c, w.woc, gco, s);
+        { Mark mk(c, s, "o_cross_proj", gemm_bytes(gco, c->es), 2.0 * M * W * c->qd); gemm(c, w.woc, gco, s); }
       }
       NormArgs n2 = na;
       n2.scale_off = dit ? base + 4 * W : base + 3 * W;
       n2.shift_off = dit ? base + 3 * W : base + 4 * W;
-      launch_norm(n2, s);
+      { Mark mk(c, s, "norm", (4.0 + c->es) * M * W, 0); launch_norm(n2, s); }
       GemmArgs g1;
       g1.A = c->y; g1.lda = W; g1.a_dtype = dt; g1.w_dtype = dt; g1.M = M; g1.K = W;
       g1.out = c->act; g1.ldo = F; g1.out_dtype = dt;
       if (dit) { g1.N = F; g1.epi = EPI_BIAS_GELU; g1.bias = w.b1; }
       else { g1.N = 2 * F; g1.epi = EPI_GEGLU; }
-      gemm(c, dit ? w.w1 : w.wgu, g1, s);
+      { Mark mk(c, s, dit ? "mlp_up" : "gate_up_proj", gemm_bytes(g1, c->es), 2.0 * M * g1.N * W); gemm(c, dit ? w.w1 : w.wgu, g1, s); }
       GemmArgs g2;
       g2.A = c->act; g2.lda = F; g2.a_dtype = dt; g2.w_dtype = dt;
       g2.M = M; g2.N = W; g2.K = F; g2.epi = EPI_RESID_GATE; g2.resid = c->h; g2.ldr = W;
       g2.bias = dit ? w.b2 : nullptr;
       g2.gate_tab = c->tab + base + 5 * W; g2.gate_stride = c->rowlen; g2.tau_row = tr;
-      gemm(c, dit ? w.w2 : w.wd, g2, s);
+      { Mark mk(c, s, dit ? "mlp_down" : "down_proj", gemm_bytes(g2, c->es), 2.0 * M * W * F); gemm(c, dit ? w.w2 : w.wd, g2, s); }
     }
     NormArgs nf;
     nf.h = c->h; nf.ldh = W; nf.M = M; nf.W = W; nf.layer_norm = dit; nf.tab = c->tab;
     nf.stride = c->rowlen; nf.tau_row = tr; nf.out = c->y; nf.ldo = W; nf.out_dtype = dt;
     nf.scale_off = a.n_layers * W6 + (dit ? W : 0);
     nf.shift_off = a.n_layers * W6 + (dit ? 0 : W);
-    launch_norm(nf, s);
+    { Mark mk(c, s, "norm", (4.0 + c->es) * M * W, 0); launch_norm(nf, s); }
     GemmArgs go;
     go.A = c->y; go.lda = W; go.a_dtype = dt; go.w_dtype = dt;
     go.M = M; go.N = D; go.K = W; go.out = c->v; go.ldo = D; go.bias = c->b_out;
-    gemm(c, c->w_out, go, s);
+    { Mark mk(c, s, "out_proj", gemm_bytes(go, c->es), 2.0 * M * W * D); gemm(c, c->w_out, go, s); }
     EulerArgs ea;
     ea.B = B; ea.H = H; ea.D = D; ea.k = k;
     ea.plan = plan + (size_t)(k - 1) * M;
@@ -467,7 +513,7 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
     ea.final_out = c->fin; ea.ghost_out = c->ghost; ea.E_out = c->E;
     ea.host_rel = c->host_rel_dev; ea.host_flags = c->host_flags_dev;
     ea.nonfinite = c->nonfinite; ea.evals = c->evals; ea.stamps = c->stamps;
-    launch_euler(ea, s);
+    { Mark mk(c, s, "euler_tr_gac", 40.0 * M * D, 0); launch_euler(ea, s); }
   }
 }
 
@@ -788,7 +834,8 @@ int uad_prepare_times(uad_ctx* c, int32_t max_budget) {
   return UAD_OK;
 }
 
-int uad_denoise(uad_ctx* c, const float* noise, const uad_schedule* sc, int32_t n_star, void* stream) {
+static int denoise_impl(uad_ctx* c, const float* noise, const uad_schedule* sc, int32_t n_star, void* stream,
+                        bool profile) {
   if (!c || !noise || !sc || !sc->budgets) return c ? fail(c, UAD_EINVAL, "null argument") : UAD_EINVAL;
   const uad_arch& a = c->a;
   if (c->in_flight) return fail(c, UAD_ESTATE, "previous chunk not finished");
@@ -860,7 +907,7 @@ int uad_denoise(uad_ctx* c, const float* noise, const uad_schedule* sc, int32_t 
   for (size_t e = 0; e < taus.size(); ++e) taur[e] = c->tau_row.at(taus[e]);
   CK(cudaMemcpyAsync(c->plan_dev, hp, PL.total, cudaMemcpyHostToDevice, s));
   CK(cudaMemcpyAsync(c->noise, noise, (size_t)M * D * 4, cudaMemcpyDefault, s));
-  if (c->use_graphs) {
+  if (c->use_graphs && !profile) {
     const auto key = std::make_pair(B, steps);
     auto it = c->graphs.find(key);
     if (it == c->graphs.end()) {
@@ -877,7 +924,11 @@ int uad_denoise(uad_ctx* c, const float* noise, const uad_schedule* sc, int32_t 
     }
     CK(cudaGraphLaunch(it->second, s));
   } else {
+    c->prof_on = profile;
+    c->prof.clear();
+    c->prof_next = 0;
     enqueue_chunk(c, B, steps, s);
+    c->prof_on = false;
     CK(cudaGetLastError());
   }
   CK(cudaEventRecord(c->ev_done, s));
@@ -888,6 +939,40 @@ int uad_denoise(uad_ctx* c, const float* noise, const uad_schedule* sc, int32_t 
   c->cur_budgets.assign(sc->budgets, sc->budgets + (size_t)B * H);
   c->cur_nstar = ns;
   return UAD_OK;
+}
+
+int uad_denoise(uad_ctx* c, const float* noise, const uad_schedule* sc, int32_t n_star, void* stream) {
+  return denoise_impl(c, noise, sc, n_star, stream, false);
+}
+
+int uad_profile_chunk(uad_ctx* c, const float* noise, const uad_schedule* sc, uad_kernel_stat* out,
+                      int32_t max_stats, int64_t timeout_us) {
+  if (!c || !out || max_stats < 1) return c ? fail(c, UAD_EINVAL, "null argument") : UAD_EINVAL;
+  int rc = denoise_impl(c, noise, sc, 0, nullptr, true);
+  if (rc) return rc;
+  rc = uad_finish(c, nullptr, nullptr, nullptr, nullptr, timeout_us);
+  if (rc && rc != UAD_ENONFINITE) return rc;
+  std::vector<std::string> names;
+  std::vector<uad_kernel_stat> st;
+  for (const auto& r : c->prof) {
+    float ms = 0.f;
+    CK(cudaEventElapsedTime(&ms, c->prof_ev[r.ev0], c->prof_ev[r.ev1]));
+    size_t j = 0;
+    while (j < names.size() && names[j] != r.name) ++j;
+    if (j == names.size()) {
+      names.push_back(r.name);
+      uad_kernel_stat z{};
+      snprintf(z.name, sizeof z.name, "%s", r.name);
+      st.push_back(z);
+    }
+    st[j].launches += 1;
+    st[j].total_ms += ms;
+    st[j].bytes += r.bytes;
+    st[j].flops += r.flops;
+  }
+  const int n = std::min((int)st.size(), (int)max_stats);
+  for (int j = 0; j < n; ++j) out[j] = st[j];
+  return n;
 }
 
 int uad_poll_released(uad_ctx* c, int32_t robot, int32_t min_ready, int64_t timeout_us, float* out,
@@ -986,6 +1071,7 @@ void uad_destroy(uad_ctx* c) {
       std::this_thread::yield();
   }
   for (auto& kv : c->graphs) cudaGraphExecDestroy(kv.second);
+  for (cudaEvent_t e : c->prof_ev) cudaEventDestroy(e);
   if (c->worker) cudaStreamDestroy(c->worker);
   if (c->ev_in) cudaEventDestroy(c->ev_in);
   if (c->ev_done) cudaEventDestroy(c->ev_done);

@@ -1,0 +1,61 @@
+"""CPU checks of bench.py's host logic: the replica (N > 1) timing reduction over gloo ranks,
+and its action-availability-latency arithmetic against the oracle's control clock."""
+import multiprocessing as mp
+import os
+import socket
+import sys
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, q):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank), UAD_BENCH_BACKEND="gloo")
+    sys.path.insert(0, ROOT)
+    import bench
+    import torch.distributed as dist
+    w, r, _ = bench.dist_setup()
+    bench.barrier(w)
+    t = bench.max_over_ranks(100.0 + 7.0 * r, w)
+    q.put((r, w, t))
+    dist.destroy_process_group()
+
+
+@pytest.mark.parametrize("world", [2])
+def test_replica_timing_takes_max_over_ranks(world):
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_rank_main, args=(r, world, port, q)) for r in range(world)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(120)
+        assert p.exitcode == 0
+    got = sorted(q.get(timeout=10) for _ in range(world))
+    assert [g[0] for g in got] == list(range(world))
+    assert all(g[1] == world for g in got)
+    assert all(g[2] == 100.0 + 7.0 * (world - 1) for g in got)
+
+
+def test_bench_aal_matches_oracle_clock():
+    sys.path.insert(0, ROOT)
+    import bench
+    from oracle.clock import aal
+    rng = np.random.default_rng(0)
+    for _ in range(50):
+        H = int(rng.integers(2, 60))
+        ready = np.sort(rng.uniform(0, 30, size=H)).tolist()
+        ready = [r if rng.random() < 0.7 else ready[0] for r in ready]
+        t_act = float(rng.uniform(0.5, 20))
+        S = int(rng.integers(1, H + 1))
+        assert bench.aal_ms(ready, t_act, S) == pytest.approx(aal(ready, t_act, S), rel=1e-12, abs=1e-12)
