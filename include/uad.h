@@ -194,6 +194,30 @@ int uad_plan_step(const int32_t* budgets, int32_t H, int32_t k, int32_t tr, int3
 /* Library version string. */
 const char* uad_version(void);
 
+/* ---- Kernel-level op: the step loop's tensor-core projection on caller buffers ------------ */
+
+/* Re-lay out one linear weight for the tensor-core projection kernel (host only, no GPU).
+ * w: host fp32 [K][N] (y = x w); out: host bf16 bit patterns, N * K values, as 128 x 64 blocks:
+ * block (n / 128, k / 64) starts at element ((n / 128) * (K / 64) + k / 64) * 8192; inside it,
+ * row n % 128 holds 64 values (128 bytes) whose eight 16-byte groups are permuted by
+ * group ^ (n % 8) -- the 128-byte-swizzled K-major shared-memory layout the tensor cores read.
+ * Values are rounded to bf16 (nearest, ties to even). Needs N % 128 == 0 and K % 64 == 0.
+ * Returns UAD_OK or UAD_EINVAL. */
+int uad_tile_weight(const float* w, int32_t K, int32_t N, uint16_t* out);
+
+/* out[M][N] = x[M][K] w + bias on the tensor cores (tcgen05, bf16 operands, fp32 accumulation):
+ * the projection kernel of every velocity-network layer (Sec. 3, Eq. 1).
+ * x: device bf16 [M][K]; w_tiled: device, the layout of uad_tile_weight; bias: device fp32 [N]
+ * or NULL; out: device fp32 [M][N]. Needs N % 128 == 0, K % 64 == 0, M >= 1.
+ * Split-K scratch (an fp32 [M][N] accumulator and per-tile counters) is allocated by the library
+ * with cudaMalloc on the first call on each device and grown on demand; it is kept until exit.
+ * Asynchronous on `stream` (a cudaStream_t, NULL = legacy stream). Calls on one device must not
+ * overlap on the GPU, since they share that scratch. Returns UAD_OK, UAD_EINVAL, UAD_ENOMEM or
+ * UAD_ECUDA. */
+int uad_linear(const void* x, const void* w_tiled, const float* bias, float* out, int32_t M,
+               int32_t N, int32_t K, void* stream);
+
+
 #ifdef __cplusplus
 }
 #endif

@@ -13,7 +13,7 @@ import numpy as np
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libuad.so")
 if not os.path.exists(LIB_PATH):
-    raise ImportError(f"{LIB_PATH} is missing: build it with `python -m paper_2609_37772_gb300.build` "
+    raise ImportError(f"{LIB_PATH} is missing: build it with `python paper_2609_37772_gb300/build.py` "
                       "(or __graft_entry__.build()); there is no fallback path")
 _lib = C.CDLL(LIB_PATH)
 
@@ -65,10 +65,24 @@ uad_launches_per_chunk = _fn("uad_launches_per_chunk", C.c_int, _P, _I32, _I32)
 uad_destroy = _fn("uad_destroy", None, _P)
 uad_plan_step = _fn("uad_plan_step", C.c_int, _P, _I32, _I32, _I32, _P, _P, _P)
 uad_profile_chunk = _fn("uad_profile_chunk", C.c_int, _P, _P, C.POINTER(uad_schedule), _P, _I32, C.c_int64)
+uad_tile_weight = _fn("uad_tile_weight", C.c_int, _P, _I32, _I32, _P)
+uad_linear = _fn("uad_linear", C.c_int, _P, _P, _P, _P, _I32, _I32, _I32, _P)
 
 EXPORTS = ["uad_version", "uad_last_error", "uad_init", "uad_set_prefix_kv", "uad_prepare_times",
            "uad_denoise", "uad_poll_released", "uad_finish", "uad_step_times",
-           "uad_launches_per_chunk", "uad_destroy", "uad_plan_step", "uad_profile_chunk"]
+           "uad_launches_per_chunk", "uad_destroy", "uad_plan_step", "uad_profile_chunk",
+           "uad_tile_weight", "uad_linear"]
+
+
+def tile_weight(w):
+    """fp32 [K][N] -> uint16 bf16 bits in the tensor-core projection layout (host only)."""
+    w = np.ascontiguousarray(w, dtype=np.float32)
+    K, N = w.shape
+    out = np.empty(N * K, dtype=np.uint16)
+    rc = uad_tile_weight(_ptr(w), K, N, _ptr(out))
+    if rc:
+        raise UADError(rc, "tile_weight: needs N % 128 == 0 and K % 64 == 0")
+    return out
 
 
 class UADError(RuntimeError):

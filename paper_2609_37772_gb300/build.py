@@ -1,6 +1,7 @@
 """Build libuad.so for sm_103a in-tree: one nvcc process per translation unit, then a link.
 
-Usable as ``python -m paper_2609_37772_gb300.build`` or via ``__graft_entry__.build()``.
+Run as ``python paper_2609_37772_gb300/build.py`` (not with -m: the package refuses to import
+without its library) or via ``__graft_entry__.build()``.
 """
 from __future__ import annotations
 

@@ -13,6 +13,8 @@
 // applies the epilogue, then clears the accumulator and counter for the next launch.
 // Every wait is bounded: on timeout the kernel records an error code and winds down.
 #include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include "uad_internal.cuh"
 
 namespace uad {
@@ -279,6 +281,31 @@ __global__ void relayout_tiled_kernel(const float* src, int K, int N, __nv_bfloa
 }
 
 }  // namespace
+
+static PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+int encode_act_tmap(CUtensorMap* m, const void* base, int K, int rows) {
+  auto enc = tmap_encoder();
+  if (!enc) return -1;
+  const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)K * 2};
+  const cuuint32_t box[2] = {kBK, kBN};
+  const cuuint32_t es[2] = {1, 1};
+  const CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                         CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? 0 : (int)r;
+}
 
 size_t gemm_tc_smem_bytes(int stages) {
   return 1024 + (size_t)stages * (kStageA + kStageB) + (2 * kTcMaxStages + 1) * 8 + 16;

@@ -12,8 +12,6 @@
 #include <thread>
 #include <vector>
 
-#include <cudaTypedefs.h>
-
 #include "../../include/uad.h"
 #include "uad_internal.cuh"
 
@@ -362,32 +360,12 @@ void gemm(uad_ctx* c, const void* w, GemmArgs g, cudaStream_t s) {
   gemm(c, l, g, s);
 }
 
-PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  if (!fn) {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
-            cudaSuccess && q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  }
-  return fn;
-}
-
 // 2-D TMA descriptor of a bf16 activation buffer [rows][K]: 64 x 64 boxes, 128-byte swizzle,
 // zero fill outside the buffer.
 int make_tmap(uad_ctx* c, const void* base, int K, int rows) {
-  auto enc = tmap_encoder();
-  if (!enc) return fail(c, UAD_ECUDA, "cuTensorMapEncodeTiled unavailable");
   CUtensorMap m;
-  const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
-  const cuuint64_t strides[1] = {(cuuint64_t)K * 2};
-  const cuuint32_t box[2] = {64, 64};
-  const cuuint32_t es[2] = {1, 1};
-  CUresult r = enc(&m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
-                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                   CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  if (r != CUDA_SUCCESS) return fail(c, UAD_ECUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
+  const int r = encode_act_tmap(&m, base, K, rows);
+  if (r) return fail(c, UAD_ECUDA, "TMA descriptor encoding failed (%d)", r);
   c->tmaps[base] = m;
   return UAD_OK;
 }

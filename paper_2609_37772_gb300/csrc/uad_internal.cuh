@@ -113,6 +113,9 @@ struct TcGemmArgs {
   int* err = nullptr;              // set to a nonzero code if a bounded wait gave up
 };
 size_t gemm_tc_smem_bytes(int stages);
+// 2-D TMA descriptor of a bf16 activation matrix [rows][K] (64 x 64 boxes, 128-byte swizzle,
+// zero fill past the last row). 0 on success.
+int encode_act_tmap(CUtensorMap* m, const void* base, int K, int rows);
 void gemm_tc_prepare();
 int gemm_tc_splits(int M, int N, int K, int sms);
 void launch_gemm_tc(const CUtensorMap* tmx, const TcGemmArgs& a, cudaStream_t s);
