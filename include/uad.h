@@ -217,6 +217,29 @@ int uad_tile_weight(const float* w, int32_t K, int32_t N, uint16_t* out);
 int uad_linear(const void* x, const void* w_tiled, const float* bias, float* out, int32_t M,
                int32_t N, int32_t K, void* stream);
 
+/* ---- The same projection op for callers that cannot allocate device memory ---------------
+ * The paper has no counterpart: this serves deployments rather than the method. A real-time
+ * controller that has finished start-up must not block on cudaMalloc (it can take unbounded
+ * time and synchronize the device, stalling the control loop), and a host framework whose
+ * caching allocator already holds the GPU's memory cannot take a stray allocation. This entry
+ * point computes exactly what uad_linear computes but allocates nothing: no cudaMalloc,
+ * cudaFree or allocating library call. Its split-K scratch is a fixed array inside the
+ * library's device image (about 4 MiB), held by every GPU that loads the library until exit.
+ *   - Limits: M * N <= UAD_LINEAR_STATIC_MAX_ELEMS and (N / 128) * ceil(M / 64) <=
+ *     UAD_LINEAR_STATIC_MAX_TILES; larger calls return UAD_ETOOBIG and launch nothing.
+ *   - The first call on a device looks up the array's device address (cudaGetSymbolAddress,
+ *     which may load the library's device code); make that first call before any stream
+ *     capture begins.
+ *   - Every call on a device shares the one array and it keeps the previous call's contents:
+ *     each call clears the part it uses (asynchronously, on `stream`) before its kernel.
+ *     Calls whose work overlaps on the GPU (different streams, or threads racing) corrupt
+ *     each other's results; order them on one stream.
+ * Arguments, layout and other errors are those of uad_linear. */
+#define UAD_ETOOBIG (-7)
+#define UAD_LINEAR_STATIC_MAX_ELEMS (1 << 20)
+#define UAD_LINEAR_STATIC_MAX_TILES 4096
+int uad_linear_static_scratch(const void* x, const void* w_tiled, const float* bias, float* out,
+                              int32_t M, int32_t N, int32_t K, void* stream);
 
 #ifdef __cplusplus
 }

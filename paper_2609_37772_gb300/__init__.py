@@ -67,11 +67,13 @@ uad_plan_step = _fn("uad_plan_step", C.c_int, _P, _I32, _I32, _I32, _P, _P, _P)
 uad_profile_chunk = _fn("uad_profile_chunk", C.c_int, _P, _P, C.POINTER(uad_schedule), _P, _I32, C.c_int64)
 uad_tile_weight = _fn("uad_tile_weight", C.c_int, _P, _I32, _I32, _P)
 uad_linear = _fn("uad_linear", C.c_int, _P, _P, _P, _P, _I32, _I32, _I32, _P)
+uad_linear_static_scratch = _fn("uad_linear_static_scratch", C.c_int, _P, _P, _P, _P, _I32, _I32, _I32, _P)
+UAD_ETOOBIG = -7
 
 EXPORTS = ["uad_version", "uad_last_error", "uad_init", "uad_set_prefix_kv", "uad_prepare_times",
            "uad_denoise", "uad_poll_released", "uad_finish", "uad_step_times",
            "uad_launches_per_chunk", "uad_destroy", "uad_plan_step", "uad_profile_chunk",
-           "uad_tile_weight", "uad_linear"]
+           "uad_tile_weight", "uad_linear", "uad_linear_static_scratch"]
 
 
 def tile_weight(w):
