@@ -1,0 +1,371 @@
+// Tensor-core attention of chunk queries over [prefix keys ; chunk keys] (grouped KV heads),
+// for bf16 experts with joint attention over the observation prefix.
+//
+// Layouts (written by the QKV projection epilogue and, for the prefix, by set_prefix):
+//   Q  [B][Hkv][G][H][dh]       queries of one KV group are the R = G*H rows of one matrix
+//   K  [B][L][Hkv][NK][dh]      keys: P prefix rows then H chunk rows (NK = P + H)
+//   Vt [B][L][Hkv][dh][NKp]     values transposed (keys contiguous), NKp = NK rounded up to 8
+// One CTA = one 128-row query tile x one 128-key chunk of one (robot, group):
+//   TMA loads Q, K, Vt tiles (128-byte swizzle); S = Q K^T on tcgen05 into TMEM; four warps
+//   read S rows, apply the 1/sqrt(dh) scale and key mask, write P = exp(S - rowmax) in bf16 into
+//   shared memory in the K-major swizzled layout; O = P Vt^T on tcgen05; O rows (unnormalised)
+//   and per-row (max, sum) go to a workspace. attn_combine merges the key chunks (the usual
+//   log-sum-exp rescaling) and writes o [B*H][Hq*dh] in bf16 for the O projection.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include "uad_internal.cuh"
+
+namespace uad {
+
+namespace {
+
+constexpr int kQT = 128, kKT = 128;
+constexpr int kMaxKeyChunks = 16;   // keys per (robot, layer) <= 2048
+constexpr uint32_t kTmemCols = 256; // S (128 columns) then O (dh <= 256 columns) in the same columns
+constexpr unsigned long long kWaitNs = 2000000000ull;
+
+__device__ __forceinline__ uint32_t su32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ unsigned long long gtime() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void mbar_init(uint64_t* b, uint32_t n) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(b)), "r"(n));
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* b, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(b)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity, int* err, int code) {
+  unsigned long long t0 = 0;
+  for (uint32_t it = 0;; ++it) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok) : "r"(su32(b)), "r"(parity) : "memory");
+    if (ok) return true;
+    if ((it & 255) == 0) {
+      const unsigned long long t = gtime();
+      if (t0 == 0) t0 = t;
+      else if (t - t0 > kWaitNs) {
+        atomicCAS(err, 0, code);
+        return false;
+      }
+    }
+  }
+}
+__device__ __forceinline__ void tma_3d(void* dst, const CUtensorMap* map, int x, int y, int z, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];"
+      ::"r"(su32(dst)), "l"(map), "r"(x), "r"(y), "r"(z), "r"(su32(bar)) : "memory");
+}
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
+         ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+// kind::f16 instruction descriptor: bf16 x bf16 -> fp32, K-major A and B, M = 128, N = n.
+__device__ __forceinline__ uint32_t idesc_m128(int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+}
+__device__ __forceinline__ void mma_bf16(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accum) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n"
+      ::"r"(d), "l"(a), "l"(b), "r"(idesc), "r"(accum));
+}
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(su32(bar)) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// smem plan for head dim dh: Q tiles (dh/64 blocks of 128 x 64), K tiles (same), Vt tiles
+// (2 blocks of dh x 64 keys), P (2 blocks of 128 x 64, aliased on Q when Q is >= 32 KB).
+__host__ __device__ __forceinline__ size_t attn_q_bytes(int dh) { return (size_t)dh * kQT * 2; }
+__host__ __device__ __forceinline__ size_t attn_p_extra(int dh) { return attn_q_bytes(dh) >= 32768 ? 0 : 32768; }
+
+template <int DH>
+__global__ void __launch_bounds__(128, 1) attn_tc_kernel(const __grid_constant__ CUtensorMap tq,
+                                                         const __grid_constant__ CUtensorMap tk,
+                                                         const __grid_constant__ CUtensorMap tv, AttnTcArgs p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  constexpr int NC = DH / 64;
+  constexpr uint32_t QB = DH * kQT * 2, KB = DH * kKT * 2, VB = DH * kKT * 2;
+  uint8_t* sQ = smem;
+  uint8_t* sK = sQ + QB;
+  uint8_t* sV = sK + KB;
+  uint8_t* sP = attn_p_extra(DH) ? sV + VB : sQ;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sV + VB + attn_p_extra(DH));
+  uint64_t *bar_qk = bars, *bar_v = bars + 1, *bar_s = bars + 2, *bar_o = bars + 3;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 4);
+
+  const int qt = blockIdx.x, kc = blockIdx.y, bg = blockIdx.z;   // bg = b * Hkv + g
+  const int b = bg / p.n_kv_heads, g = bg % p.n_kv_heads;
+  const int kvz = (b * p.n_layers + p.layer) * p.n_kv_heads + g;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 4; ++i) mbar_init(bars + i, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(tmem_slot)), "r"(kTmemCols));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  // S occupies columns [0, 128); O = P V reuses columns [0, DH) once every thread has read S
+  const uint32_t tS = tmem, tO = tmem;
+  pdl_trigger();
+  pdl_wait();
+
+  if (threadIdx.x == 0) {
+    mbar_expect_tx(bar_qk, QB + KB);
+#pragma unroll
+    for (int c = 0; c < NC; ++c) {
+      tma_3d(sQ + c * (kQT * 128), &tq, c * 64, qt * kQT, bg, bar_qk);
+      tma_3d(sK + c * (kKT * 128), &tk, c * 64, kc * kKT, kvz, bar_qk);
+    }
+    mbar_expect_tx(bar_v, VB);
+#pragma unroll
+    for (int u = 0; u < kKT / 64; ++u) tma_3d(sV + u * (DH * 128), &tv, kc * kKT + u * 64, 0, kvz, bar_v);
+  } else if (threadIdx.x == 32) {
+    if (mbar_wait(bar_qk, 0, p.err, 21)) {
+      tc_fence_after();
+      const uint32_t q0 = su32(sQ), k0 = su32(sK);
+#pragma unroll
+      for (int c = 0; c < NC; ++c)
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          mma_bf16(tS, sw128_desc(q0 + c * (kQT * 128) + 32 * k), sw128_desc(k0 + c * (kKT * 128) + 32 * k),
+                   idesc_m128(kKT), (c | k) ? 1u : 0u);
+    }
+    mma_commit(bar_s);
+  }
+  __syncwarp();
+
+  // ---- softmax over this key chunk: one query row per thread ----
+  const bool ok_s = mbar_wait(bar_s, 0, p.err, 22);
+  tc_fence_after();
+  const int row = warp * 32 + lane;
+  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+  const float c2 = p.scale_log2;             // log2(e) / sqrt(dh)
+  const int key0 = kc * kKT;
+  float mx = -INFINITY;
+  float sv[32];
+  __syncwarp();
+#pragma unroll
+  for (int cc = 0; cc < kKT / 32; ++cc) {
+    tmem_ld32(tS + lane_base + cc * 32, sv);
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      if (key0 + cc * 32 + i < p.n_keys) mx = fmaxf(mx, sv[i]);
+  }
+  float l = 0.f;
+  const int r8 = row & 7;
+#pragma unroll
+  for (int cc = 0; cc < kKT / 32; ++cc) {
+    tmem_ld32(tS + lane_base + cc * 32, sv);
+    uint32_t pk[16];
+#pragma unroll
+    for (int i = 0; i < 32; i += 2) {
+      const bool v0 = key0 + cc * 32 + i < p.n_keys, v1 = key0 + cc * 32 + i + 1 < p.n_keys;
+      const float e0 = v0 ? exp2f((sv[i] - mx) * c2) : 0.f;
+      const float e1 = v1 ? exp2f((sv[i + 1] - mx) * c2) : 0.f;
+      const __nv_bfloat162 h = __floats2bfloat162_rn(e0, e1);
+      l += __low2float(h) + __high2float(h);   // normalise by what the MMA actually sums
+      pk[i / 2] = *reinterpret_cast<const uint32_t*>(&h);
+    }
+    // 32 keys = four 16-byte granules of row `row` in P block (cc / 2), granules (cc % 2) * 4 + q
+    uint8_t* prow = sP + (cc / 2) * (kQT * 128) + row * 128;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int gidx = (cc % 2) * 4 + q;
+      *reinterpret_cast<uint4*>(prow + ((gidx ^ r8) * 16)) = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+    }
+  }
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  tc_fence_before();
+  __syncthreads();
+
+  if (threadIdx.x == 32) {
+    tc_fence_after();
+    if (ok_s && mbar_wait(bar_v, 0, p.err, 23)) {
+      const uint32_t p0 = su32(sP), v0 = su32(sV);
+#pragma unroll
+      for (int u = 0; u < kKT / 64; ++u)
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          mma_bf16(tO, sw128_desc(p0 + u * (kQT * 128) + 32 * k), sw128_desc(v0 + u * (DH * 128) + 32 * k),
+                   idesc_m128(DH), (u | k) ? 1u : 0u);
+    }
+    mma_commit(bar_o);
+  }
+  __syncwarp();
+  const bool ok_o = mbar_wait(bar_o, 0, p.err, 24);
+  tc_fence_after();
+
+  // ---- partial output row (unnormalised) + (max, sum) ----
+  const int qrow = qt * kQT + row;
+  const size_t prow_idx = ((size_t)bg * gridDim.y + kc) * p.r_pad + qrow;
+  float* po = p.part_o + prow_idx * DH;
+  __syncwarp();
+#pragma unroll
+  for (int cc = 0; cc < DH / 32; ++cc) {
+    tmem_ld32(tO + lane_base + cc * 32, sv);
+    if (ok_o && qrow < p.rows) {
+#pragma unroll
+      for (int i = 0; i < 32; i += 4)
+        *reinterpret_cast<float4*>(po + cc * 32 + i) = make_float4(sv[i], sv[i + 1], sv[i + 2], sv[i + 3]);
+    }
+  }
+  if (qrow < p.rows) {
+    p.part_ml[prow_idx * 2] = mx;
+    p.part_ml[prow_idx * 2 + 1] = l;
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols));
+}
+
+// Merge the key chunks of every query row: o = sum_c w_c O_c / sum_c w_c l_c, w_c = 2^((m_c - M) c2).
+// One CTA per (query row, robot-group), one thread per head dim; every partial is loaded
+// before any arithmetic. Writes o [(b*H + i)][(g*G + j)*dh + d] in bf16.
+__global__ void attn_combine_kernel(AttnTcArgs p, int n_chunks) {
+  constexpr int MAXC = kMaxKeyChunks;
+  pdl_trigger();
+  pdl_wait();
+  const int r = blockIdx.x, bg = blockIdx.y, d = threadIdx.x, DH = blockDim.x;
+  const int b = bg / p.n_kv_heads, g = bg % p.n_kv_heads;
+  float m[MAXC], l[MAXC], o[MAXC];
+#pragma unroll
+  for (int c = 0; c < MAXC; ++c) {
+    if (c < n_chunks) {
+      const size_t idx = ((size_t)bg * n_chunks + c) * p.r_pad + r;
+      m[c] = p.part_ml[idx * 2];
+      l[c] = p.part_ml[idx * 2 + 1];
+      o[c] = p.part_o[idx * DH + d];
+    }
+  }
+  float M = -INFINITY;
+#pragma unroll
+  for (int c = 0; c < MAXC; ++c)
+    if (c < n_chunks) M = fmaxf(M, m[c]);
+  float L = 0.f, acc = 0.f;
+#pragma unroll
+  for (int c = 0; c < MAXC; ++c) {
+    if (c < n_chunks) {
+      const float w = exp2f((m[c] - M) * p.scale_log2);
+      L = fmaf(w, l[c], L);
+      acc = fmaf(w, o[c], acc);
+    }
+  }
+  const int j = r / p.H, i = r % p.H;
+  p.out[((size_t)b * p.H + i) * p.out_ld + (size_t)(g * p.group + j) * DH + d] = __float2bfloat16_rn(acc / L);
+}
+
+// Prefix K/V of one robot (fp32 or bf16 source [L][P][Hkv][dh]) into the K and Vt caches.
+__global__ void kv_prefix_kernel(const void* k, const void* v, int src_dt, AttnTcArgs p, int robot) {
+  const int dh = p.head_dim;
+  const long long n = (long long)p.n_layers * p.prefix * p.n_kv_heads * dh;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < n; e += (long long)gridDim.x * blockDim.x) {
+    const int d = (int)(e % dh);
+    const int g = (int)((e / dh) % p.n_kv_heads);
+    const int pp = (int)((e / ((long long)dh * p.n_kv_heads)) % p.prefix);
+    const int l = (int)(e / ((long long)dh * p.n_kv_heads * p.prefix));
+    const float kv = src_dt == BF16 ? __bfloat162float(static_cast<const __nv_bfloat16*>(k)[e]) : static_cast<const float*>(k)[e];
+    const float vv = src_dt == BF16 ? __bfloat162float(static_cast<const __nv_bfloat16*>(v)[e]) : static_cast<const float*>(v)[e];
+    const size_t z = ((size_t)robot * p.n_layers + l) * p.n_kv_heads + g;
+    p.kcache[(z * p.n_keys + pp) * dh + d] = __float2bfloat16_rn(kv);
+    p.vtcache[(z * dh + d) * p.nk_pad + pp] = __float2bfloat16_rn(vv);
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* q = nullptr;
+    cudaDriverEntryPointQueryResult r;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &q, 12000, cudaEnableDefault, &r) ==
+            cudaSuccess && r == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(q);
+  }
+  return fn;
+}
+
+int tmap3(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint64_t s1, uint64_t s2,
+          uint32_t b0, uint32_t b1) {
+  auto enc = encoder();
+  if (!enc) return -1;
+  const cuuint64_t dims[3] = {d0, d1, d2};
+  const cuuint64_t strides[2] = {s1, s2};
+  const cuuint32_t box[3] = {b0, b1, 1};
+  const cuuint32_t es[3] = {1, 1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS ? 0 : -2;
+}
+
+}  // namespace
+
+size_t attn_tc_smem_bytes(int dh) {
+  return 1024 + 3 * attn_q_bytes(dh) + attn_p_extra(dh) + 4 * 8 + 16;
+}
+
+int attn_tc_prepare(AttnTcMaps* maps, const AttnTcArgs& a, int batch_max) {
+  const int dh = a.head_dim;
+  const uint64_t R = a.rows, NK = a.n_keys, NKp = a.nk_pad;
+  if (tmap3(&maps->q, a.q, dh, R, (uint64_t)batch_max * a.n_kv_heads, (uint64_t)dh * 2, R * dh * 2, 64, kQT)) return -1;
+  if (tmap3(&maps->k, a.kcache, dh, NK, (uint64_t)batch_max * a.n_layers * a.n_kv_heads, (uint64_t)dh * 2,
+            NK * dh * 2, 64, kKT)) return -1;
+  if (tmap3(&maps->vt, a.vtcache, NK, dh, (uint64_t)batch_max * a.n_layers * a.n_kv_heads, NKp * 2,
+            (uint64_t)dh * NKp * 2, 64, (uint32_t)dh)) return -1;
+  const int smem = (int)attn_tc_smem_bytes(dh);
+  if (dh == 64) cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (dh == 128) cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (dh == 256) cudaFuncSetAttribute(attn_tc_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  return 0;
+}
+
+int attn_tc_chunks(int n_keys) { return (n_keys + kKT - 1) / kKT; }
+int attn_tc_max_keys() { return kMaxKeyChunks * kKT; }
+int attn_tc_rpad(int rows) { return (rows + kQT - 1) / kQT * kQT; }
+
+void launch_attn_tc(const AttnTcMaps& maps, const AttnTcArgs& a, cudaStream_t s) {
+  dim3 grid((a.rows + kQT - 1) / kQT, attn_tc_chunks(a.n_keys), a.batch * a.n_kv_heads);
+  const size_t smem = attn_tc_smem_bytes(a.head_dim);
+  if (a.head_dim == 64) launch_k(attn_tc_kernel<64>, grid, dim3(128), smem, s, maps.q, maps.k, maps.vt, a);
+  if (a.head_dim == 128) launch_k(attn_tc_kernel<128>, grid, dim3(128), smem, s, maps.q, maps.k, maps.vt, a);
+  if (a.head_dim == 256) launch_k(attn_tc_kernel<256>, grid, dim3(128), smem, s, maps.q, maps.k, maps.vt, a);
+  launch_k(attn_combine_kernel, dim3(a.rows, a.batch * a.n_kv_heads), dim3(a.head_dim), 0, s, a,
+           attn_tc_chunks(a.n_keys));
+}
+
+void launch_kv_prefix(const void* k, const void* v, int src_dtype, const AttnTcArgs& a, int robot, cudaStream_t s) {
+  kv_prefix_kernel<<<1024, 256, 0, s>>>(k, v, src_dtype, a, robot);
+}
+
+}  // namespace uad

@@ -116,27 +116,39 @@ __device__ __forceinline__ void store_out(void* out, long long i, float v, int d
   else static_cast<float*>(out)[i] = v;
 }
 
-// Apply the epilogue to one value of row n (this thread) and token m.
-__device__ __forceinline__ void epi_one(const TcGemmArgs& p, int m, int n, float acc, bool lane_even,
-                                        float partner) {
-  switch (p.epi) {
-    case EPI_GEGLU:
-      if (lane_even) store_out(p.out, (long long)m * p.ldo + n / 2, gelu_tanh_f(acc) * partner, p.out_dtype);
-      break;
-    case EPI_RESID_GATE: {
-      const float r = acc + (p.bias ? p.bias[n] : 0.f);
-      const float gt = p.gate_tab ? p.gate_tab[(long long)p.tau_row[m] * p.gate_stride + n] : 1.f;
-      float* dst = p.resid + (long long)m * p.ldr + n;
-      *dst = fmaf(gt, r, *dst);
-      break;
+// Store one already-rotated q / k value (or a v value) of output row n, robot b, token i into
+// the tensor-core attention layouts.
+__device__ __forceinline__ void epi_qkv_store_bi(const QkvTcOut& o, int b, int i, int n, float val) {
+  if (n < o.qd + o.kvd) {
+    const int sn = n < o.qd ? n : n - o.qd;
+    const int h = sn / o.dh, r = sn % o.dh, half = o.dh / 2;
+    const int d = o.rope ? ((r & 1) ? (r >> 1) + half : (r >> 1)) : r;
+    if (n < o.qd) {
+      const int g = h / o.G, jj = h % o.G;
+      o.q[(((size_t)b * o.Hkv + g) * o.G * o.H + (size_t)jj * o.H + i) * o.dh + d] = __float2bfloat16_rn(val);
+    } else {
+      o.kcache[((((size_t)b * o.L + o.layer) * o.Hkv + h) * o.NK + o.P + i) * o.dh + d] = __float2bfloat16_rn(val);
     }
-    case EPI_BIAS_GELU:
-      store_out(p.out, (long long)m * p.ldo + n, gelu_tanh_f(acc + (p.bias ? p.bias[n] : 0.f)), p.out_dtype);
-      break;
-    default:
-      store_out(p.out, (long long)m * p.ldo + n, acc + (p.bias ? p.bias[n] : 0.f), p.out_dtype);
-      break;
+  } else {
+    const int sn = n - o.qd - o.kvd, g = sn / o.dh, d = sn % o.dh;
+    o.vtcache[((((size_t)b * o.L + o.layer) * o.Hkv + g) * o.dh + d) * o.NKp + o.P + i] = __float2bfloat16_rn(val);
   }
+}
+
+__device__ __forceinline__ void red_add_v4(float* dst, float4 v) {
+  asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(dst), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
+               : "memory");
+}
+
+// Shared-memory plan: [pipeline stages, at least 32 KB (reused as the split-K staging tile)]
+// [gate rows 32 KB][residual rows 32 KB] (residual epilogue only) [mbarriers, TMEM slot, flag].
+__host__ __device__ __forceinline__ int tc_stages(int nch, int epi) {
+  const int cap = epi == EPI_RESID_GATE ? kTcMaxStagesResid : kTcMaxStages;
+  return nch < cap ? nch : cap;
+}
+__host__ __device__ __forceinline__ size_t tc_pipe_bytes(int stages) {
+  const size_t b = (size_t)stages * (kStageA + kStageB);
+  return b < 32768 ? 32768 : b;
 }
 
 __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__ CUtensorMap tmx, TcGemmArgs p) {
@@ -145,15 +157,20 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   const int t = blockIdx.x, mt = blockIdx.y, s = blockIdx.z;
   const int KC = p.K / kBK;
   const int c0 = s * KC / p.splits, c1 = (s + 1) * KC / p.splits, nch = c1 - c0;
-  const int stages = nch < kTcMaxStages ? nch : kTcMaxStages;
+  const int stages = tc_stages(nch, p.epi);
+  const bool resid = p.epi == EPI_RESID_GATE;
   uint8_t* sA = smem;
   uint8_t* sB = smem + (size_t)stages * kStageA;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sB + (size_t)stages * kStageB);
+  float* G = reinterpret_cast<float*>(smem + tc_pipe_bytes(stages));   // [kBN][kBM] gates
+  float* R = G + kBN * kBM;                                            // [kBN][kBM] residual rows
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + tc_pipe_bytes(stages) + (resid ? 2 * kBN * kBM * 4 : 0));
   uint64_t* empty = full + kTcMaxStages;
   uint64_t* done = empty + kTcMaxStages;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
   int* last_flag = reinterpret_cast<int*>(tmem_slot + 1);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int m0 = mt * kBN;
+  const int mcount = p.M - m0 < kBN ? p.M - m0 : kBN;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < stages; ++i) {
@@ -172,14 +189,24 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
+  pdl_trigger();
   if (threadIdx.x == 0) {
-    // ---- producer: weight block (bulk copy) + activation tile (tensor map) per K chunk ----
+    // ---- producer: weight block (bulk copy) + activation tile (tensor map) per K chunk.
+    //      Weights are constant: the first ring's worth is requested before waiting for the
+    //      kernel that produces the activations. ----
     const uint64_t pol = policy_evict_first();
     const uint8_t* wt = static_cast<const uint8_t*>(p.w_tiled) + ((size_t)t * KC + c0) * kStageA;
-    int issued = 0;
-    for (int i = 0; i < nch; ++i) {
+    const int first = nch < stages ? nch : stages;
+    for (int i = 0; i < first; ++i) {
+      mbar_expect_tx(full + i, kStageA + kStageB);
+      bulk_g2s(sA + (size_t)i * kStageA, wt + (size_t)i * kStageA, kStageA, full + i, pol);
+    }
+    pdl_wait();
+    for (int i = 0; i < first; ++i) tma_2d(sB + (size_t)i * kStageB, &tmx, (c0 + i) * kBK, mt * kBN, full + i);
+    int issued = first;
+    for (int i = first; i < nch; ++i) {
       const int st = i % stages, round = i / stages;
-      if (round > 0 && !mbar_wait(empty + st, (round - 1) & 1, p.err, 11)) break;
+      if (!mbar_wait(empty + st, (round - 1) & 1, p.err, 11)) break;
       mbar_expect_tx(full + st, kStageA + kStageB);
       bulk_g2s(sA + (size_t)st * kStageA, wt + (size_t)i * kStageA, kStageA, full + st, pol);
       tma_2d(sB + (size_t)st * kStageB, &tmx, (c0 + i) * kBK, mt * kBN, full + st);
@@ -203,55 +230,146 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
       mma_commit(empty + st);
     }
     mma_commit(done);
+  } else if (resid && warp >= 2) {
+    // ---- warps 2-3 prefetch the residual epilogue's inputs while the tile is computed:
+    //      gate rows gate_tab[tau(m)][n0..n0+127] and residual rows resid[m][n0..n0+127] ----
+    pdl_wait();
+    const int tid = threadIdx.x - 64;
+    const int n0 = t * kBM;
+    for (int base = 0; base < mcount * (kBM / 4); base += 64 * 8) {
+      float4 g[8], r[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int idx = base + u * 64 + tid;
+        if (idx < mcount * (kBM / 4)) {
+          const int j = idx / (kBM / 4), c4 = idx % (kBM / 4);
+          g[u] = p.gate_tab ? __ldg(reinterpret_cast<const float4*>(
+                                  p.gate_tab + (size_t)p.tau_row[m0 + j] * p.gate_stride + n0 + c4 * 4))
+                            : make_float4(1.f, 1.f, 1.f, 1.f);
+          r[u] = *reinterpret_cast<const float4*>(p.resid + (size_t)(m0 + j) * p.ldr + n0 + c4 * 4);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int idx = base + u * 64 + tid;
+        if (idx < mcount * (kBM / 4)) {
+          const int j = idx / (kBM / 4), c4 = idx % (kBM / 4);
+          *reinterpret_cast<float4*>(G + j * kBM + c4 * 4) = g[u];
+          *reinterpret_cast<float4*>(R + j * kBM + c4 * 4) = r[u];
+        }
+      }
+    }
   }
   __syncwarp();
 
   // ---- epilogue: TMEM -> registers, one weight row (output feature) per thread ----
+  pdl_wait();
   const bool ok = mbar_wait(done, 0, p.err, 14);
   tc_fence_after();
   const int row = warp * 32 + lane;
   const int n = t * kBM + row;
-  const int m0 = mt * kBN;
-  const int mcount = p.M - m0 < kBN ? p.M - m0 : kBN;
   float v[kBN];
   __syncwarp();
 #pragma unroll
   for (int c = 0; c < kBN; c += 16) tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + c, v + c);
-  const bool even = (lane & 1) == 0;
-  if (ok && nch > 0) {
-    if (p.splits == 1) {
+  bool have = ok && nch > 0;
+  // Stage the accumulator tile in shared memory, T[token j][row]: the epilogues below are
+  // compact loops over it (neighbouring rows -- GeGLU and RoPE partners -- are one column
+  // apart), which keeps the kernel's code small.
+  float* T = reinterpret_cast<float*>(smem);                         // pipeline region is idle
 #pragma unroll
-      for (int j = 0; j < kBN; ++j) {
-        if (j < mcount) {
-          const float partner = __shfl_xor_sync(0xffffffffu, v[j], 1);
-          epi_one(p, m0 + j, n, v[j], even, partner);
-        }
+  for (int j = 0; j < kBN; ++j) T[j * kBM + row] = v[j];
+  __syncthreads();
+  if (p.splits > 1) {
+    // add the partial tile into the L2 accumulator with 16-byte reds; the last CTA of the tile
+    // reads the sum back (independent 16-byte loads) and clears it for the next launch
+    float* acc = p.acc + (size_t)m0 * p.N + t * kBM;
+    if (have) {
+      for (int idx = threadIdx.x; idx < mcount * (kBM / 4); idx += 128) {
+        const int j = idx / (kBM / 4), c4 = idx % (kBM / 4);
+        red_add_v4(acc + (size_t)j * p.N + c4 * 4, *reinterpret_cast<const float4*>(T + j * kBM + c4 * 4));
       }
-    } else {
-      float* acc = p.acc + (size_t)m0 * p.N + n;
-#pragma unroll
-      for (int j = 0; j < kBN; ++j)
-        if (j < mcount)
-          asm volatile("red.global.add.f32 [%0], %1;" ::"l"(acc + (size_t)j * p.N), "f"(v[j]) : "memory");
+    }
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      const int prev = atomicAdd(p.counters + mt * gridDim.x + t, 1);
+      *last_flag = prev == p.splits - 1;
+    }
+    __syncthreads();
+    const bool last = *last_flag;
+    have = have && last;
+    if (last) {
       __threadfence();
-      __syncthreads();
-      if (threadIdx.x == 0) {
-        const int tile = mt * gridDim.x + t;
-        const int prev = atomicAdd(p.counters + tile, 1);
-        *last_flag = prev == p.splits - 1;
+      float4 q[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        const int idx = threadIdx.x + u * 128;
+        if (idx < mcount * (kBM / 4))
+          q[u] = __ldcg(reinterpret_cast<const float4*>(acc + (size_t)(idx / (kBM / 4)) * p.N + (idx % (kBM / 4)) * 4));
       }
-      __syncthreads();
-      if (*last_flag) {
-        __threadfence();
-        for (int j = 0; j < mcount; ++j) {
-          float* a = acc + (size_t)j * p.N;
-          const float sum = __ldcg(a);
-          __stcg(a, 0.f);
-          const float partner = __shfl_xor_sync(0xffffffffu, sum, 1);
-          epi_one(p, m0 + j, n, sum, even, partner);
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        const int idx = threadIdx.x + u * 128;
+        if (idx < mcount * (kBM / 4)) {
+          const int j = idx / (kBM / 4), c4 = idx % (kBM / 4);
+          __stcg(reinterpret_cast<float4*>(acc + (size_t)j * p.N + c4 * 4), make_float4(0.f, 0.f, 0.f, 0.f));
+          *reinterpret_cast<float4*>(T + j * kBM + c4 * 4) = q[u];
         }
-        if (threadIdx.x == 0) p.counters[mt * gridDim.x + t] = 0;
       }
+      if (threadIdx.x == 0) p.counters[mt * gridDim.x + t] = 0;
+    }
+    __syncthreads();
+  }
+  if (resid) __syncthreads();   // gate / residual rows staged by warps 2-3
+  if (have) {
+    const float b = p.bias ? p.bias[n] : 0.f;
+    const float* Tr = T + row;
+    switch (p.epi) {
+      case EPI_RESID_GATE:
+#pragma unroll 4
+        for (int j = 0; j < mcount; ++j)
+          p.resid[(size_t)(m0 + j) * p.ldr + n] = fmaf(G[j * kBM + row], Tr[j * kBM] + b, R[j * kBM + row]);
+        break;
+      case EPI_GEGLU:
+        if ((lane & 1) == 0) {
+#pragma unroll 4
+          for (int j = 0; j < mcount; ++j)
+            store_out(p.out, (size_t)(m0 + j) * p.ldo + n / 2, gelu_tanh_f(Tr[j * kBM]) * Tr[j * kBM + 1],
+                      p.out_dtype);
+        }
+        break;
+      case EPI_BIAS_GELU:
+#pragma unroll 4
+        for (int j = 0; j < mcount; ++j)
+          store_out(p.out, (size_t)(m0 + j) * p.ldo + n, gelu_tanh_f(Tr[j * kBM] + b), p.out_dtype);
+        break;
+      case EPI_QKV_TC: {
+        const QkvTcOut& o = p.qkv;
+        const bool rot = o.rope && n < o.qd + o.kvd;
+        const int r = (n < o.qd ? n : n - o.qd) % o.dh;
+        // RoPE frequency of this row's pair, theta = 1e4: angle = position * 1e4^(-2j/dh)
+        const float inv = exp2f(-13.287712379549449f * (float)(2 * (r >> 1)) / (float)o.dh);
+        const float sgn = (r & 1) ? 1.f : -1.f;
+        const int pr = (r & 1) ? -1 : 1;                                   // partner column offset
+        int bi = m0 / o.H, ii = m0 % o.H;
+        for (int j = 0; j < mcount; ++j) {
+          float val = Tr[j * kBM];
+          if (rot) {
+            float sn, cs;
+            sincosf((float)(o.P + ii) * inv, &sn, &cs);
+            val = fmaf(val, cs, sgn * Tr[j * kBM + pr] * sn);
+          }
+          epi_qkv_store_bi(o, bi, ii, n, val);
+          if (++ii == o.H) { ii = 0; ++bi; }
+        }
+        break;
+      }
+      default:
+#pragma unroll 4
+        for (int j = 0; j < mcount; ++j)
+          store_out(p.out, (size_t)(m0 + j) * p.ldo + n, Tr[j * kBM] + b, p.out_dtype);
+        break;
     }
   }
   tc_fence_before();
@@ -260,7 +378,8 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
 }
 
 // ---- weight re-layout into 128 x 64 swizzled blocks --------------------------------------
-__global__ void relayout_tiled_kernel(const float* src, int K, int N, __nv_bfloat16* dst, int mult, long long off) {
+__global__ void relayout_tiled_kernel(const float* src, int K, int N, __nv_bfloat16* dst, int mult, long long off,
+                                      int rope_dh) {
   __shared__ float tt[32][33];
   const int k0 = blockIdx.y * 32, n0 = blockIdx.x * 32;
   for (int r = threadIdx.y; r < 32; r += blockDim.y) {
@@ -272,7 +391,12 @@ __global__ void relayout_tiled_kernel(const float* src, int K, int N, __nv_bfloa
   for (int r = threadIdx.y; r < 32; r += blockDim.y) {
     const int n = n0 + r, k = k0 + threadIdx.x;
     if (n >= N || k >= K) continue;
-    const long long row = (long long)n * mult + off;
+    int nn = n;
+    if (rope_dh > 0) {
+      const int h = n / rope_dh, d = n % rope_dh, half = rope_dh / 2;
+      nn = h * rope_dh + (d < half ? 2 * d : 2 * (d - half) + 1);
+    }
+    const long long row = (long long)nn * mult + off;
     const long long tile = (row / kBM) * KC + k / kBK;
     const int rr = (int)(row % kBM), kk = k % kBK;
     const int gran = (kk >> 3) ^ (rr & 7);
@@ -307,19 +431,21 @@ int encode_act_tmap(CUtensorMap* m, const void* base, int K, int rows) {
   return r == CUDA_SUCCESS ? 0 : (int)r;
 }
 
-size_t gemm_tc_smem_bytes(int stages) {
-  return 1024 + (size_t)stages * (kStageA + kStageB) + (2 * kTcMaxStages + 1) * 8 + 16;
+size_t gemm_tc_smem_bytes(int stages, int epi) {
+  return 1024 + tc_pipe_bytes(stages) + (epi == EPI_RESID_GATE ? 2 * kBN * kBM * 4 : 0) +
+         (2 * kTcMaxStages + 1) * 8 + 16;
 }
 
 void gemm_tc_prepare() {
-  cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                       (int)gemm_tc_smem_bytes(kTcMaxStages));
+  const size_t a = gemm_tc_smem_bytes(kTcMaxStages, EPI_STORE);
+  const size_t b = gemm_tc_smem_bytes(kTcMaxStagesResid, EPI_RESID_GATE);
+  cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)(a > b ? a : b));
 }
 
 int gemm_tc_splits(int M, int N, int K, int sms) {
   const int tiles = (N / kBM) * ((M + kBN - 1) / kBN);
   const int KC = K / kBK;
-  int s = (sms + tiles / 2) / tiles;
+  int s = sms / tiles;                       // one wave: never more CTAs than SMs
   if (s < 1) s = 1;
   if (s > KC) s = KC;
   return s;
@@ -328,14 +454,14 @@ int gemm_tc_splits(int M, int N, int K, int sms) {
 void launch_gemm_tc(const CUtensorMap* tmx, const TcGemmArgs& a, cudaStream_t s) {
   const int KC = a.K / kBK;
   const int per = (KC + a.splits - 1) / a.splits;
-  const int stages = per < kTcMaxStages ? per : kTcMaxStages;
   dim3 grid(a.N / kBM, (a.M + kBN - 1) / kBN, a.splits);
-  gemm_tc_kernel<<<grid, 128, gemm_tc_smem_bytes(stages), s>>>(*tmx, a);
+  launch_k(gemm_tc_kernel, grid, dim3(128), gemm_tc_smem_bytes(tc_stages(per, a.epi), a.epi), s, *tmx, a);
 }
 
-void launch_relayout_tiled(const float* src, int K, int N, void* dst, int mult, long long off, cudaStream_t s) {
+void launch_relayout_tiled(const float* src, int K, int N, void* dst, int mult, long long off, int rope_dh,
+                           cudaStream_t s) {
   dim3 grid((N + 31) / 32, (K + 31) / 32);
-  relayout_tiled_kernel<<<grid, dim3(32, 8), 0, s>>>(src, K, N, static_cast<__nv_bfloat16*>(dst), mult, off);
+  relayout_tiled_kernel<<<grid, dim3(32, 8), 0, s>>>(src, K, N, static_cast<__nv_bfloat16*>(dst), mult, off, rope_dh);
 }
 
 }  // namespace uad

@@ -4,6 +4,15 @@
 
 namespace uad {
 
+bool pdl_enabled() {
+  static int on = -1;
+  if (on < 0) {
+    const char* e = getenv("UAD_PDL");
+    on = !(e && e[0] == '0');
+  }
+  return on != 0;
+}
+
 // ------------------------------------------------------------------------------------------
 // small helpers
 // ------------------------------------------------------------------------------------------
@@ -48,6 +57,8 @@ template <int AD, int WD>
 __global__ void __launch_bounds__(256) gemm_simt_kernel(GemmArgs p) {
   __shared__ float As[32][68];
   __shared__ float Ws[32][68];
+  pdl_trigger();
+  pdl_wait();
   const int m0 = blockIdx.y * 64, n0 = blockIdx.x * 64;
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
   float acc[4][4];
@@ -117,18 +128,61 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(GemmArgs p) {
   }
 }
 
+// Projections with a tiny side (action in: K = D; action out: N = D): one CTA per token row m,
+// the row staged in shared memory, then one warp per output (long K) or one thread per output
+// (short K). out[m][n] = sum_k A[m][k] Wt[n][k] + bias[n] (+ add_rows[m % add_mod][n]), fp32.
+template <int AD, int WD>
+__global__ void __launch_bounds__(256) gemv_rows_kernel(GemmArgs p) {
+  __shared__ float a_s[kGemvMaxK];
+  pdl_trigger();
+  pdl_wait();
+  const int m = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int k = tid; k < p.K; k += 256) a_s[k] = ldf<AD>(p.A, (long long)m * p.lda + k);
+  __syncthreads();
+  float* out = static_cast<float*>(p.out) + (long long)m * p.ldo;
+  const float* add = p.add_rows ? p.add_rows + (long long)(m % p.add_mod) * p.N : nullptr;
+  if (p.K <= 64) {
+    for (int n = tid; n < p.N; n += 256) {
+      float acc = 0.f;
+      for (int k = 0; k < p.K; ++k) acc = fmaf(a_s[k], ldf<WD>(p.W, (long long)n * p.K + k), acc);
+      out[n] = acc + (p.bias ? p.bias[n] : 0.f) + (add ? add[n] : 0.f);
+    }
+  } else {
+    for (int n = warp; n < p.N; n += 8) {
+      float acc = 0.f;
+#pragma unroll 8
+      for (int k = lane; k < p.K; k += 32) acc = fmaf(a_s[k], ldf<WD>(p.W, (long long)n * p.K + k), acc);
+      acc = warp_sum(acc);
+      if (lane == 0) out[n] = acc + (p.bias ? p.bias[n] : 0.f) + (add ? add[n] : 0.f);
+    }
+  }
+}
+
+bool gemv_rows_ok(const GemmArgs& a) {
+  return a.epi == EPI_STORE && a.out_dtype == F32 && a.K <= kGemvMaxK && (a.N <= 64 || a.K <= 64);
+}
+
+void launch_gemv_rows(const GemmArgs& a, cudaStream_t s) {
+  if (a.a_dtype == F32 && a.w_dtype == F32) launch_k(gemv_rows_kernel<F32, F32>, dim3(a.M), dim3(256), 0, s, a);
+  else if (a.a_dtype == F32 && a.w_dtype == BF16) launch_k(gemv_rows_kernel<F32, BF16>, dim3(a.M), dim3(256), 0, s, a);
+  else if (a.a_dtype == BF16 && a.w_dtype == BF16) launch_k(gemv_rows_kernel<BF16, BF16>, dim3(a.M), dim3(256), 0, s, a);
+  else launch_k(gemv_rows_kernel<BF16, F32>, dim3(a.M), dim3(256), 0, s, a);
+}
+
 void launch_gemm_simt(const GemmArgs& a, cudaStream_t s) {
   dim3 grid((a.N + 63) / 64, (a.M + 63) / 64);
-  if (a.a_dtype == F32 && a.w_dtype == F32) gemm_simt_kernel<F32, F32><<<grid, 256, 0, s>>>(a);
-  else if (a.a_dtype == F32 && a.w_dtype == BF16) gemm_simt_kernel<F32, BF16><<<grid, 256, 0, s>>>(a);
-  else if (a.a_dtype == BF16 && a.w_dtype == BF16) gemm_simt_kernel<BF16, BF16><<<grid, 256, 0, s>>>(a);
-  else gemm_simt_kernel<BF16, F32><<<grid, 256, 0, s>>>(a);
+  if (a.a_dtype == F32 && a.w_dtype == F32) launch_k(gemm_simt_kernel<F32, F32>, grid, dim3(256), 0, s, a);
+  else if (a.a_dtype == F32 && a.w_dtype == BF16) launch_k(gemm_simt_kernel<F32, BF16>, grid, dim3(256), 0, s, a);
+  else if (a.a_dtype == BF16 && a.w_dtype == BF16) launch_k(gemm_simt_kernel<BF16, BF16>, grid, dim3(256), 0, s, a);
+  else launch_k(gemm_simt_kernel<BF16, F32>, grid, dim3(256), 0, s, a);
 }
 
 // ------------------------------------------------------------------------------------------
 // Adaptive norm: y = norm(h) * (1 + scale[tau]) + shift[tau]; one warp per token row.
 // ------------------------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) norm_kernel(NormArgs p) {
+  pdl_trigger();
+  pdl_wait();
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (row >= p.M) return;
   const float* r = p.h + (long long)row * p.ldh;
@@ -152,8 +206,76 @@ __global__ void __launch_bounds__(256) norm_kernel(NormArgs p) {
   }
 }
 
+// Same computation with the whole row held in registers (W = 128 * NV): every load of the row
+// and of its modulation vectors is issued before any arithmetic, so a row costs two memory
+// round trips (modulation-row index, then data) instead of one per 32 elements.
+template <int NV>
+__global__ void __launch_bounds__(256) norm_reg_kernel(NormArgs p) {
+  pdl_trigger();
+  pdl_wait();
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (row >= p.M) return;
+  const float4* r4 = reinterpret_cast<const float4*>(p.h + (long long)row * p.ldh);
+  const float* mod = p.tab ? p.tab + (long long)p.tau_row[row] * p.stride : nullptr;
+  float4 x[NV], sc[NV], sh[NV];
+#pragma unroll
+  for (int i = 0; i < NV; ++i) x[i] = r4[i * 32 + lane];
+  if (mod) {
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+      sc[i] = __ldg(reinterpret_cast<const float4*>(mod + p.scale_off) + i * 32 + lane);
+      sh[i] = __ldg(reinterpret_cast<const float4*>(mod + p.shift_off) + i * 32 + lane);
+    }
+  }
+  float mean = 0.f;
+  if (p.layer_norm) {
+    float t = 0.f;
+#pragma unroll
+    for (int i = 0; i < NV; ++i) t += (x[i].x + x[i].y) + (x[i].z + x[i].w);
+    mean = warp_sum(t) / p.W;
+  }
+  float ss = 0.f;
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    const float a = x[i].x - mean, b = x[i].y - mean, c = x[i].z - mean, d = x[i].w - mean;
+    ss = fmaf(a, a, fmaf(b, b, fmaf(c, c, fmaf(d, d, ss))));
+  }
+  const float rstd = 1.f / sqrtf(warp_sum(ss) / p.W + 1e-6f);
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    float4 y = make_float4((x[i].x - mean) * rstd, (x[i].y - mean) * rstd, (x[i].z - mean) * rstd,
+                           (x[i].w - mean) * rstd);
+    if (mod) {
+      y.x = fmaf(y.x, 1.f + sc[i].x, sh[i].x);
+      y.y = fmaf(y.y, 1.f + sc[i].y, sh[i].y);
+      y.z = fmaf(y.z, 1.f + sc[i].z, sh[i].z);
+      y.w = fmaf(y.w, 1.f + sc[i].w, sh[i].w);
+    }
+    const long long off = (long long)row * p.ldo + (i * 32 + lane) * 4;
+    if (p.out_dtype == BF16) {
+      __nv_bfloat162 lo = __floats2bfloat162_rn(y.x, y.y), hi = __floats2bfloat162_rn(y.z, y.w);
+      uint2 pk;
+      pk.x = *reinterpret_cast<uint32_t*>(&lo);
+      pk.y = *reinterpret_cast<uint32_t*>(&hi);
+      *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(p.out) + off) = pk;
+    } else {
+      *reinterpret_cast<float4*>(static_cast<float*>(p.out) + off) = y;
+    }
+  }
+}
+
 void launch_norm(const NormArgs& a, cudaStream_t s) {
-  norm_kernel<<<(a.M + 7) / 8, 256, 0, s>>>(a);
+  const int blocks = (a.M + 7) / 8;
+  const bool aligned = a.ldh % 4 == 0 && a.ldo % 4 == 0 && a.scale_off % 4 == 0 && a.shift_off % 4 == 0 &&
+                       a.stride % 4 == 0 && a.W % 128 == 0;
+  switch (aligned ? a.W / 128 : 0) {
+    case 2: launch_k(norm_reg_kernel<2>, dim3(blocks), dim3(256), 0, s, a); break;
+    case 3: launch_k(norm_reg_kernel<3>, dim3(blocks), dim3(256), 0, s, a); break;
+    case 4: launch_k(norm_reg_kernel<4>, dim3(blocks), dim3(256), 0, s, a); break;
+    case 8: launch_k(norm_reg_kernel<8>, dim3(blocks), dim3(256), 0, s, a); break;
+    case 12: launch_k(norm_reg_kernel<12>, dim3(blocks), dim3(256), 0, s, a); break;
+    default: launch_k(norm_kernel, dim3(blocks), dim3(256), 0, s, a); break;
+  }
 }
 
 // ------------------------------------------------------------------------------------------
@@ -175,6 +297,8 @@ __device__ __forceinline__ float rope_elem(const void* base, long long off, int 
 template <int DPL>
 __global__ void __launch_bounds__(128) attn_kernel(AttnArgs p) {
   extern __shared__ float sm[];
+  pdl_trigger();
+  pdl_wait();
   const int dh = DPL * 32, half = dh / 2;
   float* qs = sm;                   // [AQ][dh]
   float* ks = qs + AQ * dh;         // [AKB][dh + 1]
@@ -263,7 +387,7 @@ __global__ void __launch_bounds__(128) attn_kernel(AttnArgs p) {
 
 template <int DPL>
 static void launch_attn_dpl(const AttnArgs& a, dim3 grid, size_t smem, cudaStream_t s) {
-  attn_kernel<DPL><<<grid, 128, smem, s>>>(a);
+  launch_k(attn_kernel<DPL>, grid, dim3(128), smem, s, a);
 }
 
 size_t attention_smem_bytes(int dh) {
@@ -296,6 +420,8 @@ void launch_attention(const AttnArgs& a, cudaStream_t s) {
 // last step GAC (Eqs. 8-9). Released rows go to mapped pinned memory, then a per-step flag.
 // ------------------------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) euler_kernel(EulerArgs p) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x, tid = threadIdx.x;
   const int HD = p.H * p.D;
   const float gs = p.gstep[b];
@@ -369,10 +495,12 @@ __global__ void __launch_bounds__(256) euler_kernel(EulerArgs p) {
   }
 }
 
-void launch_euler(const EulerArgs& a, cudaStream_t s) { euler_kernel<<<a.B, 256, 0, s>>>(a); }
+void launch_euler(const EulerArgs& a, cudaStream_t s) { launch_k(euler_kernel, dim3(a.B), dim3(256), 0, s, a); }
 
 __global__ void begin_kernel(const float* noise, float* x, float* g, float* u, int n, int* nonfinite,
                              int* evals, unsigned long long* stamps) {
+  pdl_trigger();
+  pdl_wait();
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i == 0) {
     *nonfinite = 0;
@@ -389,7 +517,7 @@ __global__ void begin_kernel(const float* noise, float* x, float* g, float* u, i
 
 void launch_begin(const float* noise, float* x, float* g, float* u, int n, int* nonfinite, int* evals,
                   unsigned long long* stamps, cudaStream_t s) {
-  begin_kernel<<<(n + 255) / 256, 256, 0, s>>>(noise, x, g, u, n, nonfinite, evals, stamps);
+  launch_k(begin_kernel, dim3((n + 255) / 256), dim3(256), 0, s, noise, x, g, u, n, nonfinite, evals, stamps);
 }
 
 // ------------------------------------------------------------------------------------------

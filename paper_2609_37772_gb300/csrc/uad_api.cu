@@ -64,6 +64,10 @@ struct uad_ctx {
 
   // tensor-core GEMM: TMA descriptors of the activation buffers, split-K workspace
   std::map<const void*, CUtensorMap> tmaps;
+  // tensor-core attention (bf16 joint-attention experts): query matrix, K and Vt caches
+  bool attn_tc = false;
+  AttnTcArgs at0;                 // shapes and buffers; batch / layer set per launch
+  AttnTcMaps atmaps;
   float* tc_acc = nullptr;
   int* tc_counters = nullptr;
   int* dev_err = nullptr;
@@ -320,11 +324,11 @@ struct Mark {
       c->prof_ev.push_back(e);
     }
     c->prof.push_back({name, bytes, flops, c->prof_next, c->prof_next + 1});
-    cudaEventRecord(c->prof_ev[c->prof_next], s);
+    cudaEventRecordWithFlags(c->prof_ev[c->prof_next], s, cudaEventRecordExternal);
     c->prof_next += 2;
   }
   ~Mark() {
-    if (c->prof_on) cudaEventRecord(c->prof_ev[c->prof.back().ev1], s);
+    if (c->prof_on) cudaEventRecordWithFlags(c->prof_ev[c->prof.back().ev1], s, cudaEventRecordExternal);
   }
 };
 
@@ -342,7 +346,8 @@ double gemm_bytes(const GemmArgs& g, int wes) {
 void gemm(uad_ctx* c, const Lin& w, GemmArgs g, cudaStream_t s) {
   g.W = w.w;
   if (!w.tiled) {
-    launch_gemm_simt(g, s);
+    if (gemv_rows_ok(g)) launch_gemv_rows(g, s);
+    else launch_gemm_simt(g, s);
     return;
   }
   TcGemmArgs t;
@@ -350,7 +355,7 @@ void gemm(uad_ctx* c, const Lin& w, GemmArgs g, cudaStream_t s) {
   t.splits = gemm_tc_splits(g.M, g.N, g.K, c->sms);
   t.epi = g.epi; t.out = g.out; t.ldo = g.ldo; t.out_dtype = g.out_dtype; t.bias = g.bias;
   t.resid = g.resid; t.ldr = g.ldr; t.gate_tab = g.gate_tab; t.gate_stride = g.gate_stride;
-  t.tau_row = g.tau_row; t.acc = c->tc_acc; t.counters = c->tc_counters; t.err = c->dev_err;
+  t.tau_row = g.tau_row; t.qkv = g.qkv; t.acc = c->tc_acc; t.counters = c->tc_counters; t.err = c->dev_err;
   launch_gemm_tc(&c->tmaps.at(g.A), t, s);
 }
 
@@ -401,6 +406,15 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
       GemmArgs gq;
       gq.A = c->y; gq.lda = W; gq.a_dtype = dt; gq.w_dtype = dt;
       gq.M = M; gq.N = c->qkvd; gq.K = W; gq.out = c->qkv; gq.ldo = c->qkvd; gq.out_dtype = dt;
+      if (c->attn_tc) {
+        QkvTcOut& o = gq.qkv;
+        gq.epi = EPI_QKV_TC;
+        o.q = c->at0.q; o.kcache = c->at0.kcache; o.vtcache = c->at0.vtcache;
+        o.rope = a.rope ? c->rope_cs : nullptr;
+        o.H = H; o.P = a.prefix_len; o.NK = c->at0.n_keys; o.NKp = c->at0.nk_pad; o.dh = a.head_dim;
+        o.G = a.n_heads / a.n_kv_heads; o.Hkv = a.n_kv_heads; o.L = a.n_layers; o.layer = l;
+        o.qd = c->qd; o.kvd = c->kvd;
+      }
       { Mark mk(c, s, "qkv_proj", gemm_bytes(gq, c->es), 2.0 * M * gq.N * W); gemm(c, w.wqkv, gq, s); }
       AttnArgs at;
       at.n_heads = a.n_heads; at.n_kv_heads = a.n_kv_heads; at.head_dim = a.head_dim; at.H = H; at.B = B;
@@ -415,7 +429,14 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
         at.P = a.prefix_len; at.kp_bstride = (long long)a.n_layers * a.prefix_len * c->kvd;
         at.kp_ld = c->kvd; at.rope_cs = a.rope ? c->rope_cs : nullptr;
       }
-      {
+      if (c->attn_tc) {
+        AttnTcArgs t = c->at0;
+        t.batch = B; t.layer = l;
+        const double keys = (double)t.n_keys;
+        const double by = 2.0 * ((double)B * t.n_keys * c->kvd * 2 + (double)M * 2 * c->qd);
+        Mark mk(c, s, "attention", by, 4.0 * M * a.n_heads * keys * a.head_dim);
+        launch_attn_tc(c->atmaps, t, s);
+      } else {
         const double keys = (double)(at.P + H);
         const double by = c->es * ((double)B * at.P * c->kvd * 2 + (double)M * (2 * c->qd + 2 * c->kvd));
         Mark mk(c, s, dit ? "self_attn" : "attention", by, 4.0 * M * a.n_heads * keys * a.head_dim);
@@ -495,8 +516,8 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
   }
 }
 
-int launches_per_step(const uad_arch& a) {
-  return a.kind == UAD_KIND_DIT ? 11 * a.n_layers + 4 : 7 * a.n_layers + 4;
+int launches_per_step(const uad_arch& a, bool attn_tc) {
+  return a.kind == UAD_KIND_DIT ? 11 * a.n_layers + 4 : (attn_tc ? 8 : 7) * a.n_layers + 4;
 }
 
 }  // namespace
@@ -630,16 +651,20 @@ int uad_init(const uad_arch* arch, const float* weights, size_t n_floats, uad_ct
     l->tiled = dt == BF16 && !c->force_simt && N % 128 == 0 && K % 64 == 0;
     return dalloc(c, &l->w, (size_t)N * K * es);
   };
-  auto put = [&](const std::string& n, const Lin& l, int mult, long long off) {
-    if (l.tiled) launch_relayout_tiled(src(n), (int)T.at(n)->rows, (int)T.at(n)->cols, l.w, mult, off, s0);
+  auto put = [&](const std::string& n, const Lin& l, int mult, long long off, int rope_dh = 0) {
+    if (l.tiled) launch_relayout_tiled(src(n), (int)T.at(n)->rows, (int)T.at(n)->cols, l.w, mult, off, rope_dh, s0);
     else lin(n, l.w, mult, off);
   };
+  // tensor-core attention: bf16 joint-attention experts whose QKV projection is tiled
+  c->attn_tc = a.kind == UAD_KIND_ADARMS && dt == BF16 && !c->force_simt && c->qkvd % 128 == 0 && W % 64 == 0 &&
+              a.prefix_len + H <= attn_tc_max_keys();
+  const int qk_perm = c->attn_tc && a.rope ? a.head_dim : 0;
   for (int l = 0; l < a.n_layers; ++l) {
     const std::string p = "l" + std::to_string(l) + ".";
     LayerW& w = c->L[l];
     TRY(mklin(&w.wqkv, c->qkvd, W));
-    put(p + "wq", w.wqkv, 1, 0);
-    put(p + "wk", w.wqkv, 1, c->qd);
+    put(p + "wq", w.wqkv, 1, 0, qk_perm);
+    put(p + "wk", w.wqkv, 1, c->qd, qk_perm);
     put(p + "wv", w.wqkv, 1, c->qd + (a.kind == UAD_KIND_DIT ? c->qd : c->kvd));
     TRY(mklin(&w.wo, W, c->qd)); put(p + "wo", w.wo, 1, 0);
     if (a.kind == UAD_KIND_ADARMS) {
@@ -704,6 +729,27 @@ int uad_init(const uad_arch* arch, const float* weights, size_t n_floats, uad_ct
   for (float** p : {&c->v, &c->x, &c->g, &c->u, &c->rel, &c->fin, &c->ghost, &c->noise})
     TRY(dalloc_t(c, p, M * D));
   TRY(dalloc_t(c, &c->dev_err, 1));
+  if (c->attn_tc) {
+    AttnTcArgs& t = c->at0;
+    t.n_layers = a.n_layers; t.n_kv_heads = a.n_kv_heads; t.group = a.n_heads / a.n_kv_heads;
+    t.head_dim = a.head_dim; t.H = H; t.prefix = a.prefix_len; t.n_keys = a.prefix_len + H;
+    t.nk_pad = (t.n_keys + 7) / 8 * 8; t.rows = t.group * H; t.r_pad = attn_tc_rpad(t.rows);
+    t.scale_log2 = 1.4426950408889634f / std::sqrt((float)a.head_dim);
+    t.out_ld = c->qd; t.err = c->dev_err;
+    const size_t kvz = (size_t)a.max_batch * a.n_layers * a.n_kv_heads;
+    const int chunks = attn_tc_chunks(t.n_keys);
+    void* p;
+    TRY(dalloc(c, &p, (size_t)a.max_batch * a.n_kv_heads * t.rows * a.head_dim * 2)); t.q = (__nv_bfloat16*)p;
+    TRY(dalloc(c, &p, kvz * t.n_keys * a.head_dim * 2)); t.kcache = (__nv_bfloat16*)p;
+    TRY(dalloc(c, &p, kvz * a.head_dim * t.nk_pad * 2)); t.vtcache = (__nv_bfloat16*)p;
+    TRY(dalloc_t(c, &t.part_o, (size_t)a.max_batch * a.n_kv_heads * chunks * t.r_pad * a.head_dim));
+    TRY(dalloc_t(c, &t.part_ml, (size_t)a.max_batch * a.n_kv_heads * chunks * t.r_pad * 2));
+    t.out = (__nv_bfloat16*)c->o;
+    if (attn_tc_prepare(&c->atmaps, t, a.max_batch)) {
+      fail(c, UAD_ECUDA, "attention TMA descriptors failed");
+      TRY(UAD_ECUDA);
+    }
+  }
   if (dt == BF16 && !c->force_simt) {
     TRY(make_tmap(c, c->y, W, (int)M));
     TRY(make_tmap(c, c->o, c->qd, (int)M));
@@ -749,7 +795,24 @@ int uad_set_prefix_kv(uad_ctx* c, int32_t robot, const void* k, const void* v, i
   if (c->in_flight) return fail(c, UAD_ESTATE, "a chunk is in flight");
   const int ies = dtype == UAD_DTYPE_BF16 ? 2 : 4;
   cudaStream_t s = c->worker;
-  if (a.kind == UAD_KIND_ADARMS) {
+  if (a.kind == UAD_KIND_ADARMS && c->attn_tc) {
+    if (!v) return fail(c, UAD_EINVAL, "null prefix values");
+    const size_t n = (size_t)a.n_layers * a.prefix_len * c->kvd;
+    void *tk = nullptr, *tv = nullptr;
+    if (cudaMalloc(&tk, n * ies) != cudaSuccess) return fail(c, UAD_ENOMEM, "prefix staging");
+    if (cudaMalloc(&tv, n * ies) != cudaSuccess) { cudaFree(tk); return fail(c, UAD_ENOMEM, "prefix staging"); }
+    int rc = UAD_OK;
+    if (cudaMemcpyAsync(tk, k, n * ies, cudaMemcpyDefault, s) != cudaSuccess ||
+        cudaMemcpyAsync(tv, v, n * ies, cudaMemcpyDefault, s) != cudaSuccess)
+      rc = UAD_ECUDA;
+    else
+      launch_kv_prefix(tk, tv, dtype, c->at0, robot, s);
+    cudaError_t e = cudaStreamSynchronize(s);
+    cudaFree(tk);
+    cudaFree(tv);
+    if (rc != UAD_OK || e != cudaSuccess || cudaGetLastError() != cudaSuccess)
+      return fail(c, UAD_ECUDA, "prefix upload failed");
+  } else if (a.kind == UAD_KIND_ADARMS) {
     if (!v) return fail(c, UAD_EINVAL, "null prefix values");
     const size_t n = (size_t)a.n_layers * a.prefix_len * c->kvd;
     void* tmp = nullptr;
@@ -901,12 +964,36 @@ static int denoise_impl(uad_ctx* c, const float* noise, const uad_schedule* sc, 
       it = c->graphs.emplace(key, ex).first;
     }
     CK(cudaGraphLaunch(it->second, s));
-  } else {
-    c->prof_on = profile;
+  } else if (profile) {
+    // capture with an event-record node around every kernel, so that the event times are
+    // GPU timestamps between graph nodes (no host launch gaps)
+    c->prof_on = true;
     c->prof.clear();
     c->prof_next = 0;
+    // create the events before capture
+    {
+      int need = 2 * (1 + steps * launches_per_step(c->a, c->attn_tc)) + 8;
+      while ((int)c->prof_ev.size() < need) {
+        cudaEvent_t e;
+        CK(cudaEventCreate(&e));
+        c->prof_ev.push_back(e);
+      }
+    }
+    cudaGraph_t g = nullptr;
+    CK(cudaStreamBeginCapture(s, cudaStreamCaptureModeThreadLocal));
     enqueue_chunk(c, B, steps, s);
+    cudaError_t e = cudaStreamEndCapture(s, &g);
     c->prof_on = false;
+    if (e != cudaSuccess) return fail(c, UAD_ECUDA, "profile capture failed: %s", cudaGetErrorString(e));
+    cudaGraphExec_t ex = nullptr;
+    e = cudaGraphInstantiate(&ex, g, 0);
+    cudaGraphDestroy(g);
+    if (e != cudaSuccess) return fail(c, UAD_ECUDA, "profile instantiate failed: %s", cudaGetErrorString(e));
+    e = cudaGraphLaunch(ex, s);
+    cudaGraphExecDestroy(ex);
+    if (e != cudaSuccess) return fail(c, UAD_ECUDA, "profile launch failed: %s", cudaGetErrorString(e));
+  } else {
+    enqueue_chunk(c, B, steps, s);
     CK(cudaGetLastError());
   }
   CK(cudaEventRecord(c->ev_done, s));
@@ -1036,7 +1123,7 @@ int uad_step_times(const uad_ctx* c, double* ms, int32_t max_entries) {
 
 int uad_launches_per_chunk(const uad_ctx* c, int32_t batch, int32_t n_star) {
   if (!c || batch < 1 || n_star < 1) return UAD_EINVAL;
-  return 1 + n_star * launches_per_step(c->a);
+  return 1 + n_star * launches_per_step(c->a, c->attn_tc);
 }
 
 void uad_destroy(uad_ctx* c) {

@@ -12,6 +12,30 @@ constexpr int kFlagStride = kMaxSteps + 1;  // host flag slots per robot (steps 
 
 enum DType { F32 = 0, BF16 = 1 };
 
+// Programmatic dependent launch. Kernels of the step loop are launched so that the next kernel's
+// CTAs may start while the previous kernel drains; every kernel calls pdl_trigger() once it has
+// started and pdl_wait() before it reads anything a predecessor wrote or writes anything a
+// predecessor reads (pdl_wait returns at once for a kernel launched without the attribute).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+bool pdl_enabled();   // UAD_PDL=0 turns it off (debugging)
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_k(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                            Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = pdl_enabled() ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<Args&&>(args)...);
+}
+
 // GEMM epilogues (out[m][n] from acc = sum_k A[m][k] * Wt[n][k]).
 enum Epi {
   EPI_STORE = 0,       // out = acc (+ bias) (+ add_rows[m % add_mod][n])
@@ -19,6 +43,17 @@ enum Epi {
   EPI_RESID_GATE = 2,  // resid[m][n] += gate(m, n) * (acc + bias); gate = 1 when gate_tab is null
   EPI_GEGLU = 3,       // rows interleaved (2j = gate, 2j+1 = up): out[m][j] = gelu_tanh(g) * u
   EPI_BIAS_GELU = 4,   // out = gelu_tanh(acc + bias)
+  EPI_QKV_TC = 5,      // q/k rows pair-interleaved per head: RoPE, then scatter q -> Q, k -> K cache,
+                       // v -> Vt cache (tensor-core attention layouts, see attn_tc.cu)
+};
+
+// Where the QKV projection epilogue (EPI_QKV_TC) writes, and the RoPE table it uses.
+struct QkvTcOut {
+  __nv_bfloat16* q = nullptr;        // [B][Hkv][G*H][dh]
+  __nv_bfloat16* kcache = nullptr;   // [B][L][Hkv][NK][dh]
+  __nv_bfloat16* vtcache = nullptr;  // [B][L][Hkv][dh][NKp]
+  const float* rope = nullptr;       // [H][dh/2][2] (cos, sin) at positions P + i, or null
+  int H = 0, P = 0, NK = 0, NKp = 0, dh = 0, G = 1, Hkv = 1, L = 0, layer = 0, qd = 0, kvd = 0;
 };
 
 struct GemmArgs {
@@ -32,6 +67,7 @@ struct GemmArgs {
   float* resid = nullptr; int ldr = 0;             // EPI_RESID_GATE target, fp32
   const float* gate_tab = nullptr; int gate_stride = 0;  // gate(m, n) = gate_tab[tau_row[m] * gate_stride + n]
   const int* tau_row = nullptr;
+  QkvTcOut qkv;                                    // EPI_QKV_TC
 };
 
 struct NormArgs {
@@ -85,7 +121,10 @@ struct EulerArgs {
 };
 
 // kernels_simt.cu
+constexpr int kGemvMaxK = 8192;
 void launch_gemm_simt(const GemmArgs& a, cudaStream_t s);
+bool gemv_rows_ok(const GemmArgs& a);                     // tiny-side projection (N or K <= 64)
+void launch_gemv_rows(const GemmArgs& a, cudaStream_t s);
 void launch_norm(const NormArgs& a, cudaStream_t s);
 void launch_attention(const AttnArgs& a, cudaStream_t s);
 void launch_euler(const EulerArgs& a, cudaStream_t s);
@@ -99,7 +138,8 @@ void launch_attention_prepare(int dh);  // opt in to > 48 KB dynamic shared memo
 void launch_convert(const void* src, int src_dtype, void* dst, int dst_dtype, long long n, cudaStream_t s);
 
 // gemm_tc.cu: tcgen05 projection GEMM (bf16 operands, fp32 accumulation in TMEM)
-constexpr int kTcMaxStages = 8;
+constexpr int kTcMaxStages = 4;        // <= ~97 KB of shared memory: two CTAs fit one SM
+constexpr int kTcMaxStagesResid = 3;   // plus the staged gate / residual rows
 struct TcGemmArgs {
   const void* w_tiled = nullptr;   // [N/128][K/64] blocks of 128 x 64 bf16, 128B-swizzled K-major
   int M = 0, N = 0, K = 0, splits = 1;
@@ -108,18 +148,43 @@ struct TcGemmArgs {
   const float* bias = nullptr;
   float* resid = nullptr; int ldr = 0;
   const float* gate_tab = nullptr; int gate_stride = 0; const int* tau_row = nullptr;
+  QkvTcOut qkv;                    // EPI_QKV_TC
   float* acc = nullptr;            // split-K accumulator [M][N] fp32, zero between launches
   int* counters = nullptr;         // split-K arrival counters per output tile, zero between launches
   int* err = nullptr;              // set to a nonzero code if a bounded wait gave up
 };
-size_t gemm_tc_smem_bytes(int stages);
+size_t gemm_tc_smem_bytes(int stages, int epi);
 // 2-D TMA descriptor of a bf16 activation matrix [rows][K] (64 x 64 boxes, 128-byte swizzle,
 // zero fill past the last row). 0 on success.
 int encode_act_tmap(CUtensorMap* m, const void* base, int K, int rows);
 void gemm_tc_prepare();
 int gemm_tc_splits(int M, int N, int K, int sms);
 void launch_gemm_tc(const CUtensorMap* tmx, const TcGemmArgs& a, cudaStream_t s);
-// element (k, n) of src [K][N] -> row n * mult + off, column k of the tiled bf16 layout (K cols)
-void launch_relayout_tiled(const float* src, int K, int N, void* dst, int mult, long long off, cudaStream_t s);
+// element (k, n) of src [K][N] -> row n' * mult + off, column k of the tiled bf16 layout (K cols),
+// where n' = n, or with rope_dh > 0 the head-local pair interleave (d, d + dh/2) -> (2d, 2d + 1)
+void launch_relayout_tiled(const float* src, int K, int N, void* dst, int mult, long long off, int rope_dh,
+                           cudaStream_t s);
+
+// attn_tc.cu: tensor-core attention over [prefix ; chunk] keys
+struct AttnTcArgs {
+  int batch = 0, n_layers = 0, layer = 0, n_kv_heads = 0, group = 1, head_dim = 0, H = 0, prefix = 0;
+  int n_keys = 0, nk_pad = 0, rows = 0, r_pad = 0;
+  float scale_log2 = 0.f;              // log2(e) / sqrt(dh)
+  __nv_bfloat16* q = nullptr;          // [B][Hkv][rows][dh]
+  __nv_bfloat16* kcache = nullptr;     // [B][L][Hkv][n_keys][dh]
+  __nv_bfloat16* vtcache = nullptr;    // [B][L][Hkv][dh][nk_pad]
+  float* part_o = nullptr;             // [B*Hkv][chunks][r_pad][dh]
+  float* part_ml = nullptr;            // [B*Hkv][chunks][r_pad][2]
+  __nv_bfloat16* out = nullptr; int out_ld = 0;   // o [B*H][Hq*dh]
+  int* err = nullptr;
+};
+struct AttnTcMaps { CUtensorMap q, k, vt; };
+size_t attn_tc_smem_bytes(int dh);
+int attn_tc_prepare(AttnTcMaps* maps, const AttnTcArgs& a, int batch_max);  // 0 on success
+int attn_tc_chunks(int n_keys);
+int attn_tc_max_keys();
+int attn_tc_rpad(int rows);
+void launch_attn_tc(const AttnTcMaps& maps, const AttnTcArgs& a, cudaStream_t s);   // 2 kernels
+void launch_kv_prefix(const void* k, const void* v, int src_dtype, const AttnTcArgs& a, int robot, cudaStream_t s);
 
 }  // namespace uad
