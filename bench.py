@@ -41,6 +41,9 @@ WORKLOADS = {
     "tiny": dict(arch="tiny", batch=1, groups=[(0, 3, 5), (4, 15, 10)], t_act_ms=10.0,
                  desc="tiny fp32 expert, B=1, first 4 actions after 5 of 10 steps"),
 }
+for _k, _u in [(k, u) for k in (2, 3, 4, 6) for u in (5, 10, 20)]:
+    WORKLOADS[f"pi0-k{_k}-u{_u}"] = dict(arch="pi0", batch=1, groups=[(0, _u - 1, _k), (_u, 49, 10)], t_act_ms=10.0,
+                                         desc=f"pi0-like bf16 expert, B=1, first {_u} actions after {_k} of 10 steps, TR+GAC")
 for _b in (4, 16, 64):
     WORKLOADS[f"pi0-b{_b}"] = dict(arch="pi0", batch=_b, groups=None, t_act_ms=10.0,
                                    desc=f"pi0-like bf16 expert, B={_b} robots, schedules drawn from the sweep grid")
@@ -345,6 +348,41 @@ def run_ours(args, wl, world, rank, local):
     return 0
 
 
+def run_sweep(args):
+    """Schedule sweep on one context: AAL / first-action latency / chunk time per schedule."""
+    import torch
+    import paper_2609_37772_gb300 as uad
+    a = ARCHS["pi0"]
+    ex = uad.Expert(a, make_weights(a), max_batch=1)
+    ex.set_prefix(0, *make_prefix_kv(a))
+    ex.prepare_times(10)
+    noise = torch.from_numpy(make_noise(a, 1)).cuda()
+    stream = torch.cuda.current_stream()
+    for k, u in [(k, u) for k in (2, 3, 4, 6) for u in (5, 10, 20)] + [(10, 50)]:
+        bud = group_budgets(a.chunk_len, [(0, u - 1, k)] + ([(u, 49, 10)] if u < 50 else []))[None]
+        for _ in range(args.warmup):
+            ex.denoise(noise, bud, stream=stream)
+            ex.finish(timeout_us=60_000_000)
+        rows = []
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            ex.denoise(noise, bud, stream=stream)
+            ex.finish(timeout_us=60_000_000)
+            st = ex.step_times()
+            rows.append([float(st[int(bud[0][i]) - 1]) for i in range(a.chunk_len)])
+        e1.record(stream)
+        torch.cuda.synchronize()
+        print(json.dumps({"sweep": "pi0-like B=1", "first_group_budget": k, "first_group_size": u,
+                          "ms_per_chunk": e0.elapsed_time(e1) / args.steps,
+                          "first_action_ms": statistics.mean(r[0] for r in rows),
+                          "aal_ms_10ms_S50": statistics.mean(aal_ms(r, 10.0, 50) for r in rows),
+                          "aal_ms_10ms_S10": statistics.mean(aal_ms(r, 10.0, 10) for r in rows)}), flush=True)
+    ex.close()
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -354,7 +392,11 @@ def main():
     ap.add_argument("--workload", default="pi0-b1", choices=sorted(WORKLOADS))
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="pi0-like B=1 schedule sweep: one JSON line per (first-group budget, size)")
     args = ap.parse_args()
+    if args.sweep:
+        return run_sweep(args)
     wl = WORKLOADS[args.workload]
     world, rank, local = dist_setup()
     try:
