@@ -69,6 +69,10 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;"
       ::"r"(su32(dst)), "l"(src), "r"(bytes), "r"(su32(bar)), "l"(pol) : "memory");
 }
+__device__ __forceinline__ void bulk_g2s_plain(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               ::"r"(su32(dst)), "l"(src), "r"(bytes), "r"(su32(bar)) : "memory");
+}
 __device__ __forceinline__ void tma_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
   asm volatile(
       "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
@@ -116,32 +120,14 @@ __device__ __forceinline__ void store_out(void* out, long long i, float v, int d
   else static_cast<float*>(out)[i] = v;
 }
 
-// Store one already-rotated q / k value (or a v value) of output row n, robot b, token i into
-// the tensor-core attention layouts.
-__device__ __forceinline__ void epi_qkv_store_bi(const QkvTcOut& o, int b, int i, int n, float val) {
-  if (n < o.qd + o.kvd) {
-    const int sn = n < o.qd ? n : n - o.qd;
-    const int h = sn / o.dh, r = sn % o.dh, half = o.dh / 2;
-    const int d = o.rope ? ((r & 1) ? (r >> 1) + half : (r >> 1)) : r;
-    if (n < o.qd) {
-      const int g = h / o.G, jj = h % o.G;
-      o.q[(((size_t)b * o.Hkv + g) * o.G * o.H + (size_t)jj * o.H + i) * o.dh + d] = __float2bfloat16_rn(val);
-    } else {
-      o.kcache[((((size_t)b * o.L + o.layer) * o.Hkv + h) * o.NK + o.P + i) * o.dh + d] = __float2bfloat16_rn(val);
-    }
-  } else {
-    const int sn = n - o.qd - o.kvd, g = sn / o.dh, d = sn % o.dh;
-    o.vtcache[((((size_t)b * o.L + o.layer) * o.Hkv + g) * o.dh + d) * o.NKp + o.P + i] = __float2bfloat16_rn(val);
-  }
-}
-
 __device__ __forceinline__ void red_add_v4(float* dst, float4 v) {
   asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(dst), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
                : "memory");
 }
 
 // Shared-memory plan: [pipeline stages, at least 32 KB (reused as the split-K staging tile)]
-// [gate rows 32 KB][residual rows 32 KB] (residual epilogue only) [mbarriers, TMEM slot, flag].
+// [gate rows][residual rows] (residual epilogue only: min(M, 64) rows of 128 fp32 each)
+// [mbarriers, TMEM slot, flag].
 __host__ __device__ __forceinline__ int tc_stages(int nch, int epi) {
   const int cap = epi == EPI_RESID_GATE ? kTcMaxStagesResid : kTcMaxStages;
   return nch < cap ? nch : cap;
@@ -150,9 +136,18 @@ __host__ __device__ __forceinline__ size_t tc_pipe_bytes(int stages) {
   const size_t b = (size_t)stages * (kStageA + kStageB);
   return b < 32768 ? 32768 : b;
 }
+__host__ __device__ __forceinline__ int tc_gr_rows(int M) { return M < kBN ? M : kBN; }
+
+// Optional phase timestamps (TcGemmArgs::trace): slot i of this CTA's 16.
+#define TC_TRACE(i)                                                                                  \
+  do {                                                                                               \
+    if (p.trace)                                                                                     \
+      p.trace[((size_t)(blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x) * 16 + (i)] = gtime(); \
+  } while (0)
 
 __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__ CUtensorMap tmx, TcGemmArgs p) {
   extern __shared__ uint8_t smem_raw[];
+  if (threadIdx.x == 0) TC_TRACE(0);
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   const int t = blockIdx.x, mt = blockIdx.y, s = blockIdx.z;
   const int KC = p.K / kBK;
@@ -161,12 +156,14 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   const bool resid = p.epi == EPI_RESID_GATE;
   uint8_t* sA = smem;
   uint8_t* sB = smem + (size_t)stages * kStageA;
-  float* G = reinterpret_cast<float*>(smem + tc_pipe_bytes(stages));   // [kBN][kBM] gates
-  float* R = G + kBN * kBM;                                            // [kBN][kBM] residual rows
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + tc_pipe_bytes(stages) + (resid ? 2 * kBN * kBM * 4 : 0));
+  const int grr = tc_gr_rows(p.M);
+  float* G = reinterpret_cast<float*>(smem + tc_pipe_bytes(stages));   // [grr][kBM] gates
+  float* R = G + grr * kBM;                                            // [grr][kBM] residual rows
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + tc_pipe_bytes(stages) + (resid ? 2 * grr * kBM * 4 : 0));
   uint64_t* empty = full + kTcMaxStages;
   uint64_t* done = empty + kTcMaxStages;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  uint64_t* bar_gr = done + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_gr + 1);
   int* last_flag = reinterpret_cast<int*>(tmem_slot + 1);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int m0 = mt * kBN;
@@ -178,6 +175,7 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
       mbar_init(empty + i, 1);
     }
     mbar_init(done, 1);
+    mbar_init(bar_gr, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 0) {
@@ -188,6 +186,7 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  if (threadIdx.x == 0) TC_TRACE(1);
 
   pdl_trigger();
   if (threadIdx.x == 0) {
@@ -201,7 +200,9 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
       mbar_expect_tx(full + i, kStageA + kStageB);
       bulk_g2s(sA + (size_t)i * kStageA, wt + (size_t)i * kStageA, kStageA, full + i, pol);
     }
+    TC_TRACE(2);
     pdl_wait();
+    TC_TRACE(3);
     for (int i = 0; i < first; ++i) tma_2d(sB + (size_t)i * kStageB, &tmx, (c0 + i) * kBK, mt * kBN, full + i);
     int issued = first;
     for (int i = first; i < nch; ++i) {
@@ -222,6 +223,7 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
       const int st = i % stages, round = i / stages;
       ok = mbar_wait(full + st, round & 1, p.err, 13);
       if (!ok) break;
+      if (i == 0) TC_TRACE(4);
       tc_fence_after();
       const uint32_t a0 = su32(sA + (size_t)st * kStageA), b0 = su32(sB + (size_t)st * kStageB);
 #pragma unroll
@@ -229,35 +231,20 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
         mma_bf16(tmem, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), (i > 0 || k > 0) ? 1u : 0u);
       mma_commit(empty + st);
     }
+    TC_TRACE(5);
     mma_commit(done);
-  } else if (resid && warp >= 2) {
-    // ---- warps 2-3 prefetch the residual epilogue's inputs while the tile is computed:
-    //      gate rows gate_tab[tau(m)][n0..n0+127] and residual rows resid[m][n0..n0+127] ----
+  } else if (resid && warp == 2) {
+    // ---- warp 2 fetches the residual epilogue's inputs while the tile is computed: one 512-byte
+    //      bulk copy per token for the residual row resid[m][n0..n0+127] and for the gate row
+    //      gate_tab[tau(m)][n0..n0+127], all in flight at once ----
     pdl_wait();
-    const int tid = threadIdx.x - 64;
     const int n0 = t * kBM;
-    for (int base = 0; base < mcount * (kBM / 4); base += 64 * 8) {
-      float4 g[8], r[8];
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int idx = base + u * 64 + tid;
-        if (idx < mcount * (kBM / 4)) {
-          const int j = idx / (kBM / 4), c4 = idx % (kBM / 4);
-          g[u] = p.gate_tab ? __ldg(reinterpret_cast<const float4*>(
-                                  p.gate_tab + (size_t)p.tau_row[m0 + j] * p.gate_stride + n0 + c4 * 4))
-                            : make_float4(1.f, 1.f, 1.f, 1.f);
-          r[u] = *reinterpret_cast<const float4*>(p.resid + (size_t)(m0 + j) * p.ldr + n0 + c4 * 4);
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int idx = base + u * 64 + tid;
-        if (idx < mcount * (kBM / 4)) {
-          const int j = idx / (kBM / 4), c4 = idx % (kBM / 4);
-          *reinterpret_cast<float4*>(G + j * kBM + c4 * 4) = g[u];
-          *reinterpret_cast<float4*>(R + j * kBM + c4 * 4) = r[u];
-        }
-      }
+    if (lane == 0) mbar_expect_tx(bar_gr, (p.gate_tab ? 2u : 1u) * (uint32_t)mcount * (kBM * 4));
+    __syncwarp();
+    for (int j = lane; j < mcount; j += 32) {
+      bulk_g2s_plain(R + j * kBM, p.resid + (size_t)(m0 + j) * p.ldr + n0, kBM * 4, bar_gr);
+      if (p.gate_tab)
+        bulk_g2s_plain(G + j * kBM, p.gate_tab + (size_t)p.tau_row[m0 + j] * p.gate_stride + n0, kBM * 4, bar_gr);
     }
   }
   __syncwarp();
@@ -265,6 +252,7 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   // ---- epilogue: TMEM -> registers, one weight row (output feature) per thread ----
   pdl_wait();
   const bool ok = mbar_wait(done, 0, p.err, 14);
+  if (threadIdx.x == 64) TC_TRACE(6);
   tc_fence_after();
   const int row = warp * 32 + lane;
   const int n = t * kBM + row;
@@ -280,6 +268,7 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
 #pragma unroll
   for (int j = 0; j < kBN; ++j) T[j * kBM + row] = v[j];
   __syncthreads();
+  if (threadIdx.x == 0) TC_TRACE(7);
   if (p.splits > 1) {
     // add the partial tile into the L2 accumulator with 16-byte reds; the last CTA of the tile
     // reads the sum back (independent 16-byte loads) and clears it for the next launch
@@ -293,8 +282,10 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
     __threadfence();
     __syncthreads();
     if (threadIdx.x == 0) {
+      TC_TRACE(8);
       const int prev = atomicAdd(p.counters + mt * gridDim.x + t, 1);
       *last_flag = prev == p.splits - 1;
+      TC_TRACE(9);
     }
     __syncthreads();
     const bool last = *last_flag;
@@ -320,8 +311,9 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
       if (threadIdx.x == 0) p.counters[mt * gridDim.x + t] = 0;
     }
     __syncthreads();
+    if (threadIdx.x == 0 && last) TC_TRACE(10);
   }
-  if (resid) __syncthreads();   // gate / residual rows staged by warps 2-3
+  if (resid) mbar_wait(bar_gr, 0, p.err, 15);   // gate / residual rows fetched by warp 2
   if (have) {
     const float b = p.bias ? p.bias[n] : 0.f;
     const float* Tr = T + row;
@@ -329,7 +321,8 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
       case EPI_RESID_GATE:
 #pragma unroll 4
         for (int j = 0; j < mcount; ++j)
-          p.resid[(size_t)(m0 + j) * p.ldr + n] = fmaf(G[j * kBM + row], Tr[j * kBM] + b, R[j * kBM + row]);
+          p.resid[(size_t)(m0 + j) * p.ldr + n] =
+              fmaf(p.gate_tab ? G[j * kBM + row] : 1.f, Tr[j * kBM] + b, R[j * kBM + row]);
         break;
       case EPI_GEGLU:
         if ((lane & 1) == 0) {
@@ -345,23 +338,56 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
           store_out(p.out, (size_t)(m0 + j) * p.ldo + n, gelu_tanh_f(Tr[j * kBM] + b), p.out_dtype);
         break;
       case EPI_QKV_TC: {
+        // Destination of row n for robot b, token i is affine: dst0 + b * sb + i * si.
         const QkvTcOut& o = p.qkv;
-        const bool rot = o.rope && n < o.qd + o.kvd;
-        const int r = (n < o.qd ? n : n - o.qd) % o.dh;
-        // RoPE frequency of this row's pair, theta = 1e4: angle = position * 1e4^(-2j/dh)
-        const float inv = exp2f(-13.287712379549449f * (float)(2 * (r >> 1)) / (float)o.dh);
+        const bool isq = n < o.qd, isk = !isq && n < o.qd + o.kvd;
+        __nv_bfloat16* dst0;
+        size_t sb, si;
+        const int half = o.dh / 2;
+        int r = 0;
+        if (isq || isk) {
+          const int sn = isq ? n : n - o.qd, h = sn / o.dh;
+          r = sn % o.dh;
+          const int d = o.rope ? ((r & 1) ? (r >> 1) + half : (r >> 1)) : r;
+          if (isq) {
+            dst0 = o.q + (((size_t)(h / o.G) * o.G + (h % o.G)) * o.H) * o.dh + d;   // + b*Hkv*G*H*dh + i*dh
+            sb = (size_t)o.Hkv * o.G * o.H * o.dh;
+            si = o.dh;
+          } else {
+            dst0 = o.kcache + (((size_t)o.layer * o.Hkv + h) * o.NK + o.P) * o.dh + d;
+            sb = (size_t)o.L * o.Hkv * o.NK * o.dh;
+            si = o.dh;
+          }
+        } else {
+          const int sn = n - o.qd - o.kvd, g = sn / o.dh, d = sn % o.dh;
+          dst0 = o.vtcache + (((size_t)o.layer * o.Hkv + g) * o.dh + d) * o.NKp + o.P;
+          sb = (size_t)o.L * o.Hkv * o.dh * o.NKp;
+          si = 1;
+        }
+        const bool rot = o.rope && (isq || isk);
+        // RoPE angle of token i: (P + i) * f, f = 1e4^(-2j/dh) for this row's pair j; (cos, sin)
+        // advance from token to token by a fixed rotation (one accurate sincosf per robot).
+        const float f = exp2f(-13.287712379549449f * (float)(2 * (r >> 1)) / (float)o.dh);
+        float cd = 1.f, sd = 0.f, c = 1.f, sn = 0.f;
+        if (rot) sincosf(f, &sd, &cd);
         const float sgn = (r & 1) ? 1.f : -1.f;
-        const int pr = (r & 1) ? -1 : 1;                                   // partner column offset
+        const int pr = (r & 1) ? -1 : 1;
         int bi = m0 / o.H, ii = m0 % o.H;
+        if (rot) sincosf((float)(o.P + ii) * f, &sn, &c);
         for (int j = 0; j < mcount; ++j) {
           float val = Tr[j * kBM];
           if (rot) {
-            float sn, cs;
-            sincosf((float)(o.P + ii) * inv, &sn, &cs);
-            val = fmaf(val, cs, sgn * Tr[j * kBM + pr] * sn);
+            val = fmaf(val, c, sgn * Tr[j * kBM + pr] * sn);
+            const float c2 = c * cd - sn * sd;
+            sn = fmaf(sn, cd, c * sd);
+            c = c2;
           }
-          epi_qkv_store_bi(o, bi, ii, n, val);
-          if (++ii == o.H) { ii = 0; ++bi; }
+          dst0[bi * sb + ii * si] = __float2bfloat16_rn(val);
+          if (++ii == o.H) {
+            ii = 0;
+            ++bi;
+            if (rot) sincosf((float)o.P * f, &sn, &c);
+          }
         }
         break;
       }
@@ -374,6 +400,7 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   }
   tc_fence_before();
   __syncthreads();
+  if (threadIdx.x == 0) TC_TRACE(11);
   if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kBN));
 }
 
@@ -431,22 +458,31 @@ int encode_act_tmap(CUtensorMap* m, const void* base, int K, int rows) {
   return r == CUDA_SUCCESS ? 0 : (int)r;
 }
 
-size_t gemm_tc_smem_bytes(int stages, int epi) {
-  return 1024 + tc_pipe_bytes(stages) + (epi == EPI_RESID_GATE ? 2 * kBN * kBM * 4 : 0) +
-         (2 * kTcMaxStages + 1) * 8 + 16;
+size_t gemm_tc_smem_bytes(int stages, int epi, int M) {
+  return 1024 + tc_pipe_bytes(stages) + (epi == EPI_RESID_GATE ? 2 * (size_t)tc_gr_rows(M) * kBM * 4 : 0) +
+         (2 * kTcMaxStages + 2) * 8 + 16;
 }
 
 void gemm_tc_prepare() {
-  const size_t a = gemm_tc_smem_bytes(kTcMaxStages, EPI_STORE);
-  const size_t b = gemm_tc_smem_bytes(kTcMaxStagesResid, EPI_RESID_GATE);
+  const size_t a = gemm_tc_smem_bytes(kTcMaxStages, EPI_STORE, kBN);
+  const size_t b = gemm_tc_smem_bytes(kTcMaxStagesResid, EPI_RESID_GATE, kBN);
   cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)(a > b ? a : b));
 }
 
-int gemm_tc_splits(int M, int N, int K, int sms) {
+// K splits per output tile: one CTA per SM. Residual epilogues (small shared-memory ring) take
+// more splits, up to two CTAs per SM, so that every CTA holds its whole K range in flight (one
+// HBM round trip); for the other epilogues extra splits cost more in reduction than they save.
+int gemm_tc_splits(int M, int N, int K, int sms, int epi) {
   const int tiles = (N / kBM) * ((M + kBN - 1) / kBN);
   const int KC = K / kBK;
-  int s = sms / tiles;                       // one wave: never more CTAs than SMs
+  const int cap = kTcMaxStagesResid;
+  int s = sms / tiles;
   if (s < 1) s = 1;
+  if (epi == EPI_RESID_GATE && (KC + s - 1) / s > cap) {
+    const int need = (KC + cap - 1) / cap;
+    const int most = 2 * sms / tiles;
+    s = need < most ? need : (most > s ? most : s);
+  }
   if (s > KC) s = KC;
   return s;
 }
@@ -455,7 +491,7 @@ void launch_gemm_tc(const CUtensorMap* tmx, const TcGemmArgs& a, cudaStream_t s)
   const int KC = a.K / kBK;
   const int per = (KC + a.splits - 1) / a.splits;
   dim3 grid(a.N / kBM, (a.M + kBN - 1) / kBN, a.splits);
-  launch_k(gemm_tc_kernel, grid, dim3(128), gemm_tc_smem_bytes(tc_stages(per, a.epi), a.epi), s, *tmx, a);
+  launch_k(gemm_tc_kernel, grid, dim3(128), gemm_tc_smem_bytes(tc_stages(per, a.epi), a.epi, a.M), s, *tmx, a);
 }
 
 void launch_relayout_tiled(const float* src, int K, int N, void* dst, int mult, long long off, int rope_dh,

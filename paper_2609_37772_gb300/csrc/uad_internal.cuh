@@ -139,7 +139,7 @@ void launch_convert(const void* src, int src_dtype, void* dst, int dst_dtype, lo
 
 // gemm_tc.cu: tcgen05 projection GEMM (bf16 operands, fp32 accumulation in TMEM)
 constexpr int kTcMaxStages = 4;        // <= ~97 KB of shared memory: two CTAs fit one SM
-constexpr int kTcMaxStagesResid = 3;   // plus the staged gate / residual rows
+constexpr int kTcMaxStagesResid = 2;   // plus the staged gate / residual rows (two CTAs per SM)
 struct TcGemmArgs {
   const void* w_tiled = nullptr;   // [N/128][K/64] blocks of 128 x 64 bf16, 128B-swizzled K-major
   int M = 0, N = 0, K = 0, splits = 1;
@@ -152,13 +152,14 @@ struct TcGemmArgs {
   float* acc = nullptr;            // split-K accumulator [M][N] fp32, zero between launches
   int* counters = nullptr;         // split-K arrival counters per output tile, zero between launches
   int* err = nullptr;              // set to a nonzero code if a bounded wait gave up
+  unsigned long long* trace = nullptr;  // optional: 16 global-timer stamps per CTA (phase times)
 };
-size_t gemm_tc_smem_bytes(int stages, int epi);
+size_t gemm_tc_smem_bytes(int stages, int epi, int M);
 // 2-D TMA descriptor of a bf16 activation matrix [rows][K] (64 x 64 boxes, 128-byte swizzle,
 // zero fill past the last row). 0 on success.
 int encode_act_tmap(CUtensorMap* m, const void* base, int K, int rows);
 void gemm_tc_prepare();
-int gemm_tc_splits(int M, int N, int K, int sms);
+int gemm_tc_splits(int M, int N, int K, int sms, int epi);
 void launch_gemm_tc(const CUtensorMap* tmx, const TcGemmArgs& a, cudaStream_t s);
 // element (k, n) of src [K][N] -> row n' * mult + off, column k of the tiled bf16 layout (K cols),
 // where n' = n, or with rope_dh > 0 the head-local pair interleave (d, d + dh/2) -> (2d, 2d + 1)
