@@ -55,10 +55,23 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity, int* err
     }
   }
 }
-__device__ __forceinline__ void tma_3d(void* dst, const CUtensorMap* map, int x, int y, int z, uint64_t* bar) {
+// 3-D tensor-map load with an L2 eviction hint (evict-last keeps the observation prefix, which
+// every evaluation re-reads, resident while the weights stream past with evict-first).
+__device__ __forceinline__ void tma_3d(void* dst, const CUtensorMap* map, int x, int y, int z, uint64_t* bar,
+                                       uint64_t pol) {
   asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];"
-      ::"r"(su32(dst)), "l"(map), "r"(x), "r"(y), "r"(z), "r"(su32(bar)) : "memory");
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3, %4}], [%5], %6;"
+      ::"r"(su32(dst)), "l"(map), "r"(x), "r"(y), "r"(z), "r"(su32(bar)), "l"(pol) : "memory");
+}
+__device__ __forceinline__ uint64_t policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ void bulk_s2g(void* gdst, const void* ssrc, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;"
+               ::"l"(gdst), "r"(su32(ssrc)), "r"(bytes) : "memory");
 }
 __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
   return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
@@ -143,15 +156,16 @@ __global__ void __launch_bounds__(128, 1) attn_tc_kernel(const __grid_constant__
   pdl_wait();
 
   if (threadIdx.x == 0) {
+    const uint64_t pol = policy_evict_last();
     mbar_expect_tx(bar_qk, QB + KB);
 #pragma unroll
     for (int c = 0; c < NC; ++c) {
-      tma_3d(sQ + c * (kQT * 128), &tq, c * 64, qt * kQT, bg, bar_qk);
-      tma_3d(sK + c * (kKT * 128), &tk, c * 64, kc * kKT, kvz, bar_qk);
+      tma_3d(sQ + c * (kQT * 128), &tq, c * 64, qt * kQT, bg, bar_qk, pol);
+      tma_3d(sK + c * (kKT * 128), &tk, c * 64, kc * kKT, kvz, bar_qk, pol);
     }
     mbar_expect_tx(bar_v, VB);
 #pragma unroll
-    for (int u = 0; u < kKT / 64; ++u) tma_3d(sV + u * (DH * 128), &tv, kc * kKT + u * 64, 0, kvz, bar_v);
+    for (int u = 0; u < kKT / 64; ++u) tma_3d(sV + u * (DH * 128), &tv, kc * kKT + u * 64, 0, kvz, bar_v, pol);
   } else if (threadIdx.x == 32) {
     if (mbar_wait(bar_qk, 0, p.err, 21)) {
       tc_fence_after();
@@ -228,23 +242,28 @@ __global__ void __launch_bounds__(128, 1) attn_tc_kernel(const __grid_constant__
   const bool ok_o = mbar_wait(bar_o, 0, p.err, 24);
   tc_fence_after();
 
-  // ---- partial output row (unnormalised) + (max, sum) ----
+  // ---- partial output row (unnormalised) + (max, sum): the row is staged in shared memory (all
+  //      operand tiles are free once O is complete; rows padded by 16 bytes against bank
+  //      conflicts) and written with one 1-KB bulk copy per row ----
   const int qrow = qt * kQT + row;
   const size_t prow_idx = ((size_t)bg * gridDim.y + kc) * p.r_pad + qrow;
-  float* po = p.part_o + prow_idx * DH;
+  constexpr uint32_t pitch = DH * 4 + 16;
+  uint8_t* srow = smem + (size_t)row * pitch;
   __syncwarp();
 #pragma unroll
   for (int cc = 0; cc < DH / 32; ++cc) {
     tmem_ld32(tO + lane_base + cc * 32, sv);
-    if (ok_o && qrow < p.rows) {
 #pragma unroll
-      for (int i = 0; i < 32; i += 4)
-        *reinterpret_cast<float4*>(po + cc * 32 + i) = make_float4(sv[i], sv[i + 1], sv[i + 2], sv[i + 3]);
-    }
+    for (int i = 0; i < 32; i += 4)
+      *reinterpret_cast<float4*>(srow + (cc * 32 + i) * 4) = make_float4(sv[i], sv[i + 1], sv[i + 2], sv[i + 3]);
   }
-  if (qrow < p.rows) {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  if (ok_o && qrow < p.rows) {
+    bulk_s2g(p.part_o + prow_idx * DH, srow, DH * 4);
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
     p.part_ml[prow_idx * 2] = mx;
     p.part_ml[prow_idx * 2 + 1] = l;
+    asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
   }
   tc_fence_before();
   __syncthreads();
@@ -332,7 +351,9 @@ int tmap3(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d
 }  // namespace
 
 size_t attn_tc_smem_bytes(int dh) {
-  return 1024 + 3 * attn_q_bytes(dh) + attn_p_extra(dh) + 4 * 8 + 16;
+  const size_t tiles = 3 * attn_q_bytes(dh) + attn_p_extra(dh);
+  const size_t ostage = (size_t)kQT * (dh * 4 + 16);   // O rows staged over the free operand tiles
+  return 1024 + (tiles > ostage ? tiles : ostage) + 4 * 8 + 16;
 }
 
 int attn_tc_prepare(AttnTcMaps* maps, const AttnTcArgs& a, int batch_max) {
