@@ -138,6 +138,95 @@ __host__ __device__ __forceinline__ size_t tc_pipe_bytes(int stages) {
 }
 __host__ __device__ __forceinline__ int tc_gr_rows(int M) { return M < kBN ? M : kBN; }
 
+// Epilogue of one tile slice: T[j][row] holds the fp32 accumulator of token m0 + j (j < mcount)
+// for output row n = this thread's row; G / R hold the gate and residual rows (residual
+// epilogue). Small rolled loops keep the code compact.
+__device__ __forceinline__ void tile_epilogue(const TcGemmArgs& p, const float* T, const float* G, const float* R,
+                                              int m0, int mcount, int n, int row, int lane) {
+  const float b = p.bias ? p.bias[n] : 0.f;
+  const float* Tr = T + row;
+  switch (p.epi) {
+    case EPI_RESID_GATE:
+#pragma unroll 4
+      for (int j = 0; j < mcount; ++j)
+        p.resid[(size_t)(m0 + j) * p.ldr + n] =
+            fmaf(p.gate_tab ? G[j * kBM + row] : 1.f, Tr[j * kBM] + b, R[j * kBM + row]);
+      break;
+    case EPI_GEGLU:
+      if ((lane & 1) == 0) {
+#pragma unroll 4
+        for (int j = 0; j < mcount; ++j)
+          store_out(p.out, (size_t)(m0 + j) * p.ldo + n / 2, gelu_tanh_f(Tr[j * kBM]) * Tr[j * kBM + 1],
+                    p.out_dtype);
+      }
+      break;
+    case EPI_BIAS_GELU:
+#pragma unroll 4
+      for (int j = 0; j < mcount; ++j)
+        store_out(p.out, (size_t)(m0 + j) * p.ldo + n, gelu_tanh_f(Tr[j * kBM] + b), p.out_dtype);
+      break;
+    case EPI_QKV_TC: {
+      // Destination of row n for robot b, token i is affine: dst0 + b * sb + i * si.
+      const QkvTcOut& o = p.qkv;
+      const bool isq = n < o.qd, isk = !isq && n < o.qd + o.kvd;
+      __nv_bfloat16* dst0;
+      size_t sb, si;
+      const int half = o.dh / 2;
+      int r = 0;
+      if (isq || isk) {
+        const int sn = isq ? n : n - o.qd, h = sn / o.dh;
+        r = sn % o.dh;
+        const int d = o.rope ? ((r & 1) ? (r >> 1) + half : (r >> 1)) : r;
+        if (isq) {
+          dst0 = o.q + (((size_t)(h / o.G) * o.G + (h % o.G)) * o.H) * o.dh + d;   // + b*Hkv*G*H*dh + i*dh
+          sb = (size_t)o.Hkv * o.G * o.H * o.dh;
+          si = o.dh;
+        } else {
+          dst0 = o.kcache + (((size_t)o.layer * o.Hkv + h) * o.NK + o.P) * o.dh + d;
+          sb = (size_t)o.L * o.Hkv * o.NK * o.dh;
+          si = o.dh;
+        }
+      } else {
+        const int sn = n - o.qd - o.kvd, g = sn / o.dh, d = sn % o.dh;
+        dst0 = o.vtcache + (((size_t)o.layer * o.Hkv + g) * o.dh + d) * o.NKp + o.P;
+        sb = (size_t)o.L * o.Hkv * o.dh * o.NKp;
+        si = 1;
+      }
+      const bool rot = o.rope && (isq || isk);
+      // RoPE angle of token i: (P + i) * f, f = 1e4^(-2j/dh) for this row's pair j; (cos, sin)
+      // advance from token to token by a fixed rotation (one accurate sincosf per robot).
+      const float f = exp2f(-13.287712379549449f * (float)(2 * (r >> 1)) / (float)o.dh);
+      float cd = 1.f, sd = 0.f, c = 1.f, sn = 0.f;
+      if (rot) sincosf(f, &sd, &cd);
+      const float sgn = (r & 1) ? 1.f : -1.f;
+      const int pr = (r & 1) ? -1 : 1;
+      int bi = m0 / o.H, ii = m0 % o.H;
+      if (rot) sincosf((float)(o.P + ii) * f, &sn, &c);
+      for (int j = 0; j < mcount; ++j) {
+        float val = Tr[j * kBM];
+        if (rot) {
+          val = fmaf(val, c, sgn * Tr[j * kBM + pr] * sn);
+          const float c2 = c * cd - sn * sd;
+          sn = fmaf(sn, cd, c * sd);
+          c = c2;
+        }
+        dst0[bi * sb + ii * si] = __float2bfloat16_rn(val);
+        if (++ii == o.H) {
+          ii = 0;
+          ++bi;
+          if (rot) sincosf((float)o.P * f, &sn, &c);
+        }
+      }
+      break;
+    }
+    default:
+#pragma unroll 4
+      for (int j = 0; j < mcount; ++j)
+        store_out(p.out, (size_t)(m0 + j) * p.ldo + n, Tr[j * kBM] + b, p.out_dtype);
+      break;
+  }
+}
+
 // Optional phase timestamps (TcGemmArgs::trace): slot i of this CTA's 16.
 #define TC_TRACE(i)                                                                                  \
   do {                                                                                               \
@@ -314,94 +403,138 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
     if (threadIdx.x == 0 && last) TC_TRACE(10);
   }
   if (resid) mbar_wait(bar_gr, 0, p.err, 15);   // gate / residual rows fetched by warp 2
-  if (have) {
-    const float b = p.bias ? p.bias[n] : 0.f;
-    const float* Tr = T + row;
-    switch (p.epi) {
-      case EPI_RESID_GATE:
-#pragma unroll 4
-        for (int j = 0; j < mcount; ++j)
-          p.resid[(size_t)(m0 + j) * p.ldr + n] =
-              fmaf(p.gate_tab ? G[j * kBM + row] : 1.f, Tr[j * kBM] + b, R[j * kBM + row]);
-        break;
-      case EPI_GEGLU:
-        if ((lane & 1) == 0) {
-#pragma unroll 4
-          for (int j = 0; j < mcount; ++j)
-            store_out(p.out, (size_t)(m0 + j) * p.ldo + n / 2, gelu_tanh_f(Tr[j * kBM]) * Tr[j * kBM + 1],
-                      p.out_dtype);
-        }
-        break;
-      case EPI_BIAS_GELU:
-#pragma unroll 4
-        for (int j = 0; j < mcount; ++j)
-          store_out(p.out, (size_t)(m0 + j) * p.ldo + n, gelu_tanh_f(Tr[j * kBM] + b), p.out_dtype);
-        break;
-      case EPI_QKV_TC: {
-        // Destination of row n for robot b, token i is affine: dst0 + b * sb + i * si.
-        const QkvTcOut& o = p.qkv;
-        const bool isq = n < o.qd, isk = !isq && n < o.qd + o.kvd;
-        __nv_bfloat16* dst0;
-        size_t sb, si;
-        const int half = o.dh / 2;
-        int r = 0;
-        if (isq || isk) {
-          const int sn = isq ? n : n - o.qd, h = sn / o.dh;
-          r = sn % o.dh;
-          const int d = o.rope ? ((r & 1) ? (r >> 1) + half : (r >> 1)) : r;
-          if (isq) {
-            dst0 = o.q + (((size_t)(h / o.G) * o.G + (h % o.G)) * o.H) * o.dh + d;   // + b*Hkv*G*H*dh + i*dh
-            sb = (size_t)o.Hkv * o.G * o.H * o.dh;
-            si = o.dh;
-          } else {
-            dst0 = o.kcache + (((size_t)o.layer * o.Hkv + h) * o.NK + o.P) * o.dh + d;
-            sb = (size_t)o.L * o.Hkv * o.NK * o.dh;
-            si = o.dh;
-          }
-        } else {
-          const int sn = n - o.qd - o.kvd, g = sn / o.dh, d = sn % o.dh;
-          dst0 = o.vtcache + (((size_t)o.layer * o.Hkv + g) * o.dh + d) * o.NKp + o.P;
-          sb = (size_t)o.L * o.Hkv * o.dh * o.NKp;
-          si = 1;
-        }
-        const bool rot = o.rope && (isq || isk);
-        // RoPE angle of token i: (P + i) * f, f = 1e4^(-2j/dh) for this row's pair j; (cos, sin)
-        // advance from token to token by a fixed rotation (one accurate sincosf per robot).
-        const float f = exp2f(-13.287712379549449f * (float)(2 * (r >> 1)) / (float)o.dh);
-        float cd = 1.f, sd = 0.f, c = 1.f, sn = 0.f;
-        if (rot) sincosf(f, &sd, &cd);
-        const float sgn = (r & 1) ? 1.f : -1.f;
-        const int pr = (r & 1) ? -1 : 1;
-        int bi = m0 / o.H, ii = m0 % o.H;
-        if (rot) sincosf((float)(o.P + ii) * f, &sn, &c);
-        for (int j = 0; j < mcount; ++j) {
-          float val = Tr[j * kBM];
-          if (rot) {
-            val = fmaf(val, c, sgn * Tr[j * kBM + pr] * sn);
-            const float c2 = c * cd - sn * sd;
-            sn = fmaf(sn, cd, c * sd);
-            c = c2;
-          }
-          dst0[bi * sb + ii * si] = __float2bfloat16_rn(val);
-          if (++ii == o.H) {
-            ii = 0;
-            ++bi;
-            if (rot) sincosf((float)o.P * f, &sn, &c);
-          }
-        }
-        break;
-      }
-      default:
-#pragma unroll 4
-        for (int j = 0; j < mcount; ++j)
-          store_out(p.out, (size_t)(m0 + j) * p.ldo + n, Tr[j * kBM] + b, p.out_dtype);
-        break;
-    }
-  }
+  if (have) tile_epilogue(p, T, G, R, m0, mcount, n, row, lane);
   tc_fence_before();
   __syncthreads();
   if (threadIdx.x == 0) TC_TRACE(11);
   if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kBN));
+}
+
+// ---- wide tiles for many tokens: 128 weight rows x 256 tokens per CTA, no K split ----------
+constexpr int kWN = 256;                       // tokens per tile (MMA N)
+constexpr int kWStageB = kWN * kBK * 2;        // 32 KB activation block per stage
+constexpr int kWStages = 4;
+constexpr uint32_t kIdescWide = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kWN >> 3) << 17) |
+                                ((uint32_t)(kBM >> 4) << 24);
+
+__device__ __forceinline__ void mma_bf16_wide(uint32_t d, uint64_t a, uint64_t b, uint32_t accum) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n"
+      ::"r"(d), "l"(a), "l"(b), "r"(kIdescWide), "r"(accum));
+}
+
+__global__ void __launch_bounds__(128, 1) gemm_tc_wide_kernel(const __grid_constant__ CUtensorMap tmx, TcGemmArgs p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  const int t = blockIdx.x, mt = blockIdx.y;
+  const int KC = p.K / kBK;
+  const int stages = KC < kWStages ? KC : kWStages;
+  const bool resid = p.epi == EPI_RESID_GATE;
+  uint8_t* sA = smem;                                        // stages x 16 KB weights
+  uint8_t* sB = smem + (size_t)kWStages * kStageA;           // stages x 32 KB activations
+  // after the main loop the stage area holds the epilogue slices: T, G, R (32 KB each)
+  float* T = reinterpret_cast<float*>(smem);
+  float* G = T + kBN * kBM;
+  float* R = G + kBN * kBM;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)kWStages * (kStageA + kWStageB));
+  uint64_t* empty = full + kWStages;
+  uint64_t* done = empty + kWStages;
+  uint64_t* bar_gr = done + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_gr + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kWStages; ++i) {
+      mbar_init(full + i, 1);
+      mbar_init(empty + i, 1);
+    }
+    mbar_init(done, 1);
+    mbar_init(bar_gr, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(tmem_slot)), "r"(kWN));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_trigger();
+
+  if (threadIdx.x == 0) {
+    const uint64_t pol = policy_evict_first();
+    const uint8_t* wt = static_cast<const uint8_t*>(p.w_tiled) + (size_t)t * KC * kStageA;
+    const int first = stages;
+    for (int i = 0; i < first; ++i) {
+      mbar_expect_tx(full + i, kStageA + kWStageB);
+      bulk_g2s(sA + (size_t)i * kStageA, wt + (size_t)i * kStageA, kStageA, full + i, pol);
+    }
+    pdl_wait();
+    for (int i = 0; i < first; ++i)
+      for (int q = 0; q < kWN / kBN; ++q)
+        tma_2d(sB + (size_t)i * kWStageB + q * kStageB, &tmx, i * kBK, mt * kWN + q * kBN, full + i);
+    int issued = first;
+    for (int i = first; i < KC; ++i) {
+      const int st = i % stages, round = i / stages;
+      if (!mbar_wait(empty + st, (round - 1) & 1, p.err, 31)) break;
+      mbar_expect_tx(full + st, kStageA + kWStageB);
+      bulk_g2s(sA + (size_t)st * kStageA, wt + (size_t)i * kStageA, kStageA, full + st, pol);
+      for (int q = 0; q < kWN / kBN; ++q)
+        tma_2d(sB + (size_t)st * kWStageB + q * kStageB, &tmx, i * kBK, mt * kWN + q * kBN, full + st);
+      ++issued;
+    }
+    for (int i = issued - stages > 0 ? issued - stages : 0; i < issued; ++i)
+      mbar_wait(full + i % stages, (i / stages) & 1, p.err, 32);
+  } else if (threadIdx.x == 32) {
+    bool ok = true;
+    for (int i = 0; i < KC && ok; ++i) {
+      const int st = i % stages, round = i / stages;
+      ok = mbar_wait(full + st, round & 1, p.err, 33);
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t a0 = su32(sA + (size_t)st * kStageA), b0 = su32(sB + (size_t)st * kWStageB);
+#pragma unroll
+      for (int k = 0; k < kBK / 16; ++k)
+        mma_bf16_wide(tmem, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), (i > 0 || k > 0) ? 1u : 0u);
+      mma_commit(empty + st);
+    }
+    mma_commit(done);
+  }
+  __syncwarp();
+  pdl_wait();
+  const bool ok = mbar_wait(done, 0, p.err, 34);
+  tc_fence_after();
+  const int row = warp * 32 + lane;
+  const int n = t * kBM + row;
+  // epilogue in four slices of 64 tokens (TMEM columns [64 q, 64 q + 64))
+  for (int q = 0; q < kWN / kBN; ++q) {
+    const int m0 = mt * kWN + q * kBN;
+    if (m0 >= p.M) break;
+    const int mcount = p.M - m0 < kBN ? p.M - m0 : kBN;
+    if (resid && warp == 2) {
+      if (lane == 0) mbar_expect_tx(bar_gr, (p.gate_tab ? 2u : 1u) * (uint32_t)mcount * (kBM * 4));
+      __syncwarp();
+      for (int j = lane; j < mcount; j += 32) {
+        bulk_g2s_plain(R + j * kBM, p.resid + (size_t)(m0 + j) * p.ldr + t * kBM, kBM * 4, bar_gr);
+        if (p.gate_tab)
+          bulk_g2s_plain(G + j * kBM, p.gate_tab + (size_t)p.tau_row[m0 + j] * p.gate_stride + t * kBM, kBM * 4, bar_gr);
+      }
+    }
+    float v[kBN];
+    __syncwarp();
+#pragma unroll
+    for (int c = 0; c < kBN; c += 16) tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + q * kBN + c, v + c);
+#pragma unroll
+    for (int j = 0; j < kBN; ++j) T[j * kBM + row] = v[j];
+    __syncthreads();
+    if (resid) mbar_wait(bar_gr, q & 1, p.err, 35);
+    if (ok) tile_epilogue(p, T, G, R, m0, mcount, n, row, lane);
+    __syncthreads();
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kWN));
 }
 
 // ---- weight re-layout into 128 x 64 swizzled blocks --------------------------------------
@@ -463,10 +596,20 @@ size_t gemm_tc_smem_bytes(int stages, int epi, int M) {
          (2 * kTcMaxStages + 2) * 8 + 16;
 }
 
+static size_t gemm_tc_wide_smem_bytes() { return 1024 + (size_t)kWStages * (kStageA + kWStageB) + (2 * kWStages + 2) * 8 + 16; }
+
 void gemm_tc_prepare() {
   const size_t a = gemm_tc_smem_bytes(kTcMaxStages, EPI_STORE, kBN);
   const size_t b = gemm_tc_smem_bytes(kTcMaxStagesResid, EPI_RESID_GATE, kBN);
   cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)(a > b ? a : b));
+  cudaFuncSetAttribute(gemm_tc_wide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)gemm_tc_wide_smem_bytes());
+}
+
+// Wide tiles cut L2 re-reads of the weights (one CTA per 256 tokens instead of 64) but hold a
+// whole SM; for very wide outputs (gate/up at N = 8192) two narrow CTAs per SM overlap one
+// CTA's epilogue with the other's main loop and win.
+bool gemm_tc_use_wide(int M, int N, int sms) {
+  return M >= kWN && N <= 4096 && (N / kBM) * ((M + kWN - 1) / kWN) * 2 >= sms;
 }
 
 // K splits per output tile: one CTA per SM. Residual epilogues (small shared-memory ring) take
@@ -488,6 +631,11 @@ int gemm_tc_splits(int M, int N, int K, int sms, int epi) {
 }
 
 void launch_gemm_tc(const CUtensorMap* tmx, const TcGemmArgs& a, cudaStream_t s) {
+  if (a.wide) {
+    launch_k(gemm_tc_wide_kernel, dim3(a.N / kBM, (a.M + kWN - 1) / kWN), dim3(128), gemm_tc_wide_smem_bytes(), s,
+             *tmx, a);
+    return;
+  }
   const int KC = a.K / kBK;
   const int per = (KC + a.splits - 1) / a.splits;
   dim3 grid(a.N / kBM, (a.M + kBN - 1) / kBN, a.splits);

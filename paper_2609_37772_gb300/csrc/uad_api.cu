@@ -352,7 +352,8 @@ void gemm(uad_ctx* c, const Lin& w, GemmArgs g, cudaStream_t s) {
   }
   TcGemmArgs t;
   t.w_tiled = w.w; t.M = g.M; t.N = g.N; t.K = g.K;
-  t.splits = gemm_tc_splits(g.M, g.N, g.K, c->sms, g.epi);
+  t.wide = gemm_tc_use_wide(g.M, g.N, c->sms);
+  t.splits = t.wide ? 1 : gemm_tc_splits(g.M, g.N, g.K, c->sms, g.epi);
   t.epi = g.epi; t.out = g.out; t.ldo = g.ldo; t.out_dtype = g.out_dtype; t.bias = g.bias;
   t.resid = g.resid; t.ldr = g.ldr; t.gate_tab = g.gate_tab; t.gate_stride = g.gate_stride;
   t.tau_row = g.tau_row; t.qkv = g.qkv; t.acc = c->tc_acc; t.counters = c->tc_counters; t.err = c->dev_err;

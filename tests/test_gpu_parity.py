@@ -292,3 +292,27 @@ def test_tensor_core_gemm_matches_cuda_core_gemm(monkeypatch):
             c.close()
     for k in ("final", "ghost"):
         assert rel_err(outs[1][k], outs[0][k].astype(np.float64)) <= 5e-3, k
+
+
+def test_pi0_full_batched_16_robots_sampled():
+    """16 robots (M = 800 tokens: wide 128 x 256 projection tiles), each with its own prefix and
+    a schedule from the sweep grid; robots 0, 7 and 15 are checked against the oracle."""
+    a = ARCHS["pi0"]
+    B = 16
+    blob = make_weights(a, seed=3)
+    ex = uad.Expert(a, blob, max_batch=B)
+    try:
+        pre = [make_prefix_kv(a, robot=b, seed=3) for b in range(B)]
+        for b in range(B):
+            ex.set_prefix(b, *pre[b])
+        noise = make_noise(a, batch=B, seed=3)
+        bud = draw_sweep_schedules(a.chunk_len, B, seed=3)
+        ex.denoise(noise, bud)
+        res = ex.finish(timeout_us=TIMEOUT)
+        for b in (0, 7, 15):
+            ref = denoise(build_model(a, blob, pre[b]).velocity, noise[b], bud[b])
+            assert rel_err(res["final"][b], ref["final"]) <= TOL["bf16"]
+            assert rel_err(res["ghost"][b], ref["ghost"]) <= TOL["bf16"]
+        assert res["evals"] == 10
+    finally:
+        ex.close()
