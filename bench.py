@@ -48,9 +48,13 @@ for _b in (4, 16, 64):
     WORKLOADS[f"pi0-b{_b}"] = dict(arch="pi0", batch=_b, groups=None, t_act_ms=10.0,
                                    desc=f"pi0-like bf16 expert, B={_b} robots, schedules drawn from the sweep grid")
 
-# ncu DRAM traffic per launch of the dominant kernel class, with the sha1 of the source file it
-# was measured on (reported as null once that source changes). Filled from profiles/.
-TRAFFIC = {}
+# ncu DRAM traffic (read + write bytes) per launch of the dominant kernel class, with the source
+# file and its sha1 at measurement time (reported as null once that source changes); figures from
+# profiles/ncu_full_pi0_b1_attention_gemm.md (attention + combine kernels of one layer).
+TRAFFIC = {
+    "attention@pi0-b1": (4057856.0, "paper_2609_37772_gb300/csrc/attn_tc.cu",
+                         "3bf844d67be14408fc8fd4d1769c8209a3d970ea"),
+}
 
 
 def peaks():

@@ -46,6 +46,9 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity, int* err
         : "=r"(ok) : "r"(su32(b)), "r"(parity) : "memory");
     if (ok) return true;
     if ((it & 255) == 0) {
+      // give up at once if another wait already failed, so that one failure cannot chain
+      // into a long sequence of timeouts
+      if (*reinterpret_cast<volatile int*>(err) != 0) return false;
       const unsigned long long t = gtime();
       if (t0 == 0) t0 = t;
       else if (t - t0 > kWaitNs) {
@@ -270,6 +273,217 @@ __global__ void __launch_bounds__(128, 1) attn_tc_kernel(const __grid_constant__
   if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols));
 }
 
+// ---- two-pass attention for many query tiles: no partials, no combine --------------------
+// One CTA per (128-row query tile, robot-group). Keys in chunks of 64 through a 2-slot ring.
+// Pass 1: S = Q K_c^T on tcgen05 (double-buffered in TMEM), row maxima in registers.
+// Pass 2: S again, P = exp(S - max) in bf16 into shared memory, O += P V_c on tcgen05 (no
+// rescaling: the maxima are final), row sums of the rounded P. O / l is written in bf16.
+constexpr int kKC2 = 64;                        // keys per chunk
+constexpr uint32_t kTmem2 = 512;                // S buffers at columns [0,64) and [64,128), O at [128, 128+dh)
+
+// Warps 0-3: softmax and output (they own the four TMEM lane quadrants); warp 4: TMA producer;
+// warp 5: MMA issuer. The producer and issuer wait on the softmax warps' progress, so they must
+// not share a warp with them.
+template <int DH>
+__global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant__ CUtensorMap tq,
+                                                          const __grid_constant__ CUtensorMap tk,
+                                                          const __grid_constant__ CUtensorMap tv, AttnTcArgs p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  constexpr int NC = DH / 64;
+  constexpr uint32_t QB = DH * kQT * 2;          // Q: NC blocks of 128 x 64
+  constexpr uint32_t KB = DH * kKC2 * 2;         // one K chunk: NC blocks of 64 x 64
+  constexpr uint32_t VB = DH * kKC2 * 2;         // one Vt chunk: dh x 64 keys
+  constexpr uint32_t PB = kQT * kKC2 * 2;        // P: 128 x 64
+  uint8_t* sQ = smem;
+  uint8_t* sK = sQ + QB;                         // 2 slots
+  uint8_t* sV = sK + 2 * KB;                     // 2 slots
+  uint8_t* sP = sV + 2 * VB;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + PB);
+  uint64_t* q_full = bars;          // Q landed
+  uint64_t* kv_full = bars + 1;     // [2] chunk landed in slot
+  uint64_t* kv_empty = bars + 3;    // [2] slot free (MMAs that read it are done)
+  uint64_t* s_full = bars + 5;      // [2] S buffer written
+  uint64_t* s_empty = bars + 7;     // [2] S buffer read by the 4 warps
+  uint64_t* p_full = bars + 9;      // P written by the 4 warps
+  uint64_t* p_empty = bars + 10;    // PV MMA done reading P
+  uint64_t* o_done = bars + 11;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
+
+  const int qt = blockIdx.x, bg = blockIdx.y;
+  const int b = bg / p.n_kv_heads, g = bg % p.n_kv_heads;
+  const int kvz = (b * p.n_layers + p.layer) * p.n_kv_heads + g;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nck = (p.n_keys + kKC2 - 1) / kKC2;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(kv_full + i, 1);
+      mbar_init(kv_empty + i, 1);
+      mbar_init(s_full + i, 1);
+      mbar_init(s_empty + i, 4);
+    }
+    mbar_init(p_full, 4);
+    mbar_init(p_empty, 1);
+    mbar_init(o_done, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(tmem_slot)), "r"(kTmem2));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t tO = tmem + 2 * kKC2;
+  pdl_trigger();
+  pdl_wait();
+
+  // chunk sequence: pass 1 loads K only (n = 0..nck-1), pass 2 loads K and Vt (n = nck..2nck-1)
+  const int total = 2 * nck;
+  if (threadIdx.x == 128) {
+    const uint64_t pol = policy_evict_last();
+    mbar_expect_tx(q_full, QB);
+#pragma unroll
+    for (int c = 0; c < NC; ++c) tma_3d(sQ + c * (kQT * 128), &tq, c * 64, qt * kQT, bg, q_full, pol);
+    for (int n = 0; n < total; ++n) {
+      const int slot = n & 1, use = n >> 1;
+      if (use > 0 && !mbar_wait(kv_empty + slot, (use - 1) & 1, p.err, 41)) break;
+      const bool pass2 = n >= nck;
+      const int key0 = (pass2 ? n - nck : n) * kKC2;
+      mbar_expect_tx(kv_full + slot, pass2 ? KB + VB : KB);
+#pragma unroll
+      for (int c = 0; c < NC; ++c) tma_3d(sK + slot * KB + c * (kKC2 * 128), &tk, c * 64, key0, kvz, kv_full + slot, pol);
+      if (pass2) tma_3d(sV + slot * VB, &tv, key0, 0, kvz, kv_full + slot, pol);
+    }
+  } else if (threadIdx.x == 160) {
+    bool ok = mbar_wait(q_full, 0, p.err, 42);
+    const uint32_t q0 = su32(sQ);
+    for (int n = 0; n < total && ok; ++n) {
+      const int slot = n & 1, use = n >> 1, sb = n & 1;
+      const bool pass2 = n >= nck;
+      ok = mbar_wait(kv_full + slot, use & 1, p.err, 43);
+      if (ok && n >= 2) ok = mbar_wait(s_empty + sb, ((n >> 1) - 1) & 1, p.err, 44);
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t k0 = su32(sK + slot * KB);
+#pragma unroll
+      for (int c = 0; c < NC; ++c)
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          mma_bf16(tmem + sb * kKC2, sw128_desc(q0 + c * (kQT * 128) + 32 * k),
+                   sw128_desc(k0 + c * (kKC2 * 128) + 32 * k), idesc_m128(kKC2), (c | k) ? 1u : 0u);
+      mma_commit(s_full + sb);
+      if (!pass2) {
+        mma_commit(kv_empty + slot);
+      } else {
+        const int c2 = n - nck;
+        ok = mbar_wait(p_full, c2 & 1, p.err, 45);
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t pp = su32(sP), v0 = su32(sV + slot * VB);
+#pragma unroll
+        for (int k = 0; k < kKC2 / 16; ++k)
+          mma_bf16(tO, sw128_desc(pp + 32 * k), sw128_desc(v0 + 32 * k), idesc_m128(DH), (c2 | k) ? 1u : 0u);
+        mma_commit(kv_empty + slot);
+        mma_commit(p_empty);
+      }
+    }
+    mma_commit(o_done);
+  }
+  if (warp >= 4) {
+    // producer / issuer warps: done issuing; wait for the output stage before releasing TMEM
+    __syncthreads();
+    return;
+  }
+
+  // ---- softmax warps: one query row per thread ----
+  const int row = warp * 32 + lane;
+  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+  const float c2s = p.scale_log2;
+  float sv[32];
+  float mx = -INFINITY, l = 0.f;
+  bool ok = true;
+  for (int n = 0; n < total; ++n) {
+    const int sb = n & 1;
+    const bool pass2 = n >= nck;
+    const int key0 = (pass2 ? n - nck : n) * kKC2;
+    ok = ok && mbar_wait(s_full + sb, (n >> 1) & 1, p.err, 46);
+    tc_fence_after();
+    __syncwarp();
+    if (!pass2) {
+#pragma unroll
+      for (int cc = 0; cc < kKC2 / 32; ++cc) {
+        tmem_ld32(tmem + sb * kKC2 + lane_base + cc * 32, sv);
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          if (key0 + cc * 32 + i < p.n_keys) mx = fmaxf(mx, sv[i]);
+      }
+    } else {
+      const int c2 = n - nck;
+      if (c2 > 0) ok = ok && mbar_wait(p_empty, (c2 - 1) & 1, p.err, 47);
+      const int r8 = row & 7;
+#pragma unroll
+      for (int cc = 0; cc < kKC2 / 32; ++cc) {
+        tmem_ld32(tmem + sb * kKC2 + lane_base + cc * 32, sv);
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 32; i += 2) {
+          const bool v0 = key0 + cc * 32 + i < p.n_keys, v1 = key0 + cc * 32 + i + 1 < p.n_keys;
+          const float e0 = v0 ? exp2f((sv[i] - mx) * c2s) : 0.f;
+          const float e1 = v1 ? exp2f((sv[i + 1] - mx) * c2s) : 0.f;
+          const __nv_bfloat162 h = __floats2bfloat162_rn(e0, e1);
+          l += __low2float(h) + __high2float(h);
+          pk[i / 2] = *reinterpret_cast<const uint32_t*>(&h);
+        }
+        uint8_t* prow = sP + row * 128;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int gidx = cc * 4 + q;
+          *reinterpret_cast<uint4*>(prow + ((gidx ^ r8) * 16)) =
+              make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+        }
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(p_full)) : "memory");
+    }
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(s_empty + sb)) : "memory");
+  }
+  ok = ok && mbar_wait(o_done, 0, p.err, 48);
+  tc_fence_after();
+  __syncwarp();
+
+  // ---- o = O / l in bf16, row (j, i) of this tile -> o[(b*H + i)][(g*G + j)*dh + d] ----
+  const int qrow = qt * kQT + row;
+  const float inv = 1.f / l;
+  const int jj = qrow / p.H, ii = qrow % p.H;
+  __nv_bfloat16* orow = p.out + ((size_t)b * p.H + ii) * p.out_ld + (size_t)(g * p.group + jj) * DH;
+#pragma unroll
+  for (int cc = 0; cc < DH / 32; ++cc) {
+    tmem_ld32(tO + lane_base + cc * 32, sv);
+    if (ok && qrow < p.rows) {
+#pragma unroll
+      for (int i = 0; i < 32; i += 8) {
+        uint4 w;
+        w.x = pack_bf16(sv[i] * inv, sv[i + 1] * inv);
+        w.y = pack_bf16(sv[i + 2] * inv, sv[i + 3] * inv);
+        w.z = pack_bf16(sv[i + 4] * inv, sv[i + 5] * inv);
+        w.w = pack_bf16(sv[i + 6] * inv, sv[i + 7] * inv);
+        *reinterpret_cast<uint4*>(orow + cc * 32 + i) = w;
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();   // pairs with the producer / issuer warps' final barrier
+  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmem2));
+}
+
 // Merge the key chunks of every query row: o = sum_c w_c O_c / sum_c w_c l_c, w_c = 2^((m_c - M) c2).
 // One CTA per (query row, robot-group), one thread per head dim; every partial is loaded
 // before any arithmetic. Writes o [(b*H + i)][(g*G + j)*dh + d] in bf16.
@@ -350,6 +564,15 @@ int tmap3(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d
 
 }  // namespace
 
+size_t attn_tc2_smem_bytes(int dh) {
+  return 1024 + (size_t)dh * kQT * 2 + 4 * (size_t)dh * kKC2 * 2 + (size_t)kQT * kKC2 * 2 + 16 * 8;
+}
+
+bool attn_tc_use_two_pass(const AttnTcArgs& a) {
+  const int tiles = (a.rows + kQT - 1) / kQT * a.batch * a.n_kv_heads;
+  return tiles >= 64;
+}
+
 size_t attn_tc_smem_bytes(int dh) {
   const size_t tiles = 3 * attn_q_bytes(dh) + attn_p_extra(dh);
   const size_t ostage = (size_t)kQT * (dh * 4 + 16);   // O rows staged over the free operand tiles
@@ -364,6 +587,13 @@ int attn_tc_prepare(AttnTcMaps* maps, const AttnTcArgs& a, int batch_max) {
             NK * dh * 2, 64, kKT)) return -1;
   if (tmap3(&maps->vt, a.vtcache, NK, dh, (uint64_t)batch_max * a.n_layers * a.n_kv_heads, NKp * 2,
             (uint64_t)dh * NKp * 2, 64, (uint32_t)dh)) return -1;
+  if (tmap3(&maps->k2, a.kcache, dh, NK, (uint64_t)batch_max * a.n_layers * a.n_kv_heads, (uint64_t)dh * 2,
+            NK * dh * 2, 64, kKC2)) return -1;
+  maps->vt2 = maps->vt;   // the Vt box is already 64 keys x dh
+  const int smem2 = (int)attn_tc2_smem_bytes(dh);
+  if (dh == 64) cudaFuncSetAttribute(attn_tc2_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem2);
+  if (dh == 128) cudaFuncSetAttribute(attn_tc2_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem2);
+  if (dh == 256) cudaFuncSetAttribute(attn_tc2_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem2);
   const int smem = (int)attn_tc_smem_bytes(dh);
   if (dh == 64) cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (dh == 128) cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
@@ -376,6 +606,14 @@ int attn_tc_max_keys() { return kMaxKeyChunks * kKT; }
 int attn_tc_rpad(int rows) { return (rows + kQT - 1) / kQT * kQT; }
 
 void launch_attn_tc(const AttnTcMaps& maps, const AttnTcArgs& a, cudaStream_t s) {
+  if (attn_tc_use_two_pass(a)) {
+    dim3 grid2((a.rows + kQT - 1) / kQT, a.batch * a.n_kv_heads);
+    const size_t smem2 = attn_tc2_smem_bytes(a.head_dim);
+    if (a.head_dim == 64) launch_k(attn_tc2_kernel<64>, grid2, dim3(192), smem2, s, maps.q, maps.k2, maps.vt2, a);
+    if (a.head_dim == 128) launch_k(attn_tc2_kernel<128>, grid2, dim3(192), smem2, s, maps.q, maps.k2, maps.vt2, a);
+    if (a.head_dim == 256) launch_k(attn_tc2_kernel<256>, grid2, dim3(192), smem2, s, maps.q, maps.k2, maps.vt2, a);
+    return;
+  }
   dim3 grid((a.rows + kQT - 1) / kQT, attn_tc_chunks(a.n_keys), a.batch * a.n_kv_heads);
   const size_t smem = attn_tc_smem_bytes(a.head_dim);
   if (a.head_dim == 64) launch_k(attn_tc_kernel<64>, grid, dim3(128), smem, s, maps.q, maps.k, maps.vt, a);

@@ -50,6 +50,9 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity, int* err
         : "=r"(ok) : "r"(su32(b)), "r"(parity) : "memory");
     if (ok) return true;
     if ((it & 255) == 0) {
+      // give up at once if another wait already failed, so that one failure cannot chain
+      // into a long sequence of timeouts
+      if (*reinterpret_cast<volatile int*>(err) != 0) return false;
       const unsigned long long t = gtime();
       if (t0 == 0) t0 = t;
       else if (t - t0 > kWaitNs) {

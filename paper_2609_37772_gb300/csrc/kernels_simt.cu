@@ -453,14 +453,18 @@ __global__ void __launch_bounds__(256) euler_kernel(EulerArgs p) {
   __syncthreads();
   if (last) {
     const int T = p.tail_count[b];
+    // Eq. 8 terms (ghost - released) of early actions, staged in shared memory by all threads,
+    // then summed per dimension in token order
+    extern __shared__ float ediff[];   // [H][D]
+    for (int e = tid; e < HD; e += blockDim.x) {
+      const int i = e / p.D;
+      const long long idx = (long long)b * HD + e;
+      ediff[e] = (p.plan[b * p.H + i].flags & PF_EARLY) ? p.g[idx] - p.rel[idx] : 0.f;
+    }
+    __syncthreads();
     if (tid < p.D) {
       float E = 0.f;
-      for (int i = 0; i < p.H; ++i) {
-        if (p.plan[b * p.H + i].flags & PF_EARLY) {
-          const long long idx = (long long)b * HD + i * p.D + tid;
-          E += p.g[idx] - p.rel[idx];
-        }
-      }
+      for (int i = 0; i < p.H; ++i) E += ediff[i * p.D + tid];
       E = T > 0 ? E : 0.f;
       E_s[tid] = E;
       p.E_out[b * p.D + tid] = E;
@@ -495,7 +499,13 @@ __global__ void __launch_bounds__(256) euler_kernel(EulerArgs p) {
   }
 }
 
-void launch_euler(const EulerArgs& a, cudaStream_t s) { launch_k(euler_kernel, dim3(a.B), dim3(256), 0, s, a); }
+void launch_euler_prepare() {
+  cudaFuncSetAttribute(euler_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 256 * 64 * (int)sizeof(float));
+}
+
+void launch_euler(const EulerArgs& a, cudaStream_t s) {
+  launch_k(euler_kernel, dim3(a.B), dim3(256), (size_t)a.H * a.D * sizeof(float), s, a);
+}
 
 __global__ void begin_kernel(const float* noise, float* x, float* g, float* u, int n, int* nonfinite,
                              int* evals, unsigned long long* stamps) {

@@ -778,6 +778,7 @@ int uad_init(const uad_arch* arch, const float* weights, size_t n_floats, uad_ct
   CK(cudaEventCreateWithFlags(&c->ev_done, cudaEventDisableTiming));
   // attention kernels need more than 48 KB of dynamic shared memory: opt in once, here
   launch_attention_prepare(a.head_dim);
+  launch_euler_prepare();
   CK(cudaDeviceSynchronize());
   CK(cudaGetLastError());
 #undef TRY
@@ -1130,11 +1131,16 @@ int uad_launches_per_chunk(const uad_ctx* c, int32_t batch, int32_t n_star) {
 void uad_destroy(uad_ctx* c) {
   if (!c) return;
   if (c->in_flight && c->ev_done) {
-    // bounded wait so that no kernel still writes into memory about to be freed
+    // bounded wait so that no kernel still writes into memory about to be freed; if the chunk
+    // is still running after it, the device memory is deliberately leaked, not freed under it
     const auto t0 = std::chrono::steady_clock::now();
     while (cudaEventQuery(c->ev_done) == cudaErrorNotReady &&
            std::chrono::steady_clock::now() - t0 < std::chrono::seconds(10))
       std::this_thread::yield();
+    if (cudaEventQuery(c->ev_done) == cudaErrorNotReady) {
+      fprintf(stderr, "uad_destroy: chunk still running; device memory of this context is not freed\n");
+      return;
+    }
   }
   for (auto& kv : c->graphs) cudaGraphExecDestroy(kv.second);
   for (cudaEvent_t e : c->prof_ev) cudaEventDestroy(e);

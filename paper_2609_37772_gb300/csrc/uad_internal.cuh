@@ -128,6 +128,7 @@ void launch_gemv_rows(const GemmArgs& a, cudaStream_t s);
 void launch_norm(const NormArgs& a, cudaStream_t s);
 void launch_attention(const AttnArgs& a, cudaStream_t s);
 void launch_euler(const EulerArgs& a, cudaStream_t s);
+void launch_euler_prepare();   // shared memory for H x D GAC terms (up to 256 x 64)
 void launch_begin(const float* noise, float* x, float* g, float* u, int n, int* nonfinite, int* evals,
                   unsigned long long* stamps, cudaStream_t s);
 // dst[(n * mult + off) * K + k] = src[k * N + n]: transpose [K][N] -> rows of K, convert dtype
@@ -181,7 +182,7 @@ struct AttnTcArgs {
   __nv_bfloat16* out = nullptr; int out_ld = 0;   // o [B*H][Hq*dh]
   int* err = nullptr;
 };
-struct AttnTcMaps { CUtensorMap q, k, vt; };
+struct AttnTcMaps { CUtensorMap q, k, vt, k2, vt2; };   // k2 / vt2: 64-key boxes (two-pass kernel)
 size_t attn_tc_smem_bytes(int dh);
 int attn_tc_prepare(AttnTcMaps* maps, const AttnTcArgs& a, int batch_max);  // 0 on success
 int attn_tc_chunks(int n_keys);

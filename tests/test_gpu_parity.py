@@ -316,3 +316,26 @@ def test_pi0_full_batched_16_robots_sampled():
         assert res["evals"] == 10
     finally:
         ex.close()
+
+
+def test_two_pass_attention_many_tiles():
+    """32 robots x 2 query tiles on the small bf16 expert: the attention takes its two-pass path
+    (row maxima, then P V accumulated without rescaling); sampled robots vs the oracle."""
+    a = ARCHS["pi0_small"]
+    B = 32
+    blob = make_weights(a, seed=12)
+    ex = uad.Expert(a, blob, max_batch=B)
+    try:
+        pre = [make_prefix_kv(a, robot=b, seed=12) for b in range(B)]
+        for b in range(B):
+            ex.set_prefix(b, *pre[b])
+        noise = make_noise(a, batch=B, seed=12)
+        bud = draw_sweep_schedules(a.chunk_len, B, seed=12)
+        ex.denoise(noise, bud)
+        res = ex.finish(timeout_us=TIMEOUT)
+        for b in (0, 13, 31):
+            ref = denoise(build_model(a, blob, pre[b]).velocity, noise[b], bud[b])
+            assert rel_err(res["final"][b], ref["final"]) <= TOL["bf16"]
+            assert rel_err(res["ghost"][b], ref["ghost"]) <= TOL["bf16"]
+    finally:
+        ex.close()
