@@ -10,7 +10,9 @@
 //
 // Split-K: CTAs sharing an output tile each own a K range; they add their partial tile into
 // an fp32 accumulator in L2 (red.global.add) and the last one to arrive (per-tile counter)
-// applies the epilogue, then clears the accumulator and counter for the next launch.
+// applies the epilogue, then clears the accumulator and counter for the next launch. The
+// residual projections instead write each split's tile to a plane of its own (EPI_PARTIAL):
+// the norm that follows sums the planes in a fixed order as part of the residual update.
 // Every wait is bounded: on timeout the kernel records an error code and winds down.
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -129,32 +131,32 @@ __device__ __forceinline__ void red_add_v4(float* dst, float4 v) {
 }
 
 // Shared-memory plan: [pipeline stages, at least 32 KB (reused as the split-K staging tile)]
-// [gate rows][residual rows] (residual epilogue only: min(M, 64) rows of 128 fp32 each)
 // [mbarriers, TMEM slot, flag].
 __host__ __device__ __forceinline__ int tc_stages(int nch, int epi) {
-  const int cap = epi == EPI_RESID_GATE ? kTcMaxStagesResid : kTcMaxStages;
-  return nch < cap ? nch : cap;
+  (void)epi;
+  return nch < kTcMaxStages ? nch : kTcMaxStages;
 }
 __host__ __device__ __forceinline__ size_t tc_pipe_bytes(int stages) {
   const size_t b = (size_t)stages * (kStageA + kStageB);
   return b < 32768 ? 32768 : b;
 }
-__host__ __device__ __forceinline__ int tc_gr_rows(int M) { return M < kBN ? M : kBN; }
+
 
 // Epilogue of one tile slice: T[j][row] holds the fp32 accumulator of token m0 + j (j < mcount)
-// for output row n = this thread's row; G / R hold the gate and residual rows (residual
-// epilogue). Small rolled loops keep the code compact.
-__device__ __forceinline__ void tile_epilogue(const TcGemmArgs& p, const float* T, const float* G, const float* R,
-                                              int m0, int mcount, int n, int row, int lane) {
+// for output row n = this thread's row; `plane` is the K split (partial epilogue). Small rolled
+// loops keep the code compact.
+__device__ __forceinline__ void tile_epilogue(const TcGemmArgs& p, const float* T, int plane, int m0, int mcount,
+                                              int n, int row, int lane) {
   const float b = p.bias ? p.bias[n] : 0.f;
   const float* Tr = T + row;
   switch (p.epi) {
-    case EPI_RESID_GATE:
+    case EPI_PARTIAL: {
+      // this split's fp32 partial tile into its own plane [split][M][N]; the consumer sums
+      float* dst = static_cast<float*>(p.out) + (size_t)plane * p.M * p.N;
 #pragma unroll 4
-      for (int j = 0; j < mcount; ++j)
-        p.resid[(size_t)(m0 + j) * p.ldr + n] =
-            fmaf(p.gate_tab ? G[j * kBM + row] : 1.f, Tr[j * kBM] + b, R[j * kBM + row]);
+      for (int j = 0; j < mcount; ++j) dst[(size_t)(m0 + j) * p.N + n] = Tr[j * kBM];
       break;
+    }
     case EPI_GEGLU:
       if ((lane & 1) == 0) {
 #pragma unroll 4
@@ -245,17 +247,13 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   const int KC = p.K / kBK;
   const int c0 = s * KC / p.splits, c1 = (s + 1) * KC / p.splits, nch = c1 - c0;
   const int stages = tc_stages(nch, p.epi);
-  const bool resid = p.epi == EPI_RESID_GATE;
+  const bool partial = p.epi == EPI_PARTIAL;
   uint8_t* sA = smem;
   uint8_t* sB = smem + (size_t)stages * kStageA;
-  const int grr = tc_gr_rows(p.M);
-  float* G = reinterpret_cast<float*>(smem + tc_pipe_bytes(stages));   // [grr][kBM] gates
-  float* R = G + grr * kBM;                                            // [grr][kBM] residual rows
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + tc_pipe_bytes(stages) + (resid ? 2 * grr * kBM * 4 : 0));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + tc_pipe_bytes(stages));
   uint64_t* empty = full + kTcMaxStages;
   uint64_t* done = empty + kTcMaxStages;
-  uint64_t* bar_gr = done + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_gr + 1);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
   int* last_flag = reinterpret_cast<int*>(tmem_slot + 1);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int m0 = mt * kBN;
@@ -267,7 +265,6 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
       mbar_init(empty + i, 1);
     }
     mbar_init(done, 1);
-    mbar_init(bar_gr, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 0) {
@@ -325,19 +322,6 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
     }
     TC_TRACE(5);
     mma_commit(done);
-  } else if (resid && warp == 2) {
-    // ---- warp 2 fetches the residual epilogue's inputs while the tile is computed: one 512-byte
-    //      bulk copy per token for the residual row resid[m][n0..n0+127] and for the gate row
-    //      gate_tab[tau(m)][n0..n0+127], all in flight at once ----
-    pdl_wait();
-    const int n0 = t * kBM;
-    if (lane == 0) mbar_expect_tx(bar_gr, (p.gate_tab ? 2u : 1u) * (uint32_t)mcount * (kBM * 4));
-    __syncwarp();
-    for (int j = lane; j < mcount; j += 32) {
-      bulk_g2s_plain(R + j * kBM, p.resid + (size_t)(m0 + j) * p.ldr + n0, kBM * 4, bar_gr);
-      if (p.gate_tab)
-        bulk_g2s_plain(G + j * kBM, p.gate_tab + (size_t)p.tau_row[m0 + j] * p.gate_stride + n0, kBM * 4, bar_gr);
-    }
   }
   __syncwarp();
 
@@ -361,7 +345,7 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   for (int j = 0; j < kBN; ++j) T[j * kBM + row] = v[j];
   __syncthreads();
   if (threadIdx.x == 0) TC_TRACE(7);
-  if (p.splits > 1) {
+  if (p.splits > 1 && !partial) {
     // add the partial tile into the L2 accumulator with 16-byte reds; the last CTA of the tile
     // reads the sum back (independent 16-byte loads) and clears it for the next launch
     float* acc = p.acc + (size_t)m0 * p.N + t * kBM;
@@ -405,8 +389,18 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
     __syncthreads();
     if (threadIdx.x == 0 && last) TC_TRACE(10);
   }
-  if (resid) mbar_wait(bar_gr, 0, p.err, 15);   // gate / residual rows fetched by warp 2
-  if (have) tile_epilogue(p, T, G, R, m0, mcount, n, row, lane);
+  if (partial) {
+    // plane s of [splits][M][N]: whole rows of the tile as 16-byte stores
+    if (have) {
+      float* dst = static_cast<float*>(p.out) + (size_t)s * p.M * p.N + (size_t)m0 * p.N + t * kBM;
+      for (int idx = threadIdx.x; idx < mcount * (kBM / 4); idx += 128) {
+        const int j = idx / (kBM / 4), c4 = idx % (kBM / 4);
+        *reinterpret_cast<float4*>(dst + (size_t)j * p.N + c4 * 4) = *reinterpret_cast<const float4*>(T + j * kBM + c4 * 4);
+      }
+    }
+  } else if (have) {
+    tile_epilogue(p, T, s, m0, mcount, n, row, lane);
+  }
   tc_fence_before();
   __syncthreads();
   if (threadIdx.x == 0) TC_TRACE(11);
@@ -432,18 +426,14 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_wide_kernel(const __grid_const
   const int t = blockIdx.x, mt = blockIdx.y;
   const int KC = p.K / kBK;
   const int stages = KC < kWStages ? KC : kWStages;
-  const bool resid = p.epi == EPI_RESID_GATE;
   uint8_t* sA = smem;                                        // stages x 16 KB weights
   uint8_t* sB = smem + (size_t)kWStages * kStageA;           // stages x 32 KB activations
-  // after the main loop the stage area holds the epilogue slices: T, G, R (32 KB each)
+  // after the main loop the stage area holds the epilogue slice T (32 KB)
   float* T = reinterpret_cast<float*>(smem);
-  float* G = T + kBN * kBM;
-  float* R = G + kBN * kBM;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)kWStages * (kStageA + kWStageB));
   uint64_t* empty = full + kWStages;
   uint64_t* done = empty + kWStages;
-  uint64_t* bar_gr = done + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_gr + 1);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
@@ -452,7 +442,6 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_wide_kernel(const __grid_const
       mbar_init(empty + i, 1);
     }
     mbar_init(done, 1);
-    mbar_init(bar_gr, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 0) {
@@ -515,15 +504,6 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_wide_kernel(const __grid_const
     const int m0 = mt * kWN + q * kBN;
     if (m0 >= p.M) break;
     const int mcount = p.M - m0 < kBN ? p.M - m0 : kBN;
-    if (resid && warp == 2) {
-      if (lane == 0) mbar_expect_tx(bar_gr, (p.gate_tab ? 2u : 1u) * (uint32_t)mcount * (kBM * 4));
-      __syncwarp();
-      for (int j = lane; j < mcount; j += 32) {
-        bulk_g2s_plain(R + j * kBM, p.resid + (size_t)(m0 + j) * p.ldr + t * kBM, kBM * 4, bar_gr);
-        if (p.gate_tab)
-          bulk_g2s_plain(G + j * kBM, p.gate_tab + (size_t)p.tau_row[m0 + j] * p.gate_stride + t * kBM, kBM * 4, bar_gr);
-      }
-    }
     float v[kBN];
     __syncwarp();
 #pragma unroll
@@ -531,8 +511,7 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_wide_kernel(const __grid_const
 #pragma unroll
     for (int j = 0; j < kBN; ++j) T[j * kBM + row] = v[j];
     __syncthreads();
-    if (resid) mbar_wait(bar_gr, q & 1, p.err, 35);
-    if (ok) tile_epilogue(p, T, G, R, m0, mcount, n, row, lane);
+    if (ok) tile_epilogue(p, T, 0, m0, mcount, n, row, lane);
     __syncthreads();
   }
   tc_fence_before();
@@ -595,16 +574,16 @@ int encode_act_tmap(CUtensorMap* m, const void* base, int K, int rows) {
 }
 
 size_t gemm_tc_smem_bytes(int stages, int epi, int M) {
-  return 1024 + tc_pipe_bytes(stages) + (epi == EPI_RESID_GATE ? 2 * (size_t)tc_gr_rows(M) * kBM * 4 : 0) +
-         (2 * kTcMaxStages + 2) * 8 + 16;
+  (void)epi;
+  (void)M;
+  return 1024 + tc_pipe_bytes(stages) + (2 * kTcMaxStages + 1) * 8 + 16;
 }
 
 static size_t gemm_tc_wide_smem_bytes() { return 1024 + (size_t)kWStages * (kStageA + kWStageB) + (2 * kWStages + 2) * 8 + 16; }
 
 void gemm_tc_prepare() {
   const size_t a = gemm_tc_smem_bytes(kTcMaxStages, EPI_STORE, kBN);
-  const size_t b = gemm_tc_smem_bytes(kTcMaxStagesResid, EPI_RESID_GATE, kBN);
-  cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)(a > b ? a : b));
+  cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)a);
   cudaFuncSetAttribute(gemm_tc_wide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)gemm_tc_wide_smem_bytes());
 }
 
@@ -615,16 +594,17 @@ bool gemm_tc_use_wide(int M, int N, int sms) {
   return M >= kWN && N <= 4096 && (N / kBM) * ((M + kWN - 1) / kWN) * 2 >= sms;
 }
 
-// K splits per output tile: one CTA per SM. Residual epilogues (small shared-memory ring) take
-// more splits, up to two CTAs per SM, so that every CTA holds its whole K range in flight (one
-// HBM round trip); for the other epilogues extra splits cost more in reduction than they save.
+// K splits per output tile: one CTA per SM. Partial-plane epilogues (the consumer sums the
+// planes) take more splits, up to two CTAs per SM, so that every CTA holds its whole K range in
+// flight (one HBM round trip); where the kernel reduces in L2, extra splits cost more than they
+// save.
 int gemm_tc_splits(int M, int N, int K, int sms, int epi) {
   const int tiles = (N / kBM) * ((M + kBN - 1) / kBN);
   const int KC = K / kBK;
-  const int cap = kTcMaxStagesResid;
+  const int cap = kTcMaxStages;
   int s = sms / tiles;
   if (s < 1) s = 1;
-  if (epi == EPI_RESID_GATE && (KC + s - 1) / s > cap) {
+  if (epi == EPI_PARTIAL && (KC + s - 1) / s > cap) {
     const int need = (KC + cap - 1) / cap;
     const int most = 2 * sms / tiles;
     s = need < most ? need : (most > s ? most : s);

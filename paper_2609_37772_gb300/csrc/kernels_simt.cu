@@ -264,7 +264,94 @@ __global__ void __launch_bounds__(256) norm_reg_kernel(NormArgs p) {
   }
 }
 
+// Residual update + adaptive norm, one CTA per token row, 4 columns per thread:
+//   h += gate(tau) * (sum_s part[s] + bias);  y = norm(h) * (1 + scale[tau]) + shift[tau].
+// The K-split partial planes are summed in plane order (deterministic); all of a thread's
+// loads are issued before the arithmetic that needs them.
+__device__ __forceinline__ float block_sum(float v, float* red) {
+  v = warp_sum(v);
+  const int w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  __syncthreads();                       // red[] may still be read by the previous call
+  if ((threadIdx.x & 31) == 0) red[w] = v;
+  __syncthreads();
+  float t = 0.f;
+  for (int i = 0; i < nw; ++i) t += red[i];
+  return t;
+}
+
+__global__ void __launch_bounds__(1024) resid_norm_kernel(NormArgs p) {
+  __shared__ float red[32];
+  pdl_trigger();
+  pdl_wait();
+  const int row = blockIdx.x, c4 = threadIdx.x;
+  const bool on = c4 * 4 < p.W;
+  const int tr = p.tau_row[row];
+  float4 x = make_float4(0.f, 0.f, 0.f, 0.f), sc = x, sh = x, gt = make_float4(1.f, 1.f, 1.f, 1.f), bs = x;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  float4* h4 = reinterpret_cast<float4*>(p.h + (long long)row * p.ldh) + c4;
+  if (on) {
+    x = *h4;
+    const float* mod = p.tab ? p.tab + (long long)tr * p.stride : nullptr;
+    if (mod) {
+      sc = __ldg(reinterpret_cast<const float4*>(mod + p.scale_off) + c4);
+      sh = __ldg(reinterpret_cast<const float4*>(mod + p.shift_off) + c4);
+    }
+    if (p.rgate_tab) gt = __ldg(reinterpret_cast<const float4*>(p.rgate_tab + (long long)tr * p.stride + p.rgate_off) + c4);
+    if (p.rbias) bs = __ldg(reinterpret_cast<const float4*>(p.rbias) + c4);
+    const long long plane4 = (long long)p.M * p.W / 4;
+    const float4* pp = reinterpret_cast<const float4*>(p.part + (long long)row * p.W) + c4;
+    int i = 0;
+    for (; i + 8 <= p.n_part; i += 8) {
+      float4 q[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) q[u] = __ldcg(pp + (i + u) * plane4);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        acc.x += q[u].x; acc.y += q[u].y; acc.z += q[u].z; acc.w += q[u].w;
+      }
+    }
+    for (; i < p.n_part; ++i) {
+      const float4 q = __ldcg(pp + i * plane4);
+      acc.x += q.x; acc.y += q.y; acc.z += q.z; acc.w += q.w;
+    }
+    x.x = fmaf(gt.x, acc.x + bs.x, x.x);
+    x.y = fmaf(gt.y, acc.y + bs.y, x.y);
+    x.z = fmaf(gt.z, acc.z + bs.z, x.z);
+    x.w = fmaf(gt.w, acc.w + bs.w, x.w);
+    *h4 = x;
+  }
+  float mean = 0.f;
+  if (p.layer_norm) mean = block_sum(on ? (x.x + x.y) + (x.z + x.w) : 0.f, red) / p.W;
+  const float a = x.x - mean, b = x.y - mean, c = x.z - mean, d = x.w - mean;
+  const float ss = block_sum(on ? fmaf(a, a, fmaf(b, b, fmaf(c, c, d * d))) : 0.f, red);
+  const float rstd = 1.f / sqrtf(ss / p.W + 1e-6f);
+  if (!on) return;
+  float4 y = make_float4(a * rstd, b * rstd, c * rstd, d * rstd);
+  if (p.tab) {
+    y.x = fmaf(y.x, 1.f + sc.x, sh.x);
+    y.y = fmaf(y.y, 1.f + sc.y, sh.y);
+    y.z = fmaf(y.z, 1.f + sc.z, sh.z);
+    y.w = fmaf(y.w, 1.f + sc.w, sh.w);
+  }
+  const long long off = (long long)row * p.ldo + c4 * 4;
+  if (p.out_dtype == BF16) {
+    __nv_bfloat162 lo = __floats2bfloat162_rn(y.x, y.y), hi = __floats2bfloat162_rn(y.z, y.w);
+    uint2 pk;
+    pk.x = *reinterpret_cast<uint32_t*>(&lo);
+    pk.y = *reinterpret_cast<uint32_t*>(&hi);
+    *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(p.out) + off) = pk;
+  } else {
+    *reinterpret_cast<float4*>(static_cast<float*>(p.out) + off) = y;
+  }
+}
+
 void launch_norm(const NormArgs& a, cudaStream_t s) {
+  if (a.part) {
+    // the caller guarantees 16-byte rows: W, ldh, ldo, stride and the offsets multiples of 4
+    const int threads = ((a.W / 4 + 31) / 32) * 32;
+    launch_k(resid_norm_kernel, dim3(a.M), dim3(threads), 0, s, a);
+    return;
+  }
   const int blocks = (a.M + 7) / 8;
   const bool aligned = a.ldh % 4 == 0 && a.ldo % 4 == 0 && a.scale_off % 4 == 0 && a.shift_off % 4 == 0 &&
                        a.stride % 4 == 0 && a.W % 128 == 0;

@@ -71,6 +71,7 @@ struct uad_ctx {
   float* tc_acc = nullptr;
   int* tc_counters = nullptr;
   int* dev_err = nullptr;
+  float* part = nullptr;          // K-split partial planes of the residual projections
 
   // weights (library layout)
   float *t_w1 = nullptr, *t_b1 = nullptr, *t_w2 = nullptr, *t_b2 = nullptr;  // t_w* are dtype
@@ -332,11 +333,18 @@ struct Mark {
   }
 };
 
+// Partial planes a residual projection [M][W] x [W][K]^T writes on the tensor cores.
+size_t residual_planes(const uad_ctx* c, int M, int K) {
+  const int W = c->a.width;
+  return gemm_tc_use_wide(M, W, c->sms) ? 1 : (size_t)gemm_tc_splits(M, W, K, c->sms, EPI_PARTIAL);
+}
+
 // Algorithmic HBM bytes of one projection: weights + activations in + output (+ residual r/w).
 double gemm_bytes(const GemmArgs& g, int wes) {
   const double aes = g.a_dtype == BF16 ? 2 : 4, oes = g.out_dtype == BF16 ? 2 : 4;
   double b = (double)g.N * g.K * wes + (double)g.M * g.K * aes;
   if (g.epi == EPI_RESID_GATE) b += 8.0 * g.M * g.N;
+  else if (g.epi == EPI_PARTIAL) b += 4.0 * g.M * g.N;
   else if (g.epi == EPI_GEGLU) b += oes * g.M * (g.N / 2);
   else b += oes * (double)g.M * g.N;
   return b;
@@ -355,8 +363,7 @@ void gemm(uad_ctx* c, const Lin& w, GemmArgs g, cudaStream_t s) {
   t.wide = gemm_tc_use_wide(g.M, g.N, c->sms);
   t.splits = t.wide ? 1 : gemm_tc_splits(g.M, g.N, g.K, c->sms, g.epi);
   t.epi = g.epi; t.out = g.out; t.ldo = g.ldo; t.out_dtype = g.out_dtype; t.bias = g.bias;
-  t.resid = g.resid; t.ldr = g.ldr; t.gate_tab = g.gate_tab; t.gate_stride = g.gate_stride;
-  t.tau_row = g.tau_row; t.qkv = g.qkv; t.acc = c->tc_acc; t.counters = c->tc_counters; t.err = c->dev_err;
+  t.qkv = g.qkv; t.acc = c->tc_acc; t.counters = c->tc_counters; t.err = c->dev_err;
   launch_gemm_tc(&c->tmaps.at(g.A), t, s);
 }
 
@@ -364,6 +371,49 @@ void gemm(uad_ctx* c, const void* w, GemmArgs g, cudaStream_t s) {
   Lin l;
   l.w = const_cast<void*>(w);
   gemm(c, l, g, s);
+}
+
+// Residual update h += gate(tau) * (A W^T + bias) (gate 1 without a table). Tensor-core
+// weights: the K splits write fp32 partial planes and the update is left pending in `pend`
+// for the next norm, which sums the planes in a fixed order, applies it and normalises in one
+// pass over the row. CUDA-core weights: applied in the GEMM epilogue.
+struct PendingResid {
+  const float* part = nullptr; int n_part = 0;
+  const float* gate_tab = nullptr; int gate_off = 0;
+  const float* bias = nullptr;
+};
+
+void resid_gemm(uad_ctx* c, const Lin& w, GemmArgs g, int gate_off, const float* bias, PendingResid* pend,
+                const char* name, cudaStream_t s) {
+  const double flops = 2.0 * g.M * g.N * g.K;
+  if (w.tiled) {
+    g.epi = EPI_PARTIAL; g.out = c->part; g.ldo = g.N; g.out_dtype = F32;
+    pend->part = c->part;
+    pend->n_part = (int)residual_planes(c, g.M, g.K);
+    pend->gate_tab = gate_off >= 0 ? c->tab : nullptr;
+    pend->gate_off = gate_off;
+    pend->bias = bias;
+    Mark mk(c, s, name, gemm_bytes(g, c->es), flops);
+    gemm(c, w, g, s);
+    return;
+  }
+  g.epi = EPI_RESID_GATE; g.resid = c->h; g.ldr = g.N; g.bias = bias;
+  if (gate_off >= 0) { g.gate_tab = c->tab + gate_off; g.gate_stride = c->rowlen; }
+  Mark mk(c, s, name, gemm_bytes(g, c->es), flops);
+  gemm(c, w, g, s);
+}
+
+// Norm of the residual stream, applying (and clearing) a pending residual update first.
+void norm_after(uad_ctx* c, NormArgs n, PendingResid* pend, cudaStream_t s) {
+  double by = (4.0 + c->es) * n.M * n.W;
+  if (pend->part) {
+    n.part = pend->part; n.n_part = pend->n_part;
+    n.rgate_tab = pend->gate_tab; n.rgate_off = pend->gate_off; n.rbias = pend->bias;
+    by += 8.0 * n.M * n.W;                     // partial sum in, residual row out
+    *pend = PendingResid();
+  }
+  Mark mk(c, s, n.part ? "resid_norm" : "norm", by, 0);
+  launch_norm(n, s);
 }
 
 // 2-D TMA descriptor of a bf16 activation buffer [rows][K]: 64 x 64 boxes, 128-byte swizzle,
@@ -388,6 +438,7 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
   const bool dit = a.kind == UAD_KIND_DIT;
 
   { Mark mk(c, s, "begin", 12.0 * M * D, 0); launch_begin(c->noise, c->x, c->g, c->u, M * D, c->nonfinite, c->evals, c->stamps, s); }
+  PendingResid pend;
   for (int k = 1; k <= n_steps; ++k) {
     const int* tr = tau + (size_t)(k - 1) * M;
     GemmArgs gi;
@@ -403,7 +454,7 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
       na.stride = c->rowlen; na.tau_row = tr; na.out = c->y; na.ldo = W; na.out_dtype = dt;
       na.scale_off = dit ? base + W : base;
       na.shift_off = dit ? base : base + W;
-      { Mark mk(c, s, "norm", (4.0 + c->es) * M * W, 0); launch_norm(na, s); }
+      norm_after(c, na, &pend, s);
       GemmArgs gq;
       gq.A = c->y; gq.lda = W; gq.a_dtype = dt; gq.w_dtype = dt;
       gq.M = M; gq.N = c->qkvd; gq.K = W; gq.out = c->qkv; gq.ldo = c->qkvd; gq.out_dtype = dt;
@@ -445,13 +496,12 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
       }
       GemmArgs go;
       go.A = c->o; go.lda = c->qd; go.a_dtype = dt; go.w_dtype = dt;
-      go.M = M; go.N = W; go.K = c->qd; go.epi = EPI_RESID_GATE; go.resid = c->h; go.ldr = W;
-      go.gate_tab = c->tab + base + 2 * W; go.gate_stride = c->rowlen; go.tau_row = tr;
-      { Mark mk(c, s, "o_proj", gemm_bytes(go, c->es), 2.0 * M * W * c->qd); gemm(c, w.wo, go, s); }
+      go.M = M; go.N = W; go.K = c->qd; go.tau_row = tr;
+      resid_gemm(c, w.wo, go, base + 2 * W, nullptr, &pend, "o_proj", s);
       if (dit) {
         NormArgs nc = na;
         nc.tab = nullptr;
-        { Mark mk(c, s, "norm", (4.0 + c->es) * M * W, 0); launch_norm(nc, s); }
+        norm_after(c, nc, &pend, s);
         GemmArgs gc;
         gc.A = c->y; gc.lda = W; gc.a_dtype = dt; gc.w_dtype = dt;
         gc.M = M; gc.N = c->qd; gc.K = W; gc.out = c->qc; gc.ldo = c->qd; gc.out_dtype = dt;
@@ -470,13 +520,13 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
         }
         GemmArgs gco;
         gco.A = c->o; gco.lda = c->qd; gco.a_dtype = dt; gco.w_dtype = dt;
-        gco.M = M; gco.N = W; gco.K = c->qd; gco.epi = EPI_RESID_GATE; gco.resid = c->h; gco.ldr = W;
-        { Mark mk(c, s, "o_cross_proj", gemm_bytes(gco, c->es), 2.0 * M * W * c->qd); gemm(c, w.woc, gco, s); }
+        gco.M = M; gco.N = W; gco.K = c->qd; gco.tau_row = tr;
+        resid_gemm(c, w.woc, gco, -1, nullptr, &pend, "o_cross_proj", s);
       }
       NormArgs n2 = na;
       n2.scale_off = dit ? base + 4 * W : base + 3 * W;
       n2.shift_off = dit ? base + 3 * W : base + 4 * W;
-      { Mark mk(c, s, "norm", (4.0 + c->es) * M * W, 0); launch_norm(n2, s); }
+      norm_after(c, n2, &pend, s);
       GemmArgs g1;
       g1.A = c->y; g1.lda = W; g1.a_dtype = dt; g1.w_dtype = dt; g1.M = M; g1.K = W;
       g1.out = c->act; g1.ldo = F; g1.out_dtype = dt;
@@ -485,17 +535,15 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
       { Mark mk(c, s, dit ? "mlp_up" : "gate_up_proj", gemm_bytes(g1, c->es), 2.0 * M * g1.N * W); gemm(c, dit ? w.w1 : w.wgu, g1, s); }
       GemmArgs g2;
       g2.A = c->act; g2.lda = F; g2.a_dtype = dt; g2.w_dtype = dt;
-      g2.M = M; g2.N = W; g2.K = F; g2.epi = EPI_RESID_GATE; g2.resid = c->h; g2.ldr = W;
-      g2.bias = dit ? w.b2 : nullptr;
-      g2.gate_tab = c->tab + base + 5 * W; g2.gate_stride = c->rowlen; g2.tau_row = tr;
-      { Mark mk(c, s, dit ? "mlp_down" : "down_proj", gemm_bytes(g2, c->es), 2.0 * M * W * F); gemm(c, dit ? w.w2 : w.wd, g2, s); }
+      g2.M = M; g2.N = W; g2.K = F; g2.tau_row = tr;
+      resid_gemm(c, dit ? w.w2 : w.wd, g2, base + 5 * W, dit ? w.b2 : nullptr, &pend, dit ? "mlp_down" : "down_proj", s);
     }
     NormArgs nf;
     nf.h = c->h; nf.ldh = W; nf.M = M; nf.W = W; nf.layer_norm = dit; nf.tab = c->tab;
     nf.stride = c->rowlen; nf.tau_row = tr; nf.out = c->y; nf.ldo = W; nf.out_dtype = dt;
     nf.scale_off = a.n_layers * W6 + (dit ? W : 0);
     nf.shift_off = a.n_layers * W6 + (dit ? 0 : W);
-    { Mark mk(c, s, "norm", (4.0 + c->es) * M * W, 0); launch_norm(nf, s); }
+    norm_after(c, nf, &pend, s);
     GemmArgs go;
     go.A = c->y; go.lda = W; go.a_dtype = dt; go.w_dtype = dt;
     go.M = M; go.N = D; go.K = W; go.out = c->v; go.ldo = D; go.bias = c->b_out;
@@ -758,6 +806,11 @@ int uad_init(const uad_arch* arch, const float* weights, size_t n_floats, uad_ct
     const size_t maxN = std::max({(size_t)c->qkvd, (size_t)2 * F, (size_t)W});
     TRY(dalloc_t(c, &c->tc_acc, M * maxN));
     TRY(dalloc_t(c, &c->tc_counters, 1 << 16));
+    size_t part = 0;
+    for (int b = 1; b <= a.max_batch; ++b)
+      part = std::max({part, residual_planes(c, b * H, c->qd) * (size_t)b * H * W,
+                       residual_planes(c, b * H, F) * (size_t)b * H * W});
+    TRY(dalloc_t(c, &c->part, part));
     gemm_tc_prepare();
   }
   TRY(dalloc_t(c, &c->E, (size_t)a.max_batch * D));

@@ -40,9 +40,10 @@ inline cudaError_t launch_k(void (*kern)(KArgs...), dim3 grid, dim3 block, size_
 enum Epi {
   EPI_STORE = 0,       // out = acc (+ bias) (+ add_rows[m % add_mod][n])
   EPI_BIAS_SILU = 1,   // out = silu(acc + bias)
-  EPI_RESID_GATE = 2,  // resid[m][n] += gate(m, n) * (acc + bias); gate = 1 when gate_tab is null
+  EPI_RESID_GATE = 2,  // CUDA cores: resid[m][n] += gate(m, n) * (acc + bias); gate = 1 without gate_tab
   EPI_GEGLU = 3,       // rows interleaved (2j = gate, 2j+1 = up): out[m][j] = gelu_tanh(g) * u
   EPI_BIAS_GELU = 4,   // out = gelu_tanh(acc + bias)
+  EPI_PARTIAL = 6,     // tensor cores: K split s writes its fp32 tile to plane s of out [splits][M][N]
   EPI_QKV_TC = 5,      // q/k rows pair-interleaved per head: RoPE, then scatter q -> Q, k -> K cache,
                        // v -> Vt cache (tensor-core attention layouts, see attn_tc.cu)
 };
@@ -71,7 +72,11 @@ struct GemmArgs {
 };
 
 struct NormArgs {
-  const float* h = nullptr; int ldh = 0;   // fp32 [M][W]
+  float* h = nullptr; int ldh = 0;         // fp32 [M][W]
+  // pending residual update applied first (resid_norm): h += gate * (sum of n_part planes + bias)
+  const float* part = nullptr; int n_part = 0;   // planes [n_part][M][W]
+  const float* rgate_tab = nullptr; int rgate_off = 0;  // gate(m, c) = rgate_tab[tau_row[m] * stride + rgate_off + c]
+  const float* rbias = nullptr;            // [W]
   int M = 0, W = 0;
   int layer_norm = 0;                      // 0: RMSNorm, 1: LayerNorm (no affine)
   const float* tab = nullptr; int stride = 0; int scale_off = 0, shift_off = 0;  // modulation
@@ -125,7 +130,7 @@ constexpr int kGemvMaxK = 8192;
 void launch_gemm_simt(const GemmArgs& a, cudaStream_t s);
 bool gemv_rows_ok(const GemmArgs& a);                     // tiny-side projection (N or K <= 64)
 void launch_gemv_rows(const GemmArgs& a, cudaStream_t s);
-void launch_norm(const NormArgs& a, cudaStream_t s);
+void launch_norm(const NormArgs& a, cudaStream_t s);   // applies the pending residual if part != null
 void launch_attention(const AttnArgs& a, cudaStream_t s);
 void launch_euler(const EulerArgs& a, cudaStream_t s);
 void launch_euler_prepare();   // shared memory for H x D GAC terms (up to 256 x 64)
@@ -140,15 +145,12 @@ void launch_convert(const void* src, int src_dtype, void* dst, int dst_dtype, lo
 
 // gemm_tc.cu: tcgen05 projection GEMM (bf16 operands, fp32 accumulation in TMEM)
 constexpr int kTcMaxStages = 4;        // <= ~97 KB of shared memory: two CTAs fit one SM
-constexpr int kTcMaxStagesResid = 2;   // plus the staged gate / residual rows (two CTAs per SM)
 struct TcGemmArgs {
   const void* w_tiled = nullptr;   // [N/128][K/64] blocks of 128 x 64 bf16, 128B-swizzled K-major
   int M = 0, N = 0, K = 0, splits = 1;
   int epi = EPI_STORE;
   void* out = nullptr; int ldo = 0; int out_dtype = BF16;
   const float* bias = nullptr;
-  float* resid = nullptr; int ldr = 0;
-  const float* gate_tab = nullptr; int gate_stride = 0; const int* tau_row = nullptr;
   QkvTcOut qkv;                    // EPI_QKV_TC
   float* acc = nullptr;            // split-K accumulator [M][N] fp32, zero between launches
   int* counters = nullptr;         // split-K arrival counters per output tile, zero between launches
