@@ -1,0 +1,961 @@
+// Persistent evaluation kernel: one velocity evaluation v = F_theta(u, tau) of an adaRMS action
+// expert with few tokens (B * H <= 64) in a single launch, one CTA per SM.
+//
+// With few tokens an evaluation is a chain of about ten dependent steps per layer, each far
+// too small to fill the GPU; as separate kernels every step pays launch, drain and
+// weight-fetch latency. Here every CTA runs every step of every layer, and grid-wide barriers
+// (bounded spins on global counters) separate the steps. One producer thread per CTA streams
+// this CTA's share of every projection weight (and nothing else) through a shared-memory ring
+// without waiting for the barriers: the weights do not depend on the activations, so HBM
+// streams ahead across steps and layers while the consumers wait for their inputs.
+//
+// Steps of layer l, each followed by a grid barrier:
+//   norm1    row m (CTA m): h += gate2'(tau) * acc_d (l > 0; h = W_in u + b_in at l = 0),
+//            y = RMSNorm(h) * (1 + scale) + shift                                 (bf16)
+//   qkv      weight tiles [v T / G, (v+1) T / G) of W_qkv: acc_qkv += y W^T    (red.add, fp32)
+//   rope     row m: RoPE on q and k, q -> Q, k -> K cache, v -> Vt cache         (bf16)
+//   attn     items (robot-group, 128 query rows, 64 keys): S = Q K^T, P = exp(S - max),
+//            O = P V on tcgen05 -> partial O rows and (max, sum)
+//   combine  query rows: log-sum-exp merge of the key chunks -> o               (bf16)
+//   o        acc_o += o W_o^T
+//   norm2    row m: h += gate1(tau) * acc_o, y = adaRMS2(h)
+//   gate_up  acc_gu += y W_gu^T  (rows interleaved gate_j, up_j)
+//   act      row m: act = gelu_tanh(gate) * up                                   (bf16)
+//   down     acc_d += act W_d^T
+// then the final norm and the action-out projection v = W_out y + b_out (row m). Every
+// accumulator row is cleared by the CTA that consumes it, so the next use starts from zero.
+//
+// Warps: 0-3 = consumers (TMEM lane quadrants 0-3; row steps), 4 = weight producer (lane 0),
+// 5 = tcgen05 issuer and TMA loads of activations and attention operands (lane 0).
+// Every wait is bounded: on timeout the kernel records an error code, skips the remaining
+// work, waits (bounded) for its copies in flight and frees its tensor memory.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include "uad_internal.cuh"
+
+namespace uad {
+
+namespace {
+
+constexpr int kSlot = 16384;         // weight tile: 128 rows x 64 bf16, 128-byte swizzled
+constexpr int kATile = 8192;         // activation tile: 64 tokens x 64 bf16
+constexpr int kQT = 128, kKC = 64;   // attention: query rows per tile, keys per chunk
+constexpr int kThreads = 192;
+constexpr int kMaxRows = kStepMaxRows;   // tokens per evaluation (the N side of every MMA)
+constexpr int kMaxATiles = kStepMaxATiles;
+constexpr int kMaxRing = kStepMaxRing;
+constexpr uint32_t kTmemCols = 512;  // projection segments at 64-column steps; attention S at 0, O at 256
+constexpr unsigned long long kWaitNs = 2000000000ull;   // any single wait
+constexpr unsigned long long kDrainNs = 200000000ull;   // waiting for own copies before exit
+
+__device__ __forceinline__ uint32_t su32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ unsigned long long gtime() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void mbar_init(uint64_t* b, uint32_t n) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(b)), "r"(n));
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* b, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(b)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* b) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(b)) : "memory");
+}
+__device__ __forceinline__ bool mbar_test(uint64_t* b, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok) : "r"(su32(b)), "r"(parity) : "memory");
+  return ok != 0;
+}
+// Wait for the phase with the given parity; false at once if an error is already recorded,
+// false with *err = code after kWaitNs.
+__device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity, int* err, int code) {
+  unsigned long long t0 = 0;
+  for (uint32_t it = 0;; ++it) {
+    if (mbar_test(b, parity)) return true;
+    if ((it & 255) == 0) {
+      if (*reinterpret_cast<volatile int*>(err) != 0) return false;
+      const unsigned long long t = gtime();
+      if (t0 == 0) t0 = t;
+      else if (t - t0 > kWaitNs) {
+        atomicCAS(err, 0, code);
+        return false;
+      }
+    }
+  }
+}
+// Wait for own asynchronous work before the CTA exits: bounded by time only.
+__device__ __forceinline__ void mbar_drain(uint64_t* b, uint32_t parity) {
+  const unsigned long long t0 = gtime();
+  while (!mbar_test(b, parity))
+    if (gtime() - t0 > kDrainNs) return;
+}
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ uint64_t policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar, uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;"
+      ::"r"(su32(dst)), "l"(src), "r"(bytes), "r"(su32(bar)), "l"(pol) : "memory");
+}
+__device__ __forceinline__ void tma_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+      ::"r"(su32(dst)), "l"(map), "r"(x), "r"(y), "r"(su32(bar)) : "memory");
+}
+__device__ __forceinline__ void tma_3d(void* dst, const CUtensorMap* map, int x, int y, int z, uint64_t* bar,
+                                       uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3, %4}], [%5], %6;"
+      ::"r"(su32(dst)), "l"(map), "r"(x), "r"(y), "r"(z), "r"(su32(bar)), "l"(pol) : "memory");
+}
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row core groups 1024 B apart.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
+         ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+// kind::f16 instruction descriptor: bf16 x bf16 -> fp32, K-major A and B, M = 128, N = n.
+__device__ __forceinline__ uint32_t idesc_m128(int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+}
+__device__ __forceinline__ void mma_bf16(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accum) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n"
+      ::"r"(d), "l"(a), "l"(b), "r"(idesc), "r"(accum));
+}
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(su32(bar)) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+// TMEM base address re-read from shared memory after a barrier wait: the tensor-memory loads
+// that follow take their address from this load, so they cannot be scheduled ahead of the
+// wait (the loads have no other dependence on it).
+__device__ __forceinline__ uint32_t tmem_base_after_wait(const uint32_t* slot) {
+  uint32_t t;
+  asm volatile("ld.volatile.shared.u32 %0, [%1];" : "=r"(t) : "r"(su32(slot)) : "memory");
+  return t;
+}
+__device__ __forceinline__ void red_add_v4(float* dst, float4 v) {
+  asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(dst), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
+               : "memory");
+}
+// Named barrier among `count` threads (whole warps).
+__device__ __forceinline__ void named_sync(int id, int count) {
+  asm volatile("barrier.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+__device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ float gelu_tanh(float x) {
+  const float k0 = 0.7978845608028654f;
+  return 0.5f * x * (1.f + tanhf(k0 * (x + 0.044715f * x * x * x)));
+}
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// Shared-memory plan (1024-aligned base): [weight ring: ring x 16 KB][work area X][mbarriers,
+// TMEM slot, flags, reduction scratch]. X holds, by step, the activation tiles of a projection
+// (up to kMaxATiles x 8 KB), the attention operands Q | K | Vt | P, the staged partial O rows,
+// or the final normalised row.
+__host__ __device__ constexpr size_t step_x_bytes(int dh) {
+  const size_t a = (size_t)kMaxATiles * kATile;
+  const size_t att = (size_t)dh * kQT * 2 + 2 * (size_t)dh * kKC * 2 + (size_t)kQT * kKC * 2;
+  const size_t ost = (size_t)kQT * (dh * 4 + 16);
+  const size_t m = a > att ? a : att;
+  return m > ost ? m : ost;
+}
+constexpr size_t kTailBytes = 512;   // mbarriers (<= 2 * 12 + 8), TMEM slot, flag, scratch
+
+// Projection j of a layer: 0 = qkv, 1 = o, 2 = gate/up, 3 = down.
+__device__ __forceinline__ void proj_shape(const StepArgs& p, int j, int& N, int& K) {
+  switch (j) {
+    case 0: N = p.qkvd; K = p.W; break;
+    case 1: N = p.W; K = p.qd; break;
+    case 2: N = 2 * p.F; K = p.W; break;
+    default: N = p.W; K = p.F; break;
+  }
+}
+// Tile range of this CTA in a projection of T tiles. The split is rotated from projection to
+// projection so that the CTAs that take one tile more change every time.
+__device__ __forceinline__ void tile_range(int T, int proj, int& t0, int& t1) {
+  const int G = gridDim.x;
+  const int v = (int)((blockIdx.x + 41u * (unsigned)proj) % (unsigned)G);
+  t0 = (int)((long long)v * T / G);
+  t1 = (int)((long long)(v + 1) * T / G);
+}
+
+struct Smem {
+  uint8_t* ring;
+  uint8_t* X;
+  uint64_t *full, *empty;   // [ring]
+  uint64_t *a_full, *g_done, *q_full, *v_full, *s_full, *p_full, *o_done, *fin;
+  uint32_t* tmem_slot;
+  int* flag;
+  float* red;               // [8]
+};
+
+// Shared-memory layout of a CTA (the plan described above), from the dynamic base.
+__device__ __forceinline__ Smem smem_plan(int R, size_t xbytes) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  Smem S;
+  S.ring = base;
+  S.X = base + (size_t)R * kSlot;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(S.X + xbytes);
+  S.full = bars;
+  S.empty = bars + R;
+  S.a_full = bars + 2 * R;
+  S.g_done = S.a_full + 1;
+  S.q_full = S.a_full + 2;
+  S.v_full = S.a_full + 3;
+  S.s_full = S.a_full + 4;
+  S.p_full = S.a_full + 5;
+  S.o_done = S.a_full + 6;
+  S.fin = S.a_full + 7;
+  S.tmem_slot = reinterpret_cast<uint32_t*>(S.a_full + 8);
+  S.flag = reinterpret_cast<int*>(S.tmem_slot + 1);
+  S.red = reinterpret_cast<float*>(S.tmem_slot + 4);
+  return S;
+}
+
+// Per-thread position in the CTA's barrier and ring sequences (issuer and consumers advance
+// the same sequences in the same order).
+struct Role {
+  int slot = 0;                      // weight ring slot and its phase parity
+  uint32_t par = 0;
+  uint32_t apar = 0, gpar = 0, ipar = 0;   // a_full, g_done, per-attention-item barriers
+  int a_uses = 0, i_uses = 0;        // loads issued on a_full and on q_full / v_full
+};
+
+// Grid barrier among warps 0-3 and 5 of every CTA: every CTA arrives (also after an error, so
+// that no CTA waits for it), then thread 160 spins on the counter. Returns false once any error is
+// recorded, so that the remaining steps are skipped.
+__device__ bool grid_sync(unsigned* ctr, bool ok, int* err, const Smem& S) {
+  tc_fence_before();
+  __syncwarp();
+  named_sync(1, 160);
+  if (threadIdx.x == 160) {
+    bool good = ok && *reinterpret_cast<volatile int*>(err) == 0;
+    // release arrival: the CTA's writes (ordered before this thread by the named barrier)
+    // are visible at GPU scope to whoever observes the count
+    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ctr) : "memory");
+    if (good) {
+      const unsigned target = gridDim.x;
+      unsigned long long t0 = 0;
+      for (uint32_t it = 0;; ++it) {
+        if (ld_acquire(ctr) >= target) break;
+        if ((it & 63) == 63) {
+          if (*reinterpret_cast<volatile int*>(err) != 0) { good = false; break; }
+          const unsigned long long t = gtime();
+          if (t0 == 0) t0 = t;
+          else if (t - t0 > kWaitNs) {
+            atomicCAS(err, 0, 51);
+            good = false;
+            break;
+          }
+        }
+      }
+    }
+    // activations written by other CTAs are read next by this thread's tensor-map loads
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+    *S.flag = good ? 1 : 0;
+  }
+  __syncwarp();
+  named_sync(1, 160);
+  tc_fence_after();
+  return *reinterpret_cast<volatile int*>(S.flag) != 0;
+}
+
+// Sum over the 128 consumer threads (warps 0-3); every consumer gets the total.
+__device__ __forceinline__ float cons_sum(float v, float* red) {
+  v = warp_sum(v);
+  const int w = threadIdx.x >> 5;
+  if ((threadIdx.x & 31) == 0) red[w] = v;
+  named_sync(2, 128);
+  const float t = (red[0] + red[1]) + (red[2] + red[3]);
+  named_sync(2, 128);
+  return t;
+}
+
+// ---- row steps (consumers, one token row per CTA) ---------------------------------------
+constexpr int kMaxV4 = kStepMaxWidth / 512;   // float4 per consumer thread
+
+// h[m] (+)= ..., then y[m] = RMSNorm(h[m]) * (1 + scale) + shift in bf16. With `acc`, h[m] +=
+// gate(tau) * acc[m] (gate 1 when gate_off < 0) and acc[m] is cleared; with `in_proj`,
+// h[m] = W_in u[m] + b_in. Returns the normalised row in `ys` (fp32 of the bf16 values) when
+// ys is not null. Every load of the row (and of its modulation vectors) is issued up front.
+__device__ __noinline__ void row_norm(const StepArgs& p, int m, const float* mod, float* acc, int gate_off,
+                                      int scale_off, int shift_off, bool in_proj, float* red, float* ys) {
+  const int tid = threadIdx.x, W = p.W, nv = W / 512;
+  float4* h4 = reinterpret_cast<float4*>(p.h + (size_t)m * W);
+  float4 x[kMaxV4], sc[kMaxV4], sh[kMaxV4];
+#pragma unroll
+  for (int j = 0; j < kMaxV4; ++j) {
+    if (j >= nv) break;
+    const int c4 = tid + 128 * j;
+    sc[j] = __ldg(reinterpret_cast<const float4*>(mod + scale_off) + c4);
+    sh[j] = __ldg(reinterpret_cast<const float4*>(mod + shift_off) + c4);
+  }
+  if (in_proj) {
+    // W_in rows are D bf16 (D a multiple of 8): 16-byte loads, all issued before the FMAs
+    const float* u = p.u + (size_t)m * p.D;
+    const uint4* wi = static_cast<const uint4*>(p.w_in);
+    const int D8 = p.D / 8;
+#pragma unroll
+    for (int j = 0; j < kMaxV4; ++j) {
+      if (j >= nv) break;
+      const int c = (tid + 128 * j) * 4;
+      const float4 b = __ldg(reinterpret_cast<const float4*>(p.b_in + c));
+      float o[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll 8
+      for (int k8 = 0; k8 < D8; ++k8) {
+        uint4 wv[4];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) wv[r] = __ldg(wi + (size_t)(c + r) * D8 + k8);
+        const float4 u0 = __ldg(reinterpret_cast<const float4*>(u) + 2 * k8);
+        const float4 u1 = __ldg(reinterpret_cast<const float4*>(u) + 2 * k8 + 1);
+        const float uk[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          const __nv_bfloat162* w2 = reinterpret_cast<const __nv_bfloat162*>(&wv[r]);
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const float2 f = __bfloat1622float2(w2[q]);
+            o[r] = fmaf(uk[2 * q], f.x, fmaf(uk[2 * q + 1], f.y, o[r]));
+          }
+        }
+      }
+      x[j] = make_float4(o[0], o[1], o[2], o[3]);
+      h4[tid + 128 * j] = x[j];
+    }
+  } else {
+    float4 a[kMaxV4], g[kMaxV4];
+#pragma unroll
+    for (int j = 0; j < kMaxV4; ++j) {
+      if (j >= nv) break;
+      const int c4 = tid + 128 * j;
+      x[j] = h4[c4];
+      if (acc) {
+        a[j] = __ldcg(reinterpret_cast<const float4*>(acc + (size_t)m * W) + c4);
+        g[j] = gate_off >= 0 ? __ldg(reinterpret_cast<const float4*>(mod + gate_off) + c4) : make_float4(1.f, 1.f, 1.f, 1.f);
+      }
+    }
+    if (acc) {
+#pragma unroll
+      for (int j = 0; j < kMaxV4; ++j) {
+        if (j >= nv) break;
+        const int c4 = tid + 128 * j;
+        x[j].x = fmaf(g[j].x, a[j].x, x[j].x);
+        x[j].y = fmaf(g[j].y, a[j].y, x[j].y);
+        x[j].z = fmaf(g[j].z, a[j].z, x[j].z);
+        x[j].w = fmaf(g[j].w, a[j].w, x[j].w);
+        h4[c4] = x[j];
+      }
+    }
+  }
+  float ss = 0.f;
+#pragma unroll
+  for (int j = 0; j < kMaxV4; ++j) {
+    if (j >= nv) break;
+    ss = fmaf(x[j].x, x[j].x, fmaf(x[j].y, x[j].y, fmaf(x[j].z, x[j].z, fmaf(x[j].w, x[j].w, ss))));
+  }
+  const float rstd = 1.f / sqrtf(cons_sum(ss, red) / W + 1e-6f);
+  if (acc && !in_proj) {
+#pragma unroll
+    for (int j = 0; j < kMaxV4; ++j) {
+      if (j >= nv) break;
+      __stcg(reinterpret_cast<float4*>(acc + (size_t)m * W) + tid + 128 * j, make_float4(0.f, 0.f, 0.f, 0.f));
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < kMaxV4; ++j) {
+    if (j >= nv) break;
+    const int c4 = tid + 128 * j;
+    const float y0 = fmaf(x[j].x * rstd, 1.f + sc[j].x, sh[j].x), y1 = fmaf(x[j].y * rstd, 1.f + sc[j].y, sh[j].y);
+    const float y2 = fmaf(x[j].z * rstd, 1.f + sc[j].z, sh[j].z), y3 = fmaf(x[j].w * rstd, 1.f + sc[j].w, sh[j].w);
+    uint2 pk;
+    pk.x = pack_bf16(y0, y1);
+    pk.y = pack_bf16(y2, y3);
+    *reinterpret_cast<uint2*>(p.y + (size_t)m * W + c4 * 4) = pk;
+    if (ys) {
+      const __nv_bfloat162 lo = *reinterpret_cast<const __nv_bfloat162*>(&pk.x);
+      const __nv_bfloat162 hi = *reinterpret_cast<const __nv_bfloat162*>(&pk.y);
+      *reinterpret_cast<float4*>(ys + c4 * 4) =
+          make_float4(__low2float(lo), __high2float(lo), __low2float(hi), __high2float(hi));
+    }
+  }
+}
+
+// Elementwise steps run on the consumers of every CTA: work item w of `total` goes to thread
+// (w mod T) with T = 128 * CTAs, and each thread issues all of its loads before using any.
+constexpr int kEwBatch = 4;   // work items per thread and batch
+
+// q, k (RoPE) and v of every token into the attention layouts; acc_qkv cleared. Item = one
+// (token, q/k row pair) or one (token, v row).
+__device__ __noinline__ void ew_rope(const StepArgs& p, int l) {
+  const int dh = p.dh, half = dh / 2, npairs = (p.qd + p.kvd) / 2, per = npairs + p.kvd;
+  const int total = p.M * per, T = 128 * gridDim.x;
+  for (int base = blockIdx.x * 128 + threadIdx.x; base < total; base += kEwBatch * T) {
+    float2 a[kEwBatch], cs[kEwBatch];
+    // every load first: accumulator values and the rotation of each pair
+#pragma unroll
+    for (int u = 0; u < kEwBatch; ++u) {
+      const int w = base + u * T;
+      if (w >= total) break;
+      const int m = w / per, e = w % per;
+      const float* acc = p.acc_qkv + (size_t)m * p.qkvd;
+      if (e < npairs) {
+        a[u] = __ldcg(reinterpret_cast<const float2*>(acc) + e);
+        const int sn = 2 * e < p.qd ? 2 * e : 2 * e - p.qd;
+        cs[u] = p.rope ? __ldg(reinterpret_cast<const float2*>(p.rope_cs + (size_t)(m % p.H) * dh) + ((sn % dh) >> 1))
+                       : make_float2(1.f, 0.f);
+      } else {
+        a[u].x = __ldcg(acc + p.qd + p.kvd + (e - npairs));
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kEwBatch; ++u) {
+      const int w = base + u * T;
+      if (w >= total) break;
+      const int m = w / per, e = w % per, b = m / p.H, i = m % p.H;
+      float* acc = p.acc_qkv + (size_t)m * p.qkvd;
+      if (e < npairs) {
+        const int n = 2 * e;
+        const bool isq = n < p.qd;
+        const int sn = isq ? n : n - p.qd, hh = sn / dh, r = sn % dh;
+        // with RoPE, rows 2j, 2j+1 of a head hold dims j and j + dh/2 (pair-interleaved weights)
+        const int d0 = p.rope ? (r >> 1) : r, d1 = p.rope ? (r >> 1) + half : r + 1;
+        const float x0 = a[u].x * cs[u].x - a[u].y * cs[u].y;
+        const float x1 = a[u].y * cs[u].x + a[u].x * cs[u].y;
+        __nv_bfloat16* dst = isq ? p.q + (((size_t)b * p.n_heads + hh) * p.H + i) * dh
+                                 : p.kcache + ((((size_t)b * p.L + l) * p.n_kv_heads + hh) * p.n_keys + p.P + i) * dh;
+        dst[d0] = __float2bfloat16_rn(x0);
+        dst[d1] = __float2bfloat16_rn(x1);
+        __stcg(reinterpret_cast<float2*>(acc) + e, make_float2(0.f, 0.f));
+      } else {
+        const int ev = e - npairs, g = ev / dh, d = ev % dh;
+        p.vtcache[((((size_t)b * p.L + l) * p.n_kv_heads + g) * dh + d) * p.nk_pad + p.P + i] =
+            __float2bfloat16_rn(a[u].x);
+        __stcg(acc + p.qd + p.kvd + ev, 0.f);
+      }
+    }
+  }
+}
+
+// act[m][j] = gelu_tanh(acc_gu[m][2j]) * acc_gu[m][2j+1] for every token; acc_gu cleared.
+// Item = one float4 of acc_gu (two outputs).
+__device__ __noinline__ void ew_act(const StepArgs& p) {
+  const int per = p.F / 2, total = p.M * per, T = 128 * gridDim.x;
+  float4* acc = reinterpret_cast<float4*>(p.acc_gu);
+  uint32_t* out = reinterpret_cast<uint32_t*>(p.act);
+  for (int base = blockIdx.x * 128 + threadIdx.x; base < total; base += kEwBatch * T) {
+    float4 a[kEwBatch];
+#pragma unroll
+    for (int u = 0; u < kEwBatch; ++u) {
+      const int w = base + u * T;
+      if (w >= total) break;
+      a[u] = __ldcg(acc + w);
+    }
+#pragma unroll
+    for (int u = 0; u < kEwBatch; ++u) {
+      const int w = base + u * T;
+      if (w >= total) break;
+      out[w] = pack_bf16(gelu_tanh(a[u].x) * a[u].y, gelu_tanh(a[u].z) * a[u].w);
+      __stcg(acc + w, make_float4(0.f, 0.f, 0.f, 0.f));
+    }
+  }
+}
+
+// Merge the key chunks of the query rows assigned to this consumer warp.
+template <int DH>
+__device__ __noinline__ void combine_rows(const StepArgs& p) {
+  constexpr int E = DH / 32;
+  const int lane = threadIdx.x & 31;
+  const int gw = blockIdx.x * 4 + (threadIdx.x >> 5), nw = gridDim.x * 4;
+  const int nck = p.n_chunks, total = p.B * p.n_kv_heads * p.rows;
+  for (int idx = gw; idx < total; idx += nw) {
+    const int bg = idx / p.rows, r = idx % p.rows;
+    float mc = -INFINITY, lc = 0.f;
+    if (lane < nck) {
+      const size_t pi = ((size_t)bg * nck + lane) * p.r_pad + r;
+      mc = __ldcg(p.part_ml + pi * 2);
+      lc = __ldcg(p.part_ml + pi * 2 + 1);
+    }
+    const float M = warp_max(mc);
+    const float w = lane < nck ? exp2f((mc - M) * p.scale_log2) : 0.f;
+    const float L = warp_sum(w * lc);
+    float acc[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) acc[e] = 0.f;
+    // chunks in batches of kCB: every load of a batch is issued before the first FMA
+    constexpr int kCB = 32 / E < 16 ? 32 / E : 16;
+    for (int c0 = 0; c0 < nck; c0 += kCB) {
+      float v[kCB][E];
+#pragma unroll
+      for (int cc = 0; cc < kCB; ++cc) {
+        if (c0 + cc >= nck) break;
+        const float* src = p.part_o + (((size_t)bg * nck + c0 + cc) * p.r_pad + r) * DH;
+#pragma unroll
+        for (int e = 0; e < E; ++e) v[cc][e] = __ldcg(src + e * 32 + lane);
+      }
+#pragma unroll
+      for (int cc = 0; cc < kCB; ++cc) {
+        if (c0 + cc >= nck) break;
+        const float wc = __shfl_sync(0xffffffffu, w, c0 + cc);
+#pragma unroll
+        for (int e = 0; e < E; ++e) acc[e] = fmaf(wc, v[cc][e], acc[e]);
+      }
+    }
+    const int b = bg / p.n_kv_heads, g = bg % p.n_kv_heads, j = r / p.H, i = r % p.H;
+    __nv_bfloat16* dst = p.o + ((size_t)b * p.H + i) * p.qd + (size_t)(g * p.group + j) * DH;
+#pragma unroll
+    for (int e = 0; e < E; ++e) dst[e * 32 + lane] = __float2bfloat16_rn(acc[e] / L);
+  }
+}
+
+}  // namespace
+
+// ---- projection step: acc[m][n] += sum over this CTA's weight tiles of A[m][k] W[n][k] -----
+// Thread 160 loads the activation tiles (tensor map) and issues the MMAs against the weight
+// ring; the consumer warps add each finished 128 x 64 tile into `acc` (fp32, L2) with 16-byte
+// reds.
+__device__ __noinline__ void projection_step(const StepArgs& p, const CUtensorMap* amap, float* acc, int l, int j,
+                                             uint32_t tmem, size_t xbytes, Role& st) {
+  const Smem S = smem_plan(p.ring, xbytes);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, R = p.ring, M = p.M;
+  const bool mma = threadIdx.x == 160, cons = warp < 4;
+  int N, K, t0, t1;
+  proj_shape(p, j, N, K);
+  const int KT = K / 64;
+  tile_range((N / 128) * KT, 4 * l + j, t0, t1);
+  const int nt = t1 - t0;
+  if (nt <= 0) return;
+  if (mma) {
+    mbar_expect_tx(S.a_full, (uint32_t)nt * kATile);
+    for (int i = 0; i < nt; ++i) tma_2d(S.X + (size_t)i * kATile, amap, ((t0 + i) % KT) * 64, 0, S.a_full);
+    ++st.a_uses;
+    bool good = mbar_wait(S.a_full, st.apar, p.err, 42);
+    int seg = -1, pnb = -1;
+    for (int i = 0; i < nt && good; ++i) {
+      const int nb = (t0 + i) / KT;
+      const bool first = nb != pnb;
+      if (first) { ++seg; pnb = nb; }
+      good = mbar_wait(S.full + st.slot, st.par, p.err, 43);
+      if (!good) break;
+      tc_fence_after();
+      const uint32_t a0 = su32(S.ring + (size_t)st.slot * kSlot), b0 = su32(S.X + (size_t)i * kATile);
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        mma_bf16(tmem + seg * 64, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), idesc_m128(64),
+                 (first && k == 0) ? 0u : 1u);
+      mma_commit(S.empty + st.slot);
+      if (++st.slot == R) { st.slot = 0; st.par ^= 1u; }
+    }
+    mma_commit(S.g_done);
+  }
+  st.apar ^= 1u;
+  if (cons) {
+    const bool good = mbar_wait(S.g_done, st.gpar, p.err, 44);
+    tc_fence_after();
+    const uint32_t tm = tmem_base_after_wait(S.tmem_slot);
+    const int quad = warp & 3, row = quad * 32 + lane;
+    const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
+    // each segment's tile goes through shared memory (T[token][row], over the activation
+    // tiles, which the finished MMAs no longer read) so that the adds into L2 are 16-byte
+    // reds along the output features
+    float* T = reinterpret_cast<float*>(S.X);
+    int seg = -1, pnb = -1;
+    for (int i = 0; i < nt; ++i) {
+      const int nb = (t0 + i) / KT;
+      if (nb == pnb) continue;
+      ++seg;
+      pnb = nb;
+#pragma unroll
+      for (int q = 0; q < kMaxRows; q += 32) {
+        float v[32];
+        __syncwarp();
+        tmem_ld32(tm + lane_base + seg * 64 + q, v);
+#pragma unroll
+        for (int e = 0; e < 32; ++e) T[(q + e) * 128 + row] = v[e];
+      }
+      named_sync(2, 128);
+      if (good) {
+        float* dst = acc + nb * 128;
+        for (int idx = threadIdx.x; idx < M * 32; idx += 128) {
+          const int m = idx >> 5, c4 = idx & 31;
+          red_add_v4(dst + (size_t)m * N + 4 * c4, *reinterpret_cast<const float4*>(T + m * 128 + 4 * c4));
+        }
+      }
+      named_sync(2, 128);
+    }
+  }
+  st.gpar ^= 1u;
+}
+
+// ---- attention step: items (robot-group bg, 128-row query tile qt, 64-key chunk kc) ---------
+template <int DH>
+__device__ __noinline__ void attention_step(const StepArgs& p, const CUtensorMap* t_q, const CUtensorMap* t_k,
+                                            const CUtensorMap* t_vt, int l, uint32_t tmem, Role& st) {
+  constexpr int NC = DH / 64;
+  constexpr uint32_t QB = DH * kQT * 2, KB = DH * kKC * 2, VB = DH * kKC * 2;
+  const Smem S = smem_plan(p.ring, step_x_bytes(DH));
+  uint8_t* sQ = S.X;
+  uint8_t* sK = sQ + QB;
+  uint8_t* sV = sK + KB;
+  uint8_t* sP = sV + VB;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const bool mma = threadIdx.x == 160, cons = warp < 4;
+  const int nck = p.n_chunks, nqt = p.r_pad / kQT;
+  const int items = p.B * p.n_kv_heads * nqt * nck;
+  for (int it = blockIdx.x; it < items; it += gridDim.x) {
+    const int kc = it % nck, qt = (it / nck) % nqt, bg = it / (nck * nqt);
+    const int b = bg / p.n_kv_heads, g = bg % p.n_kv_heads;
+    const int kvz = (b * p.L + l) * p.n_kv_heads + g;
+    if (mma) {
+      const uint64_t pol = policy_evict_last();
+      mbar_expect_tx(S.q_full, QB + KB);
+#pragma unroll
+      for (int cc = 0; cc < NC; ++cc) {
+        tma_3d(sQ + cc * (kQT * 128), t_q, cc * 64, qt * kQT, bg, S.q_full, pol);
+        tma_3d(sK + cc * (kKC * 128), t_k, cc * 64, kc * kKC, kvz, S.q_full, pol);
+      }
+      mbar_expect_tx(S.v_full, VB);
+      tma_3d(sV, t_vt, kc * kKC, 0, kvz, S.v_full, pol);
+      ++st.i_uses;
+      bool good = mbar_wait(S.q_full, st.ipar, p.err, 45);
+      if (good) {
+        tc_fence_after();
+        const uint32_t q0 = su32(sQ), k0 = su32(sK);
+#pragma unroll
+        for (int cc = 0; cc < NC; ++cc)
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            mma_bf16(tmem, sw128_desc(q0 + cc * (kQT * 128) + 32 * k), sw128_desc(k0 + cc * (kKC * 128) + 32 * k),
+                     idesc_m128(kKC), (cc | k) ? 1u : 0u);
+      }
+      mma_commit(S.s_full);
+      good = good && mbar_wait(S.p_full, st.ipar, p.err, 46) && mbar_wait(S.v_full, st.ipar, p.err, 47);
+      if (good) {
+        tc_fence_after();
+        const uint32_t p0 = su32(sP), v0 = su32(sV);
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          mma_bf16(tmem + 256, sw128_desc(p0 + 32 * k), sw128_desc(v0 + 32 * k), idesc_m128(DH), k ? 1u : 0u);
+      }
+      mma_commit(S.o_done);
+    }
+    if (cons) {
+      // softmax over the chunk's 64 keys, one query row per thread
+      const bool ok_s = mbar_wait(S.s_full, st.ipar, p.err, 48);
+      tc_fence_after();
+      const uint32_t tS = tmem_base_after_wait(S.tmem_slot);
+      const int quad = warp & 3, row = quad * 32 + lane;
+      const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
+      const int key0 = kc * kKC;
+      const int nvalid = p.n_keys - key0 < kKC ? p.n_keys - key0 : kKC;
+      float sv[64];
+      __syncwarp();
+      tmem_ld32(tS + lane_base, sv);
+      tmem_ld32(tS + lane_base + 32, sv + 32);
+      float mx = -INFINITY;
+#pragma unroll
+      for (int i = 0; i < 64; ++i)
+        if (i < nvalid) mx = fmaxf(mx, sv[i]);
+      const float mxs = mx * p.scale_log2;
+      float l_sum = 0.f;
+      const int r8 = row & 7;
+      uint8_t* prow = sP + row * 128;
+#pragma unroll
+      for (int gi = 0; gi < 8; ++gi) {
+        uint32_t pk[4];
+#pragma unroll
+        for (int e = 0; e < 8; e += 2) {
+          const int i0 = gi * 8 + e;
+          const float e0 = i0 < nvalid ? exp2f(fmaf(sv[i0], p.scale_log2, -mxs)) : 0.f;
+          const float e1 = i0 + 1 < nvalid ? exp2f(fmaf(sv[i0 + 1], p.scale_log2, -mxs)) : 0.f;
+          const __nv_bfloat162 h = __floats2bfloat162_rn(e0, e1);
+          l_sum += __low2float(h) + __high2float(h);   // normalise by what the MMA sums
+          pk[e / 2] = *reinterpret_cast<const uint32_t*>(&h);
+        }
+        *reinterpret_cast<uint4*>(prow + ((gi ^ r8) * 16)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(S.p_full);
+      const bool ok_o = mbar_wait(S.o_done, st.ipar, p.err, 49);
+      tc_fence_after();
+      const uint32_t tO = tmem_base_after_wait(S.tmem_slot) + 256;
+      // unnormalised O row: staged in shared memory (the operand tiles are free once O is
+      // complete; rows padded by 16 bytes against bank conflicts), then each warp writes its
+      // 32 rows with coalesced 16-byte stores
+      const int qrow = qt * kQT + row;
+      const size_t pi = ((size_t)bg * nck + kc) * p.r_pad + qrow;
+      constexpr uint32_t pitch = DH * 4 + 16;
+      uint8_t* srow = S.X + (size_t)row * pitch;
+#pragma unroll
+      for (int q = 0; q < DH; q += 32) {
+        float ov[32];
+        __syncwarp();
+        tmem_ld32(tO + lane_base + q, ov);
+#pragma unroll
+        for (int e = 0; e < 32; e += 4)
+          *reinterpret_cast<float4*>(srow + (q + e) * 4) = make_float4(ov[e], ov[e + 1], ov[e + 2], ov[e + 3]);
+      }
+      __syncwarp();
+      if (ok_s && ok_o) {
+        const int r0 = qt * kQT + quad * 32;
+        const int nrows = p.rows - r0 < 32 ? p.rows - r0 : 32;
+        float4* dst0 = reinterpret_cast<float4*>(p.part_o + (((size_t)bg * nck + kc) * p.r_pad + r0) * DH);
+        for (int idx = lane; idx < nrows * (DH / 4); idx += 32) {
+          const int rr = idx / (DH / 4), ch = idx % (DH / 4);
+          dst0[(size_t)rr * (DH / 4) + ch] =
+              *reinterpret_cast<const float4*>(S.X + (size_t)(quad * 32 + rr) * pitch + ch * 16);
+        }
+        if (qrow < p.rows) {
+          p.part_ml[pi * 2] = mx;
+          p.part_ml[pi * 2 + 1] = l_sum;
+        }
+      }
+    }
+    st.ipar ^= 1u;
+    // the next item's operand loads overwrite this item's operands and P
+    tc_fence_before();
+    __syncwarp();
+    named_sync(1, 160);
+    tc_fence_after();
+  }
+}
+
+// Final norm and action-out projection of row m: v[m] = W_out y[m] + b_out.
+__device__ __noinline__ void final_row(const StepArgs& p, int m, const float* mod, size_t xbytes) {
+  const Smem S = smem_plan(p.ring, xbytes);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float* ys = reinterpret_cast<float*>(S.X);
+  const int W6 = 6 * p.W, fb = p.L * W6;
+  row_norm(p, m, mod, p.acc_d, fb - W6 + 5 * p.W, fb, fb + p.W, false, S.red, ys);
+  named_sync(2, 128);
+  const __nv_bfloat16* wo = static_cast<const __nv_bfloat16*>(p.w_out);
+  for (int d = warp; d < p.D; d += 4) {
+    float a = 0.f;
+    for (int k = 2 * lane; k < p.W; k += 64) {
+      const float2 wv = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(wo + (size_t)d * p.W + k));
+      a = fmaf(ys[k], wv.x, fmaf(ys[k + 1], wv.y, a));
+    }
+    a = warp_sum(a);
+    if (lane == 0) p.v[(size_t)m * p.D + d] = a + p.b_out[d];
+  }
+}
+
+template <int DH>
+__global__ void __launch_bounds__(kThreads, 1)
+    step_kernel(const __grid_constant__ CUtensorMap t_y, const __grid_constant__ CUtensorMap t_o,
+                const __grid_constant__ CUtensorMap t_act, const __grid_constant__ CUtensorMap t_q,
+                const __grid_constant__ CUtensorMap t_k, const __grid_constant__ CUtensorMap t_vt,
+                const __grid_constant__ StepArgs p) {
+  constexpr size_t XB = step_x_bytes(DH);
+  const int R = p.ring;
+  const Smem S = smem_plan(R, XB);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < R; ++i) {
+      mbar_init(S.full + i, 1);
+      mbar_init(S.empty + i, 1);
+    }
+    for (int i = 0; i < 8; ++i) mbar_init(S.a_full + i, i == 5 ? 4 : 1);   // p_full: one arrive per consumer warp
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(S.tmem_slot)), "r"(kTmemCols));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *S.tmem_slot;
+
+  if (warp == 4) {
+    // ---- weight producer: this CTA's tiles of every projection, in consumption order ----
+    if (lane == 0) {
+      const uint64_t pol = policy_evict_first();
+      int slot = 0, issued = 0;
+      uint32_t par = 0;
+      bool ok = true;
+      for (int l = 0; l < p.L && ok; ++l)
+        for (int j = 0; j < 4 && ok; ++j) {
+          int N, K, t0, t1;
+          proj_shape(p, j, N, K);
+          tile_range((N / 128) * (K / 64), 4 * l + j, t0, t1);
+          const uint8_t* w = static_cast<const uint8_t*>(p.wl[4 * l + j]);
+          for (int t = t0; t < t1; ++t) {
+            if (!mbar_wait(S.empty + slot, par ^ 1u, p.err, 41)) { ok = false; break; }
+            mbar_expect_tx(S.full + slot, kSlot);
+            bulk_g2s(S.ring + (size_t)slot * kSlot, w + (size_t)t * kSlot, kSlot, S.full + slot, pol);
+            ++issued;
+            if (++slot == R) { slot = 0; par ^= 1u; }
+          }
+        }
+      // copies still in flight land before the CTA exits
+      for (int i = issued - R > 0 ? issued - R : 0; i < issued; ++i) mbar_drain(S.full + i % R, (uint32_t)(i / R) & 1u);
+    }
+    __syncwarp();
+  } else {
+    // ---- warps 0-3: consumers; warp 5: tcgen05 issuer (thread 160) ----
+    const bool mma = threadIdx.x == 160, cons = warp < 4;
+    const int c = blockIdx.x, M = p.M, W = p.W, W6 = 6 * W;
+    Role st;
+    bool ok = true;
+    unsigned* bar = p.bars;
+    // modulation row of this CTA's token (fixed for the whole evaluation)
+    const float* mod = cons && c < M ? p.tab + (size_t)p.tau_row[c] * p.rowlen : p.tab;
+    for (int l = 0; l < p.L; ++l) {
+      const int b6 = l * W6;
+      // norm1 (layer 0: the action-in projection first)
+      if (ok && cons && c < M)
+        row_norm(p, c, mod, l > 0 ? p.acc_d : nullptr, l > 0 ? b6 - W6 + 5 * W : -1, b6, b6 + W, l == 0, S.red,
+                 nullptr);
+      ok = grid_sync(bar++, ok, p.err, S);
+      if (ok) projection_step(p, &t_y, p.acc_qkv, l, 0, tmem, XB, st);
+      ok = grid_sync(bar++, ok, p.err, S);
+      if (ok && cons) ew_rope(p, l);
+      ok = grid_sync(bar++, ok, p.err, S);
+      if (ok) attention_step<DH>(p, &t_q, &t_k, &t_vt, l, tmem, st);
+      ok = grid_sync(bar++, ok, p.err, S);
+      if (ok && cons) combine_rows<DH>(p);
+      ok = grid_sync(bar++, ok, p.err, S);
+      if (ok) projection_step(p, &t_o, p.acc_o, l, 1, tmem, XB, st);
+      ok = grid_sync(bar++, ok, p.err, S);
+      if (ok && cons && c < M)
+        row_norm(p, c, mod, p.acc_o, b6 + 2 * W, b6 + 3 * W, b6 + 4 * W, false, S.red, nullptr);
+      ok = grid_sync(bar++, ok, p.err, S);
+      if (ok) projection_step(p, &t_y, p.acc_gu, l, 2, tmem, XB, st);
+      ok = grid_sync(bar++, ok, p.err, S);
+      if (ok && cons) ew_act(p);
+      ok = grid_sync(bar++, ok, p.err, S);
+      if (ok) projection_step(p, &t_act, p.acc_d, l, 3, tmem, XB, st);
+      ok = grid_sync(bar++, ok, p.err, S);
+    }
+    if (ok && cons && c < M) final_row(p, c, mod, XB);
+    if (mma) {
+      // tensor memory is freed only after every MMA of this thread has completed, and the CTA
+      // exits only after its last operand loads have landed (they are waited for on the normal
+      // path; this matters only after an error)
+      mma_commit(S.fin);
+      mbar_drain(S.fin, 0);
+      if (st.a_uses) mbar_drain(S.a_full, (uint32_t)(st.a_uses - 1) & 1u);
+      if (st.i_uses) {
+        mbar_drain(S.q_full, (uint32_t)(st.i_uses - 1) & 1u);
+        mbar_drain(S.v_full, (uint32_t)(st.i_uses - 1) & 1u);
+      }
+    }
+    __syncwarp();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols));
+}
+
+size_t step_smem_bytes(int dh, int ring) { return 1024 + (size_t)ring * kSlot + step_x_bytes(dh) + kTailBytes; }
+
+int step_ring_slots(int dh, int smem_optin) {
+  const long long left = (long long)smem_optin - 1024 - (long long)step_x_bytes(dh) - (long long)kTailBytes;
+  long long r = left / kSlot;
+  if (r > kMaxRing) r = kMaxRing;
+  return (int)r;
+}
+
+int step_prepare(int dh, int ring, int* blocks_per_sm) {
+  const int smem = (int)step_smem_bytes(dh, ring);
+  cudaError_t e = cudaErrorInvalidValue;
+  *blocks_per_sm = 0;
+  if (dh == 64) {
+    e = cudaFuncSetAttribute(step_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, step_kernel<64>, kThreads, smem);
+  } else if (dh == 128) {
+    e = cudaFuncSetAttribute(step_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, step_kernel<128>, kThreads, smem);
+  } else if (dh == 256) {
+    e = cudaFuncSetAttribute(step_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, step_kernel<256>, kThreads, smem);
+  }
+  return e == cudaSuccess ? 0 : -1;
+}
+
+// One CTA per SM. The grid barriers need every CTA resident at once: the shared-memory plan
+// admits one CTA per SM (checked at set-up with the occupancy calculator) and the kernel is
+// launched after the previous kernel has drained, so all `grid` CTAs start together. The
+// launch is not marked cooperative: under a cooperative launch, warps other than the MMA
+// issuer read stale tensor memory for a short time after the commit-driven barrier completes.
+// Should the CTAs ever not all be resident, the bounded barrier wait reports an error
+// instead of hanging.
+int launch_step(const StepMaps& m, const StepArgs& a, int grid, cudaStream_t s) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = step_smem_bytes(a.dh, a.ring);
+  cfg.stream = s;
+  cfg.attrs = nullptr;
+  cfg.numAttrs = 0;
+  cudaError_t e = cudaErrorInvalidValue;
+  if (a.dh == 64) e = cudaLaunchKernelEx(&cfg, step_kernel<64>, m.y, m.o, m.act, m.q, m.k, m.vt, a);
+  if (a.dh == 128) e = cudaLaunchKernelEx(&cfg, step_kernel<128>, m.y, m.o, m.act, m.q, m.k, m.vt, a);
+  if (a.dh == 256) e = cudaLaunchKernelEx(&cfg, step_kernel<256>, m.y, m.o, m.act, m.q, m.k, m.vt, a);
+  return e == cudaSuccess ? 0 : -1;
+}
+
+}  // namespace uad

@@ -72,6 +72,13 @@ struct uad_ctx {
   int* tc_counters = nullptr;
   int* dev_err = nullptr;
   float* part = nullptr;          // K-split partial planes of the residual projections
+  // persistent evaluation kernel (adaRMS, bf16, B * H <= 64): one launch per step
+  bool step_ok = false;
+  bool step_off = false;          // UAD_STEP=0: per-operation kernels only
+  int step_bmax = 0;              // robots per launch
+  StepArgs st0;                   // shapes and buffers; M, B, tau_row set per launch
+  StepMaps smaps;
+  double step_bytes_w = 0, step_flops_w = 0;   // weight bytes / 2 x params per evaluation
 
   // weights (library layout)
   float *t_w1 = nullptr, *t_b1 = nullptr, *t_w2 = nullptr, *t_b2 = nullptr;  // t_w* are dtype
@@ -426,6 +433,88 @@ int make_tmap(uad_ctx* c, const void* base, int K, int rows) {
   return UAD_OK;
 }
 
+// The persistent evaluation kernel serves adaRMS experts with tensor-core attention when a
+// chunk has at most 64 tokens per launch and the work fits its shared-memory plan; otherwise
+// (and with UAD_STEP=0) every evaluation runs as per-operation kernels.
+const char* step_unfit(uad_ctx* c, int* ring) {
+  const uad_arch& a = c->a;
+  const int W = a.width, F = a.mlp_dim, dh = a.head_dim;
+  if (c->step_off) return "switched off";
+  if (!c->attn_tc || a.kind != UAD_KIND_ADARMS) return "not an adaRMS expert with tensor-core attention";
+  if (a.chunk_len > kStepMaxRows) return "chunk longer than 64 tokens";
+  if (W % 512 || W > kStepMaxWidth) return "width";
+  if (a.action_dim % 8) return "action dim";
+  if (dh != 64 && dh != 128 && dh != 256) return "head dim";
+  if ((c->at0.n_keys + 63) / 64 > kStepMaxChunks) return "too many keys";
+  const int shapes[4][2] = {{c->qkvd, W}, {W, c->qd}, {2 * F, W}, {W, F}};
+  for (auto& sh : shapes) {
+    if (sh[0] % 128 || sh[1] % 64) return "projection shape";
+    const int T = sh[0] / 128 * (sh[1] / 64);
+    if ((T + c->sms - 1) / c->sms > kStepMaxATiles) return "projection too large";
+  }
+  for (const LayerW& w : c->L)
+    if (!w.wqkv.tiled || !w.wo.tiled || !w.wgu.tiled || !w.wd.tiled) return "untiled weights";
+  int optin = 0;
+  cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, c->dev);
+  *ring = step_ring_slots(dh, optin);
+  if (*ring < 3) return "shared memory";
+  // exactly one CTA per SM, all resident together (the grid barriers rely on it)
+  int per_sm = 0;
+  if (step_prepare(dh, *ring, &per_sm) || per_sm != 1) return "occupancy";
+  return nullptr;
+}
+
+int step_setup(uad_ctx* c) {
+  const uad_arch& a = c->a;
+  int ring = 0;
+  if (step_unfit(c, &ring)) return UAD_OK;
+  const int H = a.chunk_len, W = a.width, F = a.mlp_dim, L = a.n_layers;
+  const AttnTcArgs& t = c->at0;
+  StepArgs& p = c->st0;
+  c->step_bmax = std::min(a.max_batch, kStepMaxRows / H);
+  p.H = H; p.W = W; p.F = F; p.D = a.action_dim; p.L = L;
+  p.qd = c->qd; p.kvd = c->kvd; p.qkvd = c->qkvd; p.n_heads = a.n_heads; p.n_kv_heads = a.n_kv_heads;
+  p.group = t.group; p.dh = a.head_dim; p.P = a.prefix_len; p.n_keys = t.n_keys; p.nk_pad = t.nk_pad;
+  p.rows = t.rows; p.r_pad = t.r_pad; p.n_chunks = (t.n_keys + 63) / 64;
+  p.ring = ring; p.rope = a.rope ? 1 : 0; p.scale_log2 = t.scale_log2;
+  p.tab = c->tab; p.rowlen = c->rowlen; p.u = c->u;
+  p.w_in = c->w_in; p.b_in = c->b_in; p.w_out = c->w_out; p.b_out = c->b_out; p.v = c->v; p.h = c->h;
+  p.y = static_cast<__nv_bfloat16*>(c->y); p.o = static_cast<__nv_bfloat16*>(c->o);
+  p.act = static_cast<__nv_bfloat16*>(c->act);
+  int rc;
+  const size_t R = kStepMaxRows;
+  if ((rc = dalloc_t(c, &p.acc_qkv, R * c->qkvd)) || (rc = dalloc_t(c, &p.acc_o, R * W)) ||
+      (rc = dalloc_t(c, &p.acc_gu, R * 2 * F)) || (rc = dalloc_t(c, &p.acc_d, R * W)))
+    return rc;
+  std::vector<const void*> wl;
+  for (const LayerW& w : c->L) wl.insert(wl.end(), {w.wqkv.w, w.wo.w, w.wgu.w, w.wd.w});
+  void* wd = nullptr;
+  if ((rc = dalloc(c, &wd, wl.size() * sizeof(void*)))) return rc;
+  if (cudaMemcpy(wd, wl.data(), wl.size() * sizeof(void*), cudaMemcpyHostToDevice) != cudaSuccess)
+    return fail(c, UAD_ECUDA, "weight table copy failed");
+  p.wl = static_cast<const void* const*>(wd);
+  p.q = t.q; p.kcache = t.kcache; p.vtcache = t.vtcache;
+  const size_t parts = (size_t)c->step_bmax * a.n_kv_heads * p.n_chunks * t.r_pad;
+  if ((rc = dalloc_t(c, &p.part_o, parts * a.head_dim)) || (rc = dalloc_t(c, &p.part_ml, parts * 2))) return rc;
+  p.rope_cs = c->rope_cs;
+  if ((rc = dalloc_t(c, &p.bars, (size_t)L * kStepBarriersPerLayer))) return rc;
+  p.err = c->dev_err;
+  c->smaps.y = c->tmaps.at(c->y);
+  c->smaps.o = c->tmaps.at(c->o);
+  c->smaps.act = c->tmaps.at(c->act);
+  c->smaps.q = c->atmaps.q;
+  c->smaps.k = c->atmaps.k2;
+  c->smaps.vt = c->atmaps.vt;
+  double params = (double)W * a.action_dim * 2;
+  params += (double)L * ((double)c->qkvd * W + (double)W * c->qd + 2.0 * F * W + (double)W * F);
+  c->step_bytes_w = 2.0 * params;
+  c->step_flops_w = 2.0 * params;
+  c->step_ok = true;
+  return UAD_OK;
+}
+
+bool step_path(const uad_ctx* c, int B) { return c->step_ok && B <= c->step_bmax; }
+
 // Enqueue every kernel of one chunk (begin + n_steps evaluations) for B robots.
 void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
   const uad_arch& a = c->a;
@@ -438,116 +527,138 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
   const bool dit = a.kind == UAD_KIND_DIT;
 
   { Mark mk(c, s, "begin", 12.0 * M * D, 0); launch_begin(c->noise, c->x, c->g, c->u, M * D, c->nonfinite, c->evals, c->stamps, s); }
+  const bool step = step_path(c, B);
+  if (step) {
+    // the persistent kernel's accumulators are zero between uses; clearing them per chunk keeps
+    // a chunk that ended in an error from leaking into the next one
+    const StepArgs& p = c->st0;
+    const size_t R = kStepMaxRows;
+    cudaMemsetAsync(p.acc_qkv, 0, R * c->qkvd * 4, s);
+    cudaMemsetAsync(p.acc_o, 0, R * W * 4, s);
+    cudaMemsetAsync(p.acc_gu, 0, R * 2 * F * 4, s);
+    cudaMemsetAsync(p.acc_d, 0, R * W * 4, s);
+  }
   PendingResid pend;
   for (int k = 1; k <= n_steps; ++k) {
     const int* tr = tau + (size_t)(k - 1) * M;
-    GemmArgs gi;
-    gi.A = c->u; gi.lda = D; gi.a_dtype = F32; gi.w_dtype = dt;
-    gi.M = M; gi.N = W; gi.K = D; gi.epi = EPI_STORE; gi.out = c->h; gi.ldo = W; gi.bias = c->b_in;
-    if (dit) { gi.add_rows = c->pos_code; gi.add_mod = H; }
-    { Mark mk(c, s, "in_proj", gemm_bytes(gi, c->es), 2.0 * M * W * D); gemm(c, c->w_in, gi, s); }
-    for (int l = 0; l < a.n_layers; ++l) {
-      const LayerW& w = c->L[l];
-      const int base = l * W6;
-      NormArgs na;
-      na.h = c->h; na.ldh = W; na.M = M; na.W = W; na.layer_norm = dit; na.tab = c->tab;
-      na.stride = c->rowlen; na.tau_row = tr; na.out = c->y; na.ldo = W; na.out_dtype = dt;
-      na.scale_off = dit ? base + W : base;
-      na.shift_off = dit ? base : base + W;
-      norm_after(c, na, &pend, s);
-      GemmArgs gq;
-      gq.A = c->y; gq.lda = W; gq.a_dtype = dt; gq.w_dtype = dt;
-      gq.M = M; gq.N = c->qkvd; gq.K = W; gq.out = c->qkv; gq.ldo = c->qkvd; gq.out_dtype = dt;
-      if (c->attn_tc) {
-        QkvTcOut& o = gq.qkv;
-        gq.epi = EPI_QKV_TC;
-        o.q = c->at0.q; o.kcache = c->at0.kcache; o.vtcache = c->at0.vtcache;
-        o.rope = a.rope ? c->rope_cs : nullptr;
-        o.H = H; o.P = a.prefix_len; o.NK = c->at0.n_keys; o.NKp = c->at0.nk_pad; o.dh = a.head_dim;
-        o.G = a.n_heads / a.n_kv_heads; o.Hkv = a.n_kv_heads; o.L = a.n_layers; o.layer = l;
-        o.qd = c->qd; o.kvd = c->kvd;
-      }
-      { Mark mk(c, s, "qkv_proj", gemm_bytes(gq, c->es), 2.0 * M * gq.N * W); gemm(c, w.wqkv, gq, s); }
-      AttnArgs at;
-      at.n_heads = a.n_heads; at.n_kv_heads = a.n_kv_heads; at.head_dim = a.head_dim; at.H = H; at.B = B;
-      at.q = c->qkv; at.q_ld = c->qkvd;
-      at.kc = static_cast<const char*>(c->qkv) + (size_t)c->qd * c->es;
-      at.vc = static_cast<const char*>(c->qkv) + (size_t)(c->qd + c->kvd) * c->es;
-      at.kc_ld = c->qkvd;
-      at.out = c->o; at.out_ld = c->qd; at.dtype = dt; at.scale = 1.f / std::sqrt((float)a.head_dim);
-      if (!dit) {
-        at.kp = static_cast<const char*>(c->kpre) + (size_t)l * a.prefix_len * c->kvd * c->es;
-        at.vp = static_cast<const char*>(c->vpre) + (size_t)l * a.prefix_len * c->kvd * c->es;
-        at.P = a.prefix_len; at.kp_bstride = (long long)a.n_layers * a.prefix_len * c->kvd;
-        at.kp_ld = c->kvd; at.rope_cs = a.rope ? c->rope_cs : nullptr;
-      }
-      if (c->attn_tc) {
-        AttnTcArgs t = c->at0;
-        t.batch = B; t.layer = l;
-        const double keys = (double)t.n_keys;
-        const double by = 2.0 * ((double)B * t.n_keys * c->kvd * 2 + (double)M * 2 * c->qd);
-        Mark mk(c, s, "attention", by, 4.0 * M * a.n_heads * keys * a.head_dim);
-        launch_attn_tc(c->atmaps, t, s);
-      } else {
-        const double keys = (double)(at.P + H);
-        const double by = c->es * ((double)B * at.P * c->kvd * 2 + (double)M * (2 * c->qd + 2 * c->kvd));
-        Mark mk(c, s, dit ? "self_attn" : "attention", by, 4.0 * M * a.n_heads * keys * a.head_dim);
-        launch_attention(at, s);
-      }
-      GemmArgs go;
-      go.A = c->o; go.lda = c->qd; go.a_dtype = dt; go.w_dtype = dt;
-      go.M = M; go.N = W; go.K = c->qd; go.tau_row = tr;
-      resid_gemm(c, w.wo, go, base + 2 * W, nullptr, &pend, "o_proj", s);
-      if (dit) {
-        NormArgs nc = na;
-        nc.tab = nullptr;
-        norm_after(c, nc, &pend, s);
-        GemmArgs gc;
-        gc.A = c->y; gc.lda = W; gc.a_dtype = dt; gc.w_dtype = dt;
-        gc.M = M; gc.N = c->qd; gc.K = W; gc.out = c->qc; gc.ldo = c->qd; gc.out_dtype = dt;
-        { Mark mk(c, s, "q_cross_proj", gemm_bytes(gc, c->es), 2.0 * M * c->qd * W); gemm(c, w.wqc, gc, s); }
-        AttnArgs ac;
-        ac.n_heads = a.n_heads; ac.n_kv_heads = a.n_heads; ac.head_dim = a.head_dim; ac.H = H; ac.B = B;
-        ac.q = c->qc; ac.q_ld = c->qd;
-        ac.kp = static_cast<const char*>(c->kpre) + (size_t)l * a.prefix_len * c->qd * c->es;
-        ac.vp = static_cast<const char*>(c->vpre) + (size_t)l * a.prefix_len * c->qd * c->es;
-        ac.P = a.prefix_len; ac.kp_bstride = (long long)a.n_layers * a.prefix_len * c->qd; ac.kp_ld = c->qd;
-        ac.out = c->o; ac.out_ld = c->qd; ac.dtype = dt; ac.scale = at.scale;
-        {
-          const double by = c->es * ((double)B * ac.P * c->qd * 2 + 2.0 * M * c->qd);
-          Mark mk(c, s, "cross_attn", by, 4.0 * M * a.n_heads * (double)ac.P * a.head_dim);
-          launch_attention(ac, s);
+    if (step) {
+      StepArgs p = c->st0;
+      p.M = M; p.B = B; p.tau_row = tr;
+      cudaMemsetAsync(p.bars, 0, (size_t)a.n_layers * kStepBarriersPerLayer * 4, s);
+      const double kv = 2.0 * B * a.n_layers * a.n_kv_heads * (double)p.n_keys * a.head_dim * 2;
+      const double by = c->step_bytes_w + kv + 16.0 * a.n_layers * M * W + 8.0 * M * D;
+      const double fl = c->step_flops_w * M + 4.0 * M * a.n_heads * (double)p.n_keys * a.head_dim * a.n_layers;
+      Mark mk(c, s, "step_kernel", by, fl);
+      if (launch_step(c->smaps, p, c->sms, s)) fail(c, UAD_ECUDA, "step kernel launch failed");
+    } else {
+      GemmArgs gi;
+      gi.A = c->u; gi.lda = D; gi.a_dtype = F32; gi.w_dtype = dt;
+      gi.M = M; gi.N = W; gi.K = D; gi.epi = EPI_STORE; gi.out = c->h; gi.ldo = W; gi.bias = c->b_in;
+      if (dit) { gi.add_rows = c->pos_code; gi.add_mod = H; }
+      { Mark mk(c, s, "in_proj", gemm_bytes(gi, c->es), 2.0 * M * W * D); gemm(c, c->w_in, gi, s); }
+      for (int l = 0; l < a.n_layers; ++l) {
+        const LayerW& w = c->L[l];
+        const int base = l * W6;
+        NormArgs na;
+        na.h = c->h; na.ldh = W; na.M = M; na.W = W; na.layer_norm = dit; na.tab = c->tab;
+        na.stride = c->rowlen; na.tau_row = tr; na.out = c->y; na.ldo = W; na.out_dtype = dt;
+        na.scale_off = dit ? base + W : base;
+        na.shift_off = dit ? base : base + W;
+        norm_after(c, na, &pend, s);
+        GemmArgs gq;
+        gq.A = c->y; gq.lda = W; gq.a_dtype = dt; gq.w_dtype = dt;
+        gq.M = M; gq.N = c->qkvd; gq.K = W; gq.out = c->qkv; gq.ldo = c->qkvd; gq.out_dtype = dt;
+        if (c->attn_tc) {
+          QkvTcOut& o = gq.qkv;
+          gq.epi = EPI_QKV_TC;
+          o.q = c->at0.q; o.kcache = c->at0.kcache; o.vtcache = c->at0.vtcache;
+          o.rope = a.rope ? c->rope_cs : nullptr;
+          o.H = H; o.P = a.prefix_len; o.NK = c->at0.n_keys; o.NKp = c->at0.nk_pad; o.dh = a.head_dim;
+          o.G = a.n_heads / a.n_kv_heads; o.Hkv = a.n_kv_heads; o.L = a.n_layers; o.layer = l;
+          o.qd = c->qd; o.kvd = c->kvd;
         }
-        GemmArgs gco;
-        gco.A = c->o; gco.lda = c->qd; gco.a_dtype = dt; gco.w_dtype = dt;
-        gco.M = M; gco.N = W; gco.K = c->qd; gco.tau_row = tr;
-        resid_gemm(c, w.woc, gco, -1, nullptr, &pend, "o_cross_proj", s);
+        { Mark mk(c, s, "qkv_proj", gemm_bytes(gq, c->es), 2.0 * M * gq.N * W); gemm(c, w.wqkv, gq, s); }
+        AttnArgs at;
+        at.n_heads = a.n_heads; at.n_kv_heads = a.n_kv_heads; at.head_dim = a.head_dim; at.H = H; at.B = B;
+        at.q = c->qkv; at.q_ld = c->qkvd;
+        at.kc = static_cast<const char*>(c->qkv) + (size_t)c->qd * c->es;
+        at.vc = static_cast<const char*>(c->qkv) + (size_t)(c->qd + c->kvd) * c->es;
+        at.kc_ld = c->qkvd;
+        at.out = c->o; at.out_ld = c->qd; at.dtype = dt; at.scale = 1.f / std::sqrt((float)a.head_dim);
+        if (!dit) {
+          at.kp = static_cast<const char*>(c->kpre) + (size_t)l * a.prefix_len * c->kvd * c->es;
+          at.vp = static_cast<const char*>(c->vpre) + (size_t)l * a.prefix_len * c->kvd * c->es;
+          at.P = a.prefix_len; at.kp_bstride = (long long)a.n_layers * a.prefix_len * c->kvd;
+          at.kp_ld = c->kvd; at.rope_cs = a.rope ? c->rope_cs : nullptr;
+        }
+        if (c->attn_tc) {
+          AttnTcArgs t = c->at0;
+          t.batch = B; t.layer = l;
+          const double keys = (double)t.n_keys;
+          const double by = 2.0 * ((double)B * t.n_keys * c->kvd * 2 + (double)M * 2 * c->qd);
+          Mark mk(c, s, "attention", by, 4.0 * M * a.n_heads * keys * a.head_dim);
+          launch_attn_tc(c->atmaps, t, s);
+        } else {
+          const double keys = (double)(at.P + H);
+          const double by = c->es * ((double)B * at.P * c->kvd * 2 + (double)M * (2 * c->qd + 2 * c->kvd));
+          Mark mk(c, s, dit ? "self_attn" : "attention", by, 4.0 * M * a.n_heads * keys * a.head_dim);
+          launch_attention(at, s);
+        }
+        GemmArgs go;
+        go.A = c->o; go.lda = c->qd; go.a_dtype = dt; go.w_dtype = dt;
+        go.M = M; go.N = W; go.K = c->qd; go.tau_row = tr;
+        resid_gemm(c, w.wo, go, base + 2 * W, nullptr, &pend, "o_proj", s);
+        if (dit) {
+          NormArgs nc = na;
+          nc.tab = nullptr;
+          norm_after(c, nc, &pend, s);
+          GemmArgs gc;
+          gc.A = c->y; gc.lda = W; gc.a_dtype = dt; gc.w_dtype = dt;
+          gc.M = M; gc.N = c->qd; gc.K = W; gc.out = c->qc; gc.ldo = c->qd; gc.out_dtype = dt;
+          { Mark mk(c, s, "q_cross_proj", gemm_bytes(gc, c->es), 2.0 * M * c->qd * W); gemm(c, w.wqc, gc, s); }
+          AttnArgs ac;
+          ac.n_heads = a.n_heads; ac.n_kv_heads = a.n_heads; ac.head_dim = a.head_dim; ac.H = H; ac.B = B;
+          ac.q = c->qc; ac.q_ld = c->qd;
+          ac.kp = static_cast<const char*>(c->kpre) + (size_t)l * a.prefix_len * c->qd * c->es;
+          ac.vp = static_cast<const char*>(c->vpre) + (size_t)l * a.prefix_len * c->qd * c->es;
+          ac.P = a.prefix_len; ac.kp_bstride = (long long)a.n_layers * a.prefix_len * c->qd; ac.kp_ld = c->qd;
+          ac.out = c->o; ac.out_ld = c->qd; ac.dtype = dt; ac.scale = at.scale;
+          {
+            const double by = c->es * ((double)B * ac.P * c->qd * 2 + 2.0 * M * c->qd);
+            Mark mk(c, s, "cross_attn", by, 4.0 * M * a.n_heads * (double)ac.P * a.head_dim);
+            launch_attention(ac, s);
+          }
+          GemmArgs gco;
+          gco.A = c->o; gco.lda = c->qd; gco.a_dtype = dt; gco.w_dtype = dt;
+          gco.M = M; gco.N = W; gco.K = c->qd; gco.tau_row = tr;
+          resid_gemm(c, w.woc, gco, -1, nullptr, &pend, "o_cross_proj", s);
+        }
+        NormArgs n2 = na;
+        n2.scale_off = dit ? base + 4 * W : base + 3 * W;
+        n2.shift_off = dit ? base + 3 * W : base + 4 * W;
+        norm_after(c, n2, &pend, s);
+        GemmArgs g1;
+        g1.A = c->y; g1.lda = W; g1.a_dtype = dt; g1.w_dtype = dt; g1.M = M; g1.K = W;
+        g1.out = c->act; g1.ldo = F; g1.out_dtype = dt;
+        if (dit) { g1.N = F; g1.epi = EPI_BIAS_GELU; g1.bias = w.b1; }
+        else { g1.N = 2 * F; g1.epi = EPI_GEGLU; }
+        { Mark mk(c, s, dit ? "mlp_up" : "gate_up_proj", gemm_bytes(g1, c->es), 2.0 * M * g1.N * W); gemm(c, dit ? w.w1 : w.wgu, g1, s); }
+        GemmArgs g2;
+        g2.A = c->act; g2.lda = F; g2.a_dtype = dt; g2.w_dtype = dt;
+        g2.M = M; g2.N = W; g2.K = F; g2.tau_row = tr;
+        resid_gemm(c, dit ? w.w2 : w.wd, g2, base + 5 * W, dit ? w.b2 : nullptr, &pend, dit ? "mlp_down" : "down_proj", s);
       }
-      NormArgs n2 = na;
-      n2.scale_off = dit ? base + 4 * W : base + 3 * W;
-      n2.shift_off = dit ? base + 3 * W : base + 4 * W;
-      norm_after(c, n2, &pend, s);
-      GemmArgs g1;
-      g1.A = c->y; g1.lda = W; g1.a_dtype = dt; g1.w_dtype = dt; g1.M = M; g1.K = W;
-      g1.out = c->act; g1.ldo = F; g1.out_dtype = dt;
-      if (dit) { g1.N = F; g1.epi = EPI_BIAS_GELU; g1.bias = w.b1; }
-      else { g1.N = 2 * F; g1.epi = EPI_GEGLU; }
-      { Mark mk(c, s, dit ? "mlp_up" : "gate_up_proj", gemm_bytes(g1, c->es), 2.0 * M * g1.N * W); gemm(c, dit ? w.w1 : w.wgu, g1, s); }
-      GemmArgs g2;
-      g2.A = c->act; g2.lda = F; g2.a_dtype = dt; g2.w_dtype = dt;
-      g2.M = M; g2.N = W; g2.K = F; g2.tau_row = tr;
-      resid_gemm(c, dit ? w.w2 : w.wd, g2, base + 5 * W, dit ? w.b2 : nullptr, &pend, dit ? "mlp_down" : "down_proj", s);
+      NormArgs nf;
+      nf.h = c->h; nf.ldh = W; nf.M = M; nf.W = W; nf.layer_norm = dit; nf.tab = c->tab;
+      nf.stride = c->rowlen; nf.tau_row = tr; nf.out = c->y; nf.ldo = W; nf.out_dtype = dt;
+      nf.scale_off = a.n_layers * W6 + (dit ? W : 0);
+      nf.shift_off = a.n_layers * W6 + (dit ? 0 : W);
+      norm_after(c, nf, &pend, s);
+      GemmArgs go;
+      go.A = c->y; go.lda = W; go.a_dtype = dt; go.w_dtype = dt;
+      go.M = M; go.N = D; go.K = W; go.out = c->v; go.ldo = D; go.bias = c->b_out;
+      { Mark mk(c, s, "out_proj", gemm_bytes(go, c->es), 2.0 * M * W * D); gemm(c, c->w_out, go, s); }
     }
-    NormArgs nf;
-    nf.h = c->h; nf.ldh = W; nf.M = M; nf.W = W; nf.layer_norm = dit; nf.tab = c->tab;
-    nf.stride = c->rowlen; nf.tau_row = tr; nf.out = c->y; nf.ldo = W; nf.out_dtype = dt;
-    nf.scale_off = a.n_layers * W6 + (dit ? W : 0);
-    nf.shift_off = a.n_layers * W6 + (dit ? 0 : W);
-    norm_after(c, nf, &pend, s);
-    GemmArgs go;
-    go.A = c->y; go.lda = W; go.a_dtype = dt; go.w_dtype = dt;
-    go.M = M; go.N = D; go.K = W; go.out = c->v; go.ldo = D; go.bias = c->b_out;
-    { Mark mk(c, s, "out_proj", gemm_bytes(go, c->es), 2.0 * M * W * D); gemm(c, c->w_out, go, s); }
     EulerArgs ea;
     ea.B = B; ea.H = H; ea.D = D; ea.k = k;
     ea.plan = plan + (size_t)(k - 1) * M;
@@ -565,8 +676,10 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
   }
 }
 
-int launches_per_step(const uad_arch& a, bool attn_tc) {
-  return a.kind == UAD_KIND_DIT ? 11 * a.n_layers + 4 : (attn_tc ? 8 : 7) * a.n_layers + 4;
+int launches_per_step(const uad_ctx* c, int B) {
+  const uad_arch& a = c->a;
+  if (step_path(c, B)) return 2;   // persistent evaluation kernel + Euler step
+  return a.kind == UAD_KIND_DIT ? 11 * a.n_layers + 4 : (c->attn_tc ? 8 : 7) * a.n_layers + 4;
 }
 
 }  // namespace
@@ -620,6 +733,8 @@ int uad_init(const uad_arch* arch, const float* weights, size_t n_floats, uad_ct
     if (e && e[0] == '0') c->use_graphs = false;
     e = getenv("UAD_GEMM");
     if (e && !strcmp(e, "simt")) c->force_simt = true;
+    e = getenv("UAD_STEP");
+    if (e && e[0] == '0') c->step_off = true;
   }
   int rc = UAD_OK;
 #define TRY(x)                        \
@@ -813,6 +928,7 @@ int uad_init(const uad_arch* arch, const float* weights, size_t n_floats, uad_ct
     TRY(dalloc_t(c, &c->part, part));
     gemm_tc_prepare();
   }
+  TRY(step_setup(c));
   TRY(dalloc_t(c, &c->E, (size_t)a.max_batch * D));
   TRY(dalloc_t(c, &c->nonfinite, 1));
   TRY(dalloc_t(c, &c->evals, 1));
@@ -1027,7 +1143,7 @@ static int denoise_impl(uad_ctx* c, const float* noise, const uad_schedule* sc, 
     c->prof_next = 0;
     // create the events before capture
     {
-      int need = 2 * (1 + steps * launches_per_step(c->a, c->attn_tc)) + 8;
+      int need = 2 * (1 + steps * launches_per_step(c, B)) + 8;
       while ((int)c->prof_ev.size() < need) {
         cudaEvent_t e;
         CK(cudaEventCreate(&e));
@@ -1178,7 +1294,7 @@ int uad_step_times(const uad_ctx* c, double* ms, int32_t max_entries) {
 
 int uad_launches_per_chunk(const uad_ctx* c, int32_t batch, int32_t n_star) {
   if (!c || batch < 1 || n_star < 1) return UAD_EINVAL;
-  return 1 + n_star * launches_per_step(c->a, c->attn_tc);
+  return 1 + n_star * launches_per_step(c, batch);
 }
 
 void uad_destroy(uad_ctx* c) {

@@ -193,4 +193,42 @@ int attn_tc_rpad(int rows);
 void launch_attn_tc(const AttnTcMaps& maps, const AttnTcArgs& a, cudaStream_t s);   // 2 kernels
 void launch_kv_prefix(const void* k, const void* v, int src_dtype, const AttnTcArgs& a, int robot, cudaStream_t s);
 
+// ---- persistent evaluation kernel (adaRMS experts, bf16, few tokens) ----------------------
+constexpr int kStepMaxRows = 64;      // B * H tokens per evaluation
+constexpr int kStepMaxATiles = 8;     // weight tiles per CTA and projection
+constexpr int kStepMaxRing = 12;      // weight ring slots of 16 KB
+constexpr int kStepMaxChunks = 32;    // 64-key chunks per (robot, KV head)
+constexpr int kStepBarriersPerLayer = 10;
+constexpr int kStepMaxWidth = 2048;   // model width, a multiple of 512
+struct StepArgs {
+  int M = 0, B = 0, H = 0, W = 0, F = 0, D = 0, L = 0;
+  int qd = 0, kvd = 0, qkvd = 0, n_heads = 0, n_kv_heads = 0, group = 0, dh = 0;
+  int P = 0, n_keys = 0, nk_pad = 0, rows = 0, r_pad = 0, n_chunks = 0;
+  int ring = 0;                        // weight ring slots
+  int rope = 0;                        // q/k rows pair-interleaved per head, rotated by rope_cs
+  float scale_log2 = 0.f;              // log2(e) / sqrt(dh)
+  const int* tau_row = nullptr;        // [M] modulation row of each token at this step
+  const float* tab = nullptr; int rowlen = 0;
+  const float* u = nullptr;            // [M][D] model input
+  const void* w_in = nullptr; const float* b_in = nullptr;     // bf16 [W][D]
+  const void* w_out = nullptr; const float* b_out = nullptr;   // bf16 [D][W]
+  float* v = nullptr;                  // [M][D] velocity
+  float* h = nullptr;                  // [M][W] residual stream
+  __nv_bfloat16* y = nullptr;          // [M][W] normalised rows
+  __nv_bfloat16* o = nullptr;          // [M][qd] attention output
+  __nv_bfloat16* act = nullptr;        // [M][F] MLP activation
+  float *acc_qkv = nullptr, *acc_o = nullptr, *acc_gu = nullptr, *acc_d = nullptr;  // zero between uses
+  const void* const* wl = nullptr;     // [L][4] tiled weights: qkv, o, gate/up, down
+  __nv_bfloat16 *q = nullptr, *kcache = nullptr, *vtcache = nullptr;   // tensor-core attention layouts
+  float *part_o = nullptr, *part_ml = nullptr;   // [B*Hkv][n_chunks][r_pad][dh], [..][2]
+  const float* rope_cs = nullptr;      // [H][dh/2][cos, sin]
+  unsigned* bars = nullptr;            // [L * kStepBarriersPerLayer] grid-barrier counters, zeroed per launch
+  int* err = nullptr;
+};
+struct StepMaps { CUtensorMap y, o, act, q, k, vt; };   // k: 64-key boxes
+size_t step_smem_bytes(int dh, int ring);
+int step_ring_slots(int dh, int smem_optin);           // ring slots that fit (may be < 3: unusable)
+int step_prepare(int dh, int ring, int* blocks_per_sm); // 0 on success
+int launch_step(const StepMaps& m, const StepArgs& a, int grid, cudaStream_t s);   // grid = SMs
+
 }  // namespace uad

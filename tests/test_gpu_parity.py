@@ -294,6 +294,45 @@ def test_tensor_core_gemm_matches_cuda_core_gemm(monkeypatch):
         assert rel_err(outs[1][k], outs[0][k].astype(np.float64)) <= 5e-3, k
 
 
+def test_step_kernel_matches_per_operation_kernels(monkeypatch):
+    """The persistent evaluation kernel (one launch per step, B * H <= 64) against
+    the per-operation kernels on the same bf16 operands, and both against the oracle."""
+    a = ARCHS["pi0_small"]
+    blob = make_weights(a, seed=12)
+    noise = make_noise(a, seed=12)
+    bud = group_budgets(a.chunk_len, [(0, 9, 3), (10, 29, 5), (30, a.chunk_len - 1, 8)])
+    outs, launches = [], []
+    for mode in ("0", "1"):
+        monkeypatch.setenv("UAD_STEP", mode)
+        c = Case(a, seed=12, blob=blob)
+        try:
+            launches.append(c.ex.launches_per_chunk(1, 8))
+            outs.append(c.gpu(noise, bud))
+            if mode == "1":
+                check(c, outs[-1], c.oracle(noise, bud), bud, TOL["bf16"])
+        finally:
+            c.close()
+    assert launches[1] == 1 + 2 * 8 < launches[0]
+    for k in ("final", "ghost"):
+        assert rel_err(outs[1][k], outs[0][k].astype(np.float64)) <= 5e-3, k
+    assert np.array_equal(outs[1]["polled"][0][1], outs[0]["polled"][0][1])
+
+
+def test_step_kernel_batched_robots():
+    """Four robots of 16 tokens (64 rows, the largest persistent-kernel launch), each with its
+    own prefix and schedule."""
+    a = ARCHS["pi0_small"].replace(name="pi0_small_h16", chunk_len=16)
+    B = 4
+    c = Case(a, B=B, seed=13)
+    try:
+        assert c.ex.launches_per_chunk(B, 10) == 1 + 2 * 10
+        noise = make_noise(a, batch=B, seed=13)
+        bud = draw_sweep_schedules(a.chunk_len, B, seed=13)
+        check(c, c.gpu(noise, bud), c.oracle(noise, bud), bud, TOL["bf16"])
+    finally:
+        c.close()
+
+
 def test_pi0_full_batched_16_robots_sampled():
     """16 robots (M = 800 tokens: wide 128 x 256 projection tiles), each with its own prefix and
     a schedule from the sweep grid; robots 0, 7 and 15 are checked against the oracle."""
