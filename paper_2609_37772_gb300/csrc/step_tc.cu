@@ -198,9 +198,25 @@ __device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
 }
+// Hardware approximations (MUFU): 2^x and tanh. Both feed values that are rounded to bf16
+// next (P for the P V product, the MLP activation), far coarser than their error.
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ float tanh_approx(float x) {
+  float y;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 __device__ __forceinline__ float gelu_tanh(float x) {
   const float k0 = 0.7978845608028654f;
-  return 0.5f * x * (1.f + tanhf(k0 * (x + 0.044715f * x * x * x)));
+  return 0.5f * x * (1.f + tanh_approx(k0 * (x + 0.044715f * x * x * x)));
+}
+__device__ __forceinline__ void bulk_s2g(void* gdst, const void* ssrc, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(gdst), "r"(su32(ssrc)), "r"(bytes)
+               : "memory");
 }
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
   __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
@@ -221,7 +237,7 @@ __host__ __device__ constexpr size_t step_x_bytes(int dh) {
 constexpr size_t kTailBytes = 512;   // mbarriers (<= 2 * 12 + 8), TMEM slot, flag, scratch
 
 // Projection j of a layer: 0 = qkv, 1 = o, 2 = gate/up, 3 = down.
-__device__ __forceinline__ void proj_shape(const StepArgs& p, int j, int& N, int& K) {
+__device__ __forceinline__ void proj_shape(const StepArgs& __restrict__ p, int j, int& N, int& K) {
   switch (j) {
     case 0: N = p.qkvd; K = p.W; break;
     case 1: N = p.W; K = p.qd; break;
@@ -338,7 +354,7 @@ constexpr int kMaxV4 = kStepMaxWidth / 512;   // float4 per consumer thread
 // gate(tau) * acc[m] (gate 1 when gate_off < 0) and acc[m] is cleared; with `in_proj`,
 // h[m] = W_in u[m] + b_in. Returns the normalised row in `ys` (fp32 of the bf16 values) when
 // ys is not null. Every load of the row (and of its modulation vectors) is issued up front.
-__device__ __noinline__ void row_norm(const StepArgs& p, int m, const float* mod, float* acc, int gate_off,
+__device__ __noinline__ void row_norm(const StepArgs& __restrict__ p, int m, const float* mod, float* acc, int gate_off,
                                       int scale_off, int shift_off, bool in_proj, float* red, float* ys) {
   const int tid = threadIdx.x, W = p.W, nv = W / 512;
   float4* h4 = reinterpret_cast<float4*>(p.h + (size_t)m * W);
@@ -446,7 +462,7 @@ constexpr int kEwBatch = 4;   // work items per thread and batch
 
 // q, k (RoPE) and v of every token into the attention layouts; acc_qkv cleared. Item = one
 // (token, q/k row pair) or one (token, v row).
-__device__ __noinline__ void ew_rope(const StepArgs& p, int l) {
+__device__ __noinline__ void ew_rope(const StepArgs& __restrict__ p, int l) {
   const int dh = p.dh, half = dh / 2, npairs = (p.qd + p.kvd) / 2, per = npairs + p.kvd;
   const int total = p.M * per, T = 128 * gridDim.x;
   for (int base = blockIdx.x * 128 + threadIdx.x; base < total; base += kEwBatch * T) {
@@ -498,7 +514,7 @@ __device__ __noinline__ void ew_rope(const StepArgs& p, int l) {
 
 // act[m][j] = gelu_tanh(acc_gu[m][2j]) * acc_gu[m][2j+1] for every token; acc_gu cleared.
 // Item = one float4 of acc_gu (two outputs).
-__device__ __noinline__ void ew_act(const StepArgs& p) {
+__device__ __noinline__ void ew_act(const StepArgs& __restrict__ p) {
   const int per = p.F / 2, total = p.M * per, T = 128 * gridDim.x;
   float4* acc = reinterpret_cast<float4*>(p.acc_gu);
   uint32_t* out = reinterpret_cast<uint32_t*>(p.act);
@@ -522,7 +538,7 @@ __device__ __noinline__ void ew_act(const StepArgs& p) {
 
 // Merge the key chunks of the query rows assigned to this consumer warp.
 template <int DH>
-__device__ __noinline__ void combine_rows(const StepArgs& p) {
+__device__ __noinline__ void combine_rows(const StepArgs& __restrict__ p) {
   constexpr int E = DH / 32;
   const int lane = threadIdx.x & 31;
   const int gw = blockIdx.x * 4 + (threadIdx.x >> 5), nw = gridDim.x * 4;
@@ -573,7 +589,7 @@ __device__ __noinline__ void combine_rows(const StepArgs& p) {
 // Thread 160 loads the activation tiles (tensor map) and issues the MMAs against the weight
 // ring; the consumer warps add each finished 128 x 64 tile into `acc` (fp32, L2) with 16-byte
 // reds.
-__device__ __noinline__ void projection_step(const StepArgs& p, const CUtensorMap* amap, float* acc, int l, int j,
+__device__ __noinline__ void projection_step(const StepArgs& __restrict__ p, const CUtensorMap* amap, float* acc, int l, int j,
                                              uint32_t tmem, size_t xbytes, Role& st) {
   const Smem S = smem_plan(p.ring, xbytes);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, R = p.ring, M = p.M;
@@ -648,7 +664,7 @@ __device__ __noinline__ void projection_step(const StepArgs& p, const CUtensorMa
 
 // ---- attention step: items (robot-group bg, 128-row query tile qt, 64-key chunk kc) ---------
 template <int DH>
-__device__ __noinline__ void attention_step(const StepArgs& p, const CUtensorMap* t_q, const CUtensorMap* t_k,
+__device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, const CUtensorMap* t_q, const CUtensorMap* t_k,
                                             const CUtensorMap* t_vt, int l, uint32_t tmem, Role& st) {
   constexpr int NC = DH / 64;
   constexpr uint32_t QB = DH * kQT * 2, KB = DH * kKC * 2, VB = DH * kKC * 2;
@@ -725,8 +741,8 @@ __device__ __noinline__ void attention_step(const StepArgs& p, const CUtensorMap
 #pragma unroll
         for (int e = 0; e < 8; e += 2) {
           const int i0 = gi * 8 + e;
-          const float e0 = i0 < nvalid ? exp2f(fmaf(sv[i0], p.scale_log2, -mxs)) : 0.f;
-          const float e1 = i0 + 1 < nvalid ? exp2f(fmaf(sv[i0 + 1], p.scale_log2, -mxs)) : 0.f;
+          const float e0 = i0 < nvalid ? ex2_approx(fmaf(sv[i0], p.scale_log2, -mxs)) : 0.f;
+          const float e1 = i0 + 1 < nvalid ? ex2_approx(fmaf(sv[i0 + 1], p.scale_log2, -mxs)) : 0.f;
           const __nv_bfloat162 h = __floats2bfloat162_rn(e0, e1);
           l_sum += __low2float(h) + __high2float(h);   // normalise by what the MMA sums
           pk[e / 2] = *reinterpret_cast<const uint32_t*>(&h);
@@ -741,8 +757,8 @@ __device__ __noinline__ void attention_step(const StepArgs& p, const CUtensorMap
       tc_fence_after();
       const uint32_t tO = tmem_base_after_wait(S.tmem_slot) + 256;
       // unnormalised O row: staged in shared memory (the operand tiles are free once O is
-      // complete; rows padded by 16 bytes against bank conflicts), then each warp writes its
-      // 32 rows with coalesced 16-byte stores
+      // complete; rows padded by 16 bytes against bank conflicts), then written by one bulk copy
+      // per row, complete before the step's barrier
       const int qrow = qt * kQT + row;
       const size_t pi = ((size_t)bg * nck + kc) * p.r_pad + qrow;
       constexpr uint32_t pitch = DH * 4 + 16;
@@ -756,20 +772,14 @@ __device__ __noinline__ void attention_step(const StepArgs& p, const CUtensorMap
         for (int e = 0; e < 32; e += 4)
           *reinterpret_cast<float4*>(srow + (q + e) * 4) = make_float4(ov[e], ov[e + 1], ov[e + 2], ov[e + 3]);
       }
-      __syncwarp();
-      if (ok_s && ok_o) {
-        const int r0 = qt * kQT + quad * 32;
-        const int nrows = p.rows - r0 < 32 ? p.rows - r0 : 32;
-        float4* dst0 = reinterpret_cast<float4*>(p.part_o + (((size_t)bg * nck + kc) * p.r_pad + r0) * DH);
-        for (int idx = lane; idx < nrows * (DH / 4); idx += 32) {
-          const int rr = idx / (DH / 4), ch = idx % (DH / 4);
-          dst0[(size_t)rr * (DH / 4) + ch] =
-              *reinterpret_cast<const float4*>(S.X + (size_t)(quad * 32 + rr) * pitch + ch * 16);
-        }
-        if (qrow < p.rows) {
-          p.part_ml[pi * 2] = mx;
-          p.part_ml[pi * 2 + 1] = l_sum;
-        }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      if (ok_s && ok_o && qrow < p.rows) {
+        bulk_s2g(p.part_o + pi * DH, srow, DH * 4);
+        asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+        p.part_ml[pi * 2] = mx;
+        p.part_ml[pi * 2 + 1] = l_sum;
+        asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+        asm volatile("fence.proxy.async.global;" ::: "memory");
       }
     }
     st.ipar ^= 1u;
@@ -782,7 +792,7 @@ __device__ __noinline__ void attention_step(const StepArgs& p, const CUtensorMap
 }
 
 // Final norm and action-out projection of row m: v[m] = W_out y[m] + b_out.
-__device__ __noinline__ void final_row(const StepArgs& p, int m, const float* mod, size_t xbytes) {
+__device__ __noinline__ void final_row(const StepArgs& __restrict__ p, int m, const float* mod, size_t xbytes) {
   const Smem S = smem_plan(p.ring, xbytes);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   float* ys = reinterpret_cast<float*>(S.X);
