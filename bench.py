@@ -83,6 +83,57 @@ def aal_ms(ready_ms, t_act, n_exec):
     return sum(waits) / n_exec
 
 
+def tail_blocking_ms(ready_ms, t_act, u):
+    """Wait of the first tail action (index u) under the same clock: how long execution blocks
+    once the u released actions have been executed (the quantity the U selection bounds)."""
+    request, start = 0.0, 0.0
+    for i, r in enumerate(ready_ms[:u + 1]):
+        if i > 0:
+            request = start + t_act
+        start = max(request, r)
+    return max(0.0, ready_ms[u] - request)
+
+
+def rel_l2(x, ref):
+    """||x - ref||_2 / ||ref||_2 over every element of the set."""
+    x, ref = np.asarray(x, np.float64), np.asarray(ref, np.float64)
+    n = np.linalg.norm(ref)
+    return float(np.linalg.norm(x - ref) / n) if n > 0 else float(np.linalg.norm(x - ref))
+
+
+# Variants of the diagnostic (Sec. 4.3, Fig. 3): early release alone, with Trajectory
+# Reconciliation, and with Ghost Action Correction on top.
+DIAG_VARIANTS = {"uaer": dict(tr=False, gac=False), "uaer+tr": dict(tr=True, gac=False),
+                 "uaer+tr+gac": dict(tr=True, gac=True)}
+
+
+def diagnostic_errors(final, ghost, vanilla, budgets, tr=True):
+    """Relative L2 error to vanilla inference (same noise, all tokens at N*) of the released
+    actions (N_i < N*), of their ghost actions (TR only) and of the tail (N_i = N*); arrays
+    [H, D]. Fig. 3 of the paper plots these three per setting."""
+    b = np.asarray(budgets)
+    early = b < b.max()
+    out = {}
+    if early.any():
+        out["released"] = rel_l2(np.asarray(final)[early], np.asarray(vanilla)[early])
+        if tr:
+            out["ghost"] = rel_l2(np.asarray(ghost)[early], np.asarray(vanilla)[early])
+    if (~early).any():
+        out["tail"] = rel_l2(np.asarray(final)[~early], np.asarray(vanilla)[~early])
+    return out
+
+
+def bootstrap_ci(values, reps=8000, seed=0):
+    """95% interval of the mean by resampling the units with replacement (2.5th / 97.5th
+    percentiles of the bootstrap distribution, 8,000 replicates)."""
+    v = np.asarray(values, np.float64)
+    if v.size < 2:
+        return [float(v.mean()), float(v.mean())] if v.size else [None, None]
+    idx = np.random.default_rng(seed).integers(0, v.size, size=(reps, v.size))
+    means = v[idx].mean(axis=1)
+    return [float(np.percentile(means, 2.5)), float(np.percentile(means, 97.5))]
+
+
 class Clocks:
     """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
     Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -254,7 +305,8 @@ def run_ours(args, wl, world, rank, local):
     # device-side release times of robot 0 (global timer, relative to the chunk's first kernel)
     st = np.array(step_times)                      # [K][N*]
     ready = [[float(st[c][int(bud[0][i]) - 1]) for i in range(H)] for c in range(len(st))]
-    aal = statistics.mean(aal_ms(r, wl["t_act_ms"], H) for r in ready)
+    aal_chunks = [aal_ms(r, wl["t_act_ms"], H) for r in ready]
+    aal = statistics.mean(aal_chunks)
     first = statistics.mean(r[0] for r in ready)
     ms_per_eval = statistics.mean(float(s[-1]) / n_star for s in st)
 
@@ -285,7 +337,8 @@ def run_ours(args, wl, world, rank, local):
     barrier(world)
     t_e2e = max_over_ranks(t_e2e, world)
     e2e_value = world * B * H * args.steps / t_e2e
-    aal_host = statistics.mean(aal_ms(r, wl["t_act_ms"], H) for r in host_ready)
+    aal_host_chunks = [aal_ms(r, wl["t_act_ms"], H) for r in host_ready]
+    aal_host = statistics.mean(aal_host_chunks)
     al = lambda x: (x + 15) & ~15                 # the library's plan block, uploaded per chunk
     o = al(n_star * B * H * 8)
     o = al(o + n_star * B * H * 4)
@@ -340,10 +393,13 @@ def run_ours(args, wl, world, rank, local):
         "config": {"workload": wl["desc"], "model": a.name, "global_batch": B * world, "seq_len": H,
                    "parallelism": f"replicas x{world}" if world > 1 else "none",
                    "l2": "no flush: every evaluation streams the full weight set, larger than L2"},
-        "aal_ms": aal, "first_action_ms": first, "ms_per_eval": ms_per_eval,
-        "aal_definition": "device release times, T_act = %g ms, S = H" % wl["t_act_ms"],
+        "aal_ms": aal, "aal_ci95_ms": bootstrap_ci(aal_chunks), "first_action_ms": first,
+        "ms_per_eval": ms_per_eval,
+        "aal_definition": "device release times, T_act = %g ms, S = H; 95%% CI: bootstrap over the timed "
+                          "chunks (8000 replicates)" % wl["t_act_ms"],
         "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
                 "d2h_bytes_per_step": int(d2h), "aal_ms_host": aal_host,
+                "aal_ci95_ms_host": bootstrap_ci(aal_host_chunks),
                 "first_action_ms_host": statistics.mean(r[0] for r in host_ready)},
         "roofline": roofline, "kernels": kernels, "gpu_launches": launches,
         "clocks": clk.summary(), "cpu_baseline": cpu,
@@ -383,6 +439,88 @@ def run_sweep(args):
                           "first_action_ms": statistics.mean(r[0] for r in rows),
                           "aal_ms_10ms_S50": statistics.mean(aal_ms(r, 10.0, 50) for r in rows),
                           "aal_ms_10ms_S10": statistics.mean(aal_ms(r, 10.0, 10) for r in rows)}), flush=True)
+
+    def chunk_rows(bud):
+        for _ in range(args.warmup):
+            ex.denoise(noise, bud, stream=stream)
+            ex.finish(timeout_us=60_000_000)
+        rows, ms = [], []
+        for _ in range(args.steps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            ex.denoise(noise, bud, stream=stream)
+            ex.finish(timeout_us=60_000_000)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            ms.append(e0.elapsed_time(e1))
+            st = ex.step_times()
+            rows.append([float(st[int(bud[0][i]) - 1]) for i in range(a.chunk_len)])
+        return rows, ms
+
+    # U selection at K = 1 (App. C.1): tokens 0..U-1 released after one step, the rest at N* = 10;
+    # S = 10 executed actions; tail blocking = wait of the first tail action under the clock, for
+    # the two control rates of the paper's benchmarks (80 Hz and 20 Hz).
+    S, tacts = 10, (12.5, 50.0)
+    blocking = {t: [] for t in tacts}
+    for u in range(1, S):
+        bud = group_budgets(a.chunk_len, [(0, u - 1, 1), (u, 49, 10)])[None]
+        rows, _ = chunk_rows(bud)
+        line = {"sweep": "u_select K=1 N*=10 S=10", "U": u}
+        for t in tacts:
+            b = statistics.mean(tail_blocking_ms(r, t, u) for r in rows)
+            blocking[t].append(b)
+            line[f"tail_blocking_ms_tact{t:g}"] = b
+            line[f"aal_ms_tact{t:g}"] = statistics.mean(aal_ms(r, t, S) for r in rows)
+        print(json.dumps(line), flush=True)
+    print(json.dumps({"sweep": "u_select K=1 N*=10 S=10", "rule": "smallest U with tail blocking < 0.2 ms",
+                      **{f"selected_U_tact{t:g}": next((u for u, b in zip(range(1, S), blocking[t]) if b < 0.2), None)
+                         for t in tacts}}), flush=True)
+
+    # latency against the uniform step count N = 1..10 (App. B): chunk time grows linearly in N
+    ns, chunk_ms = list(range(1, 11)), []
+    for n in ns:
+        bud = np.full((1, a.chunk_len), n, np.int32)
+        rows, ms = chunk_rows(bud)
+        chunk_ms.append(statistics.mean(ms))
+        print(json.dumps({"sweep": "uniform N", "N": n, "ms_per_chunk": chunk_ms[-1],
+                          "first_action_ms": statistics.mean(r[0] for r in rows),
+                          "aal_ms_tact12.5_S10": statistics.mean(aal_ms(r, 12.5, S) for r in rows)}), flush=True)
+    slope, intercept = np.polyfit(np.array(ns, np.float64), np.array(chunk_ms), 1)
+    print(json.dumps({"sweep": "uniform N", "fit": "ms_per_chunk = intercept + slope * N",
+                      "slope_ms_per_eval": float(slope), "intercept_ms": float(intercept)}), flush=True)
+    ex.close()
+    return 0
+
+
+def run_diagnostic(args):
+    """Relative-L2 diagnostic of Trajectory Reconciliation (Fig. 3) on the CUDA path: the
+    workload's expert at B = 1, N* = 3, urgent groups of U in {5, 10, 20} tokens at K in {1, 2},
+    every variant, against vanilla N* = 3 inference from the same noise. One JSON line each."""
+    import paper_2609_37772_gb300 as uad
+    wl = WORKLOADS[args.workload]
+    a = ARCHS[wl["arch"]]
+    ex = uad.Expert(a, make_weights(a), max_batch=1)
+    if a.kind == "dit":
+        ex.set_prefix(0, make_prefix_tokens(a, robot=0))
+    else:
+        ex.set_prefix(0, *make_prefix_kv(a, robot=0))
+    ns, H = 3, a.chunk_len
+    for seed in range(args.diag_seeds):
+        noise = make_noise(a, 1, seed=100 + seed)
+        ex.denoise(noise, np.full((1, H), ns, np.int32))
+        van = ex.finish(timeout_us=60_000_000)["final"][0]
+        for k in (1, 2):
+            for u in (5, 10, 20):
+                if u >= H:
+                    continue
+                bud = group_budgets(H, [(0, u - 1, k), (u, H - 1, ns)])
+                for name, kw in DIAG_VARIANTS.items():
+                    ex.denoise(noise, bud[None], **kw)
+                    r = ex.finish(timeout_us=60_000_000)
+                    print(json.dumps({"diagnostic": "relative L2 to vanilla", "arch": a.name, "N*": ns, "K": k,
+                                      "U": u, "variant": name, "noise_seed": 100 + seed,
+                                      **diagnostic_errors(r["final"][0], r["ghost"][0], van, bud, kw["tr"])}),
+                          flush=True)
     ex.close()
     return 0
 
@@ -397,10 +535,16 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sweep", action="store_true",
-                    help="pi0-like B=1 schedule sweep: one JSON line per (first-group budget, size)")
+                    help="pi0-like B=1 schedule sweeps: first-group budget x size, U selection at K=1, "
+                         "latency against a uniform N")
+    ap.add_argument("--diagnostic", action="store_true",
+                    help="relative L2 error to vanilla inference per variant (Fig. 3), one JSON line each")
+    ap.add_argument("--diag-seeds", type=int, default=3)
     args = ap.parse_args()
     if args.sweep:
         return run_sweep(args)
+    if args.diagnostic:
+        return run_diagnostic(args)
     wl = WORKLOADS[args.workload]
     world, rank, local = dist_setup()
     try:

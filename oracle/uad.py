@@ -22,11 +22,12 @@ from __future__ import annotations
 
 import numpy as np
 
+from . import so3
 from .plan import early_tokens, executable_tail, n_star, step_plan
 
 
 def denoise(velocity, x0, budgets, n_exec=None, tr=True, gac=True, gac_mask=None,
-            chunk_relative=False):
+            chunk_relative=False, rot_dim=None):
     """Run one action chunk.
 
     velocity   callable (u [H, D], tau [H]) -> v [H, D]
@@ -35,6 +36,8 @@ def denoise(velocity, x0, budgets, n_exec=None, tr=True, gac=True, gac_mask=None
     n_exec     S, actions executed before replanning (default H)
     tr, gac    Trajectory Reconciliation / Ghost Action Correction on or off
     gac_mask   [D] bool, True for additive dimensions (default: all additive)
+    rot_dim    first of three dimensions holding a rotation vector, corrected by composition
+               on SO(3) (so3.py; never additive whatever gac_mask says); None: no rotation
 
     Returns a dict with
       final         [H, D]  actions as handed to the controller: released actions for early
@@ -44,7 +47,8 @@ def denoise(velocity, x0, budgets, n_exec=None, tr=True, gac=True, gac_mask=None
                             without TR there is no reconciled state (ghosts exist through
                             TR, Sec. 4.3), so early rows hold the frozen action fed back
       release_step  [H]     N_i for early tokens, N* for the others (when they are available)
-      E             [D]     Eq. 8 estimate (zeros when GAC does not run)
+      E             [D]     Eq. 8 estimate (zeros when GAC does not run); on the rotation
+                            dimensions the rotation vector of the accumulated error e_R
       evals         int     evaluations of the velocity network (N*)
       tail          list    indices that GAC corrected
     """
@@ -94,7 +98,12 @@ def denoise(velocity, x0, budgets, n_exec=None, tr=True, gac=True, gac_mask=None
         tail = executable_tail(budgets, S)
         if tail:
             E = np.sum(g[early] - released[early], axis=0)
-            mask = np.ones(D, dtype=bool) if gac_mask is None else np.asarray(gac_mask, dtype=bool)
+            mask = np.ones(D, dtype=bool) if gac_mask is None else np.asarray(gac_mask, dtype=bool).copy()
+            if rot_dim is not None:
+                rd = slice(rot_dim, rot_dim + 3)
+                mask[rd] = False
+                E[rd], final[tail, rd] = so3.gac_rotation(released[early][:, rd], g[early][:, rd],
+                                                          final[tail][:, rd])
             final[np.ix_(tail, np.nonzero(mask)[0])] += E[mask] / len(tail)
     return dict(final=final, released=released, ghost=ghost, release_step=release_step,
                 E=E, evals=evals, tail=tail, n_star=ns)

@@ -59,3 +59,29 @@ def test_bench_aal_matches_oracle_clock():
         t_act = float(rng.uniform(0.5, 20))
         S = int(rng.integers(1, H + 1))
         assert bench.aal_ms(ready, t_act, S) == pytest.approx(aal(ready, t_act, S), rel=1e-12, abs=1e-12)
+
+
+def test_tail_blocking_under_the_clock():
+    """First tail action (index U) waits max(0, ready_U - request_U), request_U = start of the
+    urgent actions' execution + U * T_act (App. C.1 latency model with one release group)."""
+    import bench
+    ready = [5.0, 5.0] + [30.0] * 8
+    assert bench.tail_blocking_ms(ready, 12.5, 2) == 0.0          # 5 + 2 * 12.5 = 30: just in time
+    assert bench.tail_blocking_ms(ready, 10.0, 2) == 5.0          # 5 + 2 * 10 = 25 < 30
+    assert bench.tail_blocking_ms([4.0] + [20.0] * 9, 10.0, 1) == 6.0
+    # the model's closed form: blocking = max((N* - K) T_D - U T_act, 0) with ready times K T_D, N* T_D
+    t_d, k, ns, t_act = 1.3, 1, 10, 2.0
+    for u in range(1, 9):
+        r = [k * t_d] * u + [ns * t_d] * (10 - u)
+        assert abs(bench.tail_blocking_ms(r, t_act, u) - max((ns - k) * t_d - u * t_act, 0.0)) < 1e-12
+
+
+def test_bootstrap_interval():
+    import bench
+    lo, hi = bench.bootstrap_ci([2.0] * 7)
+    assert lo == hi == 2.0
+    v = np.random.default_rng(3).normal(10.0, 1.0, 200)
+    lo, hi = bench.bootstrap_ci(v)
+    se = v.std(ddof=1) / np.sqrt(v.size)
+    assert lo < v.mean() < hi
+    assert abs((hi - lo) - 2 * 1.96 * se) < 0.25 * (2 * 1.96 * se)   # normal-theory width within 25%

@@ -378,3 +378,26 @@ def test_two_pass_attention_many_tiles():
             assert rel_err(res["ghost"][b], ref["ghost"]) <= TOL["bf16"]
     finally:
         ex.close()
+
+
+def test_relative_l2_diagnostic_matches_oracle(tiny):
+    """The Fig. 3 diagnostic (relative L2 error to vanilla inference of released, ghost and tail
+    actions, per variant) computed from the CUDA path equals the oracle's; with K = 1 and TR the
+    tail and ghost errors vanish on both (exact recovery)."""
+    import bench
+    a = tiny.a
+    noise = make_noise(a, seed=31)
+    van_g = tiny.gpu(noise, np.full(a.chunk_len, 3), poll=False)["final"][0]
+    van_o = tiny.oracle(noise, np.full(a.chunk_len, 3), gac=False)[0]["final"]
+    for k, u in ((1, 4), (2, 6)):
+        bud = group_budgets(a.chunk_len, [(0, u - 1, k), (u, a.chunk_len - 1, 3)])
+        for name, kw in bench.DIAG_VARIANTS.items():
+            rg = tiny.gpu(noise, bud, poll=False, **kw)
+            ro = tiny.oracle(noise, bud, **kw)[0]
+            eg = bench.diagnostic_errors(rg["final"][0], rg["ghost"][0], van_g, bud, kw["tr"])
+            eo = bench.diagnostic_errors(ro["final"], ro["ghost"], van_o, bud, kw["tr"])
+            assert eg.keys() == eo.keys()
+            for key in eg:
+                assert abs(eg[key] - eo[key]) <= 1e-4 * max(1.0, eo[key]), (k, u, name, key, eg[key], eo[key])
+            if k == 1 and name == "uaer+tr":
+                assert eg["tail"] == 0.0 and eg["ghost"] == 0.0
