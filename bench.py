@@ -342,7 +342,7 @@ def run_ours(args, wl, world, rank, local):
     al = lambda x: (x + 15) & ~15                 # the library's plan block, uploaded per chunk
     o = al(n_star * B * H * 8)
     o = al(o + n_star * B * H * 4)
-    for extra in (B * 4, B * 4, B * 4, B * H * 4, D, 4):
+    for extra in (B * 4, B * 4, B * 4, B * H * 4, D, 4, 4):
         o = al(o + extra)
     plan_bytes = o
     h2d = noise_np.nbytes + plan_bytes

@@ -76,6 +76,12 @@ typedef struct uad_schedule {
   int32_t chunk_relative;  /* actions relative to the chunk start: GAC is skipped (Sec. 4.4) */
   const uint8_t* gac_mask; /* host [action_dim], 1 = additive dimension corrected by Eq. 9,
                               0 = left unchanged (rotation / gripper); NULL = all additive */
+  int32_t rot_dim;         /* first of three dimensions holding a rotation vector (axis times
+                              angle, radians) that GAC corrects by composition on SO(3)
+                              (App. C.1): E_R = product over early actions, in token order, of
+                              R(ghost) R(released)^T; every tail action R <- exp(log(E_R)/|tail|) R.
+                              These dimensions are never additive; -1 = no rotation dimensions.
+                              Must be -1 or in 0..action_dim-3 (else UAD_EINVAL). */
 } uad_schedule;
 
 typedef struct uad_stats {

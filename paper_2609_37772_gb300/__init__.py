@@ -33,7 +33,8 @@ class uad_arch(C.Structure):
 
 class uad_schedule(C.Structure):
     _fields_ = [("budgets", C.POINTER(_I32)), ("batch", _I32), ("n_exec", _I32), ("tr", _I32),
-                ("gac", _I32), ("chunk_relative", _I32), ("gac_mask", C.POINTER(C.c_uint8))]
+                ("gac", _I32), ("chunk_relative", _I32), ("gac_mask", C.POINTER(C.c_uint8)),
+                ("rot_dim", _I32)]
 
 
 class uad_stats(C.Structure):
@@ -163,17 +164,19 @@ class Expert:
     def prepare_times(self, max_budget):
         return self._check(uad_prepare_times(self.h, max_budget), "prepare_times")
 
-    def _schedule(self, budgets, n_exec, tr, gac, chunk_relative, gac_mask):
+    def _schedule(self, budgets, n_exec, tr, gac, chunk_relative, gac_mask, rot_dim=None):
         b = np.ascontiguousarray(budgets, dtype=np.int32).reshape(-1, self.H)
         m = None if gac_mask is None else np.ascontiguousarray(gac_mask, dtype=np.uint8)
         sc = uad_schedule(budgets=b.ctypes.data_as(C.POINTER(_I32)), batch=b.shape[0], n_exec=n_exec,
                           tr=int(tr), gac=int(gac), chunk_relative=int(chunk_relative),
-                          gac_mask=None if m is None else m.ctypes.data_as(C.POINTER(C.c_uint8)))
+                          gac_mask=None if m is None else m.ctypes.data_as(C.POINTER(C.c_uint8)),
+                          rot_dim=-1 if rot_dim is None else int(rot_dim))
         return sc, (b, m)
 
     def denoise(self, noise, budgets, n_exec=0, tr=True, gac=True, chunk_relative=False,
-                gac_mask=None, n_star=0, stream=None):
-        sc, keep = self._schedule(budgets, n_exec, tr, gac, chunk_relative, gac_mask)
+                gac_mask=None, n_star=0, stream=None, rot_dim=None):
+        """rot_dim: first of three rotation-vector dimensions corrected on SO(3) (None: none)."""
+        sc, keep = self._schedule(budgets, n_exec, tr, gac, chunk_relative, gac_mask, rot_dim)
         if isinstance(noise, np.ndarray):
             noise = np.ascontiguousarray(noise, dtype=np.float32)
         self._keep = noise

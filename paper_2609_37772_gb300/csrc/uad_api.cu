@@ -279,7 +279,7 @@ std::pair<int, int> reduce(int num, int den) {
 
 // Plan block layout for a call with n_steps steps and B robots (16-byte aligned sections).
 struct PlanLayout {
-  size_t plan, tau, gstep, last, tailc, tailf, mask, epoch, total;
+  size_t plan, tau, gstep, last, tailc, tailf, mask, epoch, rot, total;
 };
 PlanLayout plan_layout(int n_steps, int B, int H, int D) {
   auto al = [](size_t x) { return (x + 15) & ~(size_t)15; };
@@ -294,6 +294,7 @@ PlanLayout plan_layout(int n_steps, int B, int H, int D) {
   L.tailf = o; o = al(o + M * 4);
   L.mask = o; o = al(o + D);
   L.epoch = o; o = al(o + 4);
+  L.rot = o; o = al(o + 4);
   L.total = o;
   return L;
 }
@@ -668,6 +669,7 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
     ea.tail_flag = reinterpret_cast<const int*>(c->plan_dev + PL.tailf);
     ea.gac_mask = c->plan_dev + PL.mask;
     ea.epoch = reinterpret_cast<const int*>(c->plan_dev + PL.epoch);
+    ea.rot_dim = reinterpret_cast<const int*>(c->plan_dev + PL.rot);
     ea.v = c->v; ea.x = c->x; ea.g = c->g; ea.u = c->u; ea.rel = c->rel;
     ea.final_out = c->fin; ea.ghost_out = c->ghost; ea.E_out = c->E;
     ea.host_rel = c->host_rel_dev; ea.host_flags = c->host_flags_dev;
@@ -1056,6 +1058,8 @@ static int denoise_impl(uad_ctx* c, const float* noise, const uad_schedule* sc, 
   const int S = sc->n_exec == 0 ? H : sc->n_exec;
   if (S < 1 || S > H) return fail(c, UAD_EINVAL, "n_exec %d not in 1..H", S);
   if (sc->gac && !sc->tr && !sc->chunk_relative) return fail(c, UAD_EINVAL, "GAC needs TR");
+  if (sc->rot_dim != -1 && (sc->rot_dim < 0 || sc->rot_dim > D - 3))
+    return fail(c, UAD_EINVAL, "rot_dim %d not -1 or in 0..%d", sc->rot_dim, D - 3);
   for (int b = 0; b < B; ++b)
     if (!c->has_prefix[b]) return fail(c, UAD_EINVAL, "robot %d has no prefix", b);
   std::vector<int> ns(B, 0);
@@ -1109,6 +1113,7 @@ static int denoise_impl(uad_ctx* c, const float* noise, const uad_schedule* sc, 
   for (int d = 0; d < D; ++d) mask[d] = sc->gac_mask ? (sc->gac_mask[d] ? 1 : 0) : 1;
   c->epoch = c->epoch % 1000000000 + 1;
   *reinterpret_cast<int*>(hp + PL.epoch) = c->epoch;
+  *reinterpret_cast<int*>(hp + PL.rot) = sc->rot_dim;
 
   cudaStream_t user = static_cast<cudaStream_t>(stream);
   cudaStream_t s = c->worker;

@@ -120,6 +120,7 @@ struct EulerArgs {
   float* host_rel = nullptr;         // mapped pinned [B][H][D]
   int* host_flags = nullptr;         // mapped pinned [B][UAD_MAX_STEPS + 1]
   const int* epoch = nullptr;        // device scalar
+  const int* rot_dim = nullptr;      // device scalar: first rotation-vector dimension, -1 none
   int* nonfinite = nullptr;
   int* evals = nullptr;                  // velocity evaluations consumed this chunk
   unsigned long long* stamps = nullptr;  // [UAD_MAX_STEPS + 1], [0] = start

@@ -401,3 +401,29 @@ def test_relative_l2_diagnostic_matches_oracle(tiny):
                 assert abs(eg[key] - eo[key]) <= 1e-4 * max(1.0, eo[key]), (k, u, name, key, eg[key], eo[key])
             if k == 1 and name == "uaer+tr":
                 assert eg["tail"] == 0.0 and eg["ghost"] == 0.0
+
+
+@pytest.mark.parametrize("bud_groups", [[(0, 3, 2), (4, 15, 6)], [(0, 0, 1), (1, 5, 3), (6, 15, 7)]])
+def test_gac_on_so3_matches_oracle(tiny, bud_groups):
+    """D = 7 actions: dimensions 0-2 additive, 3-5 a rotation vector corrected by composition
+    on SO(3) (App. C.1), 6 (gripper) masked; fp32 against the fp64 oracle."""
+    a = tiny.a
+    noise = make_noise(a, seed=41)
+    bud = group_budgets(a.chunk_len, bud_groups)
+    mask = np.array([1, 1, 1, 0, 0, 0, 0], np.uint8)
+    res = tiny.gpu(noise, bud, gac_mask=mask, rot_dim=3)
+    ref = tiny.oracle(noise, bud, gac_mask=mask.astype(bool), rot_dim=3)
+    check(tiny, res, ref, bud, TOL["f32"])
+    assert np.abs(res["E"][0] - ref[0]["E"]).max() <= 1e-4 * max(1.0, np.abs(ref[0]["E"]).max())
+    # the rotation dimensions moved, the gripper did not
+    plain = tiny.oracle(noise, bud, gac_mask=mask.astype(bool))[0]
+    tail = ref[0]["tail"]
+    assert np.abs(ref[0]["final"][tail][:, 3:6] - plain["final"][tail][:, 3:6]).max() > 1e-4
+    assert np.array_equal(res["final"][0][:, 6], tiny.gpu(noise, bud, gac_mask=mask, poll=False)["final"][0][:, 6])
+
+
+def test_rot_dim_is_validated(tiny):
+    a = tiny.a
+    bud = group_budgets(a.chunk_len, [(0, 3, 2), (4, a.chunk_len - 1, 4)])
+    with pytest.raises(uad.UADError):
+        tiny.ex.denoise(make_noise(a, seed=1), bud[None], rot_dim=a.action_dim - 2)
