@@ -1,32 +1,39 @@
 // Persistent evaluation kernel: one velocity evaluation v = F_theta(u, tau) of an adaRMS action
-// expert with few tokens (B * H <= 64) in a single launch, one CTA per SM.
+// expert with few tokens in a single launch, one CTA per SM.
 //
-// With few tokens an evaluation is a chain of about ten dependent steps per layer, each far
-// too small to fill the GPU; as separate kernels every step pays launch, drain and
-// weight-fetch latency. Here every CTA runs every step of every layer, and grid-wide barriers
-// (bounded spins on global counters) separate the steps. One producer thread per CTA streams
-// this CTA's share of every projection weight (and nothing else) through a shared-memory ring
-// without waiting for the barriers: the weights do not depend on the activations, so HBM
-// streams ahead across steps and layers while the consumers wait for their inputs.
+// With few tokens an evaluation is a chain of dependent steps per layer, each far too small to
+// fill the GPU; its cost is the latency of that chain, not the weight bytes. The kernel keeps the
+// chain short: six grid barriers per layer, every elementwise step fused into the epilogue of the
+// projection that produces its input. One producer thread per CTA streams this CTA's share of
+// every projection weight through a shared-memory ring without waiting for the barriers (the
+// weights do not depend on the activations).
 //
-// Steps of layer l, each followed by a grid barrier:
-//   norm1    row m (CTA m): h += gate2'(tau) * acc_d (l > 0; h = W_in u + b_in at l = 0),
-//            y = RMSNorm(h) * (1 + scale) + shift                                 (bf16)
-//   qkv      weight tiles [v T / G, (v+1) T / G) of W_qkv: acc_qkv += y W^T    (red.add, fp32)
-//   rope     row m: RoPE on q and k, q -> Q, k -> K cache, v -> Vt cache         (bf16)
+// Factored adaptive RMSNorm. With y = RMSNorm(h) (1 + scale) + shift (per-token modulation of
+// the token's flow time), a projection of y splits as
+//     y W^T = rstd(h) * ((h (1 + scale)) W^T) + shift W^T,
+// so the producer of h writes z = h (1 + scale) (bf16) without waiting for the row norm, and the
+// shift vectors of the step's distinct flow times ride along as extra rows of z (rows M..M+S-1).
+// The consumer of the projection applies rstd (from row sums of squares accumulated by the
+// producers of h) and adds the shift row of the token's flow time.
+//
+// Phases (each ends at a grid barrier; the last CTA to finish an output block of a projection,
+// counted per block, runs that block's epilogue):
+//   in       row m: h = W_in u + b_in, sum h^2, z = h (1 + scale1); shift rows of layer 0
+//   qkv      acc += z W_qkv^T;  block epilogue: rstd * acc + shift row, RoPE, q -> Q, k -> K
+//            cache, v -> Vt cache
 //   attn     items (robot-group, 128 query rows, 64 keys): S = Q K^T, P = exp(S - max),
 //            O = P V on tcgen05 -> partial O rows and (max, sum)
-//   combine  query rows: log-sum-exp merge of the key chunks -> o               (bf16)
-//   o        acc_o += o W_o^T
-//   norm2    row m: h += gate1(tau) * acc_o, y = adaRMS2(h)
-//   gate_up  acc_gu += y W_gu^T  (rows interleaved gate_j, up_j)
-//   act      row m: act = gelu_tanh(gate) * up                                   (bf16)
-//   down     acc_d += act W_d^T
-// then the final norm and the action-out projection v = W_out y + b_out (row m). Every
-// accumulator row is cleared by the CTA that consumes it, so the next use starts from zero.
+//   combine  query rows: log-sum-exp merge of the key chunks -> o (bf16)
+//   o        acc += o W_o^T;  block epilogue: h += gate1 * acc, sum h^2, z = h (1 + scale2),
+//            shift rows of norm 2
+//   gate_up  acc += z W_gu^T;  block epilogue: rstd * acc + shift row, act = gelu_tanh(gate) up
+//   down     acc += act W_d^T;  block epilogue: h += gate2 * acc, sum h^2, z for the next
+//            layer's norm 1
+// then the final norm and the action-out projection v = W_out y + b_out (row m). The epilogue
+// that reads an accumulator block clears it, so the next use starts from zero.
 //
-// Warps: 0-3 = consumers (TMEM lane quadrants 0-3; row steps), 4 = weight producer (lane 0),
-// 5 = tcgen05 issuer and TMA loads of activations and attention operands (lane 0).
+// Warps: 0-3 = consumers (TMEM lane quadrants 0-3; epilogues and row steps), 4 = weight producer
+// (lane 0), 5 = tcgen05 issuer and TMA loads of activations and attention operands (lane 0).
 // Every wait is bounded: on timeout the kernel records an error code, skips the remaining
 // work, waits (bounded) for its copies in flight and frees its tensor memory.
 #include <cuda.h>
@@ -223,18 +230,33 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
+__device__ __forceinline__ void cp16(void* s, const void* g) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(su32(s)), "l"(g) : "memory");
+}
+__device__ __forceinline__ void cp_wait_all() {
+  asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;" ::: "memory");
+}
+__device__ __forceinline__ void st_bf16x4(__nv_bfloat16* dst, float a, float b, float c, float d) {
+  uint2 pk;
+  pk.x = pack_bf16(a, b);
+  pk.y = pack_bf16(c, d);
+  *reinterpret_cast<uint2*>(dst) = pk;
+}
+
 // Shared-memory plan (1024-aligned base): [weight ring: ring x 16 KB][work area X][mbarriers,
-// TMEM slot, flags, reduction scratch]. X holds, by step, the activation tiles of a projection
-// (up to kMaxATiles x 8 KB), the attention operands Q | K | Vt | P, the staged partial O rows,
-// or the final normalised row.
+// TMEM slot, flags, reduction scratch]. X holds, by step, the activation tiles of a projection,
+// the staged accumulator tile and the operands of its block epilogue, the attention operands
+// Q | K | Vt | P and the staged partial O rows, or the partial rows of a combine.
+constexpr size_t kEpiBytes = (size_t)kMaxRows * 512 * 2 + (size_t)3 * kStepMaxShift * 512;
 __host__ __device__ constexpr size_t step_x_bytes(int dh) {
   const size_t a = (size_t)kMaxATiles * kATile;
   const size_t att = (size_t)dh * kQT * 2 + 2 * (size_t)dh * kKC * 2 + (size_t)kQT * kKC * 2;
   const size_t ost = (size_t)kQT * (dh * 4 + 16);
-  const size_t m = a > att ? a : att;
-  return m > ost ? m : ost;
+  size_t m = a > att ? a : att;
+  m = m > ost ? m : ost;
+  return m > kEpiBytes ? m : kEpiBytes;
 }
-constexpr size_t kTailBytes = 512;   // mbarriers (<= 2 * 12 + 8), TMEM slot, flag, scratch
+constexpr size_t kTailBytes = 512;   // mbarriers (<= 2 * 12 + 8), TMEM slot, flags, scratch
 
 // Projection j of a layer: 0 = qkv, 1 = o, 2 = gate/up, 3 = down.
 __device__ __forceinline__ void proj_shape(const StepArgs& __restrict__ p, int j, int& N, int& K) {
@@ -245,14 +267,28 @@ __device__ __forceinline__ void proj_shape(const StepArgs& __restrict__ p, int j
     default: N = p.W; K = p.F; break;
   }
 }
-// Tile range of this CTA in a projection of T tiles. The split is rotated from projection to
-// projection so that the CTAs that take one tile more change every time.
-__device__ __forceinline__ void tile_range(int T, int proj, int& t0, int& t1) {
-  const int G = gridDim.x;
-  const int v = (int)((blockIdx.x + 41u * (unsigned)proj) % (unsigned)G);
-  t0 = (int)((long long)v * T / G);
-  t1 = (int)((long long)(v + 1) * T / G);
+
+// Tiles of this CTA in a projection of NB output blocks x KT k-blocks: the CTAs are split into
+// NB contiguous groups (rotated from projection to projection), group b shares block b's KT
+// k-blocks. Every CTA's tiles lie in one output block, so each CTA adds one accumulator tile.
+struct Tiles {
+  int b, k0, k1, contrib;   // output block, k-block range, CTAs that add into block b
+  int idx;                  // this CTA's index among them (its share of the block's epilogue)
+};
+__host__ __device__ __forceinline__ Tiles assign_tiles(int cta, int G, int NB, int KT, int rot) {
+  const int v = (cta + rot) % G;
+  const int b = v * NB / G;
+  const int first = (b * G + NB - 1) / NB, next = ((b + 1) * G + NB - 1) / NB;
+  const int cb = next - first, i = v - first;
+  Tiles t;
+  t.b = b;
+  t.k0 = i * KT / cb;
+  t.k1 = (i + 1) * KT / cb;
+  t.contrib = cb < KT ? cb : KT;
+  t.idx = cb <= KT ? i : t.k0;   // with more CTAs than k-blocks, each non-empty range is one k-block
+  return t;
 }
+__host__ __device__ __forceinline__ int proj_rot(int l, int j) { return 41 * (4 * l + j); }
 
 struct Smem {
   uint8_t* ring;
@@ -261,10 +297,10 @@ struct Smem {
   uint64_t *a_full, *g_done, *q_full, *v_full, *s_full, *p_full, *o_done, *fin;
   uint32_t* tmem_slot;
   int* flag;
+  int* last;
   float* red;               // [8]
 };
 
-// Shared-memory layout of a CTA (the plan described above), from the dynamic base.
 __device__ __forceinline__ Smem smem_plan(int R, size_t xbytes) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
@@ -284,6 +320,7 @@ __device__ __forceinline__ Smem smem_plan(int R, size_t xbytes) {
   S.fin = S.a_full + 7;
   S.tmem_slot = reinterpret_cast<uint32_t*>(S.a_full + 8);
   S.flag = reinterpret_cast<int*>(S.tmem_slot + 1);
+  S.last = S.flag + 1;
   S.red = reinterpret_cast<float*>(S.tmem_slot + 4);
   return S;
 }
@@ -297,10 +334,18 @@ struct Role {
   int a_uses = 0, i_uses = 0;        // loads issued on a_full and on q_full / v_full
 };
 
+// Step values shared by the CTA's threads: this step's distinct flow times and each token's.
+struct StepShared {
+  StepArgs p;
+  int nsh;                           // distinct flow times (shift rows of z)
+  int srow[kStepMaxShift];           // their modulation-table rows
+  int sidx[kMaxRows];                // token -> index of its flow time
+};
+
 // Grid barrier among warps 0-3 and 5 of every CTA: every CTA arrives (also after an error, so
 // that no CTA waits for it), then thread 160 spins on the counter. Returns false once any error is
 // recorded, so that the remaining steps are skipped.
-__device__ bool grid_sync(unsigned* ctr, bool ok, int* err, const Smem& S) {
+__device__ __noinline__ bool grid_sync(unsigned* ctr, bool ok, int* err, const Smem& S) {
   tc_fence_before();
   __syncwarp();
   named_sync(1, 160);
@@ -336,6 +381,24 @@ __device__ bool grid_sync(unsigned* ctr, bool ok, int* err, const Smem& S) {
   return *reinterpret_cast<volatile int*>(S.flag) != 0;
 }
 
+// Bounded wait until *ctr >= target (acquire); false (error recorded) on timeout or once any error
+// is recorded.
+__device__ __noinline__ int count_wait(const unsigned* ctr, unsigned target, int* err) {
+  unsigned long long t0 = 0;
+  for (uint32_t it = 0;; ++it) {
+    if (ld_acquire(ctr) >= target) return 1;
+    if ((it & 63) == 63) {
+      if (*reinterpret_cast<volatile int*>(err) != 0) return 0;
+      const unsigned long long t = gtime();
+      if (t0 == 0) t0 = t;
+      else if (t - t0 > kWaitNs) {
+        atomicCAS(err, 0, 52);
+        return 0;
+      }
+    }
+  }
+}
+
 // Sum over the 128 consumer threads (warps 0-3); every consumer gets the total.
 __device__ __forceinline__ float cons_sum(float v, float* red) {
   v = warp_sum(v);
@@ -347,47 +410,39 @@ __device__ __forceinline__ float cons_sum(float v, float* red) {
   return t;
 }
 
-// ---- row steps (consumers, one token row per CTA) ---------------------------------------
-constexpr int kMaxV4 = kStepMaxWidth / 512;   // float4 per consumer thread
+__device__ __forceinline__ float* sumsq_slot(const StepArgs& __restrict__ p, int l, int which) {
+  return reinterpret_cast<float*>(p.sync + (1 + kStepBarriersPerLayer * p.L) + (size_t)p.L * 4 * kStepMaxNB) +
+         (size_t)(2 * l + which) * kMaxRows;
+}
+__device__ __forceinline__ const float* mod_row(const StepArgs& __restrict__ p, int row) {
+  return p.tab + (size_t)row * p.rowlen;
+}
 
-// h[m] (+)= ..., then y[m] = RMSNorm(h[m]) * (1 + scale) + shift in bf16. With `acc`, h[m] +=
-// gate(tau) * acc[m] (gate 1 when gate_off < 0) and acc[m] is cleared; with `in_proj`,
-// h[m] = W_in u[m] + b_in. Returns the normalised row in `ys` (fp32 of the bf16 values) when
-// ys is not null. Every load of the row (and of its modulation vectors) is issued up front.
-__device__ __noinline__ void row_norm(const StepArgs& __restrict__ p, int m, const float* mod, float* acc, int gate_off,
-                                      int scale_off, int shift_off, bool in_proj, float* red, float* ys) {
-  const int tid = threadIdx.x, W = p.W, nv = W / 512;
-  float4* h4 = reinterpret_cast<float4*>(p.h + (size_t)m * W);
-  float4 x[kMaxV4], sc[kMaxV4], sh[kMaxV4];
-#pragma unroll
-  for (int j = 0; j < kMaxV4; ++j) {
-    if (j >= nv) break;
-    const int c4 = tid + 128 * j;
-    sc[j] = __ldg(reinterpret_cast<const float4*>(mod + scale_off) + c4);
-    sh[j] = __ldg(reinterpret_cast<const float4*>(mod + shift_off) + c4);
-  }
-  if (in_proj) {
-    // W_in rows are D bf16 (D a multiple of 8): 16-byte loads, all issued before the FMAs
-    const float* u = p.u + (size_t)m * p.D;
+// ---- phase "in": rows of layer 0 ------------------------------------------------------------
+// Token row m (CTA m < M): h = W_in u + b_in, the row's sum of squares, z = h (1 + scale1).
+// CTA M + j < M + nsh: shift row j of layer 0's first norm.
+__device__ __noinline__ void in_rows(const StepShared& __restrict__ sh, float* red) {
+  const StepArgs& p = sh.p;
+  const int c = blockIdx.x, tid = threadIdx.x, W = p.W;
+  if (c < p.M) {
+    const float* mod = mod_row(p, p.tau_row[c]);
+    const float* u = p.u + (size_t)c * p.D;
     const uint4* wi = static_cast<const uint4*>(p.w_in);
     const int D8 = p.D / 8;
-#pragma unroll
-    for (int j = 0; j < kMaxV4; ++j) {
-      if (j >= nv) break;
-      const int c = (tid + 128 * j) * 4;
-      const float4 b = __ldg(reinterpret_cast<const float4*>(p.b_in + c));
+    float ss = 0.f;
+#pragma unroll 1
+    for (int c4 = tid; c4 < W / 4; c4 += 128) {
+      const float4 b = __ldg(reinterpret_cast<const float4*>(p.b_in) + c4);
       float o[4] = {b.x, b.y, b.z, b.w};
-#pragma unroll 8
+#pragma unroll 1
       for (int k8 = 0; k8 < D8; ++k8) {
-        uint4 wv[4];
-#pragma unroll
-        for (int r = 0; r < 4; ++r) wv[r] = __ldg(wi + (size_t)(c + r) * D8 + k8);
         const float4 u0 = __ldg(reinterpret_cast<const float4*>(u) + 2 * k8);
         const float4 u1 = __ldg(reinterpret_cast<const float4*>(u) + 2 * k8 + 1);
         const float uk[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
 #pragma unroll
         for (int r = 0; r < 4; ++r) {
-          const __nv_bfloat162* w2 = reinterpret_cast<const __nv_bfloat162*>(&wv[r]);
+          const uint4 wv = __ldg(wi + (size_t)(4 * c4 + r) * D8 + k8);
+          const __nv_bfloat162* w2 = reinterpret_cast<const __nv_bfloat162*>(&wv);
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
             const float2 f = __bfloat1622float2(w2[q]);
@@ -395,156 +450,208 @@ __device__ __noinline__ void row_norm(const StepArgs& __restrict__ p, int m, con
           }
         }
       }
-      x[j] = make_float4(o[0], o[1], o[2], o[3]);
-      h4[tid + 128 * j] = x[j];
+      const float4 x = make_float4(o[0], o[1], o[2], o[3]);
+      reinterpret_cast<float4*>(p.h + (size_t)c * W)[c4] = x;
+      ss = fmaf(x.x, x.x, fmaf(x.y, x.y, fmaf(x.z, x.z, fmaf(x.w, x.w, ss))));
+      const float4 s = __ldg(reinterpret_cast<const float4*>(mod) + c4);
+      st_bf16x4(p.z + (size_t)c * W + 4 * c4, x.x * (1.f + s.x), x.y * (1.f + s.y), x.z * (1.f + s.z),
+                x.w * (1.f + s.w));
     }
-  } else {
-    float4 a[kMaxV4], g[kMaxV4];
-#pragma unroll
-    for (int j = 0; j < kMaxV4; ++j) {
-      if (j >= nv) break;
-      const int c4 = tid + 128 * j;
-      x[j] = h4[c4];
-      if (acc) {
-        a[j] = __ldcg(reinterpret_cast<const float4*>(acc + (size_t)m * W) + c4);
-        g[j] = gate_off >= 0 ? __ldg(reinterpret_cast<const float4*>(mod + gate_off) + c4) : make_float4(1.f, 1.f, 1.f, 1.f);
-      }
-    }
-    if (acc) {
-#pragma unroll
-      for (int j = 0; j < kMaxV4; ++j) {
-        if (j >= nv) break;
-        const int c4 = tid + 128 * j;
-        x[j].x = fmaf(g[j].x, a[j].x, x[j].x);
-        x[j].y = fmaf(g[j].y, a[j].y, x[j].y);
-        x[j].z = fmaf(g[j].z, a[j].z, x[j].z);
-        x[j].w = fmaf(g[j].w, a[j].w, x[j].w);
-        h4[c4] = x[j];
-      }
-    }
-  }
-  float ss = 0.f;
-#pragma unroll
-  for (int j = 0; j < kMaxV4; ++j) {
-    if (j >= nv) break;
-    ss = fmaf(x[j].x, x[j].x, fmaf(x[j].y, x[j].y, fmaf(x[j].z, x[j].z, fmaf(x[j].w, x[j].w, ss))));
-  }
-  const float rstd = 1.f / sqrtf(cons_sum(ss, red) / W + 1e-6f);
-  if (acc && !in_proj) {
-#pragma unroll
-    for (int j = 0; j < kMaxV4; ++j) {
-      if (j >= nv) break;
-      __stcg(reinterpret_cast<float4*>(acc + (size_t)m * W) + tid + 128 * j, make_float4(0.f, 0.f, 0.f, 0.f));
-    }
-  }
-#pragma unroll
-  for (int j = 0; j < kMaxV4; ++j) {
-    if (j >= nv) break;
-    const int c4 = tid + 128 * j;
-    const float y0 = fmaf(x[j].x * rstd, 1.f + sc[j].x, sh[j].x), y1 = fmaf(x[j].y * rstd, 1.f + sc[j].y, sh[j].y);
-    const float y2 = fmaf(x[j].z * rstd, 1.f + sc[j].z, sh[j].z), y3 = fmaf(x[j].w * rstd, 1.f + sc[j].w, sh[j].w);
-    uint2 pk;
-    pk.x = pack_bf16(y0, y1);
-    pk.y = pack_bf16(y2, y3);
-    *reinterpret_cast<uint2*>(p.y + (size_t)m * W + c4 * 4) = pk;
-    if (ys) {
-      const __nv_bfloat162 lo = *reinterpret_cast<const __nv_bfloat162*>(&pk.x);
-      const __nv_bfloat162 hi = *reinterpret_cast<const __nv_bfloat162*>(&pk.y);
-      *reinterpret_cast<float4*>(ys + c4 * 4) =
-          make_float4(__low2float(lo), __high2float(lo), __low2float(hi), __high2float(hi));
+    ss = cons_sum(ss, red);
+    if (tid == 0) sumsq_slot(p, 0, 0)[c] = ss;
+  } else if (c < p.M + sh.nsh) {
+    const float* shift = mod_row(p, sh.srow[c - p.M]) + W;
+#pragma unroll 1
+    for (int c4 = tid; c4 < W / 4; c4 += 128) {
+      const float4 s = __ldg(reinterpret_cast<const float4*>(shift) + c4);
+      st_bf16x4(p.z + (size_t)c * W + 4 * c4, s.x, s.y, s.z, s.w);
     }
   }
 }
 
-// Elementwise steps run on the consumers of every CTA: work item w of `total` goes to thread
-// (w mod T) with T = 128 * CTAs, and each thread issues all of its loads before using any.
-constexpr int kEwBatch = 4;   // work items per thread and batch
+// ---- block epilogues --------------------------------------------------------------------------
+// Every CTA that added into output block b finishes its share of the block's token rows,
+// [r0, r1), once all of them have arrived. A[m][128] (row m of the block at A + 128 m) holds the
+// staged accumulator rows; each CTA clears the rows it read. The shift rows M..M+nsh-1, which
+// every share reads, are cleared in a later phase (clear_shift_rows).
+__device__ __forceinline__ void stage_rows(float* A, const float* src, int N, int c0, int r0, int r1) {
+#pragma unroll 1
+  for (int i = threadIdx.x; i < (r1 - r0) * 32; i += 128) {
+    const int m = r0 + (i >> 5);
+    cp16(A + m * 128 + (i & 31) * 4, src + (size_t)m * N + c0 + (i & 31) * 4);
+  }
+}
+__device__ __forceinline__ void clear_rows(float* acc, int N, int c0, int r0, int r1) {
+#pragma unroll 1
+  for (int i = threadIdx.x; i < (r1 - r0) * 32; i += 128)
+    __stcg(reinterpret_cast<float4*>(acc + (size_t)(r0 + (i >> 5)) * N + c0) + (i & 31), make_float4(0.f, 0.f, 0.f, 0.f));
+}
+// Clears the shift rows of the qkv accumulator (this layer) and of the gate/up accumulator
+// (previous layer); every CTA's consumers take a strided share.
+__device__ __forceinline__ void clear_shift_rows(const StepShared& __restrict__ sh, bool qkv, bool gu) {
+  const StepArgs& p = sh.p;
+  const int nq = qkv ? sh.nsh * p.qkvd / 4 : 0, ng = gu ? sh.nsh * 2 * p.F / 4 : 0;
+  const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 1
+  for (int i = blockIdx.x * 128 + threadIdx.x; i < nq + ng; i += gridDim.x * 128) {
+    if (i < nq) __stcg(reinterpret_cast<float4*>(p.acc_qkv + (size_t)p.M * p.qkvd) + i, zero);
+    else __stcg(reinterpret_cast<float4*>(p.acc_gu + (size_t)p.M * 2 * p.F) + (i - nq), zero);
+  }
+}
 
-// q, k (RoPE) and v of every token into the attention layouts; acc_qkv cleared. Item = one
-// (token, q/k row pair) or one (token, v row).
-__device__ __noinline__ void ew_rope(const StepArgs& __restrict__ p, int l) {
-  const int dh = p.dh, half = dh / 2, npairs = (p.qd + p.kvd) / 2, per = npairs + p.kvd;
-  const int total = p.M * per, T = 128 * gridDim.x;
-  for (int base = blockIdx.x * 128 + threadIdx.x; base < total; base += kEwBatch * T) {
-    float2 a[kEwBatch], cs[kEwBatch];
-    // every load first: accumulator values and the rotation of each pair
+// qkv block b, rows [r0, r1): value = rstd(h_m) * acc[m] + acc[M + sidx[m]]; RoPE on q/k
+// pairs; q -> Q, k -> K cache, v -> Vt cache (bf16). Lane owns 4 consecutive features (two
+// RoPE pairs), whose (cos, sin) are staged per row next to the accumulator rows.
+__device__ __noinline__ void epi_qkv(const StepShared& __restrict__ sh, int l, int b, int r0, int r1, uint8_t* X) {
+  const StepArgs& p = sh.p;
+  const int M = p.M, warp = threadIdx.x >> 5, lane = threadIdx.x & 31, c0 = b * 128;
+  float* A = reinterpret_cast<float*>(X);
+  float* CS = A + kMaxRows * 128;           // [m][lane][cos0, sin0, cos1, sin1]
+  float* rs = CS + kMaxRows * 128;
+  stage_rows(A, p.acc_qkv, p.qkvd, c0, r0, r1);
+  stage_rows(A, p.acc_qkv, p.qkvd, c0, M, M + sh.nsh);
+  const int dh = p.dh, half = dh / 2, n = c0 + 4 * lane;
+  const bool qk = n < p.qd + p.kvd;
+  const int sn = n < p.qd ? n : n - p.qd;
+  if (qk && p.rope) {
+#pragma unroll 1
+    for (int m = r0 + warp; m < r1; m += 4)
+      cp16(CS + m * 128 + 4 * lane, p.rope_cs + (size_t)(m % p.H) * dh + ((sn % dh) >> 1) * 2);
+  }
+  const float* s1 = sumsq_slot(p, l, 0);
+  for (int m = r0 + threadIdx.x; m < r1; m += 128) rs[m] = rsqrtf(__ldcg(s1 + m) / p.W + 1e-6f);
+  cp_wait_all();
+  clear_rows(p.acc_qkv, p.qkvd, c0, r0, r1);
+  named_sync(2, 128);
+#pragma unroll 1
+  for (int m = r0 + warp; m < r1; m += 4) {
+    const float r = rs[m];
+    const float4 a = *reinterpret_cast<const float4*>(A + m * 128 + 4 * lane);
+    const float4 s = *reinterpret_cast<const float4*>(A + (M + sh.sidx[m]) * 128 + 4 * lane);
+    const float v[4] = {fmaf(r, a.x, s.x), fmaf(r, a.y, s.y), fmaf(r, a.z, s.z), fmaf(r, a.w, s.w)};
+    const int rb = m / p.H, i = m % p.H;
+    if (qk) {
+      const bool isq = n < p.qd;
+      const int hh = sn / dh;
+      __nv_bfloat16* dst = isq ? p.q + (((size_t)rb * p.n_heads + hh) * p.H + i) * dh
+                               : p.kcache + ((((size_t)rb * p.L + l) * p.n_kv_heads + hh) * p.n_keys + p.P + i) * dh;
+      const float4 cs = p.rope ? *reinterpret_cast<const float4*>(CS + m * 128 + 4 * lane) : make_float4(1.f, 0.f, 1.f, 0.f);
 #pragma unroll
-    for (int u = 0; u < kEwBatch; ++u) {
-      const int w = base + u * T;
-      if (w >= total) break;
-      const int m = w / per, e = w % per;
-      const float* acc = p.acc_qkv + (size_t)m * p.qkvd;
-      if (e < npairs) {
-        a[u] = __ldcg(reinterpret_cast<const float2*>(acc) + e);
-        const int sn = 2 * e < p.qd ? 2 * e : 2 * e - p.qd;
-        cs[u] = p.rope ? __ldg(reinterpret_cast<const float2*>(p.rope_cs + (size_t)(m % p.H) * dh) + ((sn % dh) >> 1))
-                       : make_float2(1.f, 0.f);
-      } else {
-        a[u].x = __ldcg(acc + p.qd + p.kvd + (e - npairs));
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < kEwBatch; ++u) {
-      const int w = base + u * T;
-      if (w >= total) break;
-      const int m = w / per, e = w % per, b = m / p.H, i = m % p.H;
-      float* acc = p.acc_qkv + (size_t)m * p.qkvd;
-      if (e < npairs) {
-        const int n = 2 * e;
-        const bool isq = n < p.qd;
-        const int sn = isq ? n : n - p.qd, hh = sn / dh, r = sn % dh;
+      for (int e = 0; e < 4; e += 2) {
+        const int rr = (sn + e) % dh;
+        const float c = e ? cs.z : cs.x, si = e ? cs.w : cs.y;
         // with RoPE, rows 2j, 2j+1 of a head hold dims j and j + dh/2 (pair-interleaved weights)
-        const int d0 = p.rope ? (r >> 1) : r, d1 = p.rope ? (r >> 1) + half : r + 1;
-        const float x0 = a[u].x * cs[u].x - a[u].y * cs[u].y;
-        const float x1 = a[u].y * cs[u].x + a[u].x * cs[u].y;
-        __nv_bfloat16* dst = isq ? p.q + (((size_t)b * p.n_heads + hh) * p.H + i) * dh
-                                 : p.kcache + ((((size_t)b * p.L + l) * p.n_kv_heads + hh) * p.n_keys + p.P + i) * dh;
-        dst[d0] = __float2bfloat16_rn(x0);
-        dst[d1] = __float2bfloat16_rn(x1);
-        __stcg(reinterpret_cast<float2*>(acc) + e, make_float2(0.f, 0.f));
-      } else {
-        const int ev = e - npairs, g = ev / dh, d = ev % dh;
-        p.vtcache[((((size_t)b * p.L + l) * p.n_kv_heads + g) * dh + d) * p.nk_pad + p.P + i] =
-            __float2bfloat16_rn(a[u].x);
-        __stcg(acc + p.qd + p.kvd + ev, 0.f);
+        const int d0 = p.rope ? (rr >> 1) : rr, d1 = p.rope ? (rr >> 1) + half : rr + 1;
+        dst[d0] = __float2bfloat16_rn(v[e] * c - v[e + 1] * si);
+        dst[d1] = __float2bfloat16_rn(v[e + 1] * c + v[e] * si);
+      }
+    } else {
+      const int ev = n - p.qd - p.kvd;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int g = (ev + e) / dh, d = (ev + e) % dh;
+        p.vtcache[((((size_t)rb * p.L + l) * p.n_kv_heads + g) * dh + d) * p.nk_pad + p.P + i] = __float2bfloat16_rn(v[e]);
       }
     }
   }
 }
 
-// act[m][j] = gelu_tanh(acc_gu[m][2j]) * acc_gu[m][2j+1] for every token; acc_gu cleared.
-// Item = one float4 of acc_gu (two outputs).
-__device__ __noinline__ void ew_act(const StepArgs& __restrict__ p) {
-  const int per = p.F / 2, total = p.M * per, T = 128 * gridDim.x;
-  float4* acc = reinterpret_cast<float4*>(p.acc_gu);
-  uint32_t* out = reinterpret_cast<uint32_t*>(p.act);
-  for (int base = blockIdx.x * 128 + threadIdx.x; base < total; base += kEwBatch * T) {
-    float4 a[kEwBatch];
-#pragma unroll
-    for (int u = 0; u < kEwBatch; ++u) {
-      const int w = base + u * T;
-      if (w >= total) break;
-      a[u] = __ldcg(acc + w);
+// gate/up block b (rows interleaved gate_j, up_j), rows [r0, r1): act[m][j] = gelu_tanh(gate) * up
+// with gate, up = rstd(h_m) * acc[m] + acc[M + sidx[m]].
+__device__ __noinline__ void epi_geglu(const StepShared& __restrict__ sh, int l, int b, int r0, int r1, uint8_t* X) {
+  const StepArgs& p = sh.p;
+  const int M = p.M, warp = threadIdx.x >> 5, lane = threadIdx.x & 31, c0 = b * 128;
+  float* A = reinterpret_cast<float*>(X);
+  float* rs = A + kMaxRows * 128;
+  stage_rows(A, p.acc_gu, 2 * p.F, c0, r0, r1);
+  stage_rows(A, p.acc_gu, 2 * p.F, c0, M, M + sh.nsh);
+  const float* s2 = sumsq_slot(p, l, 1);
+  for (int m = r0 + threadIdx.x; m < r1; m += 128) rs[m] = rsqrtf(__ldcg(s2 + m) / p.W + 1e-6f);
+  cp_wait_all();
+  clear_rows(p.acc_gu, 2 * p.F, c0, r0, r1);
+  named_sync(2, 128);
+#pragma unroll 1
+  for (int m = r0 + warp; m < r1; m += 4) {
+    const float r = rs[m];
+    const float4 a = *reinterpret_cast<const float4*>(A + m * 128 + 4 * lane);
+    const float4 s = *reinterpret_cast<const float4*>(A + (M + sh.sidx[m]) * 128 + 4 * lane);
+    const float g0 = fmaf(r, a.x, s.x), u0 = fmaf(r, a.y, s.y), g1 = fmaf(r, a.z, s.z), u1 = fmaf(r, a.w, s.w);
+    reinterpret_cast<uint32_t*>(p.act + (size_t)m * p.F + b * 64)[lane] = pack_bf16(gelu_tanh(g0) * u0, gelu_tanh(g1) * u1);
+  }
+}
+
+// o / down block b, rows [r0, r1): h[m] += gate(tau_m) * acc[m] on the block's 128 features, the
+// rows' partial sums of squares into `ss_out`, and (unless next_mod < 0) z[m] = h (1 + scale); the
+// first share also writes the block's shift rows of the next norm (modulation offsets next_mod =
+// scale, next_mod + W = shift).
+__device__ __noinline__ void epi_resid(const StepShared& __restrict__ sh, float* acc, int gate_off, int next_mod,
+                                       float* ss_out, int b, int r0, int r1, bool first, uint8_t* X) {
+  const StepArgs& p = sh.p;
+  const int M = p.M, W = p.W, nsh = sh.nsh, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float* A = reinterpret_cast<float*>(X);
+  float* Hs = A + kMaxRows * 128;
+  float* G = Hs + kMaxRows * 128;           // [nsh][128] gates, then scales, then shifts
+  float* Sc = G + kStepMaxShift * 128;
+  float* Sh = Sc + kStepMaxShift * 128;
+  const int tid = threadIdx.x, c0 = b * 128;
+  stage_rows(A, acc, W, c0, r0, r1);
+  stage_rows(Hs, p.h, W, c0, r0, r1);
+  const int nv = next_mod >= 0 ? 3 : 1;
+#pragma unroll 1
+  for (int i = tid; i < nv * nsh * 32; i += 128) {
+    const int kind = i / (nsh * 32), j = (i / 32) % nsh, q = i & 31;
+    const int off = kind == 0 ? gate_off : next_mod + (kind - 1) * W;
+    cp16(G + (kind * kStepMaxShift + j) * 128 + q * 4, mod_row(p, sh.srow[j]) + off + c0 + q * 4);
+  }
+  cp_wait_all();
+  clear_rows(acc, W, c0, r0, r1);
+  named_sync(2, 128);
+#pragma unroll 1
+  for (int m = r0 + warp; m < r1; m += 4) {
+    const int j = sh.sidx[m];
+    const float4 a = *reinterpret_cast<const float4*>(A + m * 128 + 4 * lane);
+    float4 h = *reinterpret_cast<const float4*>(Hs + m * 128 + 4 * lane);
+    const float4 g = *reinterpret_cast<const float4*>(G + j * 128 + 4 * lane);
+    h.x = fmaf(g.x, a.x, h.x);
+    h.y = fmaf(g.y, a.y, h.y);
+    h.z = fmaf(g.z, a.z, h.z);
+    h.w = fmaf(g.w, a.w, h.w);
+    reinterpret_cast<float4*>(p.h + (size_t)m * W + c0)[lane] = h;
+    const float ss = warp_sum(fmaf(h.x, h.x, fmaf(h.y, h.y, fmaf(h.z, h.z, h.w * h.w))));
+    if (lane == 0) atomicAdd(ss_out + m, ss);
+    if (next_mod >= 0) {
+      const float4 s = *reinterpret_cast<const float4*>(Sc + j * 128 + 4 * lane);
+      st_bf16x4(p.z + (size_t)m * W + c0 + 4 * lane, h.x * (1.f + s.x), h.y * (1.f + s.y), h.z * (1.f + s.z),
+                h.w * (1.f + s.w));
     }
-#pragma unroll
-    for (int u = 0; u < kEwBatch; ++u) {
-      const int w = base + u * T;
-      if (w >= total) break;
-      out[w] = pack_bf16(gelu_tanh(a[u].x) * a[u].y, gelu_tanh(a[u].z) * a[u].w);
-      __stcg(acc + w, make_float4(0.f, 0.f, 0.f, 0.f));
+  }
+  if (next_mod >= 0 && first) {
+#pragma unroll 1
+    for (int j = warp; j < nsh; j += 4) {
+      const float4 s = *reinterpret_cast<const float4*>(Sh + j * 128 + 4 * lane);
+      st_bf16x4(p.z + (size_t)(M + j) * W + c0 + 4 * lane, s.x, s.y, s.z, s.w);
     }
   }
 }
 
-// Merge the key chunks of the query rows assigned to this consumer warp.
+// Merge the key chunks of the query rows assigned to this consumer warp: the warp stages the
+// row's partial O of every chunk in shared memory (one round of loads), then combines.
 template <int DH>
-__device__ __noinline__ void combine_rows(const StepArgs& __restrict__ p) {
+__device__ __noinline__ void combine_rows(const StepArgs& __restrict__ p, uint8_t* X) {
   constexpr int E = DH / 32;
-  const int lane = threadIdx.x & 31;
-  const int gw = blockIdx.x * 4 + (threadIdx.x >> 5), nw = gridDim.x * 4;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int gw = blockIdx.x * 4 + w, nw = gridDim.x * 4;
   const int nck = p.n_chunks, total = p.B * p.n_kv_heads * p.rows;
+  float* buf = reinterpret_cast<float*>(X) + (size_t)w * kStepMaxChunks * DH;
+#pragma unroll 1
   for (int idx = gw; idx < total; idx += nw) {
     const int bg = idx / p.rows, r = idx % p.rows;
+    const float* src = p.part_o + ((size_t)bg * nck * p.r_pad + r) * DH;
+#pragma unroll 1
+    for (int i = lane; i < nck * (DH / 4); i += 32) {
+      const int cc = i / (DH / 4), q = i % (DH / 4);
+      cp16(buf + cc * DH + q * 4, src + (size_t)cc * p.r_pad * DH + q * 4);
+    }
     float mc = -INFINITY, lc = 0.f;
     if (lane < nck) {
       const size_t pi = ((size_t)bg * nck + lane) * p.r_pad + r;
@@ -552,34 +659,25 @@ __device__ __noinline__ void combine_rows(const StepArgs& __restrict__ p) {
       lc = __ldcg(p.part_ml + pi * 2 + 1);
     }
     const float M = warp_max(mc);
-    const float w = lane < nck ? exp2f((mc - M) * p.scale_log2) : 0.f;
-    const float L = warp_sum(w * lc);
+    const float wgt = lane < nck ? exp2f((mc - M) * p.scale_log2) : 0.f;
+    const float L = warp_sum(wgt * lc);
+    cp_wait_all();
+    __syncwarp();
     float acc[E];
 #pragma unroll
     for (int e = 0; e < E; ++e) acc[e] = 0.f;
-    // chunks in batches of kCB: every load of a batch is issued before the first FMA
-    constexpr int kCB = 32 / E < 16 ? 32 / E : 16;
-    for (int c0 = 0; c0 < nck; c0 += kCB) {
-      float v[kCB][E];
+#pragma unroll 2
+    for (int cc = 0; cc < nck; ++cc) {
+      const float wc = __shfl_sync(0xffffffffu, wgt, cc);
 #pragma unroll
-      for (int cc = 0; cc < kCB; ++cc) {
-        if (c0 + cc >= nck) break;
-        const float* src = p.part_o + (((size_t)bg * nck + c0 + cc) * p.r_pad + r) * DH;
-#pragma unroll
-        for (int e = 0; e < E; ++e) v[cc][e] = __ldcg(src + e * 32 + lane);
-      }
-#pragma unroll
-      for (int cc = 0; cc < kCB; ++cc) {
-        if (c0 + cc >= nck) break;
-        const float wc = __shfl_sync(0xffffffffu, w, c0 + cc);
-#pragma unroll
-        for (int e = 0; e < E; ++e) acc[e] = fmaf(wc, v[cc][e], acc[e]);
-      }
+      for (int e = 0; e < E; ++e) acc[e] = fmaf(wc, buf[cc * DH + e * 32 + lane], acc[e]);
     }
+    __syncwarp();
     const int b = bg / p.n_kv_heads, g = bg % p.n_kv_heads, j = r / p.H, i = r % p.H;
     __nv_bfloat16* dst = p.o + ((size_t)b * p.H + i) * p.qd + (size_t)(g * p.group + j) * DH;
+    const float invL = 1.f / L;
 #pragma unroll
-    for (int e = 0; e < E; ++e) dst[e * 32 + lane] = __float2bfloat16_rn(acc[e] / L);
+    for (int e = 0; e < E; ++e) dst[e * 32 + lane] = __float2bfloat16_rn(acc[e] * invL);
   }
 }
 
@@ -587,39 +685,37 @@ __device__ __noinline__ void combine_rows(const StepArgs& __restrict__ p) {
 
 // ---- projection step: acc[m][n] += sum over this CTA's weight tiles of A[m][k] W[n][k] -----
 // Thread 160 loads the activation tiles (tensor map) and issues the MMAs against the weight
-// ring; the consumer warps add each finished 128 x 64 tile into `acc` (fp32, L2) with 16-byte
-// reds.
-__device__ __noinline__ void projection_step(const StepArgs& __restrict__ p, const CUtensorMap* amap, float* acc, int l, int j,
+// ring; the consumer warps add the finished 128 x 64 tile into `acc` (fp32, L2) with 16-byte
+// reds, then count the block's arrival; the last of its CTAs runs the block's epilogue.
+__device__ __noinline__ void projection_step(const StepShared& __restrict__ sh, const CUtensorMap* amap, int l, int j,
                                              uint32_t tmem, size_t xbytes, Role& st) {
+  const StepArgs& p = sh.p;
   const Smem S = smem_plan(p.ring, xbytes);
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, R = p.ring, M = p.M;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const bool mma = threadIdx.x == 160, cons = warp < 4;
-  int N, K, t0, t1;
+  int N, K;
   proj_shape(p, j, N, K);
   const int KT = K / 64;
-  tile_range((N / 128) * KT, 4 * l + j, t0, t1);
-  const int nt = t1 - t0;
+  const Tiles tl = assign_tiles(blockIdx.x, gridDim.x, N / 128, KT, proj_rot(l, j));
+  const int nt = tl.k1 - tl.k0;
   if (nt <= 0) return;
+  float* acc = j == 0 ? p.acc_qkv : j == 1 ? p.acc_o : j == 2 ? p.acc_gu : p.acc_d;
+  const int R = (j == 0 || j == 2) ? p.M + sh.nsh : p.M;   // rows added: tokens (+ shift rows)
   if (mma) {
     mbar_expect_tx(S.a_full, (uint32_t)nt * kATile);
-    for (int i = 0; i < nt; ++i) tma_2d(S.X + (size_t)i * kATile, amap, ((t0 + i) % KT) * 64, 0, S.a_full);
+    for (int i = 0; i < nt; ++i) tma_2d(S.X + (size_t)i * kATile, amap, (tl.k0 + i) * 64, 0, S.a_full);
     ++st.a_uses;
     bool good = mbar_wait(S.a_full, st.apar, p.err, 42);
-    int seg = -1, pnb = -1;
     for (int i = 0; i < nt && good; ++i) {
-      const int nb = (t0 + i) / KT;
-      const bool first = nb != pnb;
-      if (first) { ++seg; pnb = nb; }
       good = mbar_wait(S.full + st.slot, st.par, p.err, 43);
       if (!good) break;
       tc_fence_after();
       const uint32_t a0 = su32(S.ring + (size_t)st.slot * kSlot), b0 = su32(S.X + (size_t)i * kATile);
 #pragma unroll
       for (int k = 0; k < 4; ++k)
-        mma_bf16(tmem + seg * 64, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), idesc_m128(64),
-                 (first && k == 0) ? 0u : 1u);
+        mma_bf16(tmem, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), idesc_m128(64), (i | k) ? 1u : 0u);
       mma_commit(S.empty + st.slot);
-      if (++st.slot == R) { st.slot = 0; st.par ^= 1u; }
+      if (++st.slot == p.ring) { st.slot = 0; st.par ^= 1u; }
     }
     mma_commit(S.g_done);
   }
@@ -630,33 +726,47 @@ __device__ __noinline__ void projection_step(const StepArgs& __restrict__ p, con
     const uint32_t tm = tmem_base_after_wait(S.tmem_slot);
     const int quad = warp & 3, row = quad * 32 + lane;
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
-    // each segment's tile goes through shared memory (T[token][row], over the activation
-    // tiles, which the finished MMAs no longer read) so that the adds into L2 are 16-byte
-    // reds along the output features
+    // the tile goes through shared memory (T[token][row], over the activation tiles, which the
+    // finished MMAs no longer read) so that the adds into L2 are 16-byte reds along the features
     float* T = reinterpret_cast<float*>(S.X);
-    int seg = -1, pnb = -1;
-    for (int i = 0; i < nt; ++i) {
-      const int nb = (t0 + i) / KT;
-      if (nb == pnb) continue;
-      ++seg;
-      pnb = nb;
+#pragma unroll 1
+    for (int q = 0; q < R; q += 32) {
+      float v[32];
+      __syncwarp();
+      tmem_ld32(tm + lane_base + q, v);
 #pragma unroll
-      for (int q = 0; q < kMaxRows; q += 32) {
-        float v[32];
-        __syncwarp();
-        tmem_ld32(tm + lane_base + seg * 64 + q, v);
-#pragma unroll
-        for (int e = 0; e < 32; ++e) T[(q + e) * 128 + row] = v[e];
+      for (int e = 0; e < 32; ++e) T[(q + e) * 128 + row] = v[e];
+    }
+    named_sync(2, 128);
+    if (good) {
+      float* dst = acc + tl.b * 128;
+#pragma unroll 4
+      for (int idx = threadIdx.x; idx < R * 32; idx += 128) {
+        const int m = idx >> 5, c4 = idx & 31;
+        red_add_v4(dst + (size_t)m * N + 4 * c4, *reinterpret_cast<const float4*>(T + m * 128 + 4 * c4));
       }
-      named_sync(2, 128);
+    }
+    named_sync(2, 128);
+    if (threadIdx.x == 0) {
+      // arrive on the block (release: this CTA's reds, ordered before by the named barrier), then
+      // wait until every CTA of the block has arrived (acquire: their reds)
+      int go = 0;
       if (good) {
-        float* dst = acc + nb * 128;
-        for (int idx = threadIdx.x; idx < M * 32; idx += 128) {
-          const int m = idx >> 5, c4 = idx & 31;
-          red_add_v4(dst + (size_t)m * N + 4 * c4, *reinterpret_cast<const float4*>(T + m * 128 + 4 * c4));
-        }
+        unsigned* ctr = p.sync + (1 + kStepBarriersPerLayer * p.L) + (size_t)(4 * l + j) * kStepMaxNB + tl.b;
+        asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ctr) : "memory");
+        go = count_wait(ctr, (unsigned)tl.contrib, p.err);
       }
-      named_sync(2, 128);
+      *S.last = go;
+    }
+    named_sync(2, 128);
+    if (*reinterpret_cast<volatile int*>(S.last)) {
+      const int W6 = 6 * p.W, b6 = l * W6, M = p.M;
+      const int r0 = tl.idx * M / tl.contrib, r1 = (tl.idx + 1) * M / tl.contrib;
+      if (j == 0) epi_qkv(sh, l, tl.b, r0, r1, S.X);
+      else if (j == 2) epi_geglu(sh, l, tl.b, r0, r1, S.X);
+      else if (j == 1) epi_resid(sh, p.acc_o, b6 + 2 * p.W, b6 + 3 * p.W, sumsq_slot(p, l, 1), tl.b, r0, r1, tl.idx == 0, S.X);
+      else epi_resid(sh, p.acc_d, b6 + 5 * p.W, l + 1 < p.L ? b6 + W6 : -1, sumsq_slot(p, l + 1, 0), tl.b, r0, r1,
+                     tl.idx == 0, S.X);
     }
   }
   st.gpar ^= 1u;
@@ -791,19 +901,29 @@ __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, cons
   }
 }
 
-// Final norm and action-out projection of row m: v[m] = W_out y[m] + b_out.
-__device__ __noinline__ void final_row(const StepArgs& __restrict__ p, int m, const float* mod, size_t xbytes) {
-  const Smem S = smem_plan(p.ring, xbytes);
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  float* ys = reinterpret_cast<float*>(S.X);
-  const int W6 = 6 * p.W, fb = p.L * W6;
-  row_norm(p, m, mod, p.acc_d, fb - W6 + 5 * p.W, fb, fb + p.W, false, S.red, ys);
+// Final norm and action-out projection of row m: y = RMSNorm(h) (1 + scale) + shift (rounded to
+// bf16 like every projection input), v[m] = W_out y + b_out.
+__device__ __noinline__ void final_row(const StepArgs& __restrict__ p, int m, float* ys) {
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, W = p.W;
+  const float* mod = mod_row(p, p.tau_row[m]) + (size_t)p.L * 6 * W;
+  const float rstd = rsqrtf(__ldcg(sumsq_slot(p, p.L, 0) + m) / W + 1e-6f);
+#pragma unroll 1
+  for (int c4 = tid; c4 < W / 4; c4 += 128) {
+    const float4 h = __ldcg(reinterpret_cast<const float4*>(p.h + (size_t)m * W) + c4);
+    const float4 sc = __ldg(reinterpret_cast<const float4*>(mod) + c4);
+    const float4 sf = __ldg(reinterpret_cast<const float4*>(mod + W) + c4);
+    const __nv_bfloat162 lo = __floats2bfloat162_rn(fmaf(h.x * rstd, 1.f + sc.x, sf.x), fmaf(h.y * rstd, 1.f + sc.y, sf.y));
+    const __nv_bfloat162 hi = __floats2bfloat162_rn(fmaf(h.z * rstd, 1.f + sc.z, sf.z), fmaf(h.w * rstd, 1.f + sc.w, sf.w));
+    reinterpret_cast<float4*>(ys)[c4] = make_float4(__low2float(lo), __high2float(lo), __low2float(hi), __high2float(hi));
+  }
   named_sync(2, 128);
   const __nv_bfloat16* wo = static_cast<const __nv_bfloat16*>(p.w_out);
+#pragma unroll 1
   for (int d = warp; d < p.D; d += 4) {
     float a = 0.f;
-    for (int k = 2 * lane; k < p.W; k += 64) {
-      const float2 wv = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(wo + (size_t)d * p.W + k));
+#pragma unroll 4
+    for (int k = 2 * lane; k < W; k += 64) {
+      const float2 wv = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(wo + (size_t)d * W + k));
       a = fmaf(ys[k], wv.x, fmaf(ys[k + 1], wv.y, a));
     }
     a = warp_sum(a);
@@ -813,21 +933,33 @@ __device__ __noinline__ void final_row(const StepArgs& __restrict__ p, int m, co
 
 template <int DH>
 __global__ void __launch_bounds__(kThreads, 1)
-    step_kernel(const __grid_constant__ CUtensorMap t_y, const __grid_constant__ CUtensorMap t_o,
+    step_kernel(const __grid_constant__ CUtensorMap t_z, const __grid_constant__ CUtensorMap t_o,
                 const __grid_constant__ CUtensorMap t_act, const __grid_constant__ CUtensorMap t_q,
                 const __grid_constant__ CUtensorMap t_k, const __grid_constant__ CUtensorMap t_vt,
-                const __grid_constant__ StepArgs p) {
+                const __grid_constant__ StepArgs p_in) {
   constexpr size_t XB = step_x_bytes(DH);
-  const int R = p.ring;
+  // the arguments and this step's flow-time rows live in shared memory for the whole launch
+  __shared__ StepShared sh;
+  const int R = p_in.ring;
   const Smem S = smem_plan(R, XB);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
+    sh.p = p_in;
+    int n = __ldg(p_in.sinfo);
+    n = n < kStepMaxShift ? n : kStepMaxShift;
+    n = n < kMaxRows - p_in.M ? n : kMaxRows - p_in.M;
+    sh.nsh = n > 0 ? n : 0;
+    for (int i = 0; i < kStepMaxShift; ++i) sh.srow[i] = __ldg(p_in.sinfo + 1 + i);
     for (int i = 0; i < R; ++i) {
       mbar_init(S.full + i, 1);
       mbar_init(S.empty + i, 1);
     }
     for (int i = 0; i < 8; ++i) mbar_init(S.a_full + i, i == 5 ? 4 : 1);   // p_full: one arrive per consumer warp
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (threadIdx.x < kMaxRows) {
+    const int si = threadIdx.x < p_in.M ? __ldg(p_in.sidx + threadIdx.x) : 0;
+    sh.sidx[threadIdx.x] = si >= 0 && si < kStepMaxShift ? si : 0;
   }
   if (warp == 0) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(S.tmem_slot)), "r"(kTmemCols));
@@ -836,6 +968,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  const StepArgs& p = sh.p;
   const uint32_t tmem = *S.tmem_slot;
 
   if (warp == 4) {
@@ -847,11 +980,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int l = 0; l < p.L && ok; ++l)
         for (int j = 0; j < 4 && ok; ++j) {
-          int N, K, t0, t1;
+          int N, K;
           proj_shape(p, j, N, K);
-          tile_range((N / 128) * (K / 64), 4 * l + j, t0, t1);
-          const uint8_t* w = static_cast<const uint8_t*>(p.wl[4 * l + j]);
-          for (int t = t0; t < t1; ++t) {
+          const int KT = K / 64;
+          const Tiles tl = assign_tiles(blockIdx.x, gridDim.x, N / 128, KT, proj_rot(l, j));
+          const uint8_t* w = static_cast<const uint8_t*>(p.wl[4 * l + j]) + ((size_t)tl.b * KT + tl.k0) * kSlot;
+          for (int t = 0; t < tl.k1 - tl.k0; ++t) {
             if (!mbar_wait(S.empty + slot, par ^ 1u, p.err, 41)) { ok = false; break; }
             mbar_expect_tx(S.full + slot, kSlot);
             bulk_g2s(S.ring + (size_t)slot * kSlot, w + (size_t)t * kSlot, kSlot, S.full + slot, pol);
@@ -866,40 +1000,30 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else {
     // ---- warps 0-3: consumers; warp 5: tcgen05 issuer (thread 160) ----
     const bool mma = threadIdx.x == 160, cons = warp < 4;
-    const int c = blockIdx.x, M = p.M, W = p.W, W6 = 6 * W;
     Role st;
     bool ok = true;
-    unsigned* bar = p.bars;
-    // modulation row of this CTA's token (fixed for the whole evaluation)
-    const float* mod = cons && c < M ? p.tab + (size_t)p.tau_row[c] * p.rowlen : p.tab;
+    unsigned* bar = p.sync;
+    if (cons) in_rows(sh, S.red);
+    ok = grid_sync(bar++, ok, p.err, S);
     for (int l = 0; l < p.L; ++l) {
-      const int b6 = l * W6;
-      // norm1 (layer 0: the action-in projection first)
-      if (ok && cons && c < M)
-        row_norm(p, c, mod, l > 0 ? p.acc_d : nullptr, l > 0 ? b6 - W6 + 5 * W : -1, b6, b6 + W, l == 0, S.red,
-                 nullptr);
-      ok = grid_sync(bar++, ok, p.err, S);
-      if (ok) projection_step(p, &t_y, p.acc_qkv, l, 0, tmem, XB, st);
-      ok = grid_sync(bar++, ok, p.err, S);
-      if (ok && cons) ew_rope(p, l);
+      if (ok) projection_step(sh, &t_z, l, 0, tmem, XB, st);
       ok = grid_sync(bar++, ok, p.err, S);
       if (ok) attention_step<DH>(p, &t_q, &t_k, &t_vt, l, tmem, st);
       ok = grid_sync(bar++, ok, p.err, S);
-      if (ok && cons) combine_rows<DH>(p);
+      if (ok && cons) {
+        clear_shift_rows(sh, true, l > 0);
+        combine_rows<DH>(p, S.X);
+      }
       ok = grid_sync(bar++, ok, p.err, S);
-      if (ok) projection_step(p, &t_o, p.acc_o, l, 1, tmem, XB, st);
+      if (ok) projection_step(sh, &t_o, l, 1, tmem, XB, st);
       ok = grid_sync(bar++, ok, p.err, S);
-      if (ok && cons && c < M)
-        row_norm(p, c, mod, p.acc_o, b6 + 2 * W, b6 + 3 * W, b6 + 4 * W, false, S.red, nullptr);
+      if (ok) projection_step(sh, &t_z, l, 2, tmem, XB, st);
       ok = grid_sync(bar++, ok, p.err, S);
-      if (ok) projection_step(p, &t_y, p.acc_gu, l, 2, tmem, XB, st);
-      ok = grid_sync(bar++, ok, p.err, S);
-      if (ok && cons) ew_act(p);
-      ok = grid_sync(bar++, ok, p.err, S);
-      if (ok) projection_step(p, &t_act, p.acc_d, l, 3, tmem, XB, st);
+      if (ok) projection_step(sh, &t_act, l, 3, tmem, XB, st);
       ok = grid_sync(bar++, ok, p.err, S);
     }
-    if (ok && cons && c < M) final_row(p, c, mod, XB);
+    if (ok && cons) clear_shift_rows(sh, false, true);
+    if (ok && cons && (int)blockIdx.x < p.M) final_row(p, blockIdx.x, reinterpret_cast<float*>(S.X));
     if (mma) {
       // tensor memory is freed only after every MMA of this thread has completed, and the CTA
       // exits only after its last operand loads have landed (they are waited for on the normal
@@ -923,10 +1047,25 @@ __global__ void __launch_bounds__(kThreads, 1)
 size_t step_smem_bytes(int dh, int ring) { return 1024 + (size_t)ring * kSlot + step_x_bytes(dh) + kTailBytes; }
 
 int step_ring_slots(int dh, int smem_optin) {
-  const long long left = (long long)smem_optin - 1024 - (long long)step_x_bytes(dh) - (long long)kTailBytes;
+  // the kernel's static shared memory (arguments and flow-time rows) comes off the top
+  const long long left = (long long)smem_optin - (long long)sizeof(StepShared) - 1024 - (long long)step_x_bytes(dh) -
+                         (long long)kTailBytes;
   long long r = left / kSlot;
   if (r > kMaxRing) r = kMaxRing;
   return (int)r;
+}
+
+int step_max_tiles(int ctas, const int (*shapes)[2], int n) {
+  int most = 0;
+  for (int s = 0; s < n; ++s) {
+    const int NB = shapes[s][0] / 128, KT = shapes[s][1] / 64;
+    if (NB < 1 || NB > ctas || NB > kStepMaxNB) return 0;
+    for (int c = 0; c < ctas; ++c) {
+      const Tiles t = assign_tiles(c, ctas, NB, KT, 0);
+      most = t.k1 - t.k0 > most ? t.k1 - t.k0 : most;
+    }
+  }
+  return most;
 }
 
 int step_prepare(int dh, int ring, int* blocks_per_sm) {
@@ -962,9 +1101,9 @@ int launch_step(const StepMaps& m, const StepArgs& a, int grid, cudaStream_t s) 
   cfg.attrs = nullptr;
   cfg.numAttrs = 0;
   cudaError_t e = cudaErrorInvalidValue;
-  if (a.dh == 64) e = cudaLaunchKernelEx(&cfg, step_kernel<64>, m.y, m.o, m.act, m.q, m.k, m.vt, a);
-  if (a.dh == 128) e = cudaLaunchKernelEx(&cfg, step_kernel<128>, m.y, m.o, m.act, m.q, m.k, m.vt, a);
-  if (a.dh == 256) e = cudaLaunchKernelEx(&cfg, step_kernel<256>, m.y, m.o, m.act, m.q, m.k, m.vt, a);
+  if (a.dh == 64) e = cudaLaunchKernelEx(&cfg, step_kernel<64>, m.z, m.o, m.act, m.q, m.k, m.vt, a);
+  if (a.dh == 128) e = cudaLaunchKernelEx(&cfg, step_kernel<128>, m.z, m.o, m.act, m.q, m.k, m.vt, a);
+  if (a.dh == 256) e = cudaLaunchKernelEx(&cfg, step_kernel<256>, m.z, m.o, m.act, m.q, m.k, m.vt, a);
   return e == cudaSuccess ? 0 : -1;
 }
 

@@ -10,6 +10,7 @@
 #include <numeric>
 #include <string>
 #include <thread>
+#include <tuple>
 #include <vector>
 
 #include "../../include/uad.h"
@@ -128,7 +129,7 @@ struct uad_ctx {
 
   cudaStream_t worker = nullptr;
   cudaEvent_t ev_in = nullptr, ev_done = nullptr;
-  std::map<std::pair<int, int>, cudaGraphExec_t> graphs;
+  std::map<std::tuple<int, int, int>, cudaGraphExec_t> graphs;   // (robots, N*, persistent kernel)
 
   // in-flight chunk
   bool in_flight = false;
@@ -279,7 +280,7 @@ std::pair<int, int> reduce(int num, int den) {
 
 // Plan block layout for a call with n_steps steps and B robots (16-byte aligned sections).
 struct PlanLayout {
-  size_t plan, tau, gstep, last, tailc, tailf, mask, epoch, rot, total;
+  size_t plan, tau, sidx, sinfo, gstep, last, tailc, tailf, mask, epoch, rot, total;
 };
 PlanLayout plan_layout(int n_steps, int B, int H, int D) {
   auto al = [](size_t x) { return (x + 15) & ~(size_t)15; };
@@ -288,6 +289,8 @@ PlanLayout plan_layout(int n_steps, int B, int H, int D) {
   size_t o = 0;
   L.plan = o; o = al(o + n_steps * M * sizeof(PlanTok));
   L.tau = o; o = al(o + n_steps * M * 4);
+  L.sidx = o; o = al(o + n_steps * M * 4);                        // persistent kernel: token -> flow time
+  L.sinfo = o; o = al(o + n_steps * (1 + kStepMaxShift) * 4);     // count, rows of distinct flow times
   L.gstep = o; o = al(o + B * 4);
   L.last = o; o = al(o + B * 4);
   L.tailc = o; o = al(o + B * 4);
@@ -448,11 +451,10 @@ const char* step_unfit(uad_ctx* c, int* ring) {
   if (dh != 64 && dh != 128 && dh != 256) return "head dim";
   if ((c->at0.n_keys + 63) / 64 > kStepMaxChunks) return "too many keys";
   const int shapes[4][2] = {{c->qkvd, W}, {W, c->qd}, {2 * F, W}, {W, F}};
-  for (auto& sh : shapes) {
+  for (auto& sh : shapes)
     if (sh[0] % 128 || sh[1] % 64) return "projection shape";
-    const int T = sh[0] / 128 * (sh[1] / 64);
-    if ((T + c->sms - 1) / c->sms > kStepMaxATiles) return "projection too large";
-  }
+  const int most = step_max_tiles(c->sms, shapes, 4);
+  if (most < 1 || most > kStepMaxATiles) return "projection too large";
   for (const LayerW& w : c->L)
     if (!w.wqkv.tiled || !w.wo.tiled || !w.wgu.tiled || !w.wd.tiled) return "untiled weights";
   int optin = 0;
@@ -480,7 +482,7 @@ int step_setup(uad_ctx* c) {
   p.ring = ring; p.rope = a.rope ? 1 : 0; p.scale_log2 = t.scale_log2;
   p.tab = c->tab; p.rowlen = c->rowlen; p.u = c->u;
   p.w_in = c->w_in; p.b_in = c->b_in; p.w_out = c->w_out; p.b_out = c->b_out; p.v = c->v; p.h = c->h;
-  p.y = static_cast<__nv_bfloat16*>(c->y); p.o = static_cast<__nv_bfloat16*>(c->o);
+  p.o = static_cast<__nv_bfloat16*>(c->o);
   p.act = static_cast<__nv_bfloat16*>(c->act);
   int rc;
   const size_t R = kStepMaxRows;
@@ -498,9 +500,14 @@ int step_setup(uad_ctx* c) {
   const size_t parts = (size_t)c->step_bmax * a.n_kv_heads * p.n_chunks * t.r_pad;
   if ((rc = dalloc_t(c, &p.part_o, parts * a.head_dim)) || (rc = dalloc_t(c, &p.part_ml, parts * 2))) return rc;
   p.rope_cs = c->rope_cs;
-  if ((rc = dalloc_t(c, &p.bars, (size_t)L * kStepBarriersPerLayer))) return rc;
+  if ((rc = dalloc_t(c, &p.sync, step_sync_words(L)))) return rc;
+  // projection input rows z: tokens, then the step's shift rows (a tensor map of all 64 rows)
+  void* z = nullptr;
+  if ((rc = dalloc(c, &z, (size_t)kStepMaxRows * W * 2))) return rc;
+  p.z = static_cast<__nv_bfloat16*>(z);
+  if ((rc = make_tmap(c, z, W, kStepMaxRows))) return rc;
   p.err = c->dev_err;
-  c->smaps.y = c->tmaps.at(c->y);
+  c->smaps.z = c->tmaps.at(z);
   c->smaps.o = c->tmaps.at(c->o);
   c->smaps.act = c->tmaps.at(c->act);
   c->smaps.q = c->atmaps.q;
@@ -516,8 +523,14 @@ int step_setup(uad_ctx* c) {
 
 bool step_path(const uad_ctx* c, int B) { return c->step_ok && B <= c->step_bmax; }
 
+// Whether a chunk runs on the persistent kernel: it serves the batch and every step has room
+// for its distinct flow times next to the tokens (set by the host plan).
+bool chunk_uses_step(const uad_ctx* c, int B, int max_shift) {
+  return step_path(c, B) && max_shift <= kStepMaxShift && B * c->a.chunk_len + max_shift <= kStepMaxRows;
+}
+
 // Enqueue every kernel of one chunk (begin + n_steps evaluations) for B robots.
-void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
+void enqueue_chunk(uad_ctx* c, int B, int n_steps, bool step, cudaStream_t s) {
   const uad_arch& a = c->a;
   const int H = a.chunk_len, D = a.action_dim, W = a.width, M = B * H, F = a.mlp_dim;
   const int dt = a.dtype;
@@ -528,7 +541,6 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
   const bool dit = a.kind == UAD_KIND_DIT;
 
   { Mark mk(c, s, "begin", 12.0 * M * D, 0); launch_begin(c->noise, c->x, c->g, c->u, M * D, c->nonfinite, c->evals, c->stamps, s); }
-  const bool step = step_path(c, B);
   if (step) {
     // the persistent kernel's accumulators are zero between uses; clearing them per chunk keeps
     // a chunk that ended in an error from leaking into the next one
@@ -545,7 +557,9 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, cudaStream_t s) {
     if (step) {
       StepArgs p = c->st0;
       p.M = M; p.B = B; p.tau_row = tr;
-      cudaMemsetAsync(p.bars, 0, (size_t)a.n_layers * kStepBarriersPerLayer * 4, s);
+      p.sidx = reinterpret_cast<const int*>(c->plan_dev + PL.sidx) + (size_t)(k - 1) * M;
+      p.sinfo = reinterpret_cast<const int*>(c->plan_dev + PL.sinfo) + (size_t)(k - 1) * (1 + kStepMaxShift);
+      cudaMemsetAsync(p.sync, 0, step_sync_words(a.n_layers) * 4, s);
       const double kv = 2.0 * B * a.n_layers * a.n_kv_heads * (double)p.n_keys * a.head_dim * 2;
       const double by = c->step_bytes_w + kv + 16.0 * a.n_layers * M * W + 8.0 * M * D;
       const double fl = c->step_flops_w * M + 4.0 * M * a.n_heads * (double)p.n_keys * a.head_dim * a.n_layers;
@@ -1122,15 +1136,39 @@ static int denoise_impl(uad_ctx* c, const float* noise, const uad_schedule* sc, 
   int rc = fill_times(c, need, s);
   if (rc) return rc;
   for (size_t e = 0; e < taus.size(); ++e) taur[e] = c->tau_row.at(taus[e]);
+  // persistent kernel: each step's distinct flow times (their table rows) and each token's index
+  int max_shift = 0;
+  {
+    int* sidx = reinterpret_cast<int*>(hp + PL.sidx);
+    int* sinfo = reinterpret_cast<int*>(hp + PL.sinfo);
+    for (int k = 0; k < steps; ++k) {
+      int* info = sinfo + (size_t)k * (1 + kStepMaxShift);
+      int n = 0;
+      for (int m = 0; m < M; ++m) {
+        const int row = taur[(size_t)k * M + m];
+        int j = 0;
+        while (j < n && info[1 + j] != row) ++j;
+        if (j == n) {
+          if (n < kStepMaxShift) info[1 + n] = row;
+          ++n;
+        }
+        sidx[(size_t)k * M + m] = j < kStepMaxShift ? j : 0;
+      }
+      for (int j = n; j < kStepMaxShift; ++j) info[1 + j] = 0;
+      info[0] = std::min(n, kStepMaxShift);
+      max_shift = std::max(max_shift, n);
+    }
+  }
+  const bool use_step = chunk_uses_step(c, B, max_shift);
   CK(cudaMemcpyAsync(c->plan_dev, hp, PL.total, cudaMemcpyHostToDevice, s));
   CK(cudaMemcpyAsync(c->noise, noise, (size_t)M * D * 4, cudaMemcpyDefault, s));
   if (c->use_graphs && !profile) {
-    const auto key = std::make_pair(B, steps);
+    const auto key = std::make_tuple(B, steps, use_step ? 1 : 0);
     auto it = c->graphs.find(key);
     if (it == c->graphs.end()) {
       cudaGraph_t g = nullptr;
       CK(cudaStreamBeginCapture(s, cudaStreamCaptureModeThreadLocal));
-      enqueue_chunk(c, B, steps, s);
+      enqueue_chunk(c, B, steps, use_step, s);
       cudaError_t e = cudaStreamEndCapture(s, &g);
       if (e != cudaSuccess) return fail(c, UAD_ECUDA, "graph capture failed: %s", cudaGetErrorString(e));
       cudaGraphExec_t ex = nullptr;
@@ -1157,7 +1195,7 @@ static int denoise_impl(uad_ctx* c, const float* noise, const uad_schedule* sc, 
     }
     cudaGraph_t g = nullptr;
     CK(cudaStreamBeginCapture(s, cudaStreamCaptureModeThreadLocal));
-    enqueue_chunk(c, B, steps, s);
+    enqueue_chunk(c, B, steps, use_step, s);
     cudaError_t e = cudaStreamEndCapture(s, &g);
     c->prof_on = false;
     if (e != cudaSuccess) return fail(c, UAD_ECUDA, "profile capture failed: %s", cudaGetErrorString(e));
@@ -1169,7 +1207,7 @@ static int denoise_impl(uad_ctx* c, const float* noise, const uad_schedule* sc, 
     cudaGraphExecDestroy(ex);
     if (e != cudaSuccess) return fail(c, UAD_ECUDA, "profile launch failed: %s", cudaGetErrorString(e));
   } else {
-    enqueue_chunk(c, B, steps, s);
+    enqueue_chunk(c, B, steps, use_step, s);
     CK(cudaGetLastError());
   }
   CK(cudaEventRecord(c->ev_done, s));

@@ -195,12 +195,19 @@ void launch_attn_tc(const AttnTcMaps& maps, const AttnTcArgs& a, cudaStream_t s)
 void launch_kv_prefix(const void* k, const void* v, int src_dtype, const AttnTcArgs& a, int robot, cudaStream_t s);
 
 // ---- persistent evaluation kernel (adaRMS experts, bf16, few tokens) ----------------------
-constexpr int kStepMaxRows = 64;      // B * H tokens per evaluation
+constexpr int kStepMaxRows = 64;      // tokens + distinct flow times per evaluation (MMA N side)
+constexpr int kStepMaxShift = 16;     // distinct flow times per evaluation
 constexpr int kStepMaxATiles = 8;     // weight tiles per CTA and projection
 constexpr int kStepMaxRing = 12;      // weight ring slots of 16 KB
 constexpr int kStepMaxChunks = 32;    // 64-key chunks per (robot, KV head)
-constexpr int kStepBarriersPerLayer = 10;
+constexpr int kStepMaxNB = 64;        // 128-row output blocks per projection
+constexpr int kStepBarriersPerLayer = 6;
 constexpr int kStepMaxWidth = 2048;   // model width, a multiple of 512
+// Per-launch synchronisation block (zeroed before every launch): grid-barrier counters,
+// per-output-block arrival counters, row sums of squares of the residual stream.
+__host__ __device__ constexpr size_t step_sync_words(int L) {
+  return (size_t)(1 + kStepBarriersPerLayer * L) + (size_t)L * 4 * kStepMaxNB + (size_t)(L + 1) * 2 * kStepMaxRows;
+}
 struct StepArgs {
   int M = 0, B = 0, H = 0, W = 0, F = 0, D = 0, L = 0;
   int qd = 0, kvd = 0, qkvd = 0, n_heads = 0, n_kv_heads = 0, group = 0, dh = 0;
@@ -209,13 +216,15 @@ struct StepArgs {
   int rope = 0;                        // q/k rows pair-interleaved per head, rotated by rope_cs
   float scale_log2 = 0.f;              // log2(e) / sqrt(dh)
   const int* tau_row = nullptr;        // [M] modulation row of each token at this step
+  const int* sidx = nullptr;           // [M] index of each token's flow time among the step's distinct ones
+  const int* sinfo = nullptr;          // [1 + kStepMaxShift]: count of distinct flow times, their rows
   const float* tab = nullptr; int rowlen = 0;
   const float* u = nullptr;            // [M][D] model input
   const void* w_in = nullptr; const float* b_in = nullptr;     // bf16 [W][D]
   const void* w_out = nullptr; const float* b_out = nullptr;   // bf16 [D][W]
   float* v = nullptr;                  // [M][D] velocity
   float* h = nullptr;                  // [M][W] residual stream
-  __nv_bfloat16* y = nullptr;          // [M][W] normalised rows
+  __nv_bfloat16* z = nullptr;          // [kStepMaxRows][W] projection input rows (see step_tc.cu)
   __nv_bfloat16* o = nullptr;          // [M][qd] attention output
   __nv_bfloat16* act = nullptr;        // [M][F] MLP activation
   float *acc_qkv = nullptr, *acc_o = nullptr, *acc_gu = nullptr, *acc_d = nullptr;  // zero between uses
@@ -223,13 +232,17 @@ struct StepArgs {
   __nv_bfloat16 *q = nullptr, *kcache = nullptr, *vtcache = nullptr;   // tensor-core attention layouts
   float *part_o = nullptr, *part_ml = nullptr;   // [B*Hkv][n_chunks][r_pad][dh], [..][2]
   const float* rope_cs = nullptr;      // [H][dh/2][cos, sin]
-  unsigned* bars = nullptr;            // [L * kStepBarriersPerLayer] grid-barrier counters, zeroed per launch
+  unsigned* sync = nullptr;            // step_sync_words(L) words, zeroed per launch
   int* err = nullptr;
 };
-struct StepMaps { CUtensorMap y, o, act, q, k, vt; };   // k: 64-key boxes
+struct StepMaps { CUtensorMap z, o, act, q, k, vt; };   // k: 64-key boxes
 size_t step_smem_bytes(int dh, int ring);
 int step_ring_slots(int dh, int smem_optin);           // ring slots that fit (may be < 3: unusable)
 int step_prepare(int dh, int ring, int* blocks_per_sm); // 0 on success
+// Tiles per CTA of the largest projection under the kernel's tile assignment (grid = `ctas`):
+// every CTA's tiles of a projection lie in one 128-row output block. 0 if a projection has
+// more output blocks than CTAs or than kStepMaxNB.
+int step_max_tiles(int ctas, const int (*shapes)[2], int n);
 int launch_step(const StepMaps& m, const StepArgs& a, int grid, cudaStream_t s);   // grid = SMs
 
 }  // namespace uad

@@ -295,7 +295,7 @@ def test_tensor_core_gemm_matches_cuda_core_gemm(monkeypatch):
 
 
 def test_step_kernel_matches_per_operation_kernels(monkeypatch):
-    """The persistent evaluation kernel (one launch per step, B * H <= 64) against
+    """The persistent evaluation kernel (one launch per step, few tokens) against
     the per-operation kernels on the same bf16 operands, and both against the oracle."""
     a = ARCHS["pi0_small"]
     blob = make_weights(a, seed=12)
@@ -318,16 +318,37 @@ def test_step_kernel_matches_per_operation_kernels(monkeypatch):
     assert np.array_equal(outs[1]["polled"][0][1], outs[0]["polled"][0][1])
 
 
+def kernel_names(c, noise, bud):
+    return {r["name"] for r in c.ex.profile(noise, bud)}
+
+
 def test_step_kernel_batched_robots():
-    """Four robots of 16 tokens (64 rows, the largest persistent-kernel launch), each with its
-    own prefix and schedule."""
+    """Three robots of 16 tokens, each with its own prefix and schedule, on the persistent kernel
+    (48 token rows plus one projection row per distinct flow time of a step)."""
     a = ARCHS["pi0_small"].replace(name="pi0_small_h16", chunk_len=16)
-    B = 4
+    B = 3
     c = Case(a, B=B, seed=13)
     try:
         assert c.ex.launches_per_chunk(B, 10) == 1 + 2 * 10
         noise = make_noise(a, batch=B, seed=13)
         bud = draw_sweep_schedules(a.chunk_len, B, seed=13)
+        assert "step_kernel" in kernel_names(c, noise, bud)
+        check(c, c.gpu(noise, bud), c.oracle(noise, bud), bud, TOL["bf16"])
+    finally:
+        c.close()
+
+
+def test_full_rows_fall_back_to_per_operation_kernels():
+    """Four robots of 16 tokens fill all 64 rows of the persistent kernel, leaving no room for
+    the per-flow-time rows: the chunk runs on the per-operation kernels, with the same results."""
+    a = ARCHS["pi0_small"].replace(name="pi0_small_h16", chunk_len=16)
+    B = 4
+    c = Case(a, B=B, seed=14)
+    try:
+        noise = make_noise(a, batch=B, seed=14)
+        bud = draw_sweep_schedules(a.chunk_len, B, seed=14)
+        names = kernel_names(c, noise, bud)
+        assert "step_kernel" not in names and "qkv_proj" in names
         check(c, c.gpu(noise, bud), c.oracle(noise, bud), bud, TOL["bf16"])
     finally:
         c.close()
