@@ -251,7 +251,7 @@ constexpr size_t kEpiBytes = (size_t)kMaxRows * 512 * 2 + (size_t)3 * kStepMaxSh
 __host__ __device__ constexpr size_t step_x_bytes(int dh) {
   const size_t a = (size_t)kMaxATiles * kATile;
   const size_t att = (size_t)dh * kQT * 2 + 2 * (size_t)dh * kKC * 2 + (size_t)kQT * kKC * 2;
-  const size_t ost = (size_t)kQT * (dh * 4 + 16);
+  const size_t ost = (size_t)kQT * (dh * 2 + 16);
   size_t m = a > att ? a : att;
   m = m > ost ? m : ost;
   return m > kEpiBytes ? m : kEpiBytes;
@@ -288,7 +288,7 @@ __host__ __device__ __forceinline__ Tiles assign_tiles(int cta, int G, int NB, i
   t.idx = cb <= KT ? i : t.k0;   // with more CTAs than k-blocks, each non-empty range is one k-block
   return t;
 }
-__host__ __device__ __forceinline__ int proj_rot(int l, int j) { return 41 * (4 * l + j); }
+__host__ __device__ __forceinline__ int proj_rot(int j) { return 41 * j; }
 
 struct Smem {
   uint8_t* ring;
@@ -299,6 +299,7 @@ struct Smem {
   int* flag;
   int* last;
   float* red;               // [8]
+  uint64_t* cbar;           // [4] per consumer warp: staging of a combine's partial rows
 };
 
 __device__ __forceinline__ Smem smem_plan(int R, size_t xbytes) {
@@ -322,6 +323,7 @@ __device__ __forceinline__ Smem smem_plan(int R, size_t xbytes) {
   S.flag = reinterpret_cast<int*>(S.tmem_slot + 1);
   S.last = S.flag + 1;
   S.red = reinterpret_cast<float*>(S.tmem_slot + 4);
+  S.cbar = reinterpret_cast<uint64_t*>(S.red + 8);
   return S;
 }
 
@@ -332,6 +334,8 @@ struct Role {
   uint32_t par = 0;
   uint32_t apar = 0, gpar = 0, ipar = 0;   // a_full, g_done, per-attention-item barriers
   int a_uses = 0, i_uses = 0;        // loads issued on a_full and on q_full / v_full
+  uint32_t cpar = 0;                 // this consumer warp's combine barrier
+  int c_uses = 0;
 };
 
 // Step values shared by the CTA's threads: this step's distinct flow times and each token's.
@@ -340,6 +344,8 @@ struct StepShared {
   int nsh;                           // distinct flow times (shift rows of z)
   int srow[kStepMaxShift];           // their modulation-table rows
   int sidx[kMaxRows];                // token -> index of its flow time
+  Tiles tiles[4];                    // this CTA's tiles of the qkv, o, gate/up, down projections
+  int fused_combine;                 // idle CTAs of the attention step merge the key chunks
 };
 
 // Grid barrier among warps 0-3 and 5 of every CTA: every CTA arrives (also after an error, so
@@ -413,6 +419,11 @@ __device__ __forceinline__ float cons_sum(float v, float* red) {
 __device__ __forceinline__ float* sumsq_slot(const StepArgs& __restrict__ p, int l, int which) {
   return reinterpret_cast<float*>(p.sync + (1 + kStepBarriersPerLayer * p.L) + (size_t)p.L * 4 * kStepMaxNB) +
          (size_t)(2 * l + which) * kMaxRows;
+}
+// Count of finished key chunks of query tile t (robot-group x 128-row tile) in layer l.
+__device__ __forceinline__ unsigned* qtile_ctr(const StepArgs& __restrict__ p, int l, int t) {
+  return p.sync + (1 + kStepBarriersPerLayer * p.L) + (size_t)p.L * 4 * kStepMaxNB + (size_t)(p.L + 1) * 2 * kMaxRows +
+         (size_t)l * kStepMaxQTiles + t;
 }
 __device__ __forceinline__ const float* mod_row(const StepArgs& __restrict__ p, int row) {
   return p.tab + (size_t)row * p.rowlen;
@@ -634,51 +645,103 @@ __device__ __noinline__ void epi_resid(const StepShared& __restrict__ sh, float*
   }
 }
 
-// Merge the key chunks of the query rows assigned to this consumer warp: the warp stages the
-// row's partial O of every chunk in shared memory (one round of loads), then combines.
+// Merge the key chunks of query rows (one warp): lane c < n_chunks copies chunk c's partial row
+// into shared memory with one bulk copy (up to two rows at once), the weights exp(max_c - max)
+// and the total sum are formed meanwhile, then each lane loads its dims of every chunk before
+// accumulating. Lane owns dims 2 lane + 64 e, e < DH / 64. Rows r0, r0 + step, ... < r1 of
+// robot-group bg.
 template <int DH>
-__device__ __noinline__ void combine_rows(const StepArgs& __restrict__ p, uint8_t* X) {
-  constexpr int E = DH / 32;
-  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  const int gw = blockIdx.x * 4 + w, nw = gridDim.x * 4;
-  const int nck = p.n_chunks, total = p.B * p.n_kv_heads * p.rows;
-  float* buf = reinterpret_cast<float*>(X) + (size_t)w * kStepMaxChunks * DH;
+__device__ __forceinline__ void combine_rows_warp(const StepArgs& __restrict__ p, int bg, int r0, int r1, int step,
+                                                  __nv_bfloat16* buf, uint64_t* bar, Role& st) {
+  constexpr int E = DH / 64, kG = 8;
+  const int lane = threadIdx.x & 31, nck = p.n_chunks;
+  constexpr int kRows = 2;                  // rows staged at once (two when n_chunks <= 16)
+  const int batch = nck * kRows <= kStepMaxChunks ? kRows : 1;
 #pragma unroll 1
-  for (int idx = gw; idx < total; idx += nw) {
-    const int bg = idx / p.rows, r = idx % p.rows;
-    const float* src = p.part_o + ((size_t)bg * nck * p.r_pad + r) * DH;
-#pragma unroll 1
-    for (int i = lane; i < nck * (DH / 4); i += 32) {
-      const int cc = i / (DH / 4), q = i % (DH / 4);
-      cp16(buf + cc * DH + q * 4, src + (size_t)cc * p.r_pad * DH + q * 4);
-    }
-    float mc = -INFINITY, lc = 0.f;
+  for (int rb = r0; rb < r1; rb += batch * step) {
+    int nr = 0;
+    for (int r = rb; r < r1 && nr < batch; r += step) ++nr;
+    if (lane == 0) mbar_expect_tx(bar, (uint32_t)(nr * nck * DH * 2));
+    __syncwarp();
     if (lane < nck) {
-      const size_t pi = ((size_t)bg * nck + lane) * p.r_pad + r;
-      mc = __ldcg(p.part_ml + pi * 2);
-      lc = __ldcg(p.part_ml + pi * 2 + 1);
+      // partial rows written by other CTAs (acquired through the chunk count) are read next by
+      // this lane's bulk copies
+      asm volatile("fence.proxy.async.global;" ::: "memory");
+      for (int k = 0; k < nr; ++k) {
+        const __nv_bfloat16* src = p.part_o + (((size_t)bg * nck + lane) * p.r_pad + rb + k * step) * DH;
+        asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                     ::"r"(su32(buf + ((size_t)k * nck + lane) * DH)), "l"(src), "r"(DH * 2), "r"(su32(bar)) : "memory");
+      }
     }
-    const float M = warp_max(mc);
-    const float wgt = lane < nck ? exp2f((mc - M) * p.scale_log2) : 0.f;
-    const float L = warp_sum(wgt * lc);
-    cp_wait_all();
-    __syncwarp();
-    float acc[E];
+    ++st.c_uses;
+    float mc[kRows], lc[kRows];
 #pragma unroll
-    for (int e = 0; e < E; ++e) acc[e] = 0.f;
-#pragma unroll 2
-    for (int cc = 0; cc < nck; ++cc) {
-      const float wc = __shfl_sync(0xffffffffu, wgt, cc);
+    for (int k = 0; k < kRows; ++k) {
+      mc[k] = -INFINITY;
+      lc[k] = 0.f;
+      if (k < nr && lane < nck) {
+        const size_t pi = ((size_t)bg * nck + lane) * p.r_pad + rb + k * step;
+        mc[k] = __ldcg(p.part_ml + pi * 2);
+        lc[k] = __ldcg(p.part_ml + pi * 2 + 1);
+      }
+    }
+    float wgt[kRows], invL[kRows];
 #pragma unroll
-      for (int e = 0; e < E; ++e) acc[e] = fmaf(wc, buf[cc * DH + e * 32 + lane], acc[e]);
+    for (int k = 0; k < kRows; ++k) {
+      const float M = warp_max(mc[k]);
+      wgt[k] = lane < nck && k < nr ? exp2f((mc[k] - M) * p.scale_log2) : 0.f;
+      invL[k] = 1.f / warp_sum(wgt[k] * lc[k]);
+    }
+    const bool ok = mbar_wait(bar, st.cpar, p.err, 53);
+    st.cpar ^= 1u;
+#pragma unroll 1
+    for (int k = 0; k < nr && ok; ++k) {
+      const int r = rb + k * step;
+      const __nv_bfloat16* row = buf + (size_t)k * nck * DH;
+      const float wk = k ? wgt[1] : wgt[0], ik = k ? invL[1] : invL[0];
+      float2 acc[E];
+#pragma unroll
+      for (int e = 0; e < E; ++e) acc[e] = make_float2(0.f, 0.f);
+#pragma unroll 1
+      for (int c0 = 0; c0 < nck; c0 += kG) {
+        __nv_bfloat162 v[kG][E];
+#pragma unroll
+        for (int g = 0; g < kG; ++g)
+#pragma unroll
+          for (int e = 0; e < E; ++e)
+            v[g][e] = c0 + g < nck ? *reinterpret_cast<const __nv_bfloat162*>(row + (c0 + g) * DH + 64 * e + 2 * lane)
+                                   : __floats2bfloat162_rn(0.f, 0.f);
+#pragma unroll
+        for (int g = 0; g < kG; ++g) {
+          const float wc = __shfl_sync(0xffffffffu, wk, (c0 + g) & 31);
+#pragma unroll
+          for (int e = 0; e < E; ++e) {
+            const float2 f = __bfloat1622float2(v[g][e]);
+            acc[e].x = fmaf(wc, f.x, acc[e].x);
+            acc[e].y = fmaf(wc, f.y, acc[e].y);
+          }
+        }
+      }
+      const int b = bg / p.n_kv_heads, g = bg % p.n_kv_heads, j = r / p.H, i = r % p.H;
+      __nv_bfloat16* dst = p.o + ((size_t)b * p.H + i) * p.qd + (size_t)(g * p.group + j) * DH;
+#pragma unroll
+      for (int e = 0; e < E; ++e)
+        *reinterpret_cast<uint32_t*>(dst + 64 * e + 2 * lane) = pack_bf16(acc[e].x * ik, acc[e].y * ik);
     }
     __syncwarp();
-    const int b = bg / p.n_kv_heads, g = bg % p.n_kv_heads, j = r / p.H, i = r % p.H;
-    __nv_bfloat16* dst = p.o + ((size_t)b * p.H + i) * p.qd + (size_t)(g * p.group + j) * DH;
-    const float invL = 1.f / L;
-#pragma unroll
-    for (int e = 0; e < E; ++e) dst[e * 32 + lane] = __float2bfloat16_rn(acc[e] * invL);
+    if (!ok) break;
   }
+}
+
+// Combine step (when the attention step does not merge the chunks itself): query rows over all
+// consumer warps of the grid.
+template <int DH>
+__device__ __noinline__ void combine_rows(const StepArgs& __restrict__ p, uint8_t* X, uint64_t* bar, Role& st) {
+  const int w = threadIdx.x >> 5, gw = blockIdx.x * 4 + w, nw = gridDim.x * 4;
+  __nv_bfloat16* buf = reinterpret_cast<__nv_bfloat16*>(X) + (size_t)w * kStepMaxChunks * DH;
+  const int total = p.B * p.n_kv_heads * p.rows;
+#pragma unroll 1
+  for (int idx = gw; idx < total; idx += nw) combine_rows_warp<DH>(p, idx / p.rows, idx % p.rows, idx % p.rows + 1, 1, buf, bar, st);
 }
 
 }  // namespace
@@ -693,12 +756,10 @@ __device__ __noinline__ void projection_step(const StepShared& __restrict__ sh, 
   const Smem S = smem_plan(p.ring, xbytes);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const bool mma = threadIdx.x == 160, cons = warp < 4;
-  int N, K;
-  proj_shape(p, j, N, K);
-  const int KT = K / 64;
-  const Tiles tl = assign_tiles(blockIdx.x, gridDim.x, N / 128, KT, proj_rot(l, j));
+  const Tiles tl = sh.tiles[j];
   const int nt = tl.k1 - tl.k0;
   if (nt <= 0) return;
+  const int N = j == 0 ? p.qkvd : j == 2 ? 2 * p.F : p.W;
   float* acc = j == 0 ? p.acc_qkv : j == 1 ? p.acc_o : j == 2 ? p.acc_gu : p.acc_d;
   const int R = (j == 0 || j == 2) ? p.M + sh.nsh : p.M;   // rows added: tokens (+ shift rows)
   if (mma) {
@@ -775,7 +836,7 @@ __device__ __noinline__ void projection_step(const StepShared& __restrict__ sh, 
 // ---- attention step: items (robot-group bg, 128-row query tile qt, 64-key chunk kc) ---------
 template <int DH>
 __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, const CUtensorMap* t_q, const CUtensorMap* t_k,
-                                            const CUtensorMap* t_vt, int l, uint32_t tmem, Role& st) {
+                                            const CUtensorMap* t_vt, int l, uint32_t tmem, Role& st, bool fused) {
   constexpr int NC = DH / 64;
   constexpr uint32_t QB = DH * kQT * 2, KB = DH * kKC * 2, VB = DH * kKC * 2;
   const Smem S = smem_plan(p.ring, step_x_bytes(DH));
@@ -787,6 +848,23 @@ __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, cons
   const bool mma = threadIdx.x == 160, cons = warp < 4;
   const int nck = p.n_chunks, nqt = p.r_pad / kQT;
   const int items = p.B * p.n_kv_heads * nqt * nck;
+  if (fused && (int)blockIdx.x >= items) {
+    // CTAs without an item merge the key chunks: each takes a share of one query tile's rows
+    // and starts once all chunks of that tile have finished
+    if (cons) {
+      const int ncomb = gridDim.x - items, ci = (int)blockIdx.x - items, QT = p.B * p.n_kv_heads * nqt;
+      const int t = ci * QT / ncomb, first = (t * ncomb + QT - 1) / QT, next = ((t + 1) * ncomb + QT - 1) / QT;
+      const int bg = t / nqt, qt = t % nqt, rows = min(kQT, p.rows - qt * kQT);
+      const int r0 = qt * kQT + (ci - first) * rows / (next - first), r1 = qt * kQT + (ci - first + 1) * rows / (next - first);
+      if (threadIdx.x == 0) *S.last = count_wait(qtile_ctr(p, l, t), (unsigned)nck, p.err);
+      named_sync(2, 128);
+      if (*reinterpret_cast<volatile int*>(S.last)) {
+        __nv_bfloat16* buf = reinterpret_cast<__nv_bfloat16*>(S.X) + (size_t)warp * kStepMaxChunks * DH;
+        combine_rows_warp<DH>(p, bg, r0 + warp, r1, 4, buf, S.cbar + warp, st);
+      }
+    }
+    return;
+  }
   for (int it = blockIdx.x; it < items; it += gridDim.x) {
     const int kc = it % nck, qt = (it / nck) % nqt, bg = it / (nck * nqt);
     const int b = bg / p.n_kv_heads, g = bg % p.n_kv_heads;
@@ -866,31 +944,37 @@ __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, cons
       const bool ok_o = mbar_wait(S.o_done, st.ipar, p.err, 49);
       tc_fence_after();
       const uint32_t tO = tmem_base_after_wait(S.tmem_slot) + 256;
-      // unnormalised O row: staged in shared memory (the operand tiles are free once O is
-      // complete; rows padded by 16 bytes against bank conflicts), then written by one bulk copy
-      // per row, complete before the step's barrier
+      // unnormalised O row in bf16: staged in shared memory (the operand tiles are free once O
+      // is complete; rows padded by 16 bytes against bank conflicts), then written by one bulk
+      // copy per row, complete before the chunk is counted
       const int qrow = qt * kQT + row;
       const size_t pi = ((size_t)bg * nck + kc) * p.r_pad + qrow;
-      constexpr uint32_t pitch = DH * 4 + 16;
+      constexpr uint32_t pitch = DH * 2 + 16;
       uint8_t* srow = S.X + (size_t)row * pitch;
-#pragma unroll
+#pragma unroll 2
       for (int q = 0; q < DH; q += 32) {
         float ov[32];
         __syncwarp();
         tmem_ld32(tO + lane_base + q, ov);
 #pragma unroll
-        for (int e = 0; e < 32; e += 4)
-          *reinterpret_cast<float4*>(srow + (q + e) * 4) = make_float4(ov[e], ov[e + 1], ov[e + 2], ov[e + 3]);
+        for (int e = 0; e < 32; e += 8)
+          *reinterpret_cast<uint4*>(srow + (q + e) * 2) = make_uint4(pack_bf16(ov[e], ov[e + 1]), pack_bf16(ov[e + 2], ov[e + 3]),
+                                                                     pack_bf16(ov[e + 4], ov[e + 5]), pack_bf16(ov[e + 6], ov[e + 7]));
       }
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       if (ok_s && ok_o && qrow < p.rows) {
-        bulk_s2g(p.part_o + pi * DH, srow, DH * 4);
+        bulk_s2g(p.part_o + pi * DH, srow, DH * 2);
         asm volatile("cp.async.bulk.commit_group;" ::: "memory");
         p.part_ml[pi * 2] = mx;
         p.part_ml[pi * 2 + 1] = l_sum;
         asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
         asm volatile("fence.proxy.async.global;" ::: "memory");
       }
+      // count the chunk for its query tile (release: every consumer's rows, ordered before by the
+      // named barrier)
+      named_sync(2, 128);
+      if (threadIdx.x == 0 && ok_s && ok_o)
+        asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(qtile_ctr(p, l, bg * nqt + qt)) : "memory");
     }
     st.ipar ^= 1u;
     // the next item's operand loads overwrite this item's operands and P
@@ -955,11 +1039,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(S.empty + i, 1);
     }
     for (int i = 0; i < 8; ++i) mbar_init(S.a_full + i, i == 5 ? 4 : 1);   // p_full: one arrive per consumer warp
+    for (int i = 0; i < 4; ++i) mbar_init(S.cbar + i, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (threadIdx.x < kMaxRows) {
     const int si = threadIdx.x < p_in.M ? __ldg(p_in.sidx + threadIdx.x) : 0;
     sh.sidx[threadIdx.x] = si >= 0 && si < kStepMaxShift ? si : 0;
+  }
+  if (threadIdx.x == 68) {
+    const int items = p_in.B * p_in.n_kv_heads * (p_in.r_pad / kQT) * p_in.n_chunks;
+    const int qtiles = p_in.B * p_in.n_kv_heads * (p_in.r_pad / kQT);
+    sh.fused_combine = (int)gridDim.x - items >= (qtiles > 16 ? qtiles : 16) ? 1 : 0;
+  }
+  if (threadIdx.x >= 64 && threadIdx.x < 68) {
+    const int j = threadIdx.x - 64;
+    int N, K;
+    proj_shape(p_in, j, N, K);
+    sh.tiles[j] = assign_tiles(blockIdx.x, gridDim.x, N / 128, K / 64, proj_rot(j));
   }
   if (warp == 0) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(S.tmem_slot)), "r"(kTmemCols));
@@ -982,9 +1078,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int j = 0; j < 4 && ok; ++j) {
           int N, K;
           proj_shape(p, j, N, K);
-          const int KT = K / 64;
-          const Tiles tl = assign_tiles(blockIdx.x, gridDim.x, N / 128, KT, proj_rot(l, j));
-          const uint8_t* w = static_cast<const uint8_t*>(p.wl[4 * l + j]) + ((size_t)tl.b * KT + tl.k0) * kSlot;
+          const Tiles tl = sh.tiles[j];
+          const uint8_t* w = static_cast<const uint8_t*>(p.wl[4 * l + j]) + ((size_t)tl.b * (K / 64) + tl.k0) * kSlot;
           for (int t = 0; t < tl.k1 - tl.k0; ++t) {
             if (!mbar_wait(S.empty + slot, par ^ 1u, p.err, 41)) { ok = false; break; }
             mbar_expect_tx(S.full + slot, kSlot);
@@ -1008,13 +1103,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int l = 0; l < p.L; ++l) {
       if (ok) projection_step(sh, &t_z, l, 0, tmem, XB, st);
       ok = grid_sync(bar++, ok, p.err, S);
-      if (ok) attention_step<DH>(p, &t_q, &t_k, &t_vt, l, tmem, st);
-      ok = grid_sync(bar++, ok, p.err, S);
-      if (ok && cons) {
-        clear_shift_rows(sh, true, l > 0);
-        combine_rows<DH>(p, S.X);
+      if (ok) {
+        if (cons) clear_shift_rows(sh, true, l > 0);
+        attention_step<DH>(p, &t_q, &t_k, &t_vt, l, tmem, st, sh.fused_combine != 0);
       }
       ok = grid_sync(bar++, ok, p.err, S);
+      if (!sh.fused_combine) {
+        if (ok && cons) combine_rows<DH>(p, S.X, S.cbar + warp, st);
+        ok = grid_sync(bar++, ok, p.err, S);
+      }
       if (ok) projection_step(sh, &t_o, l, 1, tmem, XB, st);
       ok = grid_sync(bar++, ok, p.err, S);
       if (ok) projection_step(sh, &t_z, l, 2, tmem, XB, st);
@@ -1024,6 +1121,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (ok && cons) clear_shift_rows(sh, false, true);
     if (ok && cons && (int)blockIdx.x < p.M) final_row(p, blockIdx.x, reinterpret_cast<float*>(S.X));
+    // a consumer warp exits only after its last combine copies have landed
+    if (cons && st.c_uses) mbar_drain(S.cbar + warp, (uint32_t)(st.c_uses - 1) & 1u);
     if (mma) {
       // tensor memory is freed only after every MMA of this thread has completed, and the CTA
       // exits only after its last operand loads have landed (they are waited for on the normal

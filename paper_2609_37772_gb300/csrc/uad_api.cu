@@ -450,6 +450,8 @@ const char* step_unfit(uad_ctx* c, int* ring) {
   if (a.action_dim % 8) return "action dim";
   if (dh != 64 && dh != 128 && dh != 256) return "head dim";
   if ((c->at0.n_keys + 63) / 64 > kStepMaxChunks) return "too many keys";
+  const int bmax = std::min(a.max_batch, kStepMaxRows / a.chunk_len);
+  if (bmax * a.n_kv_heads * (c->at0.r_pad / 128) > kStepMaxQTiles) return "too many query tiles";
   const int shapes[4][2] = {{c->qkvd, W}, {W, c->qd}, {2 * F, W}, {W, F}};
   for (auto& sh : shapes)
     if (sh[0] % 128 || sh[1] % 64) return "projection shape";

@@ -201,12 +201,15 @@ constexpr int kStepMaxATiles = 8;     // weight tiles per CTA and projection
 constexpr int kStepMaxRing = 12;      // weight ring slots of 16 KB
 constexpr int kStepMaxChunks = 32;    // 64-key chunks per (robot, KV head)
 constexpr int kStepMaxNB = 64;        // 128-row output blocks per projection
+constexpr int kStepMaxQTiles = 64;    // (robot, KV head, 128-row query tile) triples per evaluation
 constexpr int kStepBarriersPerLayer = 6;
 constexpr int kStepMaxWidth = 2048;   // model width, a multiple of 512
 // Per-launch synchronisation block (zeroed before every launch): grid-barrier counters,
-// per-output-block arrival counters, row sums of squares of the residual stream.
+// per-output-block arrival counters, row sums of squares of the residual stream, per-query-tile
+// counts of finished attention chunks.
 __host__ __device__ constexpr size_t step_sync_words(int L) {
-  return (size_t)(1 + kStepBarriersPerLayer * L) + (size_t)L * 4 * kStepMaxNB + (size_t)(L + 1) * 2 * kStepMaxRows;
+  return (size_t)(1 + kStepBarriersPerLayer * L) + (size_t)L * 4 * kStepMaxNB + (size_t)(L + 1) * 2 * kStepMaxRows +
+         (size_t)L * kStepMaxQTiles;
 }
 struct StepArgs {
   int M = 0, B = 0, H = 0, W = 0, F = 0, D = 0, L = 0;
@@ -230,7 +233,8 @@ struct StepArgs {
   float *acc_qkv = nullptr, *acc_o = nullptr, *acc_gu = nullptr, *acc_d = nullptr;  // zero between uses
   const void* const* wl = nullptr;     // [L][4] tiled weights: qkv, o, gate/up, down
   __nv_bfloat16 *q = nullptr, *kcache = nullptr, *vtcache = nullptr;   // tensor-core attention layouts
-  float *part_o = nullptr, *part_ml = nullptr;   // [B*Hkv][n_chunks][r_pad][dh], [..][2]
+  __nv_bfloat16* part_o = nullptr;     // [B*Hkv][n_chunks][r_pad][dh] unnormalised partial O rows
+  float* part_ml = nullptr;            // [B*Hkv][n_chunks][r_pad][2] (max, sum) of each partial row
   const float* rope_cs = nullptr;      // [H][dh/2][cos, sin]
   unsigned* sync = nullptr;            // step_sync_words(L) words, zeroed per launch
   int* err = nullptr;
