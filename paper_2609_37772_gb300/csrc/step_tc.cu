@@ -48,7 +48,12 @@ namespace {
 constexpr int kSlot = 16384;         // weight tile: 128 rows x 64 bf16, 128-byte swizzled
 constexpr int kATile = 8192;         // activation tile: 64 tokens x 64 bf16
 constexpr int kQT = 128, kKC = 64;   // attention: query rows per tile, keys per chunk
-constexpr int kThreads = 192;
+constexpr int kConsWarps = 8;                      // consumer warps 0-7
+constexpr int kCons = 32 * kConsWarps;              // consumer threads
+constexpr int kProdWarp = kConsWarps;               // weight producer (lane 0)
+constexpr int kMmaThread = 32 * (kConsWarps + 1);   // tcgen05 issuer and TMA loads (lane 0 of the last warp)
+constexpr int kThreads = kMmaThread + 32;
+constexpr int kSyncThreads = kCons + 32;            // consumers and the issuer's warp
 constexpr int kMaxRows = kStepMaxRows;   // tokens per evaluation (the N side of every MMA)
 constexpr int kMaxATiles = kStepMaxATiles;
 constexpr int kMaxRing = kStepMaxRing;
@@ -299,7 +304,7 @@ struct Smem {
   int* flag;
   int* last;
   float* red;               // [8]
-  uint64_t* cbar;           // [4] per consumer warp: staging of a combine's partial rows
+  uint64_t* cbar;           // [kConsWarps] per consumer warp: staging of a combine's partial rows
 };
 
 __device__ __forceinline__ Smem smem_plan(int R, size_t xbytes) {
@@ -348,14 +353,14 @@ struct StepShared {
   int fused_combine;                 // idle CTAs of the attention step merge the key chunks
 };
 
-// Grid barrier among warps 0-3 and 5 of every CTA: every CTA arrives (also after an error, so
-// that no CTA waits for it), then thread 160 spins on the counter. Returns false once any error is
+// Grid barrier among the consumer warps and the issuer's warp of every CTA: every CTA arrives (also
+// after an error, so that no CTA waits for it), then the issuer thread spins on the counter. Returns false once any error is
 // recorded, so that the remaining steps are skipped.
 __device__ __noinline__ bool grid_sync(unsigned* ctr, bool ok, int* err, const Smem& S) {
   tc_fence_before();
   __syncwarp();
-  named_sync(1, 160);
-  if (threadIdx.x == 160) {
+  named_sync(1, kSyncThreads);
+  if (threadIdx.x == kMmaThread) {
     bool good = ok && *reinterpret_cast<volatile int*>(err) == 0;
     // release arrival: the CTA's writes (ordered before this thread by the named barrier)
     // are visible at GPU scope to whoever observes the count
@@ -382,7 +387,7 @@ __device__ __noinline__ bool grid_sync(unsigned* ctr, bool ok, int* err, const S
     *S.flag = good ? 1 : 0;
   }
   __syncwarp();
-  named_sync(1, 160);
+  named_sync(1, kSyncThreads);
   tc_fence_after();
   return *reinterpret_cast<volatile int*>(S.flag) != 0;
 }
@@ -405,14 +410,16 @@ __device__ __noinline__ int count_wait(const unsigned* ctr, unsigned target, int
   }
 }
 
-// Sum over the 128 consumer threads (warps 0-3); every consumer gets the total.
+// Sum over the consumer threads; every consumer gets the total.
 __device__ __forceinline__ float cons_sum(float v, float* red) {
   v = warp_sum(v);
   const int w = threadIdx.x >> 5;
   if ((threadIdx.x & 31) == 0) red[w] = v;
-  named_sync(2, 128);
-  const float t = (red[0] + red[1]) + (red[2] + red[3]);
-  named_sync(2, 128);
+  named_sync(2, kCons);
+  float t = 0.f;
+#pragma unroll
+  for (int i = 0; i < kConsWarps; ++i) t += red[i];
+  named_sync(2, kCons);
   return t;
 }
 
@@ -442,7 +449,7 @@ __device__ __noinline__ void in_rows(const StepShared& __restrict__ sh, float* r
     const int D8 = p.D / 8;
     float ss = 0.f;
 #pragma unroll 1
-    for (int c4 = tid; c4 < W / 4; c4 += 128) {
+    for (int c4 = tid; c4 < W / 4; c4 += kCons) {
       const float4 b = __ldg(reinterpret_cast<const float4*>(p.b_in) + c4);
       float o[4] = {b.x, b.y, b.z, b.w};
 #pragma unroll 1
@@ -473,7 +480,7 @@ __device__ __noinline__ void in_rows(const StepShared& __restrict__ sh, float* r
   } else if (c < p.M + sh.nsh) {
     const float* shift = mod_row(p, sh.srow[c - p.M]) + W;
 #pragma unroll 1
-    for (int c4 = tid; c4 < W / 4; c4 += 128) {
+    for (int c4 = tid; c4 < W / 4; c4 += kCons) {
       const float4 s = __ldg(reinterpret_cast<const float4*>(shift) + c4);
       st_bf16x4(p.z + (size_t)c * W + 4 * c4, s.x, s.y, s.z, s.w);
     }
@@ -487,14 +494,14 @@ __device__ __noinline__ void in_rows(const StepShared& __restrict__ sh, float* r
 // every share reads, are cleared in a later phase (clear_shift_rows).
 __device__ __forceinline__ void stage_rows(float* A, const float* src, int N, int c0, int r0, int r1) {
 #pragma unroll 1
-  for (int i = threadIdx.x; i < (r1 - r0) * 32; i += 128) {
+  for (int i = threadIdx.x; i < (r1 - r0) * 32; i += kCons) {
     const int m = r0 + (i >> 5);
     cp16(A + m * 128 + (i & 31) * 4, src + (size_t)m * N + c0 + (i & 31) * 4);
   }
 }
 __device__ __forceinline__ void clear_rows(float* acc, int N, int c0, int r0, int r1) {
 #pragma unroll 1
-  for (int i = threadIdx.x; i < (r1 - r0) * 32; i += 128)
+  for (int i = threadIdx.x; i < (r1 - r0) * 32; i += kCons)
     __stcg(reinterpret_cast<float4*>(acc + (size_t)(r0 + (i >> 5)) * N + c0) + (i & 31), make_float4(0.f, 0.f, 0.f, 0.f));
 }
 // Clears the shift rows of the qkv accumulator (this layer) and of the gate/up accumulator
@@ -504,7 +511,7 @@ __device__ __forceinline__ void clear_shift_rows(const StepShared& __restrict__ 
   const int nq = qkv ? sh.nsh * p.qkvd / 4 : 0, ng = gu ? sh.nsh * 2 * p.F / 4 : 0;
   const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll 1
-  for (int i = blockIdx.x * 128 + threadIdx.x; i < nq + ng; i += gridDim.x * 128) {
+  for (int i = blockIdx.x * kCons + threadIdx.x; i < nq + ng; i += gridDim.x * kCons) {
     if (i < nq) __stcg(reinterpret_cast<float4*>(p.acc_qkv + (size_t)p.M * p.qkvd) + i, zero);
     else __stcg(reinterpret_cast<float4*>(p.acc_gu + (size_t)p.M * 2 * p.F) + (i - nq), zero);
   }
@@ -526,16 +533,16 @@ __device__ __noinline__ void epi_qkv(const StepShared& __restrict__ sh, int l, i
   const int sn = n < p.qd ? n : n - p.qd;
   if (qk && p.rope) {
 #pragma unroll 1
-    for (int m = r0 + warp; m < r1; m += 4)
+    for (int m = r0 + warp; m < r1; m += kConsWarps)
       cp16(CS + m * 128 + 4 * lane, p.rope_cs + (size_t)(m % p.H) * dh + ((sn % dh) >> 1) * 2);
   }
   const float* s1 = sumsq_slot(p, l, 0);
-  for (int m = r0 + threadIdx.x; m < r1; m += 128) rs[m] = rsqrtf(__ldcg(s1 + m) / p.W + 1e-6f);
+  for (int m = r0 + threadIdx.x; m < r1; m += kCons) rs[m] = rsqrtf(__ldcg(s1 + m) / p.W + 1e-6f);
   cp_wait_all();
   clear_rows(p.acc_qkv, p.qkvd, c0, r0, r1);
-  named_sync(2, 128);
+  named_sync(2, kCons);
 #pragma unroll 1
-  for (int m = r0 + warp; m < r1; m += 4) {
+  for (int m = r0 + warp; m < r1; m += kConsWarps) {
     const float r = rs[m];
     const float4 a = *reinterpret_cast<const float4*>(A + m * 128 + 4 * lane);
     const float4 s = *reinterpret_cast<const float4*>(A + (M + sh.sidx[m]) * 128 + 4 * lane);
@@ -577,12 +584,12 @@ __device__ __noinline__ void epi_geglu(const StepShared& __restrict__ sh, int l,
   stage_rows(A, p.acc_gu, 2 * p.F, c0, r0, r1);
   stage_rows(A, p.acc_gu, 2 * p.F, c0, M, M + sh.nsh);
   const float* s2 = sumsq_slot(p, l, 1);
-  for (int m = r0 + threadIdx.x; m < r1; m += 128) rs[m] = rsqrtf(__ldcg(s2 + m) / p.W + 1e-6f);
+  for (int m = r0 + threadIdx.x; m < r1; m += kCons) rs[m] = rsqrtf(__ldcg(s2 + m) / p.W + 1e-6f);
   cp_wait_all();
   clear_rows(p.acc_gu, 2 * p.F, c0, r0, r1);
-  named_sync(2, 128);
+  named_sync(2, kCons);
 #pragma unroll 1
-  for (int m = r0 + warp; m < r1; m += 4) {
+  for (int m = r0 + warp; m < r1; m += kConsWarps) {
     const float r = rs[m];
     const float4 a = *reinterpret_cast<const float4*>(A + m * 128 + 4 * lane);
     const float4 s = *reinterpret_cast<const float4*>(A + (M + sh.sidx[m]) * 128 + 4 * lane);
@@ -609,16 +616,16 @@ __device__ __noinline__ void epi_resid(const StepShared& __restrict__ sh, float*
   stage_rows(Hs, p.h, W, c0, r0, r1);
   const int nv = next_mod >= 0 ? 3 : 1;
 #pragma unroll 1
-  for (int i = tid; i < nv * nsh * 32; i += 128) {
+  for (int i = tid; i < nv * nsh * 32; i += kCons) {
     const int kind = i / (nsh * 32), j = (i / 32) % nsh, q = i & 31;
     const int off = kind == 0 ? gate_off : next_mod + (kind - 1) * W;
     cp16(G + (kind * kStepMaxShift + j) * 128 + q * 4, mod_row(p, sh.srow[j]) + off + c0 + q * 4);
   }
   cp_wait_all();
   clear_rows(acc, W, c0, r0, r1);
-  named_sync(2, 128);
+  named_sync(2, kCons);
 #pragma unroll 1
-  for (int m = r0 + warp; m < r1; m += 4) {
+  for (int m = r0 + warp; m < r1; m += kConsWarps) {
     const int j = sh.sidx[m];
     const float4 a = *reinterpret_cast<const float4*>(A + m * 128 + 4 * lane);
     float4 h = *reinterpret_cast<const float4*>(Hs + m * 128 + 4 * lane);
@@ -638,7 +645,7 @@ __device__ __noinline__ void epi_resid(const StepShared& __restrict__ sh, float*
   }
   if (next_mod >= 0 && first) {
 #pragma unroll 1
-    for (int j = warp; j < nsh; j += 4) {
+    for (int j = warp; j < nsh; j += kConsWarps) {
       const float4 s = *reinterpret_cast<const float4*>(Sh + j * 128 + 4 * lane);
       st_bf16x4(p.z + (size_t)(M + j) * W + c0 + 4 * lane, s.x, s.y, s.z, s.w);
     }
@@ -737,7 +744,7 @@ __device__ __forceinline__ void combine_rows_warp(const StepArgs& __restrict__ p
 // consumer warps of the grid.
 template <int DH>
 __device__ __noinline__ void combine_rows(const StepArgs& __restrict__ p, uint8_t* X, uint64_t* bar, Role& st) {
-  const int w = threadIdx.x >> 5, gw = blockIdx.x * 4 + w, nw = gridDim.x * 4;
+  const int w = threadIdx.x >> 5, gw = blockIdx.x * kConsWarps + w, nw = gridDim.x * kConsWarps;
   __nv_bfloat16* buf = reinterpret_cast<__nv_bfloat16*>(X) + (size_t)w * kStepMaxChunks * DH;
   const int total = p.B * p.n_kv_heads * p.rows;
 #pragma unroll 1
@@ -755,7 +762,7 @@ __device__ __noinline__ void projection_step(const StepShared& __restrict__ sh, 
   const StepArgs& p = sh.p;
   const Smem S = smem_plan(p.ring, xbytes);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const bool mma = threadIdx.x == 160, cons = warp < 4;
+  const bool mma = threadIdx.x == kMmaThread, cons = warp < kConsWarps;
   const Tiles tl = sh.tiles[j];
   const int nt = tl.k1 - tl.k0;
   if (nt <= 0) return;
@@ -791,23 +798,23 @@ __device__ __noinline__ void projection_step(const StepShared& __restrict__ sh, 
     // finished MMAs no longer read) so that the adds into L2 are 16-byte reds along the features
     float* T = reinterpret_cast<float*>(S.X);
 #pragma unroll 1
-    for (int q = 0; q < R; q += 32) {
+    for (int q = (warp >> 2) * 32; q < R; q += 64) {   // warps 4-7 take tokens 32-63
       float v[32];
       __syncwarp();
       tmem_ld32(tm + lane_base + q, v);
 #pragma unroll
       for (int e = 0; e < 32; ++e) T[(q + e) * 128 + row] = v[e];
     }
-    named_sync(2, 128);
+    named_sync(2, kCons);
     if (good) {
       float* dst = acc + tl.b * 128;
 #pragma unroll 4
-      for (int idx = threadIdx.x; idx < R * 32; idx += 128) {
+      for (int idx = threadIdx.x; idx < R * 32; idx += kCons) {
         const int m = idx >> 5, c4 = idx & 31;
         red_add_v4(dst + (size_t)m * N + 4 * c4, *reinterpret_cast<const float4*>(T + m * 128 + 4 * c4));
       }
     }
-    named_sync(2, 128);
+    named_sync(2, kCons);
     if (threadIdx.x == 0) {
       // arrive on the block (release: this CTA's reds, ordered before by the named barrier), then
       // wait until every CTA of the block has arrived (acquire: their reds)
@@ -819,7 +826,7 @@ __device__ __noinline__ void projection_step(const StepShared& __restrict__ sh, 
       }
       *S.last = go;
     }
-    named_sync(2, 128);
+    named_sync(2, kCons);
     if (*reinterpret_cast<volatile int*>(S.last)) {
       const int W6 = 6 * p.W, b6 = l * W6, M = p.M;
       const int r0 = tl.idx * M / tl.contrib, r1 = (tl.idx + 1) * M / tl.contrib;
@@ -845,7 +852,7 @@ __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, cons
   uint8_t* sV = sK + KB;
   uint8_t* sP = sV + VB;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const bool mma = threadIdx.x == 160, cons = warp < 4;
+  const bool mma = threadIdx.x == kMmaThread, cons = warp < kConsWarps;
   const int nck = p.n_chunks, nqt = p.r_pad / kQT;
   const int items = p.B * p.n_kv_heads * nqt * nck;
   if (fused && (int)blockIdx.x >= items) {
@@ -857,10 +864,10 @@ __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, cons
       const int bg = t / nqt, qt = t % nqt, rows = min(kQT, p.rows - qt * kQT);
       const int r0 = qt * kQT + (ci - first) * rows / (next - first), r1 = qt * kQT + (ci - first + 1) * rows / (next - first);
       if (threadIdx.x == 0) *S.last = count_wait(qtile_ctr(p, l, t), (unsigned)nck, p.err);
-      named_sync(2, 128);
+      named_sync(2, kCons);
       if (*reinterpret_cast<volatile int*>(S.last)) {
         __nv_bfloat16* buf = reinterpret_cast<__nv_bfloat16*>(S.X) + (size_t)warp * kStepMaxChunks * DH;
-        combine_rows_warp<DH>(p, bg, r0 + warp, r1, 4, buf, S.cbar + warp, st);
+        combine_rows_warp<DH>(p, bg, r0 + warp, r1, kConsWarps, buf, S.cbar + warp, st);
       }
     }
     return;
@@ -903,44 +910,47 @@ __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, cons
       mma_commit(S.o_done);
     }
     if (cons) {
-      // softmax over the chunk's 64 keys, one query row per thread
-      const bool ok_s = mbar_wait(S.s_full, st.ipar, p.err, 48);
-      tc_fence_after();
-      const uint32_t tS = tmem_base_after_wait(S.tmem_slot);
-      const int quad = warp & 3, row = quad * 32 + lane;
+      // warps 0-3: softmax over the chunk's 64 keys, one query row per thread; all warps then
+      // read out O, warps 0-3 the first half of its columns and warps 4-7 the second
+      const int quad = warp & 3, half = warp >> 2, row = quad * 32 + lane;
       const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
-      const int key0 = kc * kKC;
-      const int nvalid = p.n_keys - key0 < kKC ? p.n_keys - key0 : kKC;
-      float sv[64];
-      __syncwarp();
-      tmem_ld32(tS + lane_base, sv);
-      tmem_ld32(tS + lane_base + 32, sv + 32);
-      float mx = -INFINITY;
+      bool ok_s = true;
+      float mx = -INFINITY, l_sum = 0.f;
+      if (half == 0) {
+        ok_s = mbar_wait(S.s_full, st.ipar, p.err, 48);
+        tc_fence_after();
+        const uint32_t tS = tmem_base_after_wait(S.tmem_slot);
+        const int key0 = kc * kKC;
+        const int nvalid = p.n_keys - key0 < kKC ? p.n_keys - key0 : kKC;
+        float sv[64];
+        __syncwarp();
+        tmem_ld32(tS + lane_base, sv);
+        tmem_ld32(tS + lane_base + 32, sv + 32);
 #pragma unroll
-      for (int i = 0; i < 64; ++i)
-        if (i < nvalid) mx = fmaxf(mx, sv[i]);
-      const float mxs = mx * p.scale_log2;
-      float l_sum = 0.f;
-      const int r8 = row & 7;
-      uint8_t* prow = sP + row * 128;
+        for (int i = 0; i < 64; ++i)
+          if (i < nvalid) mx = fmaxf(mx, sv[i]);
+        const float mxs = mx * p.scale_log2;
+        const int r8 = row & 7;
+        uint8_t* prow = sP + row * 128;
 #pragma unroll
-      for (int gi = 0; gi < 8; ++gi) {
-        uint32_t pk[4];
+        for (int gi = 0; gi < 8; ++gi) {
+          uint32_t pk[4];
 #pragma unroll
-        for (int e = 0; e < 8; e += 2) {
-          const int i0 = gi * 8 + e;
-          const float e0 = i0 < nvalid ? ex2_approx(fmaf(sv[i0], p.scale_log2, -mxs)) : 0.f;
-          const float e1 = i0 + 1 < nvalid ? ex2_approx(fmaf(sv[i0 + 1], p.scale_log2, -mxs)) : 0.f;
-          const __nv_bfloat162 h = __floats2bfloat162_rn(e0, e1);
-          l_sum += __low2float(h) + __high2float(h);   // normalise by what the MMA sums
-          pk[e / 2] = *reinterpret_cast<const uint32_t*>(&h);
+          for (int e = 0; e < 8; e += 2) {
+            const int i0 = gi * 8 + e;
+            const float e0 = i0 < nvalid ? ex2_approx(fmaf(sv[i0], p.scale_log2, -mxs)) : 0.f;
+            const float e1 = i0 + 1 < nvalid ? ex2_approx(fmaf(sv[i0 + 1], p.scale_log2, -mxs)) : 0.f;
+            const __nv_bfloat162 h = __floats2bfloat162_rn(e0, e1);
+            l_sum += __low2float(h) + __high2float(h);   // normalise by what the MMA sums
+            pk[e / 2] = *reinterpret_cast<const uint32_t*>(&h);
+          }
+          *reinterpret_cast<uint4*>(prow + ((gi ^ r8) * 16)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
         }
-        *reinterpret_cast<uint4*>(prow + ((gi ^ r8) * 16)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(S.p_full);
       }
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(S.p_full);
       const bool ok_o = mbar_wait(S.o_done, st.ipar, p.err, 49);
       tc_fence_after();
       const uint32_t tO = tmem_base_after_wait(S.tmem_slot) + 256;
@@ -951,8 +961,8 @@ __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, cons
       const size_t pi = ((size_t)bg * nck + kc) * p.r_pad + qrow;
       constexpr uint32_t pitch = DH * 2 + 16;
       uint8_t* srow = S.X + (size_t)row * pitch;
-#pragma unroll 2
-      for (int q = 0; q < DH; q += 32) {
+#pragma unroll 1
+      for (int q = half * (DH / 2); q < (half + 1) * (DH / 2); q += 32) {
         float ov[32];
         __syncwarp();
         tmem_ld32(tO + lane_base + q, ov);
@@ -962,7 +972,8 @@ __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, cons
                                                                      pack_bf16(ov[e + 4], ov[e + 5]), pack_bf16(ov[e + 6], ov[e + 7]));
       }
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      if (ok_s && ok_o && qrow < p.rows) {
+      named_sync(2, kCons);   // both halves of every row staged
+      if (half == 0 && ok_s && ok_o && qrow < p.rows) {
         bulk_s2g(p.part_o + pi * DH, srow, DH * 2);
         asm volatile("cp.async.bulk.commit_group;" ::: "memory");
         p.part_ml[pi * 2] = mx;
@@ -972,7 +983,7 @@ __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, cons
       }
       // count the chunk for its query tile (release: every consumer's rows, ordered before by the
       // named barrier)
-      named_sync(2, 128);
+      named_sync(2, kCons);
       if (threadIdx.x == 0 && ok_s && ok_o)
         asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(qtile_ctr(p, l, bg * nqt + qt)) : "memory");
     }
@@ -980,7 +991,7 @@ __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, cons
     // the next item's operand loads overwrite this item's operands and P
     tc_fence_before();
     __syncwarp();
-    named_sync(1, 160);
+    named_sync(1, kSyncThreads);
     tc_fence_after();
   }
 }
@@ -992,7 +1003,7 @@ __device__ __noinline__ void final_row(const StepArgs& __restrict__ p, int m, fl
   const float* mod = mod_row(p, p.tau_row[m]) + (size_t)p.L * 6 * W;
   const float rstd = rsqrtf(__ldcg(sumsq_slot(p, p.L, 0) + m) / W + 1e-6f);
 #pragma unroll 1
-  for (int c4 = tid; c4 < W / 4; c4 += 128) {
+  for (int c4 = tid; c4 < W / 4; c4 += kCons) {
     const float4 h = __ldcg(reinterpret_cast<const float4*>(p.h + (size_t)m * W) + c4);
     const float4 sc = __ldg(reinterpret_cast<const float4*>(mod) + c4);
     const float4 sf = __ldg(reinterpret_cast<const float4*>(mod + W) + c4);
@@ -1000,10 +1011,10 @@ __device__ __noinline__ void final_row(const StepArgs& __restrict__ p, int m, fl
     const __nv_bfloat162 hi = __floats2bfloat162_rn(fmaf(h.z * rstd, 1.f + sc.z, sf.z), fmaf(h.w * rstd, 1.f + sc.w, sf.w));
     reinterpret_cast<float4*>(ys)[c4] = make_float4(__low2float(lo), __high2float(lo), __low2float(hi), __high2float(hi));
   }
-  named_sync(2, 128);
+  named_sync(2, kCons);
   const __nv_bfloat16* wo = static_cast<const __nv_bfloat16*>(p.w_out);
 #pragma unroll 1
-  for (int d = warp; d < p.D; d += 4) {
+  for (int d = warp; d < p.D; d += kConsWarps) {
     float a = 0.f;
 #pragma unroll 4
     for (int k = 2 * lane; k < W; k += 64) {
@@ -1039,7 +1050,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(S.empty + i, 1);
     }
     for (int i = 0; i < 8; ++i) mbar_init(S.a_full + i, i == 5 ? 4 : 1);   // p_full: one arrive per consumer warp
-    for (int i = 0; i < 4; ++i) mbar_init(S.cbar + i, 1);
+    for (int i = 0; i < kConsWarps; ++i) mbar_init(S.cbar + i, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (threadIdx.x < kMaxRows) {
@@ -1067,7 +1078,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const StepArgs& p = sh.p;
   const uint32_t tmem = *S.tmem_slot;
 
-  if (warp == 4) {
+  if (warp == kProdWarp) {
     // ---- weight producer: this CTA's tiles of every projection, in consumption order ----
     if (lane == 0) {
       const uint64_t pol = policy_evict_first();
@@ -1093,8 +1104,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncwarp();
   } else {
-    // ---- warps 0-3: consumers; warp 5: tcgen05 issuer (thread 160) ----
-    const bool mma = threadIdx.x == 160, cons = warp < 4;
+    // ---- consumer warps; the last warp: tcgen05 issuer (its lane 0) ----
+    const bool mma = threadIdx.x == kMmaThread, cons = warp < kConsWarps;
     Role st;
     bool ok = true;
     unsigned* bar = p.sync;
