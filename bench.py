@@ -50,10 +50,10 @@ for _b in (4, 16, 64):
 
 # ncu DRAM traffic (read + write bytes) per launch of the dominant kernel class, with the source
 # file and its sha1 at measurement time (reported as null once that source changes); figures from
-# profiles/ncu_full_pi0_b1_attention_gemm.md (attention + combine kernels of one layer).
+# profiles/ncu_full_pi0_b1_step_kernel.md (one step-kernel launch = one evaluation).
 TRAFFIC = {
-    "attention@pi0-b1": (4057856.0, "paper_2609_37772_gb300/csrc/attn_tc.cu",
-                         "3bf844d67be14408fc8fd4d1769c8209a3d970ea"),
+    "step_kernel@pi0-b1": (641493760.0 + 3616512.0, "paper_2609_37772_gb300/csrc/step_tc.cu",
+                           "456626f0768504a95025e1de87d3f7ebe6b96468"),
 }
 
 
@@ -135,36 +135,57 @@ def bootstrap_ci(values, reps=8000, seed=0):
 
 
 class Clocks:
-    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+    """nvidia-smi sampling (every 50 ms) of SM clocks and throttle reasons; summary() keeps the
+    samples that arrived between start() and stop(), the timed region."""
     Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
     def __init__(self, index):
-        self.index, self.p = index, None
+        self.index, self.p, self.lines, self.t0, self.t1 = index, None, [], None, None
 
     def __enter__(self):
+        import threading
         try:
             self.p = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
-                                       "--format=csv,noheader,nounits", "-lms", "200"],
+                                       "--format=csv,noheader,nounits", "-lms", "50"],
                                       stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.p = None
+            return self
+
+        def reader():
+            for line in self.p.stdout:
+                self.lines.append((time.perf_counter(), line))
+        self.th = threading.Thread(target=reader, daemon=True)
+        self.th.start()
+        deadline = time.perf_counter() + 5.0
+        while not self.lines and time.perf_counter() < deadline and self.p.poll() is None:
+            time.sleep(0.01)                     # sampler running before the timed region starts
         return self
 
+    def start(self):
+        self.t0 = time.perf_counter()
+
+    def stop(self):
+        self.t1 = time.perf_counter() + 0.06     # a sample taken at the end arrives a little later
+        time.sleep(0.06)
+
     def __exit__(self, *exc):
-        self.out = ""
         if self.p:
             self.p.terminate()
             try:
-                self.out, _ = self.p.communicate(timeout=5)
+                self.p.wait(timeout=5)
             except subprocess.TimeoutExpired:
                 self.p.kill()
+            self.th.join(timeout=5)
 
     def summary(self):
         sm, mx, reasons = [], 0.0, set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for line in (self.out or "").splitlines():
+        for t, line in self.lines:
+            if self.t0 is not None and not (self.t0 <= t <= (self.t1 or t)):
+                continue
             f = [x.strip() for x in line.split(",")]
             if len(f) < 9:
                 continue
@@ -177,7 +198,7 @@ class Clocks:
                 if v.lower().startswith("active"):
                     reasons.add(n)
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx or None,
-                "reasons": sorted(reasons), "samples": len(sm)}
+                "reasons": sorted(reasons), "samples": len(sm), "interval_ms": 50}
 
 
 def dist_setup():
@@ -290,12 +311,14 @@ def run_ours(args, wl, world, rank, local):
     with Clocks(local) as clk:
         barrier(world)
         torch.cuda.synchronize()
+        clk.start()
         e0.record(stream)
         for _ in range(args.steps):
             step()
             step_times.append(ex.step_times())
         e1.record(stream)
         torch.cuda.synchronize()
+        clk.stop()
         barrier(world)
     ms_total = e0.elapsed_time(e1)
     ms_total_max = max_over_ranks(ms_total, world, dev if world > 1 and os.environ.get("UAD_BENCH_BACKEND", "nccl") == "nccl" else "cpu")
