@@ -294,6 +294,15 @@ __host__ __device__ __forceinline__ Tiles assign_tiles(int cta, int G, int NB, i
   return t;
 }
 __host__ __device__ __forceinline__ int proj_rot(int j) { return 41 * j; }
+// Epilogue shares of a projection: the sum over output blocks of their contributing CTAs.
+__host__ __device__ __forceinline__ int proj_shares(int G, int NB, int KT) {
+  int n = 0;
+  for (int b = 0; b < NB; ++b) {
+    const int cb = ((b + 1) * G + NB - 1) / NB - (b * G + NB - 1) / NB;
+    n += cb < KT ? cb : KT;
+  }
+  return n;
+}
 
 struct Smem {
   uint8_t* ring;
@@ -350,7 +359,9 @@ struct StepShared {
   int srow[kStepMaxShift];           // their modulation-table rows
   int sidx[kMaxRows];                // token -> index of its flow time
   Tiles tiles[4];                    // this CTA's tiles of the qkv, o, gate/up, down projections
-  int fused_combine;                 // idle CTAs of the attention step merge the key chunks
+  int fused_combine;                 // idle CTAs of the attention step merge the key chunks; the
+                                     // phases of a layer then wait on counts, not grid barriers
+  unsigned shares[4];                // epilogue shares of qkv, o, gate/up; [3] = merging CTAs
 };
 
 // Grid barrier among the consumer warps and the issuer's warp of every CTA: every CTA arrives (also
@@ -410,6 +421,27 @@ __device__ __noinline__ int count_wait(const unsigned* ctr, unsigned target, int
   }
 }
 
+// Phase boundary inside a layer when the phases wait on counts: the CTA's consumers and issuer
+// meet (tensor memory and the work area are free again), the issuer waits until *ctr reaches
+// `target` (acquire: the outputs this phase reads), then they meet again, so that every thread's
+// loads come after the acquire. Returns false once any error is recorded.
+__device__ __noinline__ bool phase_wait(const unsigned* ctr, unsigned target, bool ok, int* err, const Smem& S) {
+  tc_fence_before();
+  __syncwarp();
+  named_sync(1, kSyncThreads);
+  if (threadIdx.x == kMmaThread) {
+    bool good = ok && *reinterpret_cast<volatile int*>(err) == 0;
+    if (good) good = count_wait(ctr, target, err) != 0;
+    // outputs written by other CTAs are read next by this thread's tensor-map loads
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+    *S.flag = good ? 1 : 0;
+  }
+  __syncwarp();
+  named_sync(1, kSyncThreads);
+  tc_fence_after();
+  return *reinterpret_cast<volatile int*>(S.flag) != 0;
+}
+
 // Sum over the consumer threads; every consumer gets the total.
 __device__ __forceinline__ float cons_sum(float v, float* red) {
   v = warp_sum(v);
@@ -431,6 +463,12 @@ __device__ __forceinline__ float* sumsq_slot(const StepArgs& __restrict__ p, int
 __device__ __forceinline__ unsigned* qtile_ctr(const StepArgs& __restrict__ p, int l, int t) {
   return p.sync + (1 + kStepBarriersPerLayer * p.L) + (size_t)p.L * 4 * kStepMaxNB + (size_t)(p.L + 1) * 2 * kMaxRows +
          (size_t)l * kStepMaxQTiles + t;
+}
+// Count of finished epilogue shares of projection j (0 qkv, 1 o, 2 gate/up) of layer l; j = 3:
+// count of CTAs that finished their chunk merges.
+__device__ __forceinline__ unsigned* done_ctr(const StepArgs& __restrict__ p, int l, int j) {
+  return p.sync + (1 + kStepBarriersPerLayer * p.L) + (size_t)p.L * 4 * kStepMaxNB + (size_t)(p.L + 1) * 2 * kMaxRows +
+         (size_t)p.L * kStepMaxQTiles + (size_t)l * 4 + j;
 }
 __device__ __forceinline__ const float* mod_row(const StepArgs& __restrict__ p, int row) {
   return p.tab + (size_t)row * p.rowlen;
@@ -835,6 +873,12 @@ __device__ __noinline__ void projection_step(const StepShared& __restrict__ sh, 
       else if (j == 1) epi_resid(sh, p.acc_o, b6 + 2 * p.W, b6 + 3 * p.W, sumsq_slot(p, l, 1), tl.b, r0, r1, tl.idx == 0, S.X);
       else epi_resid(sh, p.acc_d, b6 + 5 * p.W, l + 1 < p.L ? b6 + W6 : -1, sumsq_slot(p, l + 1, 0), tl.b, r0, r1,
                      tl.idx == 0, S.X);
+      if (j < 3) {
+        // count this share (release: every consumer's epilogue stores, ordered before by the
+        // named barrier) for the phase that reads the projection's output
+        named_sync(2, kCons);
+        if (threadIdx.x == 0) asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(done_ctr(p, l, j)) : "memory");
+      }
     }
   }
   st.gpar ^= 1u;
@@ -868,6 +912,8 @@ __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, cons
       if (*reinterpret_cast<volatile int*>(S.last)) {
         __nv_bfloat16* buf = reinterpret_cast<__nv_bfloat16*>(S.X) + (size_t)warp * kStepMaxChunks * DH;
         combine_rows_warp<DH>(p, bg, r0 + warp, r1, kConsWarps, buf, S.cbar + warp, st);
+        named_sync(2, kCons);
+        if (threadIdx.x == 0) asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(done_ctr(p, l, 3)) : "memory");
       }
     }
     return;
@@ -1061,6 +1107,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int items = p_in.B * p_in.n_kv_heads * (p_in.r_pad / kQT) * p_in.n_chunks;
     const int qtiles = p_in.B * p_in.n_kv_heads * (p_in.r_pad / kQT);
     sh.fused_combine = (int)gridDim.x - items >= (qtiles > 16 ? qtiles : 16) ? 1 : 0;
+    sh.shares[3] = (unsigned)((int)gridDim.x - items);
+  }
+  if (threadIdx.x >= 72 && threadIdx.x < 75) {
+    const int j = threadIdx.x - 72;
+    int N, K;
+    proj_shape(p_in, j, N, K);
+    sh.shares[j] = (unsigned)proj_shares(gridDim.x, N / 128, K / 64);
   }
   if (threadIdx.x >= 64 && threadIdx.x < 68) {
     const int j = threadIdx.x - 64;
@@ -1112,25 +1165,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (cons) in_rows(sh, S.red);
     ok = grid_sync(bar++, ok, p.err, S);
     for (int l = 0; l < p.L; ++l) {
+      const bool df = sh.fused_combine != 0;   // phases inside the layer wait on counts
       if (ok) projection_step(sh, &t_z, l, 0, tmem, XB, st);
-      ok = grid_sync(bar++, ok, p.err, S);
-      if (ok) {
-        if (cons) clear_shift_rows(sh, true, l > 0);
-        attention_step<DH>(p, &t_q, &t_k, &t_vt, l, tmem, st, sh.fused_combine != 0);
-      }
-      ok = grid_sync(bar++, ok, p.err, S);
-      if (!sh.fused_combine) {
+      ok = df ? phase_wait(done_ctr(p, l, 0), sh.shares[0], ok, p.err, S) : grid_sync(bar++, ok, p.err, S);
+      if (ok) attention_step<DH>(p, &t_q, &t_k, &t_vt, l, tmem, st, df);
+      if (df) {
+        ok = phase_wait(done_ctr(p, l, 3), sh.shares[3], ok, p.err, S);
+      } else {
+        ok = grid_sync(bar++, ok, p.err, S);
         if (ok && cons) combine_rows<DH>(p, S.X, S.cbar + warp, st);
         ok = grid_sync(bar++, ok, p.err, S);
       }
       if (ok) projection_step(sh, &t_o, l, 1, tmem, XB, st);
-      ok = grid_sync(bar++, ok, p.err, S);
+      ok = df ? phase_wait(done_ctr(p, l, 1), sh.shares[1], ok, p.err, S) : grid_sync(bar++, ok, p.err, S);
       if (ok) projection_step(sh, &t_z, l, 2, tmem, XB, st);
-      ok = grid_sync(bar++, ok, p.err, S);
+      ok = df ? phase_wait(done_ctr(p, l, 2), sh.shares[2], ok, p.err, S) : grid_sync(bar++, ok, p.err, S);
+      // the shift rows of this layer's qkv and gate/up sums have been read by now
+      if (ok && cons) clear_shift_rows(sh, true, true);
       if (ok) projection_step(sh, &t_act, l, 3, tmem, XB, st);
       ok = grid_sync(bar++, ok, p.err, S);
     }
-    if (ok && cons) clear_shift_rows(sh, false, true);
     if (ok && cons && (int)blockIdx.x < p.M) final_row(p, blockIdx.x, reinterpret_cast<float*>(S.X));
     // a consumer warp exits only after its last combine copies have landed
     if (cons && st.c_uses) mbar_drain(S.cbar + warp, (uint32_t)(st.c_uses - 1) & 1u);

@@ -206,10 +206,11 @@ constexpr int kStepBarriersPerLayer = 6;
 constexpr int kStepMaxWidth = 2048;   // model width, a multiple of 512
 // Per-launch synchronisation block (zeroed before every launch): grid-barrier counters,
 // per-output-block arrival counters, row sums of squares of the residual stream, per-query-tile
-// counts of finished attention chunks.
+// counts of finished attention chunks, per-layer counts of finished epilogue shares (qkv, o,
+// gate/up) and chunk merges.
 __host__ __device__ constexpr size_t step_sync_words(int L) {
   return (size_t)(1 + kStepBarriersPerLayer * L) + (size_t)L * 4 * kStepMaxNB + (size_t)(L + 1) * 2 * kStepMaxRows +
-         (size_t)L * kStepMaxQTiles;
+         (size_t)L * kStepMaxQTiles + (size_t)L * 4;
 }
 struct StepArgs {
   int M = 0, B = 0, H = 0, W = 0, F = 0, D = 0, L = 0;
