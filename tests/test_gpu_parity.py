@@ -338,6 +338,22 @@ def test_step_kernel_batched_robots():
         c.close()
 
 
+def test_step_kernel_many_attention_items():
+    """Eight KV heads over a 1900-token prefix: 240 attention items leave too few idle CTAs to merge
+    the key chunks inside the attention step, so the persistent kernel merges them in a step of its
+    own and separates every phase by a grid barrier."""
+    a = ARCHS["pi0_small"].replace(name="mha_long_prefix", width=512, n_heads=8, n_kv_heads=8, head_dim=64,
+                                   mlp_dim=1024, chunk_len=16, prefix_len=1900)
+    c = Case(a, seed=15)
+    try:
+        noise = make_noise(a, seed=15)
+        bud = group_budgets(a.chunk_len, [(0, 3, 3), (4, 9, 5), (10, 15, 8)])
+        assert "step_kernel" in kernel_names(c, noise, bud[None])
+        check(c, c.gpu(noise, bud), c.oracle(noise, bud), bud, TOL["bf16"])
+    finally:
+        c.close()
+
+
 def test_full_rows_fall_back_to_per_operation_kernels():
     """Four robots of 16 tokens fill all 64 rows of the persistent kernel, leaving no room for
     the per-flow-time rows: the chunk runs on the per-operation kernels, with the same results."""
