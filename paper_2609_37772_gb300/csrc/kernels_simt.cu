@@ -472,6 +472,159 @@ __global__ void __launch_bounds__(128) attn_kernel(AttnArgs p) {
   }
 }
 
+// ------------------------------------------------------------------------------------------
+// Attention for few queries over few keys (bf16 operands, head dim 64, at most kFewKeys keys):
+// CTA = (16 queries, one query head, one robot), 256 threads. Every key and value of the head is
+// loaded into shared memory at once (16-byte loads), the whole score block S = Q K^T is formed
+// (thread = key), each query row takes an exact softmax (warp = two rows), and O = P V is one
+// pass (thread = (query, 4 dims)). Used for the DiT head's chunk self-attention and its
+// cross-attention to the observation prefix, where a key-by-key online softmax is bound by
+// the latency of its serial key blocks.
+// ------------------------------------------------------------------------------------------
+constexpr int kFewKeys = 512, kFewDh = 64, kFewQ = 16;
+constexpr int kFewKPitch = kFewDh + 2;   // bf16 per key row: rows 33 words apart, no bank conflicts
+
+__device__ __forceinline__ uint32_t pack_bf16_pair(float a, float b) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+__global__ void __launch_bounds__(256) attn_few_kernel(AttnArgs p) {
+  extern __shared__ float sm[];
+  pdl_trigger();
+  pdl_wait();
+  constexpr int dh = kFewDh, half = dh / 2;
+  const int n_keys = p.P + (p.kc ? p.H : 0);
+  float* qs = sm;                                       // [16][dh]
+  float* ss = qs + kFewQ * dh;                          // [16][n_keys] scores, then probabilities
+  __nv_bfloat16* ks = reinterpret_cast<__nv_bfloat16*>(ss + kFewQ * kFewKeys);   // [n_keys][kFewKPitch]
+  __nv_bfloat16* vs = ks + (size_t)kFewKeys * kFewKPitch;                          // [n_keys][dh]
+  const int b = blockIdx.z, hq = blockIdx.y, i0 = blockIdx.x * kFewQ;
+  const int g = hq / (p.n_heads / p.n_kv_heads);
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  // keys and values: 8 bf16 per 16-byte load, every load issued before any use
+#pragma unroll 4
+  for (int e = tid; e < n_keys * (dh / 8); e += 256) {
+    const int j = e / (dh / 8), c8 = e % (dh / 8);
+    uint4 kv, vv;
+    if (j < p.P) {
+      const long long off = b * p.kp_bstride + (long long)j * p.kp_ld + g * dh + c8 * 8;
+      kv = *reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(p.kp) + off);
+      vv = *reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(p.vp) + off);
+    } else {
+      const long long off = (long long)(b * p.H + j - p.P) * p.kc_ld + g * dh + c8 * 8;
+      kv = *reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(p.kc) + off);
+      vv = *reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(p.vc) + off);
+    }
+    uint32_t* kd = reinterpret_cast<uint32_t*>(ks + (size_t)j * kFewKPitch + c8 * 8);
+    kd[0] = kv.x;
+    kd[1] = kv.y;
+    kd[2] = kv.z;
+    kd[3] = kv.w;
+    *reinterpret_cast<uint4*>(vs + (size_t)j * dh + c8 * 8) = vv;
+  }
+  for (int e = tid; e < kFewQ * dh; e += 256) {
+    const int qi = e / dh, d = e % dh, i = i0 + qi;
+    float val = 0.f;
+    if (i < p.H) {
+      const long long off = (long long)(b * p.H + i) * p.q_ld + hq * dh;
+      val = p.rope_cs ? rope_elem(p.q, off, d, half, p.rope_cs + (long long)i * dh, BF16)
+                      : ldf_rt(p.q, off + d, BF16);
+    }
+    qs[qi * dh + d] = val * p.scale;
+  }
+  __syncthreads();
+  // chunk keys carry RoPE like the queries (prefix keys come rotated)
+  if (p.rope_cs && p.kc) {
+    for (int e = tid; e < p.H * half; e += 256) {
+      const int jj = e / half, d = e % half;
+      __nv_bfloat16* kr = ks + (size_t)(p.P + jj) * kFewKPitch;
+      const float* cs = p.rope_cs + (long long)jj * dh;
+      const float x0 = __bfloat162float(kr[d]), x1 = __bfloat162float(kr[d + half]);
+      kr[d] = __float2bfloat16_rn(x0 * cs[2 * d] - x1 * cs[2 * d + 1]);
+      kr[d + half] = __float2bfloat16_rn(x1 * cs[2 * d] + x0 * cs[2 * d + 1]);
+    }
+    __syncthreads();
+  }
+  // scores: thread = key, all 16 queries
+  for (int j = tid; j < n_keys; j += 256) {
+    float kf[dh];
+    const __nv_bfloat162* kr = reinterpret_cast<const __nv_bfloat162*>(ks + (size_t)j * kFewKPitch);
+#pragma unroll
+    for (int d2 = 0; d2 < dh / 2; ++d2) {
+      const float2 f = __bfloat1622float2(kr[d2]);
+      kf[2 * d2] = f.x;
+      kf[2 * d2 + 1] = f.y;
+    }
+#pragma unroll 4
+    for (int q = 0; q < kFewQ; ++q) {
+      const float4* q4 = reinterpret_cast<const float4*>(qs + q * dh);
+      float a0 = 0.f, a1 = 0.f;
+#pragma unroll
+      for (int d4 = 0; d4 < dh / 4; d4 += 2) {
+        const float4 x = q4[d4], y = q4[d4 + 1];
+        a0 = fmaf(x.x, kf[4 * d4], fmaf(x.y, kf[4 * d4 + 1], fmaf(x.z, kf[4 * d4 + 2], fmaf(x.w, kf[4 * d4 + 3], a0))));
+        a1 = fmaf(y.x, kf[4 * d4 + 4], fmaf(y.y, kf[4 * d4 + 5], fmaf(y.z, kf[4 * d4 + 6], fmaf(y.w, kf[4 * d4 + 7], a1))));
+      }
+      ss[q * kFewKeys + j] = a0 + a1;
+    }
+  }
+  __syncthreads();
+  // softmax per query row (warp w: rows 2w, 2w + 1); 1 / sum kept in qs[q * dh]
+  for (int q = 2 * warp; q < 2 * warp + 2; ++q) {
+    float* row = ss + q * kFewKeys;
+    float mx = -INFINITY;
+    for (int j = lane; j < n_keys; j += 32) mx = fmaxf(mx, row[j]);
+    mx = warp_max(mx);
+    float sum = 0.f;
+    for (int j = lane; j < n_keys; j += 32) {
+      const float e = expf(row[j] - mx);
+      row[j] = e;
+      sum += e;
+    }
+    sum = warp_sum(sum);
+    __syncwarp();
+    if (lane == 0) qs[q * dh] = 1.f / sum;
+  }
+  __syncthreads();
+  // O = P V: thread = (query q, dims 4 c .. 4 c + 3)
+  {
+    const int q = tid / (dh / 4), c = tid % (dh / 4);
+    const float* row = ss + q * kFewKeys;
+    float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+    for (int j = 0; j < n_keys; ++j) {
+      const float pj = row[j];
+      const __nv_bfloat162* v2 = reinterpret_cast<const __nv_bfloat162*>(vs + (size_t)j * dh + 4 * c);
+      const float2 v0 = __bfloat1622float2(v2[0]), v1 = __bfloat1622float2(v2[1]);
+      o.x = fmaf(pj, v0.x, o.x);
+      o.y = fmaf(pj, v0.y, o.y);
+      o.z = fmaf(pj, v1.x, o.z);
+      o.w = fmaf(pj, v1.y, o.w);
+    }
+    const int i = i0 + q;
+    if (i < p.H) {
+      const float inv = qs[q * dh];
+      __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(p.out) + (long long)(b * p.H + i) * p.out_ld + hq * dh + 4 * c;
+      uint2 pk;
+      pk.x = pack_bf16_pair(o.x * inv, o.y * inv);
+      pk.y = pack_bf16_pair(o.z * inv, o.w * inv);
+      *reinterpret_cast<uint2*>(dst) = pk;
+    }
+  }
+}
+
+size_t attn_few_smem_bytes() {
+  return sizeof(float) * (kFewQ * kFewDh + kFewQ * kFewKeys) + 2 * (size_t)kFewKeys * (kFewKPitch + kFewDh);
+}
+
+bool attn_few_ok(const AttnArgs& a) {
+  const int n_keys = a.P + (a.kc ? a.H : 0);
+  const bool aligned = a.kp_ld % 8 == 0 && a.kc_ld % 8 == 0 && a.q_ld % 8 == 0 && a.out_ld % 4 == 0;
+  return a.dtype == BF16 && a.head_dim == kFewDh && n_keys <= kFewKeys && n_keys >= 1 && aligned &&
+         (a.kp_bstride % 8) == 0 && (a.n_heads * a.head_dim) % 8 == 0;
+}
+
 template <int DPL>
 static void launch_attn_dpl(const AttnArgs& a, dim3 grid, size_t smem, cudaStream_t s) {
   launch_k(attn_kernel<DPL>, grid, dim3(128), smem, s, a);
@@ -484,6 +637,7 @@ size_t attention_smem_bytes(int dh) {
 void launch_attention_prepare(int dh) {
   const int smem = (int)attention_smem_bytes(dh);
   const cudaFuncAttribute at = cudaFuncAttributeMaxDynamicSharedMemorySize;
+  cudaFuncSetAttribute(attn_few_kernel, at, (int)attn_few_smem_bytes());
   if (dh == 64) cudaFuncSetAttribute(attn_kernel<2>, at, smem);
   if (dh == 128) cudaFuncSetAttribute(attn_kernel<4>, at, smem);
   if (dh == 256) cudaFuncSetAttribute(attn_kernel<8>, at, smem);
@@ -491,6 +645,10 @@ void launch_attention_prepare(int dh) {
 
 void launch_attention(const AttnArgs& a, cudaStream_t s) {
   const int dh = a.head_dim;
+  if (attn_few_ok(a)) {
+    launch_k(attn_few_kernel, dim3((a.H + kFewQ - 1) / kFewQ, a.n_heads, a.B), dim3(256), attn_few_smem_bytes(), s, a);
+    return;
+  }
   const size_t smem = attention_smem_bytes(dh);
   dim3 grid((a.H + AQ - 1) / AQ, a.n_heads, a.B);
   switch (dh) {
