@@ -52,8 +52,8 @@ for _b in (4, 16, 64):
 # file and its sha1 at measurement time (reported as null once that source changes); figures from
 # profiles/ncu_full_pi0_b1_step_kernel.md (one step-kernel launch = one evaluation).
 TRAFFIC = {
-    "step_kernel@pi0-b1": (641493760.0 + 3616512.0, "paper_2609_37772_gb300/csrc/step_tc.cu",
-                           "456626f0768504a95025e1de87d3f7ebe6b96468"),
+    "step_kernel@pi0-b1": (641484544.0 + 3697408.0, "paper_2609_37772_gb300/csrc/step_tc.cu",
+                           "0c228215f78c12fd13e78ae0c4b0f9d9e1986c4b"),
 }
 
 
