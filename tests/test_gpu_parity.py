@@ -193,6 +193,30 @@ def test_errors_are_reported(tiny):
     tiny.ex.finish(timeout_us=TIMEOUT)
 
 
+def test_timeouts_leave_the_chunk_in_flight(tiny):
+    """A delayed chunk (the caller's stream is held by a bounded sleep kernel before the library's
+    work may start): poll and finish with short deadlines return UAD_ETIMEDOUT without waiting and
+    leave the chunk in flight, a new observation is refused while it is in flight, and a later
+    finish returns the complete chunk."""
+    a = tiny.a
+    noise = make_noise(a)
+    bud = group_budgets(a.chunk_len, [(0, 3, 5), (4, a.chunk_len - 1, 10)])
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):
+        torch.cuda._sleep(400_000_000)        # ~0.2 s of GPU time on the caller's stream
+    tiny.ex.denoise(noise, bud[None], stream=stream)
+    rc, _, ready, _ = tiny.ex.poll(0, min_ready=1, timeout_us=1000)
+    assert rc == uad.UAD_ETIMEDOUT and not ready.any()
+    res = tiny.ex.finish(timeout_us=1000, check=False)
+    assert res["rc"] == uad.UAD_ETIMEDOUT
+    with pytest.raises(uad.UADError) as ei:
+        tiny.ex.set_prefix(0, *make_prefix_kv(a))
+    assert ei.value.code == uad.UAD_ESTATE
+    res = tiny.ex.finish(timeout_us=TIMEOUT)
+    assert res["rc"] == uad.UAD_OK and res["evals"] == 10
+    torch.cuda.synchronize()
+
+
 def test_nonfinite_is_reported(tiny):
     a = tiny.a
     noise = make_noise(a)
