@@ -24,6 +24,11 @@ definition, so the composition below is this project's stated architecture:
         y = LN(h)(1+scale2)+shift2 ; h += gate2 * (gelu_tanh(y W1 + b1) W2 + b2)
         (LN: no affine, eps 1e-6; the DiT input adds a sinusoidal position code of index i)
   input / output: h = x Win + bin ; v = Norm_final(h)(1+scale_f)+shift_f) Wout + bout
+  "concat" (SmolVLA-style: the token's time embedding is given to it before the action MLP,
+  App. C.1): e = sinusoid(tau) as above (no time MLP), a = x Win + bin,
+        h = SiLU(a Wia + e Wit + bi) Wo_in + bo_in  (the MLP over [a ; e]),
+        layers as "adarms" with RMSNorm unmodulated and ungated residuals,
+        v = RMSNorm(h) Wout + bout
 
 Everything here is fp64 on the (bf16-exact, for bf16 archs) weights. Library primitives
 used as steps: numpy matmul, exp, sin, cos, tanh.
@@ -123,6 +128,8 @@ class Model:
     def time_cond(self, tau):
         w = self.w
         e = sinusoid(tau, self.a.width, TIME_SCALE)
+        if self.a.kind == "concat":
+            return e
         return silu(silu(e @ w["t_w1"] + w["t_b1"]) @ w["t_w2"] + w["t_b2"])
 
     # -- the velocity field --------------------------------------------------------------------
@@ -134,6 +141,12 @@ class Model:
         H, W = u.shape[0], a.width
         c = self.time_cond(tau)
         h = u @ w["in_w"] + w["in_b"]
+        if a.kind == "concat":
+            # the action MLP over the token's action embedding and its own time embedding
+            h = silu(h @ w["ti_wa"] + c @ w["ti_wt"] + w["ti_b"]) @ w["to_w"] + w["to_b"]
+            for l in range(a.n_layers):
+                h = self._layer(l, h, c)
+            return rms_norm(h) @ w["out_w"] + w["out_b"]
         if a.kind == "dit":
             h = h + sinusoid(np.arange(H), W, 1.0)
         for l in range(a.n_layers):
@@ -150,6 +163,18 @@ class Model:
     def _layer(self, l, h, c):
         a, w, p = self.a, self.w, f"l{l}."
         H, W, hq, hkv, dh = h.shape[0], a.width, a.n_heads, a.n_kv_heads, a.head_dim
+        if a.kind == "concat":
+            y = rms_norm(h)
+            q = (y @ w[p + "wq"]).reshape(H, hq, dh)
+            k = (y @ w[p + "wk"]).reshape(H, hkv, dh)
+            v = (y @ w[p + "wv"]).reshape(H, hkv, dh)
+            if a.rope:
+                pos = a.prefix_len + np.arange(H)
+                q, k = rope(q, pos), rope(k, pos)
+            o = attention(q, np.concatenate([self.kpre[l], k]), np.concatenate([self.vpre[l], v]))
+            h = h + o.reshape(H, hq * dh) @ w[p + "wo"]
+            y = rms_norm(h)
+            return h + (gelu_tanh(y @ w[p + "wg"]) * (y @ w[p + "wu"])) @ w[p + "wd"]
         if a.kind == "adarms":
             m = c @ w[p + "mod1_w"] + w[p + "mod1_b"]
             scale, shift, gate = m[:, :W], m[:, W:2 * W], m[:, 2 * W:]

@@ -154,3 +154,77 @@ def test_k1_exact_recovery_with_the_network():
     assert np.array_equal(uad["final"][4:], van["final"][4:])
     assert not np.array_equal(uad["final"][:4], van["final"][:4])
     assert uad["evals"] == van["evals"] == ns
+
+
+# ---- SmolVLA-style time conditioning: the time embedding joins the action MLP (App. C.1) --------
+def _concat0():
+    return ARCHS["tiny_concat"].replace(n_layers=0, chunk_len=5)
+
+
+def test_concat_input_mlp_closed_form():
+    """Zero layers, identity MLP weights and a constant action embedding: v = RMSNorm(SiLU(a0 +
+    e(tau))) Wout + bout with e(tau)_j = sin(1000 tau 10^(-4 j / (W/2))) for j < W/2 and the
+    matching cos above; e is written out here from its definition."""
+    a = _concat0()
+    W, D = a.width, a.action_dim
+    rng = np.random.default_rng(11)
+    a0 = rng.normal(size=W)
+    w = {"in_w": np.zeros((D, W)), "in_b": a0, "ti_wa": np.eye(W), "ti_wt": np.eye(W), "ti_b": np.zeros(W),
+         "to_w": np.eye(W), "to_b": np.zeros(W), "out_w": rng.normal(size=(W, D)) * 0.1, "out_b": rng.normal(size=D)}
+    m = Model(a, blob_from_weights(a, w))
+    tau = np.array([0.0, 0.1, 0.25, 0.5, 0.9])
+    v = m.velocity(rng.normal(size=(a.chunk_len, D)), tau)
+    half = W // 2
+    for i, t in enumerate(tau):
+        e = np.array([np.sin(1000.0 * t * 10000.0 ** (-j / half)) for j in range(half)] +
+                     [np.cos(1000.0 * t * 10000.0 ** (-j / half)) for j in range(half)])
+        x = a0.astype(np.float32).astype(np.float64) + e
+        g = x / (1.0 + np.exp(-x))
+        y = g / np.sqrt(np.mean(g * g) + 1e-6)
+        ref = y @ w["out_w"].astype(np.float32).astype(np.float64) + w["out_b"].astype(np.float32)
+        np.testing.assert_allclose(v[i], ref, rtol=1e-6, atol=1e-7)
+
+
+def test_concat_time_conditioning_is_per_token():
+    """Without layers a token's velocity depends on its own state and flow time only."""
+    a = _concat0()
+    m = Model(a, make_weights(a, seed=12))
+    u = make_noise(a, seed=12)[0]
+    t1 = np.array([0.0, 0.2, 0.4, 0.6, 0.8])
+    t2 = t1.copy(); t2[2] = 0.95
+    v1, v2 = m.velocity(u, t1), m.velocity(u, t2)
+    assert np.abs(v1[2] - v2[2]).max() > 1e-4
+    np.testing.assert_array_equal(np.delete(v1, 2, 0), np.delete(v2, 2, 0))
+
+
+def test_concat_layer_is_the_adarms_layer_without_modulation():
+    """A "concat" layer equals an "adarms" layer whose modulation is scale = shift = 0 and
+    gate = 1 for every token (plain RMSNorm, ungated residuals)."""
+    ac = ARCHS["tiny_concat"].replace(n_layers=1, rope=True, n_kv_heads=2)
+    aa = ARCHS["tiny"].replace(n_layers=1, rope=True, n_kv_heads=2)
+    wc = split_blob(ac, make_weights(ac, seed=13))
+    wa = split_blob(aa, make_weights(aa, seed=13))
+    W = aa.width
+    for n in ("wq", "wk", "wv", "wo", "wg", "wu", "wd"):
+        wa["l0." + n] = wc["l0." + n]
+    for n in ("l0.mod1", "l0.mod2"):
+        wa[n + "_w"] = np.zeros_like(wa[n + "_w"])
+        wa[n + "_b"] = np.concatenate([np.zeros(2 * W), np.ones(W)])
+    kv = make_prefix_kv(ac, seed=13)
+    mc = Model(ac, blob_from_weights(ac, wc)); mc.set_prefix_kv(*kv)
+    ma = Model(aa, blob_from_weights(aa, wa)); ma.set_prefix_kv(*kv)
+    h = np.random.default_rng(13).normal(size=(ac.chunk_len, W))
+    tau = np.linspace(0.0, 0.9, ac.chunk_len)
+    np.testing.assert_allclose(mc._layer(0, h, mc.time_cond(tau)), ma._layer(0, h, ma.time_cond(tau)),
+                               rtol=1e-12, atol=1e-12)
+
+
+def test_k1_exact_recovery_with_the_concat_network():
+    """Sec. 4.3 with the SmolVLA-style expert: K = 1 tail and ghosts equal vanilla bit for bit."""
+    from oracle.uad import denoise
+    a = ARCHS["tiny_concat"]
+    m = Model(a, make_weights(a)); m.set_prefix_kv(*make_prefix_kv(a))
+    x0 = make_noise(a)[0]
+    van = denoise(m.velocity, x0, [10] * a.chunk_len)
+    uad = denoise(m.velocity, x0, [1] * 4 + [10] * (a.chunk_len - 4), gac=False)
+    assert np.array_equal(uad["ghost"], van["final"]) and np.array_equal(uad["final"][4:], van["final"][4:])

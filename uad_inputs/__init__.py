@@ -37,6 +37,8 @@ class Arch:
     name: str
     kind: str            # "adarms": joint attention over prefix KV + chunk, adaptive RMSNorm
                          # "dit":    chunk self-attention + cross-attention, adaLN-zero
+                         # "concat": joint attention, plain RMSNorm; each token's time embedding
+                         #           joins its action embedding in the input MLP (SmolVLA-style)
     dtype: str           # "f32" or "bf16" (weights / GEMM operands)
     n_layers: int
     width: int
@@ -67,6 +69,10 @@ ARCHS = {
     "pi0_small": Arch("pi0_small", "adarms", "bf16", 2, 512, 4, 1, 128, 1536, 32, 50, 200, rope=True),
     "dit_small": Arch("dit_small", "dit", "bf16", 2, 384, 6, 6, 64, 1536, 32, 16, 72, prefix_width=256),
     "tiny_f32_rope": Arch("tiny_f32_rope", "adarms", "f32", 2, 256, 4, 2, 64, 1024, 7, 16, 64, rope=True),
+    # Time embedding concatenated with the action embedding before the input MLP (App. C.1's
+    # SmolVLA variant): fp32 tiny and a bf16 small expert with GQA and RoPE.
+    "tiny_concat": Arch("tiny_concat", "concat", "f32", 2, 256, 4, 4, 64, 1024, 7, 16, 64),
+    "concat_small": Arch("concat_small", "concat", "bf16", 2, 512, 8, 2, 64, 1536, 32, 50, 120, rope=True),
 }
 
 
@@ -77,10 +83,19 @@ def weight_specs(a: Arch):
     order (scale, shift, gate) for "adarms" and (shift1, scale1, gate1, shift2, scale2,
     gate2) for "dit"; the final norm's modulation is (scale, shift) / (shift, scale).
     The gate/up and q/k/v projections are separate tensors here; the library re-lays them
-    out internally.
+    out internally. "concat" has no time MLP and no modulation: its input MLP takes the action
+    embedding (ti_wa) and the sinusoidal time embedding (ti_wt) side by side, then to_w.
     """
     W, D, F = a.width, a.action_dim, a.mlp_dim
     q, kv = a.n_heads * a.head_dim, a.n_kv_heads * a.head_dim
+    if a.kind == "concat":
+        s = [("in_w", (D, W)), ("in_b", (W,)), ("ti_wa", (W, W)), ("ti_wt", (W, W)), ("ti_b", (W,)),
+             ("to_w", (W, W)), ("to_b", (W,))]
+        for l in range(a.n_layers):
+            p = f"l{l}."
+            s += [(p + "wq", (W, q)), (p + "wk", (W, kv)), (p + "wv", (W, kv)), (p + "wo", (q, W)),
+                  (p + "wg", (W, F)), (p + "wu", (W, F)), (p + "wd", (F, W))]
+        return s + [("out_w", (W, D)), ("out_b", (D,))]
     s = [("t_w1", (W, W)), ("t_b1", (W,)), ("t_w2", (W, W)), ("t_b2", (W,)),
          ("in_w", (D, W)), ("in_b", (W,))]
     for l in range(a.n_layers):
