@@ -40,6 +40,9 @@ extern "C" {
 
 #define UAD_KIND_ADARMS 0    /* joint attention over prefix KV + chunk, adaptive RMSNorm */
 #define UAD_KIND_DIT 1       /* chunk self-attention + cross-attention, adaLN-zero */
+#define UAD_KIND_CONCAT 2    /* joint attention as ADARMS with plain RMSNorm; each token's time
+                                embedding joins its action embedding in the input MLP (App. C.1,
+                                the SmolVLA variant) */
 
 #define UAD_DTYPE_F32 0
 #define UAD_DTYPE_BF16 1
@@ -103,6 +106,11 @@ typedef struct uad_ctx uad_ctx;
  *                        wqc[W][Hq*dh] wkc wvc[Pw][Hq*dh] woc[Hq*dh][W]
  *                        w1[W][F] b1[F] w2[F][W] b2[W]
  *     modf_w[W][2W] modf_b[2W] out_w[W][D] out_b[D]
+ *   CONCAT instead: in_w[D][W] in_b[W] ti_wa[W][W] ti_wt[W][W] ti_b[W] to_w[W][W] to_b[W],
+ *     per layer wq wk wv wo wg wu wd (shapes as ADARMS), out_w[W][D] out_b[D]; the input is
+ *     h = SiLU((u in_w + in_b) ti_wa + e(tau) ti_wt + ti_b) to_w + to_b with e the token's
+ *     sinusoidal time embedding, every norm is RMSNorm without modulation and residuals are
+ *     ungated.
  *   Modulation vectors are (scale, shift, gate) for ADARMS and (shift1, scale1, gate1,
  *   shift2, scale2, gate2) for DiT; the final one is (scale, shift) / (shift, scale).
  *   For bf16 architectures every weight is rounded to bf16 (nearest, ties to even).

@@ -18,7 +18,7 @@ if not os.path.exists(LIB_PATH):
 _lib = C.CDLL(LIB_PATH)
 
 UAD_OK, UAD_EINVAL, UAD_ESTATE, UAD_ENOMEM, UAD_ECUDA, UAD_ETIMEDOUT, UAD_ENONFINITE = 0, -22, -1, -12, -5, -110, -33
-KIND = {"adarms": 0, "dit": 1}
+KIND = {"adarms": 0, "dit": 1, "concat": 2}
 DTYPE = {"f32": 0, "bf16": 1}
 MAX_STEPS = 64
 

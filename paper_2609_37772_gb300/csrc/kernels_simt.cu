@@ -625,6 +625,26 @@ bool attn_few_ok(const AttnArgs& a) {
          (a.kp_bstride % 8) == 0 && (a.n_heads * a.head_dim) % 8 == 0;
 }
 
+__global__ void add_tau_silu_kernel(const float* __restrict__ x, const float* __restrict__ tab, int stride, int off,
+                                    const int* __restrict__ tau_row, int M, int N, void* y, int dt) {
+  pdl_trigger();
+  pdl_wait();
+  const long long total = (long long)M * N;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total; e += (long long)gridDim.x * blockDim.x) {
+    const int m = (int)(e / N), n = (int)(e % N);
+    const float v = x[e] + tab[(size_t)tau_row[m] * stride + off + n];
+    stf(y, e, v / (1.f + expf(-v)), dt);
+  }
+}
+
+void launch_add_tau_silu(const float* x, const float* tab, int stride, int off, const int* tau_row, int M, int N,
+                         void* y, int dt, cudaStream_t s) {
+  const long long total = (long long)M * N;
+  int blocks = (int)((total + 255) / 256);
+  if (blocks > 1024) blocks = 1024;
+  launch_k(add_tau_silu_kernel, dim3(blocks), dim3(256), 0, s, x, tab, stride, off, tau_row, M, N, y, dt);
+}
+
 template <int DPL>
 static void launch_attn_dpl(const AttnArgs& a, dim3 grid, size_t smem, cudaStream_t s) {
   launch_k(attn_kernel<DPL>, grid, dim3(128), smem, s, a);

@@ -699,7 +699,15 @@ template <int DH>
 __device__ __forceinline__ void combine_rows_warp(const StepArgs& __restrict__ p, int bg, int r0, int r1, int step,
                                                   __nv_bfloat16* buf, uint64_t* bar, Role& st) {
   constexpr int E = DH / 64, kG = 8;
-  const int lane = threadIdx.x & 31, nck = p.n_chunks;
+  // the arguments this routine uses, in registers (the asm statements below clobber memory, which
+  // would otherwise make every use reload them)
+  const int lane = threadIdx.x & 31, nck = p.n_chunks, r_pad = p.r_pad, H = p.H, qd = p.qd;
+  const int nkv = p.n_kv_heads, group = p.group;
+  const float scale_log2 = p.scale_log2;
+  const __nv_bfloat16* __restrict__ part_o = p.part_o;
+  const float* __restrict__ part_ml = p.part_ml;
+  __nv_bfloat16* __restrict__ o_out = p.o;
+  int* err = p.err;
   constexpr int kRows = 2;                  // rows staged at once (two when n_chunks <= 16)
   const int batch = nck * kRows <= kStepMaxChunks ? kRows : 1;
 #pragma unroll 1
@@ -713,7 +721,7 @@ __device__ __forceinline__ void combine_rows_warp(const StepArgs& __restrict__ p
       // this lane's bulk copies
       asm volatile("fence.proxy.async.global;" ::: "memory");
       for (int k = 0; k < nr; ++k) {
-        const __nv_bfloat16* src = p.part_o + (((size_t)bg * nck + lane) * p.r_pad + rb + k * step) * DH;
+        const __nv_bfloat16* src = part_o + (((size_t)bg * nck + lane) * r_pad + rb + k * step) * DH;
         asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
                      ::"r"(su32(buf + ((size_t)k * nck + lane) * DH)), "l"(src), "r"(DH * 2), "r"(su32(bar)) : "memory");
       }
@@ -725,19 +733,19 @@ __device__ __forceinline__ void combine_rows_warp(const StepArgs& __restrict__ p
       mc[k] = -INFINITY;
       lc[k] = 0.f;
       if (k < nr && lane < nck) {
-        const size_t pi = ((size_t)bg * nck + lane) * p.r_pad + rb + k * step;
-        mc[k] = __ldcg(p.part_ml + pi * 2);
-        lc[k] = __ldcg(p.part_ml + pi * 2 + 1);
+        const size_t pi = ((size_t)bg * nck + lane) * r_pad + rb + k * step;
+        mc[k] = __ldcg(part_ml + pi * 2);
+        lc[k] = __ldcg(part_ml + pi * 2 + 1);
       }
     }
     float wgt[kRows], invL[kRows];
 #pragma unroll
     for (int k = 0; k < kRows; ++k) {
       const float M = warp_max(mc[k]);
-      wgt[k] = lane < nck && k < nr ? exp2f((mc[k] - M) * p.scale_log2) : 0.f;
+      wgt[k] = lane < nck && k < nr ? exp2f((mc[k] - M) * scale_log2) : 0.f;
       invL[k] = 1.f / warp_sum(wgt[k] * lc[k]);
     }
-    const bool ok = mbar_wait(bar, st.cpar, p.err, 53);
+    const bool ok = mbar_wait(bar, st.cpar, err, 53);
     st.cpar ^= 1u;
 #pragma unroll 1
     for (int k = 0; k < nr && ok; ++k) {
@@ -767,8 +775,8 @@ __device__ __forceinline__ void combine_rows_warp(const StepArgs& __restrict__ p
           }
         }
       }
-      const int b = bg / p.n_kv_heads, g = bg % p.n_kv_heads, j = r / p.H, i = r % p.H;
-      __nv_bfloat16* dst = p.o + ((size_t)b * p.H + i) * p.qd + (size_t)(g * p.group + j) * DH;
+      const int b = bg / nkv, g = bg % nkv, j = r / H, i = r % H;
+      __nv_bfloat16* dst = o_out + ((size_t)b * H + i) * qd + (size_t)(g * group + j) * DH;
 #pragma unroll
       for (int e = 0; e < E; ++e)
         *reinterpret_cast<uint32_t*>(dst + 64 * e + 2 * lane) = pack_bf16(acc[e].x * ik, acc[e].y * ik);

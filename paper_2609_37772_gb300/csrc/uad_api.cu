@@ -86,6 +86,9 @@ struct uad_ctx {
   void* w_in = nullptr; float* b_in = nullptr;   // [W][D]
   void* w_out = nullptr; float* b_out = nullptr; // [D][W]
   void* w_mod = nullptr; float* b_mod = nullptr; // [rowlen][W], all layers' modulation + final
+  // time-concatenating expert (UAD_KIND_CONCAT): input MLP; e(tau) W_it + b_it sits in the table
+  void* w_it = nullptr; float* b_it = nullptr;   // [W][W] (table fill)
+  Lin w_ia, w_io; float* b_io = nullptr;          // [W][W] projections of the input MLP
   std::vector<LayerW> L;
 
   // time conditioning
@@ -194,6 +197,17 @@ std::vector<Tensor> blob_layout(const uad_arch& a) {
   };
   const long long W = a.width, D = a.action_dim, F = a.mlp_dim;
   const long long q = (long long)a.n_heads * a.head_dim, kv = (long long)a.n_kv_heads * a.head_dim;
+  if (a.kind == UAD_KIND_CONCAT) {
+    add("in_w", D, W); add("in_b", 1, W);
+    add("ti_wa", W, W); add("ti_wt", W, W); add("ti_b", 1, W); add("to_w", W, W); add("to_b", 1, W);
+    for (int l = 0; l < a.n_layers; ++l) {
+      const std::string p = "l" + std::to_string(l) + ".";
+      add(p + "wq", W, q); add(p + "wk", W, kv); add(p + "wv", W, kv); add(p + "wo", q, W);
+      add(p + "wg", W, F); add(p + "wu", W, F); add(p + "wd", F, W);
+    }
+    add("out_w", W, D); add("out_b", 1, D);
+    return t;
+  }
   add("t_w1", W, W); add("t_b1", 1, W); add("t_w2", W, W); add("t_b2", 1, W);
   add("in_w", D, W); add("in_b", 1, W);
   for (int l = 0; l < a.n_layers; ++l) {
@@ -217,7 +231,7 @@ std::vector<Tensor> blob_layout(const uad_arch& a) {
 
 int validate_arch(const uad_arch& a, std::string& why) {
   auto bad = [&](const char* m) { why = m; return UAD_EINVAL; };
-  if (a.kind != UAD_KIND_ADARMS && a.kind != UAD_KIND_DIT) return bad("kind");
+  if (a.kind != UAD_KIND_ADARMS && a.kind != UAD_KIND_DIT && a.kind != UAD_KIND_CONCAT) return bad("kind");
   if (a.dtype != UAD_DTYPE_F32 && a.dtype != UAD_DTYPE_BF16) return bad("dtype");
   if (a.n_layers < 0 || a.n_layers > 256) return bad("n_layers");
   if (a.width < 32 || a.width % 32 || a.width > 8192) return bad("width (multiple of 32, <= 8192)");
@@ -248,8 +262,12 @@ void sinusoid_row(double t, int width, double scale, float* out) {
   }
 }
 
+// Offset in a table row of the time half of the time-concatenating expert's input MLP.
+int concat_off(const uad_ctx* c) { return c->a.n_layers * 6 * c->a.width + 2 * c->a.width; }
+
 // Fill time-conditioning rows for new flow times (App. C.1): time MLP then every layer's
-// modulation Linear, one GEMM each over all new times.
+// modulation Linear, one GEMM each over all new times; for the time-concatenating expert also
+// e(tau) W_it + b_it.
 int fill_times(uad_ctx* c, const std::vector<std::pair<int, int>>& fr, cudaStream_t s) {
   if (fr.empty()) return UAD_OK;
   const int n = (int)fr.size(), W = c->a.width;
@@ -267,6 +285,14 @@ int fill_times(uad_ctx* c, const std::vector<std::pair<int, int>>& fr, cudaStrea
   g.A = c->tc2; g.W = c->w_mod; g.N = c->rowlen; g.epi = EPI_STORE; g.bias = c->b_mod;
   g.out = c->tab + (size_t)c->tab_rows * c->rowlen; g.ldo = c->rowlen;
   launch_gemm_simt(g, s);
+  if (c->a.kind == UAD_KIND_CONCAT) {
+    // the time half of the input MLP: e(tau) W_it + b_it after the (constant) modulation
+    GemmArgs t;
+    t.A = c->temb; t.lda = W; t.a_dtype = F32; t.W = c->w_it; t.w_dtype = c->a.dtype;
+    t.M = n; t.N = W; t.K = W; t.epi = EPI_STORE; t.bias = c->b_it;
+    t.out = c->tab + (size_t)c->tab_rows * c->rowlen + concat_off(c); t.ldo = c->rowlen;
+    launch_gemm_simt(t, s);
+  }
   CK(cudaGetLastError());
   for (int r = 0; r < n; ++r) c->tau_row[fr[r]] = c->tab_rows + r;
   c->tab_rows += n;
@@ -573,6 +599,20 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, bool step, cudaStream_t s) {
       gi.M = M; gi.N = W; gi.K = D; gi.epi = EPI_STORE; gi.out = c->h; gi.ldo = W; gi.bias = c->b_in;
       if (dit) { gi.add_rows = c->pos_code; gi.add_mod = H; }
       { Mark mk(c, s, "in_proj", gemm_bytes(gi, c->es), 2.0 * M * W * D); gemm(c, c->w_in, gi, s); }
+      if (a.kind == UAD_KIND_CONCAT) {
+        // the input MLP over [action embedding ; time embedding] (App. C.1, SmolVLA): the time
+        // half e(tau) W_it + b_it is a table slice per flow time
+        launch_convert(c->h, F32, c->y, dt, (long long)M * W, s);
+        GemmArgs ga;
+        ga.A = c->y; ga.lda = W; ga.a_dtype = dt; ga.w_dtype = dt;
+        ga.M = M; ga.N = W; ga.K = W; ga.epi = EPI_STORE; ga.out = c->h; ga.ldo = W; ga.out_dtype = F32;
+        { Mark mk(c, s, "in_mlp_a", gemm_bytes(ga, c->es), 2.0 * M * W * W); gemm(c, c->w_ia, ga, s); }
+        { Mark mk(c, s, "in_mlp_silu", 12.0 * M * W, 0); launch_add_tau_silu(c->h, c->tab, c->rowlen, concat_off(c), tr, M, W, c->y, dt, s); }
+        GemmArgs go;
+        go.A = c->y; go.lda = W; go.a_dtype = dt; go.w_dtype = dt;
+        go.M = M; go.N = W; go.K = W; go.epi = EPI_STORE; go.out = c->h; go.ldo = W; go.out_dtype = F32; go.bias = c->b_io;
+        { Mark mk(c, s, "in_mlp_out", gemm_bytes(go, c->es), 2.0 * M * W * W); gemm(c, c->w_io, go, s); }
+      }
       for (int l = 0; l < a.n_layers; ++l) {
         const LayerW& w = c->L[l];
         const int base = l * W6;
@@ -697,7 +737,8 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, bool step, cudaStream_t s) {
 int launches_per_step(const uad_ctx* c, int B) {
   const uad_arch& a = c->a;
   if (step_path(c, B)) return 2;   // persistent evaluation kernel + Euler step
-  return a.kind == UAD_KIND_DIT ? 11 * a.n_layers + 4 : (c->attn_tc ? 8 : 7) * a.n_layers + 4;
+  return a.kind == UAD_KIND_DIT ? 11 * a.n_layers + 4
+                                 : (c->attn_tc ? 8 : 7) * a.n_layers + 4 + (a.kind == UAD_KIND_CONCAT ? 4 : 0);
 }
 
 }  // namespace
@@ -773,7 +814,7 @@ int uad_init(const uad_arch* arch, const float* weights, size_t n_floats, uad_ct
   c->qd = a.n_heads * a.head_dim;
   c->kvd = a.n_kv_heads * a.head_dim;
   c->qkvd = a.kind == UAD_KIND_DIT ? 3 * c->qd : c->qd + 2 * c->kvd;
-  c->rowlen = a.n_layers * 6 * W + 2 * W;
+  c->rowlen = a.n_layers * 6 * W + 2 * W + (a.kind == UAD_KIND_CONCAT ? W : 0);
   c->mmax = a.max_batch * H;
   const int es = c->es;
 
@@ -798,7 +839,29 @@ int uad_init(const uad_arch* arch, const float* weights, size_t n_floats, uad_ct
     return cudaMemcpy(*dst, src(n), T.at(n)->cols * 4, cudaMemcpyDeviceToDevice) == cudaSuccess
                ? UAD_OK : fail(c, UAD_ECUDA, "copy %s", n.c_str());
   };
-  {
+  const bool concat = a.kind == UAD_KIND_CONCAT;
+  if (concat) {
+    // no time MLP and no modulation: zero weights, and biases scale = shift = 0, gate = 1, so
+    // that the adaptive norms are plain RMSNorm and the residuals ungated
+    void* p;
+    TRY(dalloc(c, &p, (size_t)W * W * es)); c->t_w1 = (float*)p;
+    TRY(dalloc(c, &p, (size_t)W * W * es)); c->t_w2 = (float*)p;
+    TRY(dalloc_t(c, &c->t_b1, (size_t)W)); TRY(dalloc_t(c, &c->t_b2, (size_t)W));
+    TRY(dalloc(c, &c->w_in, (size_t)W * D * es)); lin("in_w", c->w_in, 1, 0);
+    TRY(vec("in_b", &c->b_in));
+    TRY(dalloc(c, &c->w_out, (size_t)W * D * es)); lin("out_w", c->w_out, 1, 0);
+    TRY(vec("out_b", &c->b_out));
+    TRY(dalloc(c, &c->w_mod, (size_t)c->rowlen * W * es));
+    TRY(dalloc_t(c, &c->b_mod, (size_t)c->rowlen));
+    std::vector<float> bm((size_t)c->rowlen, 0.f);
+    for (int l = 0; l < a.n_layers; ++l)
+      for (int half = 0; half < 2; ++half)
+        std::fill(bm.begin() + (size_t)l * 6 * W + half * 3 * W + 2 * W, bm.begin() + (size_t)l * 6 * W + half * 3 * W + 3 * W, 1.f);
+    CK(cudaMemcpy(c->b_mod, bm.data(), bm.size() * 4, cudaMemcpyHostToDevice));
+    TRY(dalloc(c, &c->w_it, (size_t)W * W * es)); lin("ti_wt", c->w_it, 1, 0);
+    TRY(vec("ti_b", &c->b_it));
+    TRY(vec("to_b", &c->b_io));
+  } else {
     void* p;
     TRY(dalloc(c, &p, (size_t)W * W * es)); c->t_w1 = (float*)p; lin("t_w1", p, 1, 0);
     TRY(dalloc(c, &p, (size_t)W * W * es)); c->t_w2 = (float*)p; lin("t_w2", p, 1, 0);
@@ -838,7 +901,7 @@ int uad_init(const uad_arch* arch, const float* weights, size_t n_floats, uad_ct
     else lin(n, l.w, mult, off);
   };
   // tensor-core attention: bf16 joint-attention experts whose QKV projection is tiled
-  c->attn_tc = a.kind == UAD_KIND_ADARMS && dt == BF16 && !c->force_simt && c->qkvd % 128 == 0 && W % 64 == 0 &&
+  c->attn_tc = a.kind != UAD_KIND_DIT && dt == BF16 && !c->force_simt && c->qkvd % 128 == 0 && W % 64 == 0 &&
               a.prefix_len + H <= attn_tc_max_keys();
   const int qk_perm = c->attn_tc && a.rope ? a.head_dim : 0;
   for (int l = 0; l < a.n_layers; ++l) {
@@ -849,7 +912,7 @@ int uad_init(const uad_arch* arch, const float* weights, size_t n_floats, uad_ct
     put(p + "wk", w.wqkv, 1, c->qd, qk_perm);
     put(p + "wv", w.wqkv, 1, c->qd + (a.kind == UAD_KIND_DIT ? c->qd : c->kvd));
     TRY(mklin(&w.wo, W, c->qd)); put(p + "wo", w.wo, 1, 0);
-    if (a.kind == UAD_KIND_ADARMS) {
+    if (a.kind != UAD_KIND_DIT) {
       TRY(mklin(&w.wgu, 2 * F, W));
       put(p + "wg", w.wgu, 2, 0);
       put(p + "wu", w.wgu, 2, 1);
@@ -864,6 +927,10 @@ int uad_init(const uad_arch* arch, const float* weights, size_t n_floats, uad_ct
       TRY(vec(p + "b1", &w.b1)); TRY(vec(p + "b2", &w.b2));
     }
   }
+  if (concat) {
+    TRY(mklin(&c->w_ia, W, W)); put("ti_wa", c->w_ia, 1, 0);
+    TRY(mklin(&c->w_io, W, W)); put("to_w", c->w_io, 1, 0);
+  }
   if (cudaDeviceSynchronize() != cudaSuccess || cudaGetLastError() != cudaSuccess) {
     fail(c, UAD_ECUDA, "weight re-layout failed");
     TRY(UAD_ECUDA);
@@ -877,7 +944,7 @@ int uad_init(const uad_arch* arch, const float* weights, size_t n_floats, uad_ct
   TRY(dalloc_t(c, &c->temb, (size_t)c->tab_cap * W));
   TRY(dalloc_t(c, &c->tc1, (size_t)c->tab_cap * W));
   TRY(dalloc_t(c, &c->tc2, (size_t)c->tab_cap * W));
-  if (a.kind == UAD_KIND_ADARMS && a.rope) {
+  if (a.kind != UAD_KIND_DIT && a.rope) {
     const int dh = a.head_dim, half = dh / 2;
     std::vector<float> cs((size_t)H * dh);
     for (int i = 0; i < H; ++i)
@@ -984,7 +1051,7 @@ int uad_set_prefix_kv(uad_ctx* c, int32_t robot, const void* k, const void* v, i
   if (c->in_flight) return fail(c, UAD_ESTATE, "a chunk is in flight");
   const int ies = dtype == UAD_DTYPE_BF16 ? 2 : 4;
   cudaStream_t s = c->worker;
-  if (a.kind == UAD_KIND_ADARMS && c->attn_tc) {
+  if (a.kind != UAD_KIND_DIT && c->attn_tc) {
     if (!v) return fail(c, UAD_EINVAL, "null prefix values");
     const size_t n = (size_t)a.n_layers * a.prefix_len * c->kvd;
     void *tk = nullptr, *tv = nullptr;
@@ -1001,7 +1068,7 @@ int uad_set_prefix_kv(uad_ctx* c, int32_t robot, const void* k, const void* v, i
     cudaFree(tv);
     if (rc != UAD_OK || e != cudaSuccess || cudaGetLastError() != cudaSuccess)
       return fail(c, UAD_ECUDA, "prefix upload failed");
-  } else if (a.kind == UAD_KIND_ADARMS) {
+  } else if (a.kind != UAD_KIND_DIT) {
     if (!v) return fail(c, UAD_EINVAL, "null prefix values");
     const size_t n = (size_t)a.n_layers * a.prefix_len * c->kvd;
     void* tmp = nullptr;

@@ -143,6 +143,10 @@ void launch_relayout(const float* src, int K, int N, void* dst, int dtype, int m
 size_t attention_smem_bytes(int dh);
 void launch_attention_prepare(int dh);  // opt in to > 48 KB dynamic shared memory (call once)
 void launch_convert(const void* src, int src_dtype, void* dst, int dst_dtype, long long n, cudaStream_t s);
+// y[m][n] = SiLU(x[m][n] + tab[tau_row[m] * stride + off + n]) in dtype dt (the input MLP of the
+// time-concatenating expert: the table holds e(tau) W_it + b_it per flow time)
+void launch_add_tau_silu(const float* x, const float* tab, int stride, int off, const int* tau_row, int M, int N,
+                         void* y, int dt, cudaStream_t s);
 
 // gemm_tc.cu: tcgen05 projection GEMM (bf16 operands, fp32 accumulation in TMEM)
 constexpr int kTcMaxStages = 4;        // <= ~97 KB of shared memory: two CTAs fit one SM

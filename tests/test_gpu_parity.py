@@ -275,6 +275,21 @@ def test_batched_robots_own_schedules():
         c.close()
 
 
+@pytest.mark.parametrize("name", ["tiny_concat", "concat_small"])
+def test_time_concatenating_expert(name):
+    """SmolVLA-style per-action time conditioning (App. C.1: each token's time embedding joins its
+    action embedding before the action MLP), fp32 on CUDA cores and bf16 on the tensor cores."""
+    a = ARCHS[name]
+    c = Case(a, seed=16)
+    try:
+        noise = make_noise(a, seed=16)
+        H = a.chunk_len
+        bud = group_budgets(H, [(0, 3, 4), (4, H // 2, 7), (H // 2 + 1, H - 1, 10)])
+        check(c, c.gpu(noise, bud), c.oracle(noise, bud), bud, TOL[a.dtype])
+    finally:
+        c.close()
+
+
 # ---- full-size workloads -----------------------------------------------------------------------
 def test_pi0_full_three_groups():
     """pi0-like bf16 expert, B = 1, groups 0-9 @ 4, 10-24 @ 7, 25-49 @ 10 (all outputs)."""
