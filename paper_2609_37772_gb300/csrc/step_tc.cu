@@ -3,8 +3,8 @@
 //
 // With few tokens an evaluation is a chain of dependent steps per layer, each far too small to
 // fill the GPU; its cost is the latency of that chain, not the weight bytes. The kernel keeps the
-// chain short: six grid barriers per layer, every elementwise step fused into the epilogue of the
-// projection that produces its input. One producer thread per CTA streams this CTA's share of
+// chain short: every elementwise step is fused into the epilogue of the projection that produces
+// its input, and the phases of a layer wait on completion counts rather than grid barriers. One producer thread per CTA streams this CTA's share of
 // every projection weight through a shared-memory ring without waiting for the barriers (the
 // weights do not depend on the activations).
 //
@@ -16,8 +16,8 @@
 // The consumer of the projection applies rstd (from row sums of squares accumulated by the
 // producers of h) and adds the shift row of the token's flow time.
 //
-// Phases (each ends at a grid barrier; the last CTA to finish an output block of a projection,
-// counted per block, runs that block's epilogue):
+// Phases (the CTAs that add into an output block of a projection count their arrivals on the
+// block; each of them then runs the block's epilogue for a share of its rows):
 //   in       row m: h = W_in u + b_in, sum h^2, z = h (1 + scale1); shift rows of layer 0
 //   qkv      acc += z W_qkv^T;  block epilogue: rstd * acc + shift row, RoPE, q -> Q, k -> K
 //            cache, v -> Vt cache
@@ -32,8 +32,8 @@
 // then the final norm and the action-out projection v = W_out y + b_out (row m). The epilogue
 // that reads an accumulator block clears it, so the next use starts from zero.
 //
-// Warps: 0-3 = consumers (TMEM lane quadrants 0-3; epilogues and row steps), 4 = weight producer
-// (lane 0), 5 = tcgen05 issuer and TMA loads of activations and attention operands (lane 0).
+// Warps: 0-7 = consumers (tensor-memory readout, epilogues, row steps, chunk merges), 8 = weight
+// producer (lane 0), 9 = tcgen05 issuer and TMA loads of activations and attention operands (lane 0).
 // Every wait is bounded: on timeout the kernel records an error code, skips the remaining
 // work, waits (bounded) for its copies in flight and frees its tensor memory.
 #include <cuda.h>
@@ -80,6 +80,14 @@ __device__ __forceinline__ bool mbar_test(uint64_t* b, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok) : "r"(su32(b)), "r"(parity) : "memory");
+  return ok != 0;
+}
+// Non-blocking test of the phase with the given parity (returns at once).
+__device__ __forceinline__ bool mbar_peek(uint64_t* b, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
       : "=r"(ok) : "r"(su32(b)), "r"(parity) : "memory");
   return ok != 0;
 }
@@ -358,6 +366,8 @@ struct StepShared {
   int nsh;                           // distinct flow times (shift rows of z)
   int srow[kStepMaxShift];           // their modulation-table rows
   int sidx[kMaxRows];                // token -> index of its flow time
+  uint8_t row_b[kMaxRows];           // token -> its robot (row / H)
+  uint8_t row_i[kMaxRows];           // token -> its position in the chunk (row % H)
   Tiles tiles[4];                    // this CTA's tiles of the qkv, o, gate/up, down projections
   int fused_combine;                 // idle CTAs of the attention step merge the key chunks; the
                                      // phases of a layer then wait on counts, not grid barriers
@@ -557,7 +567,8 @@ __device__ __forceinline__ void clear_shift_rows(const StepShared& __restrict__ 
 
 // qkv block b, rows [r0, r1): value = rstd(h_m) * acc[m] + acc[M + sidx[m]]; RoPE on q/k
 // pairs; q -> Q, k -> K cache, v -> Vt cache (bf16). Lane owns 4 consecutive features (two
-// RoPE pairs), whose (cos, sin) are staged per row next to the accumulator rows.
+// RoPE pairs), whose (cos, sin) are staged per row next to the accumulator rows. DH = head dim.
+template <int DH>
 __device__ __noinline__ void epi_qkv(const StepShared& __restrict__ sh, int l, int b, int r0, int r1, uint8_t* X) {
   const StepArgs& p = sh.p;
   const int M = p.M, warp = threadIdx.x >> 5, lane = threadIdx.x & 31, c0 = b * 128;
@@ -566,13 +577,16 @@ __device__ __noinline__ void epi_qkv(const StepShared& __restrict__ sh, int l, i
   float* rs = CS + kMaxRows * 128;
   stage_rows(A, p.acc_qkv, p.qkvd, c0, r0, r1);
   stage_rows(A, p.acc_qkv, p.qkvd, c0, M, M + sh.nsh);
-  const int dh = p.dh, half = dh / 2, n = c0 + 4 * lane;
-  const bool qk = n < p.qd + p.kvd;
-  const int sn = n < p.qd ? n : n - p.qd;
+  constexpr int half = DH / 2;
+  const int n = c0 + 4 * lane;
+  const bool qk = n < p.qd + p.kvd, isq = n < p.qd;
+  const int sn = isq ? n : n - p.qd;             // feature within q, or within k
+  const int hh = sn / DH, rr0 = sn % DH;         // head and dim of the lane's first feature
+  const int ev = n - p.qd - p.kvd;               // feature within v
   if (qk && p.rope) {
 #pragma unroll 1
     for (int m = r0 + warp; m < r1; m += kConsWarps)
-      cp16(CS + m * 128 + 4 * lane, p.rope_cs + (size_t)(m % p.H) * dh + ((sn % dh) >> 1) * 2);
+      cp16(CS + m * 128 + 4 * lane, p.rope_cs + (size_t)sh.row_i[m] * DH + (rr0 >> 1) * 2);
   }
   const float* s1 = sumsq_slot(p, l, 0);
   for (int m = r0 + threadIdx.x; m < r1; m += kCons) rs[m] = rsqrtf(__ldcg(s1 + m) / p.W + 1e-6f);
@@ -585,29 +599,25 @@ __device__ __noinline__ void epi_qkv(const StepShared& __restrict__ sh, int l, i
     const float4 a = *reinterpret_cast<const float4*>(A + m * 128 + 4 * lane);
     const float4 s = *reinterpret_cast<const float4*>(A + (M + sh.sidx[m]) * 128 + 4 * lane);
     const float v[4] = {fmaf(r, a.x, s.x), fmaf(r, a.y, s.y), fmaf(r, a.z, s.z), fmaf(r, a.w, s.w)};
-    const int rb = m / p.H, i = m % p.H;
+    const int rb = sh.row_b[m], i = sh.row_i[m];
     if (qk) {
-      const bool isq = n < p.qd;
-      const int hh = sn / dh;
-      __nv_bfloat16* dst = isq ? p.q + (((size_t)rb * p.n_heads + hh) * p.H + i) * dh
-                               : p.kcache + ((((size_t)rb * p.L + l) * p.n_kv_heads + hh) * p.n_keys + p.P + i) * dh;
+      __nv_bfloat16* dst = isq ? p.q + (((size_t)rb * p.n_heads + hh) * p.H + i) * DH
+                               : p.kcache + ((((size_t)rb * p.L + l) * p.n_kv_heads + hh) * p.n_keys + p.P + i) * DH;
       const float4 cs = p.rope ? *reinterpret_cast<const float4*>(CS + m * 128 + 4 * lane) : make_float4(1.f, 0.f, 1.f, 0.f);
 #pragma unroll
       for (int e = 0; e < 4; e += 2) {
-        const int rr = (sn + e) % dh;
+        const int rr = rr0 + e;   // the lane's 4 features lie in one head (DH is a multiple of 4)
         const float c = e ? cs.z : cs.x, si = e ? cs.w : cs.y;
-        // with RoPE, rows 2j, 2j+1 of a head hold dims j and j + dh/2 (pair-interleaved weights)
+        // with RoPE, rows 2j, 2j+1 of a head hold dims j and j + DH/2 (pair-interleaved weights)
         const int d0 = p.rope ? (rr >> 1) : rr, d1 = p.rope ? (rr >> 1) + half : rr + 1;
         dst[d0] = __float2bfloat16_rn(v[e] * c - v[e + 1] * si);
         dst[d1] = __float2bfloat16_rn(v[e + 1] * c + v[e] * si);
       }
     } else {
-      const int ev = n - p.qd - p.kvd;
+      const int g = ev / DH, d = ev % DH;   // the lane's 4 features lie in one head
+      __nv_bfloat16* dst = p.vtcache + ((((size_t)rb * p.L + l) * p.n_kv_heads + g) * DH + d) * p.nk_pad + p.P + i;
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int g = (ev + e) / dh, d = (ev + e) % dh;
-        p.vtcache[((((size_t)rb * p.L + l) * p.n_kv_heads + g) * dh + d) * p.nk_pad + p.P + i] = __float2bfloat16_rn(v[e]);
-      }
+      for (int e = 0; e < 4; ++e) dst[(size_t)e * p.nk_pad] = __float2bfloat16_rn(v[e]);
     }
   }
 }
@@ -800,9 +810,11 @@ __device__ __noinline__ void combine_rows(const StepArgs& __restrict__ p, uint8_
 }  // namespace
 
 // ---- projection step: acc[m][n] += sum over this CTA's weight tiles of A[m][k] W[n][k] -----
-// Thread 160 loads the activation tiles (tensor map) and issues the MMAs against the weight
+// The issuer thread loads the activation tiles (tensor map) and issues the MMAs against the weight
 // ring; the consumer warps add the finished 128 x 64 tile into `acc` (fp32, L2) with 16-byte
-// reds, then count the block's arrival; the last of its CTAs runs the block's epilogue.
+// reds and count the block's arrival; once every CTA of the block has arrived, each runs the
+// block's epilogue for its share of the rows.
+template <int DH>
 __device__ __noinline__ void projection_step(const StepShared& __restrict__ sh, const CUtensorMap* amap, int l, int j,
                                              uint32_t tmem, size_t xbytes, Role& st) {
   const StepArgs& p = sh.p;
@@ -819,17 +831,24 @@ __device__ __noinline__ void projection_step(const StepShared& __restrict__ sh, 
     mbar_expect_tx(S.a_full, (uint32_t)nt * kATile);
     for (int i = 0; i < nt; ++i) tma_2d(S.X + (size_t)i * kATile, amap, (tl.k0 + i) * 64, 0, S.a_full);
     ++st.a_uses;
+    // the next weight tile's barrier is tested (without blocking) before the current tile's MMAs
+    // are issued, so that the test's latency overlaps the issue
+    bool ready = mbar_peek(S.full + st.slot, st.par);
     bool good = mbar_wait(S.a_full, st.apar, p.err, 42);
     for (int i = 0; i < nt && good; ++i) {
-      good = mbar_wait(S.full + st.slot, st.par, p.err, 43);
-      if (!good) break;
+      if (!ready) {
+        good = mbar_wait(S.full + st.slot, st.par, p.err, 43);
+        if (!good) break;
+      }
       tc_fence_after();
-      const uint32_t a0 = su32(S.ring + (size_t)st.slot * kSlot), b0 = su32(S.X + (size_t)i * kATile);
+      const int cur = st.slot;
+      if (++st.slot == p.ring) { st.slot = 0; st.par ^= 1u; }
+      ready = i + 1 < nt && mbar_peek(S.full + st.slot, st.par);
+      const uint32_t a0 = su32(S.ring + (size_t)cur * kSlot), b0 = su32(S.X + (size_t)i * kATile);
 #pragma unroll
       for (int k = 0; k < 4; ++k)
         mma_bf16(tmem, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), idesc_m128(64), (i | k) ? 1u : 0u);
-      mma_commit(S.empty + st.slot);
-      if (++st.slot == p.ring) { st.slot = 0; st.par ^= 1u; }
+      mma_commit(S.empty + cur);
     }
     mma_commit(S.g_done);
   }
@@ -876,7 +895,7 @@ __device__ __noinline__ void projection_step(const StepShared& __restrict__ sh, 
     if (*reinterpret_cast<volatile int*>(S.last)) {
       const int W6 = 6 * p.W, b6 = l * W6, M = p.M;
       const int r0 = tl.idx * M / tl.contrib, r1 = (tl.idx + 1) * M / tl.contrib;
-      if (j == 0) epi_qkv(sh, l, tl.b, r0, r1, S.X);
+      if (j == 0) epi_qkv<DH>(sh, l, tl.b, r0, r1, S.X);
       else if (j == 2) epi_geglu(sh, l, tl.b, r0, r1, S.X);
       else if (j == 1) epi_resid(sh, p.acc_o, b6 + 2 * p.W, b6 + 3 * p.W, sumsq_slot(p, l, 1), tl.b, r0, r1, tl.idx == 0, S.X);
       else epi_resid(sh, p.acc_d, b6 + 5 * p.W, l + 1 < p.L ? b6 + W6 : -1, sumsq_slot(p, l + 1, 0), tl.b, r0, r1,
@@ -1110,6 +1129,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x < kMaxRows) {
     const int si = threadIdx.x < p_in.M ? __ldg(p_in.sidx + threadIdx.x) : 0;
     sh.sidx[threadIdx.x] = si >= 0 && si < kStepMaxShift ? si : 0;
+    sh.row_b[threadIdx.x] = (uint8_t)(threadIdx.x / p_in.H);
+    sh.row_i[threadIdx.x] = (uint8_t)(threadIdx.x % p_in.H);
   }
   if (threadIdx.x == 68) {
     const int items = p_in.B * p_in.n_kv_heads * (p_in.r_pad / kQT) * p_in.n_chunks;
@@ -1174,7 +1195,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     ok = grid_sync(bar++, ok, p.err, S);
     for (int l = 0; l < p.L; ++l) {
       const bool df = sh.fused_combine != 0;   // phases inside the layer wait on counts
-      if (ok) projection_step(sh, &t_z, l, 0, tmem, XB, st);
+      if (ok) projection_step<DH>(sh, &t_z, l, 0, tmem, XB, st);
       ok = df ? phase_wait(done_ctr(p, l, 0), sh.shares[0], ok, p.err, S) : grid_sync(bar++, ok, p.err, S);
       if (ok) attention_step<DH>(p, &t_q, &t_k, &t_vt, l, tmem, st, df);
       if (df) {
@@ -1184,13 +1205,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (ok && cons) combine_rows<DH>(p, S.X, S.cbar + warp, st);
         ok = grid_sync(bar++, ok, p.err, S);
       }
-      if (ok) projection_step(sh, &t_o, l, 1, tmem, XB, st);
+      if (ok) projection_step<DH>(sh, &t_o, l, 1, tmem, XB, st);
       ok = df ? phase_wait(done_ctr(p, l, 1), sh.shares[1], ok, p.err, S) : grid_sync(bar++, ok, p.err, S);
-      if (ok) projection_step(sh, &t_z, l, 2, tmem, XB, st);
+      if (ok) projection_step<DH>(sh, &t_z, l, 2, tmem, XB, st);
       ok = df ? phase_wait(done_ctr(p, l, 2), sh.shares[2], ok, p.err, S) : grid_sync(bar++, ok, p.err, S);
       // the shift rows of this layer's qkv and gate/up sums have been read by now
       if (ok && cons) clear_shift_rows(sh, true, true);
-      if (ok) projection_step(sh, &t_act, l, 3, tmem, XB, st);
+      if (ok) projection_step<DH>(sh, &t_act, l, 3, tmem, XB, st);
       ok = grid_sync(bar++, ok, p.err, S);
     }
     if (ok && cons && (int)blockIdx.x < p.M) final_row(p, blockIdx.x, reinterpret_cast<float*>(S.X));
