@@ -423,7 +423,6 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
 // ---- wide tiles for many tokens: 128 weight rows x 256 tokens per CTA, no K split ----------
 constexpr int kWN = 256;                       // tokens per tile (MMA N)
 constexpr int kWStageB = kWN * kBK * 2;        // 32 KB activation block per stage
-constexpr int kWStages = 4;
 constexpr uint32_t kIdescWide = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kWN >> 3) << 17) |
                                 ((uint32_t)(kBM >> 4) << 24);
 
@@ -433,7 +432,11 @@ __device__ __forceinline__ void mma_bf16_wide(uint32_t d, uint64_t a, uint64_t b
       ::"r"(d), "l"(a), "l"(b), "r"(kIdescWide), "r"(accum));
 }
 
-__global__ void __launch_bounds__(128, 1) gemm_tc_wide_kernel(const __grid_constant__ CUtensorMap tmx, TcGemmArgs p) {
+// STAGES pipeline stages of 48 KB; MINB CTAs per SM (two with two stages: one CTA's epilogue then
+// overlaps the other's main loop, which pays when there are more tiles than SMs).
+template <int STAGES, int MINB>
+__global__ void __launch_bounds__(128, MINB) gemm_tc_wide_kernel(const __grid_constant__ CUtensorMap tmx, TcGemmArgs p) {
+  constexpr int kWStages = STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   const int t = blockIdx.x, mt = blockIdx.y;
@@ -592,19 +595,24 @@ size_t gemm_tc_smem_bytes(int stages, int epi, int M) {
   return 1024 + tc_pipe_bytes(stages) + (2 * kTcMaxStages + 1) * 8 + 16;
 }
 
-static size_t gemm_tc_wide_smem_bytes() { return 1024 + (size_t)kWStages * (kStageA + kWStageB) + (2 * kWStages + 2) * 8 + 16; }
+static size_t gemm_tc_wide_smem_bytes(int stages) { return 1024 + (size_t)stages * (kStageA + kWStageB) + (2 * stages + 2) * 8 + 16; }
 
 void gemm_tc_prepare() {
   const size_t a = gemm_tc_smem_bytes(kTcMaxStages, EPI_STORE, kBN);
   cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)a);
-  cudaFuncSetAttribute(gemm_tc_wide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)gemm_tc_wide_smem_bytes());
+  cudaFuncSetAttribute(gemm_tc_wide_kernel<4, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)gemm_tc_wide_smem_bytes(4));
+  cudaFuncSetAttribute(gemm_tc_wide_kernel<2, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)gemm_tc_wide_smem_bytes(2));
 }
 
-// Wide tiles cut L2 re-reads of the weights (one CTA per 256 tokens instead of 64) but hold a
-// whole SM; for very wide outputs (gate/up at N = 8192) two narrow CTAs per SM overlap one
-// CTA's epilogue with the other's main loop and win.
-bool gemm_tc_use_wide(int M, int N, int sms) {
-  return M >= kWN && N <= 4096 && (N / kBM) * ((M + kWN - 1) / kWN) * 2 >= sms;
+// Wide tiles (MMA N = 256 tokens) run the tensor cores near their rate and cut L2 re-reads of
+// the weights (one CTA per 256 tokens instead of 64). Returns 0 (narrow tiles), 1 (four stages,
+// one CTA per SM) or 2 (two stages, two CTAs per SM: with at least as many tiles as SMs, one
+// CTA's epilogue then overlaps the other's main loop).
+int gemm_tc_use_wide(int M, int N, int sms) {
+  if (M < kWN || N > 8192) return 0;
+  const int tiles = (N / kBM) * ((M + kWN - 1) / kWN);
+  if (tiles * 2 < sms) return 0;
+  return tiles >= sms ? 2 : 1;
 }
 
 // K splits per output tile: one CTA per SM. Partial-plane epilogues (the consumer sums the
@@ -628,8 +636,9 @@ int gemm_tc_splits(int M, int N, int K, int sms, int epi) {
 
 void launch_gemm_tc(const CUtensorMap* tmx, const TcGemmArgs& a, cudaStream_t s) {
   if (a.wide) {
-    launch_k(gemm_tc_wide_kernel, dim3(a.N / kBM, (a.M + kWN - 1) / kWN), dim3(128), gemm_tc_wide_smem_bytes(), s,
-             *tmx, a);
+    const dim3 grid(a.N / kBM, (a.M + kWN - 1) / kWN);
+    if (a.wide == 2) launch_k(gemm_tc_wide_kernel<2, 2>, grid, dim3(128), gemm_tc_wide_smem_bytes(2), s, *tmx, a);
+    else launch_k(gemm_tc_wide_kernel<4, 1>, grid, dim3(128), gemm_tc_wide_smem_bytes(4), s, *tmx, a);
     return;
   }
   const int KC = a.K / kBK;
