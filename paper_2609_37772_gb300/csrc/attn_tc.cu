@@ -275,12 +275,15 @@ __global__ void __launch_bounds__(128, 1) attn_tc_kernel(const __grid_constant__
 }
 
 // ---- two-pass attention for many query tiles: no partials, no combine --------------------
-// One CTA per (128-row query tile, robot-group). Keys in chunks of 64 through a 2-slot ring.
-// Pass 1: S = Q K_c^T on tcgen05 (double-buffered in TMEM), row maxima in registers.
+// One CTA per (128-row query tile, robot-group). Keys in chunks of 128 (S = Q K^T with MMA N = 128,
+// twice the tensor rate of 64-key chunks). Shared memory: Q, two 64 KB regions, P.
+// Pass 1: S = Q K_c^T on tcgen05 (double-buffered in TMEM), row maxima in registers; K chunks
+// alternate between the two regions.
 // Pass 2: S again, P = exp(S - max) in bf16 into shared memory, O += P V_c on tcgen05 (no
-// rescaling: the maxima are final), row sums of the rounded P. O / l is written in bf16.
-constexpr int kKC2 = 64;                        // keys per chunk
-constexpr uint32_t kTmem2 = 512;                // S buffers at columns [0,64) and [64,128), O at [128, 128+dh)
+// rescaling: the maxima are final), row sums of the rounded P; K in region 0, Vt in region 1.
+// O / l is written in bf16.
+constexpr int kKC2 = 128;                       // keys per chunk
+constexpr uint32_t kTmem2 = 512;                // S buffers at columns [0,128) and [128,256), O at [256, 256+dh)
 
 // Warps 0-3: softmax and output (they own the four TMEM lane quadrants); warp 4: TMA producer;
 // warp 5: MMA issuer. The producer and issuer wait on the softmax warps' progress, so they must
@@ -292,18 +295,18 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   constexpr int NC = DH / 64;
-  constexpr uint32_t QB = DH * kQT * 2;          // Q: NC blocks of 128 x 64
-  constexpr uint32_t KB = DH * kKC2 * 2;         // one K chunk: NC blocks of 64 x 64
-  constexpr uint32_t VB = DH * kKC2 * 2;         // one Vt chunk: dh x 64 keys
-  constexpr uint32_t PB = kQT * kKC2 * 2;        // P: 128 x 64
+  constexpr uint32_t QB = DH * kQT * 2;          // Q: NC blocks of 128 rows x 64
+  constexpr uint32_t RB = DH * kKC2 * 2;         // a K chunk (NC blocks of 128 keys x 64) or a Vt
+                                                 // chunk (2 blocks of dh x 64 keys)
+  constexpr uint32_t PB = kQT * kKC2 * 2;        // P: 2 blocks of 128 rows x 64 keys
+  constexpr uint32_t VBLK = DH * 128;            // one Vt block: dh rows x 64 keys
   uint8_t* sQ = smem;
-  uint8_t* sK = sQ + QB;                         // 2 slots
-  uint8_t* sV = sK + 2 * KB;                     // 2 slots
-  uint8_t* sP = sV + 2 * VB;
+  uint8_t* sR = sQ + QB;                         // regions 0 and 1
+  uint8_t* sP = sR + 2 * RB;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sP + PB);
   uint64_t* q_full = bars;          // Q landed
-  uint64_t* kv_full = bars + 1;     // [2] chunk landed in slot
-  uint64_t* kv_empty = bars + 3;    // [2] slot free (MMAs that read it are done)
+  uint64_t* full = bars + 1;        // [2] region loaded
+  uint64_t* empty = bars + 3;       // [2] region free (the MMAs that read it are done)
   uint64_t* s_full = bars + 5;      // [2] S buffer written
   uint64_t* s_empty = bars + 7;     // [2] S buffer read by the 4 warps
   uint64_t* p_full = bars + 9;      // P written by the 4 warps
@@ -320,8 +323,8 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
     for (int i = 0; i < 2; ++i) {
-      mbar_init(kv_full + i, 1);
-      mbar_init(kv_empty + i, 1);
+      mbar_init(full + i, 1);
+      mbar_init(empty + i, 1);
       mbar_init(s_full + i, 1);
       mbar_init(s_empty + i, 4);
     }
@@ -342,34 +345,48 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
   pdl_trigger();
   pdl_wait();
 
-  // chunk sequence: pass 1 loads K only (n = 0..nck-1), pass 2 loads K and Vt (n = nck..2nck-1)
-  const int total = 2 * nck;
+  // load sequence: pass 1 K chunk n into region n & 1 (n < nck); pass 2 K chunk c into region 0,
+  // then Vt chunk c into region 1. Producer and issuer count the uses of each region alike.
   if (threadIdx.x == 128) {
     const uint64_t pol = policy_evict_last();
     mbar_expect_tx(q_full, QB);
 #pragma unroll
     for (int c = 0; c < NC; ++c) tma_3d(sQ + c * (kQT * 128), &tq, c * 64, qt * kQT, bg, q_full, pol);
-    for (int n = 0; n < total; ++n) {
-      const int slot = n & 1, use = n >> 1;
-      if (use > 0 && !mbar_wait(kv_empty + slot, (use - 1) & 1, p.err, 41)) break;
+    int use0 = 0, use1 = 0;   // loads into regions 0 and 1
+    bool ok = true;
+    for (int n = 0; n < 2 * nck && ok; ++n) {
       const bool pass2 = n >= nck;
-      const int key0 = (pass2 ? n - nck : n) * kKC2;
-      mbar_expect_tx(kv_full + slot, pass2 ? KB + VB : KB);
+      const int ch = pass2 ? n - nck : n;
+      for (int part = 0; part < (pass2 ? 2 : 1) && ok; ++part) {
+        const int r = pass2 ? part : (n & 1);
+        const int u = r ? use1++ : use0++;
+        if (u > 0) ok = mbar_wait(empty + r, (u - 1) & 1, p.err, 41);
+        if (!ok) break;
+        uint8_t* dst = sR + r * RB;
+        mbar_expect_tx(full + r, RB);
+        if (part == 0) {
 #pragma unroll
-      for (int c = 0; c < NC; ++c) tma_3d(sK + slot * KB + c * (kKC2 * 128), &tk, c * 64, key0, kvz, kv_full + slot, pol);
-      if (pass2) tma_3d(sV + slot * VB, &tv, key0, 0, kvz, kv_full + slot, pol);
+          for (int c = 0; c < NC; ++c) tma_3d(dst + c * (kKC2 * 128), &tk, c * 64, ch * kKC2, kvz, full + r, pol);
+        } else {
+#pragma unroll
+          for (int kb = 0; kb < 2; ++kb) tma_3d(dst + kb * VBLK, &tv, ch * kKC2 + kb * 64, 0, kvz, full + r, pol);
+        }
+      }
     }
   } else if (threadIdx.x == 160) {
     bool ok = mbar_wait(q_full, 0, p.err, 42);
     const uint32_t q0 = su32(sQ);
-    for (int n = 0; n < total && ok; ++n) {
-      const int slot = n & 1, use = n >> 1, sb = n & 1;
+    int use0 = 0, use1 = 0;   // waits on regions 0 and 1, in the producer's order
+    for (int n = 0; n < 2 * nck && ok; ++n) {
+      const int sb = n & 1;
       const bool pass2 = n >= nck;
-      ok = mbar_wait(kv_full + slot, use & 1, p.err, 43);
+      const int rk = pass2 ? 0 : (n & 1);
+      const int u = rk ? use1++ : use0++;
+      ok = mbar_wait(full + rk, u & 1, p.err, 43);
       if (ok && n >= 2) ok = mbar_wait(s_empty + sb, ((n >> 1) - 1) & 1, p.err, 44);
       if (!ok) break;
       tc_fence_after();
-      const uint32_t k0 = su32(sK + slot * KB);
+      const uint32_t k0 = su32(sR + rk * RB);
 #pragma unroll
       for (int c = 0; c < NC; ++c)
 #pragma unroll
@@ -377,18 +394,19 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
           mma_bf16(tmem + sb * kKC2, sw128_desc(q0 + c * (kQT * 128) + 32 * k),
                    sw128_desc(k0 + c * (kKC2 * 128) + 32 * k), idesc_m128(kKC2), (c | k) ? 1u : 0u);
       mma_commit(s_full + sb);
-      if (!pass2) {
-        mma_commit(kv_empty + slot);
-      } else {
+      mma_commit(empty + rk);
+      if (pass2) {
         const int c2 = n - nck;
-        ok = mbar_wait(p_full, c2 & 1, p.err, 45);
+        ok = mbar_wait(p_full, c2 & 1, p.err, 45) && mbar_wait(full + 1, use1 & 1, p.err, 46);
+        ++use1;
         if (!ok) break;
         tc_fence_after();
-        const uint32_t pp = su32(sP), v0 = su32(sV + slot * VB);
+        const uint32_t pp = su32(sP), v0 = su32(sR + RB);
 #pragma unroll
         for (int k = 0; k < kKC2 / 16; ++k)
-          mma_bf16(tO, sw128_desc(pp + 32 * k), sw128_desc(v0 + 32 * k), idesc_m128(DH), (c2 | k) ? 1u : 0u);
-        mma_commit(kv_empty + slot);
+          mma_bf16(tO, sw128_desc(pp + (k >> 2) * (kQT * 128) + 32 * (k & 3)), sw128_desc(v0 + (k >> 2) * VBLK + 32 * (k & 3)),
+                   idesc_m128(DH), (c2 | k) ? 1u : 0u);
+        mma_commit(empty + 1);
         mma_commit(p_empty);
       }
     }
@@ -407,15 +425,16 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
   float sv[32];
   float mx = -INFINITY, l = 0.f;
   bool ok = true;
-  for (int n = 0; n < total; ++n) {
+  const int r8 = row & 7;
+  for (int n = 0; n < 2 * nck; ++n) {
     const int sb = n & 1;
     const bool pass2 = n >= nck;
     const int key0 = (pass2 ? n - nck : n) * kKC2;
-    ok = ok && mbar_wait(s_full + sb, (n >> 1) & 1, p.err, 46);
+    ok = ok && mbar_wait(s_full + sb, (n >> 1) & 1, p.err, 47);
     tc_fence_after();
     __syncwarp();
     if (!pass2) {
-#pragma unroll
+#pragma unroll 1
       for (int cc = 0; cc < kKC2 / 32; ++cc) {
         tmem_ld32(tmem + sb * kKC2 + lane_base + cc * 32, sv);
 #pragma unroll
@@ -424,25 +443,26 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
       }
     } else {
       const int c2 = n - nck;
-      if (c2 > 0) ok = ok && mbar_wait(p_empty, (c2 - 1) & 1, p.err, 47);
-      const int r8 = row & 7;
-#pragma unroll
+      if (c2 > 0) ok = ok && mbar_wait(p_empty, (c2 - 1) & 1, p.err, 48);
+      const float mxs = mx * c2s;
+#pragma unroll 1
       for (int cc = 0; cc < kKC2 / 32; ++cc) {
         tmem_ld32(tmem + sb * kKC2 + lane_base + cc * 32, sv);
         uint32_t pk[16];
 #pragma unroll
         for (int i = 0; i < 32; i += 2) {
           const bool v0 = key0 + cc * 32 + i < p.n_keys, v1 = key0 + cc * 32 + i + 1 < p.n_keys;
-          const float e0 = v0 ? exp2f((sv[i] - mx) * c2s) : 0.f;
-          const float e1 = v1 ? exp2f((sv[i + 1] - mx) * c2s) : 0.f;
+          const float e0 = v0 ? exp2f(fmaf(sv[i], c2s, -mxs)) : 0.f;
+          const float e1 = v1 ? exp2f(fmaf(sv[i + 1], c2s, -mxs)) : 0.f;
           const __nv_bfloat162 h = __floats2bfloat162_rn(e0, e1);
           l += __low2float(h) + __high2float(h);
           pk[i / 2] = *reinterpret_cast<const uint32_t*>(&h);
         }
-        uint8_t* prow = sP + row * 128;
+        // keys 32 cc .. 32 cc + 31: P block cc / 2, 16-byte groups 4 (cc % 2) .. + 3
+        uint8_t* prow = sP + (cc >> 1) * (kQT * 128) + row * 128;
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-          const int gidx = cc * 4 + q;
+          const int gidx = (cc & 1) * 4 + q;
           *reinterpret_cast<uint4*>(prow + ((gidx ^ r8) * 16)) =
               make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
         }
@@ -456,7 +476,7 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
     __syncwarp();
     if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(s_empty + sb)) : "memory");
   }
-  ok = ok && mbar_wait(o_done, 0, p.err, 48);
+  ok = ok && mbar_wait(o_done, 0, p.err, 49);
   tc_fence_after();
   __syncwarp();
 
@@ -566,7 +586,7 @@ int tmap3(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d
 }  // namespace
 
 size_t attn_tc2_smem_bytes(int dh) {
-  return 1024 + (size_t)dh * kQT * 2 + 4 * (size_t)dh * kKC2 * 2 + (size_t)kQT * kKC2 * 2 + 16 * 8;
+  return 1024 + (size_t)dh * kQT * 2 + 2 * (size_t)dh * kKC2 * 2 + (size_t)kQT * kKC2 * 2 + 16 * 8;
 }
 
 bool attn_tc_use_two_pass(const AttnTcArgs& a) {
@@ -588,9 +608,11 @@ int attn_tc_prepare(AttnTcMaps* maps, const AttnTcArgs& a, int batch_max) {
             NK * dh * 2, 64, kKT)) return -1;
   if (tmap3(&maps->vt, a.vtcache, NK, dh, (uint64_t)batch_max * a.n_layers * a.n_kv_heads, NKp * 2,
             (uint64_t)dh * NKp * 2, 64, (uint32_t)dh)) return -1;
+  // 64-key K boxes for the persistent step kernel's attention items; the two-pass kernel loads
+  // 128-key K chunks through `k` and Vt in 64-key boxes
   if (tmap3(&maps->k2, a.kcache, dh, NK, (uint64_t)batch_max * a.n_layers * a.n_kv_heads, (uint64_t)dh * 2,
-            NK * dh * 2, 64, kKC2)) return -1;
-  maps->vt2 = maps->vt;   // the Vt box is already 64 keys x dh
+            NK * dh * 2, 64, 64)) return -1;
+  maps->vt2 = maps->vt;
   const int smem2 = (int)attn_tc2_smem_bytes(dh);
   if (dh == 64) cudaFuncSetAttribute(attn_tc2_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem2);
   if (dh == 128) cudaFuncSetAttribute(attn_tc2_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem2);
@@ -610,9 +632,9 @@ void launch_attn_tc(const AttnTcMaps& maps, const AttnTcArgs& a, cudaStream_t s)
   if (attn_tc_use_two_pass(a)) {
     dim3 grid2((a.rows + kQT - 1) / kQT, a.batch * a.n_kv_heads);
     const size_t smem2 = attn_tc2_smem_bytes(a.head_dim);
-    if (a.head_dim == 64) launch_k(attn_tc2_kernel<64>, grid2, dim3(192), smem2, s, maps.q, maps.k2, maps.vt2, a);
-    if (a.head_dim == 128) launch_k(attn_tc2_kernel<128>, grid2, dim3(192), smem2, s, maps.q, maps.k2, maps.vt2, a);
-    if (a.head_dim == 256) launch_k(attn_tc2_kernel<256>, grid2, dim3(192), smem2, s, maps.q, maps.k2, maps.vt2, a);
+    if (a.head_dim == 64) launch_k(attn_tc2_kernel<64>, grid2, dim3(192), smem2, s, maps.q, maps.k, maps.vt2, a);
+    if (a.head_dim == 128) launch_k(attn_tc2_kernel<128>, grid2, dim3(192), smem2, s, maps.q, maps.k, maps.vt2, a);
+    if (a.head_dim == 256) launch_k(attn_tc2_kernel<256>, grid2, dim3(192), smem2, s, maps.q, maps.k, maps.vt2, a);
     return;
   }
   dim3 grid((a.rows + kQT - 1) / kQT, attn_tc_chunks(a.n_keys), a.batch * a.n_kv_heads);

@@ -190,7 +190,7 @@ struct AttnTcArgs {
   __nv_bfloat16* out = nullptr; int out_ld = 0;   // o [B*H][Hq*dh]
   int* err = nullptr;
 };
-struct AttnTcMaps { CUtensorMap q, k, vt, k2, vt2; };   // k2 / vt2: 64-key boxes (two-pass kernel)
+struct AttnTcMaps { CUtensorMap q, k, vt, k2, vt2; };   // k: 128-key boxes; k2 / vt2: 64-key boxes (step kernel)
 size_t attn_tc_smem_bytes(int dh);
 int attn_tc_prepare(AttnTcMaps* maps, const AttnTcArgs& a, int batch_max);  // 0 on success
 int attn_tc_chunks(int n_keys);
