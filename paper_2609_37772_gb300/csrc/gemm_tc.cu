@@ -420,23 +420,24 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kBN));
 }
 
-// ---- wide tiles for many tokens: 128 weight rows x 256 tokens per CTA, no K split ----------
-constexpr int kWN = 256;                       // tokens per tile (MMA N)
-constexpr int kWStageB = kWN * kBK * 2;        // 32 KB activation block per stage
-constexpr uint32_t kIdescWide = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kWN >> 3) << 17) |
-                                ((uint32_t)(kBM >> 4) << 24);
-
-__device__ __forceinline__ void mma_bf16_wide(uint32_t d, uint64_t a, uint64_t b, uint32_t accum) {
+// ---- wide tiles for many tokens: 128 weight rows x TN tokens per CTA, no K split ------------
+__device__ __forceinline__ void mma_bf16_idesc(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accum) {
   asm volatile(
       "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n"
-      ::"r"(d), "l"(a), "l"(b), "r"(kIdescWide), "r"(accum));
+      ::"r"(d), "l"(a), "l"(b), "r"(idesc), "r"(accum));
 }
 
-// STAGES pipeline stages of 48 KB; MINB CTAs per SM (two with two stages: one CTA's epilogue then
-// overlaps the other's main loop, which pays when there are more tiles than SMs).
-template <int STAGES, int MINB>
+// TN tokens per tile (MMA N = 128 or 256); STAGES pipeline stages of 16 KB + TN x 128 B; MINB CTAs
+// per SM (more than one: one CTA's epilogue overlaps another's main loop, which pays when there
+// are at least as many tiles as SMs).
+template <int TN, int STAGES, int MINB>
 __global__ void __launch_bounds__(128, MINB) gemm_tc_wide_kernel(const __grid_constant__ CUtensorMap tmx, TcGemmArgs p) {
+  constexpr int kWN = TN;
   constexpr int kWStages = STAGES;
+  constexpr int kWStageB = kWN * kBK * 2;
+  constexpr uint32_t kIdescWide = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kWN >> 3) << 17) |
+                                  ((uint32_t)(kBM >> 4) << 24);
+  static_assert(STAGES * (kStageA + kWStageB) >= kBM * kBN * 4, "the stage area holds the epilogue slice");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   const int t = blockIdx.x, mt = blockIdx.y;
@@ -504,7 +505,7 @@ __global__ void __launch_bounds__(128, MINB) gemm_tc_wide_kernel(const __grid_co
       const uint32_t a0 = su32(sA + (size_t)st * kStageA), b0 = su32(sB + (size_t)st * kWStageB);
 #pragma unroll
       for (int k = 0; k < kBK / 16; ++k)
-        mma_bf16_wide(tmem, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), (i > 0 || k > 0) ? 1u : 0u);
+        mma_bf16_idesc(tmem, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), kIdescWide, (i > 0 || k > 0) ? 1u : 0u);
       mma_commit(empty + st);
     }
     mma_commit(done);
@@ -595,25 +596,37 @@ size_t gemm_tc_smem_bytes(int stages, int epi, int M) {
   return 1024 + tc_pipe_bytes(stages) + (2 * kTcMaxStages + 1) * 8 + 16;
 }
 
-static size_t gemm_tc_wide_smem_bytes(int stages) { return 1024 + (size_t)stages * (kStageA + kWStageB) + (2 * stages + 2) * 8 + 16; }
+static size_t gemm_tc_wide_smem_bytes(int tn, int stages) {
+  return 1024 + (size_t)stages * (kStageA + (size_t)tn * kBK * 2) + (2 * stages + 2) * 8 + 16;
+}
 
 void gemm_tc_prepare() {
   const size_t a = gemm_tc_smem_bytes(kTcMaxStages, EPI_STORE, kBN);
   cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)a);
-  cudaFuncSetAttribute(gemm_tc_wide_kernel<4, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)gemm_tc_wide_smem_bytes(4));
-  cudaFuncSetAttribute(gemm_tc_wide_kernel<2, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)gemm_tc_wide_smem_bytes(2));
+  cudaFuncSetAttribute(gemm_tc_wide_kernel<256, 4, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)gemm_tc_wide_smem_bytes(256, 4));
+  cudaFuncSetAttribute(gemm_tc_wide_kernel<256, 2, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)gemm_tc_wide_smem_bytes(256, 2));
+  cudaFuncSetAttribute(gemm_tc_wide_kernel<128, 4, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)gemm_tc_wide_smem_bytes(128, 4));
+  cudaFuncSetAttribute(gemm_tc_wide_kernel<128, 3, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)gemm_tc_wide_smem_bytes(128, 3));
 }
 
-// Wide tiles (MMA N = 256 tokens) run the tensor cores near their rate and cut L2 re-reads of
-// the weights (one CTA per 256 tokens instead of 64). Returns 0 (narrow tiles), 1 (four stages,
-// one CTA per SM) or 2 (two stages, two CTAs per SM: with at least as many tiles as SMs, one
-// CTA's epilogue then overlaps the other's main loop).
+// Wide tiles (MMA N = 256 or 128 tokens) run the tensor cores near their rate (N = 64 runs at a
+// third of it) and cut L2 re-reads of the weights. Returns 0 (narrow 128 x 64 tiles with K
+// splits), or the wide form: 1 = 256 tokens, four stages, one CTA per SM; 2 = 256 tokens, two
+// stages, two CTAs per SM (with at least as many tiles as SMs, one CTA's epilogue overlaps the
+// other's main loop); 3 = 128 tokens, four stages, one CTA per SM; 4 = 128 tokens, three stages,
+// two CTAs per SM. 256-token tiles while they fill 60% of the SMs, else 128-token tiles while
+// those fill half of them (measured on the pi0-like projections from 200 to 3200 tokens: with
+// fewer than 256 tokens the narrow tiles win).
 int gemm_tc_use_wide(int M, int N, int sms) {
-  if (M < kWN || N > 8192) return 0;
-  const int tiles = (N / kBM) * ((M + kWN - 1) / kWN);
-  if (tiles * 2 < sms) return 0;
-  return tiles >= sms ? 2 : 1;
+  if (M < 256 || N > 8192) return 0;
+  const int t256 = (N / kBM) * ((M + 255) / 256), t128 = (N / kBM) * ((M + 127) / 128);
+  if (t256 >= sms) return 2;
+  if (t256 * 5 >= sms * 3) return 1;
+  if (t128 >= sms) return 4;
+  if (t128 * 2 >= sms) return 3;
+  return 0;
 }
+int gemm_tc_wide_tokens(int wide) { return wide >= 3 ? 128 : 256; }
 
 // K splits per output tile: one CTA per SM. Partial-plane epilogues (the consumer sums the
 // planes) take more splits, up to two CTAs per SM, so that every CTA holds its whole K range in
@@ -636,9 +649,14 @@ int gemm_tc_splits(int M, int N, int K, int sms, int epi) {
 
 void launch_gemm_tc(const CUtensorMap* tmx, const TcGemmArgs& a, cudaStream_t s) {
   if (a.wide) {
-    const dim3 grid(a.N / kBM, (a.M + kWN - 1) / kWN);
-    if (a.wide == 2) launch_k(gemm_tc_wide_kernel<2, 2>, grid, dim3(128), gemm_tc_wide_smem_bytes(2), s, *tmx, a);
-    else launch_k(gemm_tc_wide_kernel<4, 1>, grid, dim3(128), gemm_tc_wide_smem_bytes(4), s, *tmx, a);
+    const int tn = gemm_tc_wide_tokens(a.wide);
+    const dim3 grid(a.N / kBM, (a.M + tn - 1) / tn);
+    switch (a.wide) {
+      case 1: launch_k(gemm_tc_wide_kernel<256, 4, 1>, grid, dim3(128), gemm_tc_wide_smem_bytes(256, 4), s, *tmx, a); break;
+      case 2: launch_k(gemm_tc_wide_kernel<256, 2, 2>, grid, dim3(128), gemm_tc_wide_smem_bytes(256, 2), s, *tmx, a); break;
+      case 3: launch_k(gemm_tc_wide_kernel<128, 4, 1>, grid, dim3(128), gemm_tc_wide_smem_bytes(128, 4), s, *tmx, a); break;
+      default: launch_k(gemm_tc_wide_kernel<128, 3, 2>, grid, dim3(128), gemm_tc_wide_smem_bytes(128, 3), s, *tmx, a); break;
+    }
     return;
   }
   const int KC = a.K / kBK;
