@@ -184,55 +184,50 @@ __device__ __forceinline__ void tile_epilogue(const TcGemmArgs& p, const float* 
         store_out(p.out, (size_t)(m0 + j) * p.ldo + n, gelu_tanh_f(Tr[j * kBM] + b), p.out_dtype);
       break;
     case EPI_QKV_TC: {
-      // Destination of row n for robot b, token i is affine: dst0 + b * sb + i * si.
       const QkvTcOut& o = p.qkv;
-      const bool isq = n < o.qd, isk = !isq && n < o.qd + o.kvd;
-      __nv_bfloat16* dst0;
-      size_t sb, si;
-      const int half = o.dh / 2;
-      int r = 0;
-      if (isq || isk) {
-        const int sn = isq ? n : n - o.qd, h = sn / o.dh;
-        r = sn % o.dh;
-        const int d = o.rope ? ((r & 1) ? (r >> 1) + half : (r >> 1)) : r;
-        if (isq) {
-          dst0 = o.q + (((size_t)(h / o.G) * o.G + (h % o.G)) * o.H) * o.dh + d;   // + b*Hkv*G*H*dh + i*dh
-          sb = (size_t)o.Hkv * o.G * o.H * o.dh;
-          si = o.dh;
-        } else {
-          dst0 = o.kcache + (((size_t)o.layer * o.Hkv + h) * o.NK + o.P) * o.dh + d;
-          sb = (size_t)o.L * o.Hkv * o.NK * o.dh;
-          si = o.dh;
+      const int n0 = n - row;   // the tile's first output row; q, k and v each span whole tiles
+      if (n0 < o.qd + o.kvd) {
+        // q or k rows: tokens over the warps, lane owns 4 consecutive rows (two RoPE pairs, with
+        // rows 2j, 2j + 1 of a head holding dims j and j + dh/2), so that each token's features
+        // go out as contiguous runs; (cos, sin) of the token's position from the table
+        const bool isq = n0 < o.qd;
+        const int sn = (isq ? n0 : n0 - o.qd) + 4 * lane;
+        const int h = sn / o.dh, r = sn % o.dh, half = o.dh / 2;
+        __nv_bfloat16* base = isq ? o.q + ((size_t)(h / o.G) * o.G + (h % o.G)) * o.H * o.dh
+                                  : o.kcache + (((size_t)o.layer * o.Hkv + h) * o.NK + o.P) * o.dh;
+        const size_t sb = isq ? (size_t)o.Hkv * o.G * o.H * o.dh : (size_t)o.L * o.Hkv * o.NK * o.dh;
+        for (int j = row >> 5; j < mcount; j += kBM / 32) {
+          const int m = m0 + j, bi = m / o.H, ii = m - bi * o.H;
+          const float4 v = *reinterpret_cast<const float4*>(T + j * kBM + 4 * lane);
+          __nv_bfloat16* dst = base + bi * sb + (size_t)ii * o.dh;
+          if (o.rope) {
+            const float4 cs = *reinterpret_cast<const float4*>(o.rope + (size_t)ii * o.dh + r);
+            const int d = r >> 1;
+            *reinterpret_cast<__nv_bfloat162*>(dst + d) =
+                __floats2bfloat162_rn(v.x * cs.x - v.y * cs.y, v.z * cs.z - v.w * cs.w);
+            *reinterpret_cast<__nv_bfloat162*>(dst + d + half) =
+                __floats2bfloat162_rn(v.y * cs.x + v.x * cs.y, v.w * cs.z + v.z * cs.w);
+          } else {
+            *reinterpret_cast<__nv_bfloat162*>(dst + r) = __floats2bfloat162_rn(v.x, v.y);
+            *reinterpret_cast<__nv_bfloat162*>(dst + r + 2) = __floats2bfloat162_rn(v.z, v.w);
+          }
         }
       } else {
-        const int sn = n - o.qd - o.kvd, g = sn / o.dh, d = sn % o.dh;
-        dst0 = o.vtcache + (((size_t)o.layer * o.Hkv + g) * o.dh + d) * o.NKp + o.P;
-        sb = (size_t)o.L * o.Hkv * o.dh * o.NKp;
-        si = 1;
-      }
-      const bool rot = o.rope && (isq || isk);
-      // RoPE angle of token i: (P + i) * f, f = 1e4^(-2j/dh) for this row's pair j; (cos, sin)
-      // advance from token to token by a fixed rotation (one accurate sincosf per robot).
-      const float f = exp2f(-13.287712379549449f * (float)(2 * (r >> 1)) / (float)o.dh);
-      float cd = 1.f, sd = 0.f, c = 1.f, sn = 0.f;
-      if (rot) sincosf(f, &sd, &cd);
-      const float sgn = (r & 1) ? 1.f : -1.f;
-      const int pr = (r & 1) ? -1 : 1;
-      int bi = m0 / o.H, ii = m0 % o.H;
-      if (rot) sincosf((float)(o.P + ii) * f, &sn, &c);
-      for (int j = 0; j < mcount; ++j) {
-        float val = Tr[j * kBM];
-        if (rot) {
-          val = fmaf(val, c, sgn * Tr[j * kBM + pr] * sn);
-          const float c2 = c * cd - sn * sd;
-          sn = fmaf(sn, cd, c * sd);
-          c = c2;
-        }
-        dst0[bi * sb + ii * si] = __float2bfloat16_rn(val);
-        if (++ii == o.H) {
-          ii = 0;
-          ++bi;
-          if (rot) sincosf((float)o.P * f, &sn, &c);
+        // v rows: lane owns a token and reads 4 head dims of it at once; each store instruction
+        // then writes 32 consecutive keys of one head dim of Vt (keys contiguous)
+        const int sv0 = n0 - o.qd - o.kvd;   // the tile's first v feature
+        const size_t sb = (size_t)o.L * o.Hkv * o.dh * o.NKp;
+        for (int it = row >> 5; it < (kBM / 4) * 2; it += kBM / 32) {
+          const int r4 = 4 * (it >> 1), j = 32 * (it & 1) + lane;
+          if (j >= mcount) continue;
+          const int m = m0 + j, bi = m / o.H, ii = m - bi * o.H;
+          const float4 v = *reinterpret_cast<const float4*>(T + j * kBM + r4);
+          const int sn = sv0 + r4, g = sn / o.dh, d = sn % o.dh;   // 4 dims of one head
+          __nv_bfloat16* dst = o.vtcache + bi * sb + (((size_t)o.layer * o.Hkv + g) * o.dh + d) * o.NKp + o.P + ii;
+          dst[0] = __float2bfloat16_rn(v.x);
+          dst[o.NKp] = __float2bfloat16_rn(v.y);
+          dst[2 * (size_t)o.NKp] = __float2bfloat16_rn(v.z);
+          dst[3 * (size_t)o.NKp] = __float2bfloat16_rn(v.w);
         }
       }
       break;

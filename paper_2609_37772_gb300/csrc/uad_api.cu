@@ -900,9 +900,10 @@ int uad_init(const uad_arch* arch, const float* weights, size_t n_floats, uad_ct
     if (l.tiled) launch_relayout_tiled(src(n), (int)T.at(n)->rows, (int)T.at(n)->cols, l.w, mult, off, rope_dh, s0);
     else lin(n, l.w, mult, off);
   };
-  // tensor-core attention: bf16 joint-attention experts whose QKV projection is tiled
-  c->attn_tc = a.kind != UAD_KIND_DIT && dt == BF16 && !c->force_simt && c->qkvd % 128 == 0 && W % 64 == 0 &&
-              a.prefix_len + H <= attn_tc_max_keys();
+  // tensor-core attention: bf16 joint-attention experts whose QKV projection is tiled (q, k and v
+  // each whole 128-row tiles: the projection's epilogue writes each tile in one layout)
+  c->attn_tc = a.kind != UAD_KIND_DIT && dt == BF16 && !c->force_simt && c->qd % 128 == 0 && c->kvd % 128 == 0 &&
+              W % 64 == 0 && a.prefix_len + H <= attn_tc_max_keys();
   const int qk_perm = c->attn_tc && a.rope ? a.head_dim : 0;
   for (int l = 0; l < a.n_layers; ++l) {
     const std::string p = "l" + std::to_string(l) + ".";
