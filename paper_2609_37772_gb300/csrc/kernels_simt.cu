@@ -345,8 +345,99 @@ __global__ void __launch_bounds__(1024) resid_norm_kernel(NormArgs p) {
   }
 }
 
+// The same with one warp per token row and the whole row in registers (W = 128 * NV): the row's
+// h, planes, gate and modulation vectors are all loaded before the arithmetic that needs them,
+// and its sums are warp reductions (no CTA barrier), so a row costs two memory round trips (the
+// modulation-row index, then the data). The planes are summed in plane order as above.
+template <int NV>
+__global__ void __launch_bounds__(256) resid_norm_reg_kernel(NormArgs p) {
+  pdl_trigger();
+  pdl_wait();
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (row >= p.M) return;
+  const int tr = p.tau_row[row];
+  float4* h4 = reinterpret_cast<float4*>(p.h + (long long)row * p.ldh);
+  const float4* pp = reinterpret_cast<const float4*>(p.part + (long long)row * p.W);
+  const long long plane4 = (long long)p.M * p.W / 4;
+  const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f), one = make_float4(1.f, 1.f, 1.f, 1.f);
+  float4 x[NV], acc[NV], gt[NV], sc[NV], sh[NV];
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    x[i] = h4[i * 32 + lane];
+    acc[i] = p.n_part > 0 ? __ldcg(pp + i * 32 + lane) : zero;
+  }
+  const float* mod = p.tab ? p.tab + (long long)tr * p.stride : nullptr;
+  const float4* g4 = p.rgate_tab ? reinterpret_cast<const float4*>(p.rgate_tab + (long long)tr * p.stride + p.rgate_off) : nullptr;
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    gt[i] = g4 ? __ldg(g4 + i * 32 + lane) : one;
+    sc[i] = mod ? __ldg(reinterpret_cast<const float4*>(mod + p.scale_off) + i * 32 + lane) : zero;
+    sh[i] = mod ? __ldg(reinterpret_cast<const float4*>(mod + p.shift_off) + i * 32 + lane) : zero;
+  }
+  for (int sp = 1; sp < p.n_part; ++sp) {
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+      const float4 q = __ldcg(pp + sp * plane4 + i * 32 + lane);
+      acc[i].x += q.x;
+      acc[i].y += q.y;
+      acc[i].z += q.z;
+      acc[i].w += q.w;
+    }
+  }
+  float t = 0.f;
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    const float4 bs = p.rbias ? __ldg(reinterpret_cast<const float4*>(p.rbias) + i * 32 + lane) : zero;
+    x[i].x = fmaf(gt[i].x, acc[i].x + bs.x, x[i].x);
+    x[i].y = fmaf(gt[i].y, acc[i].y + bs.y, x[i].y);
+    x[i].z = fmaf(gt[i].z, acc[i].z + bs.z, x[i].z);
+    x[i].w = fmaf(gt[i].w, acc[i].w + bs.w, x[i].w);
+    h4[i * 32 + lane] = x[i];
+    t += (x[i].x + x[i].y) + (x[i].z + x[i].w);
+  }
+  const float mean = p.layer_norm ? warp_sum(t) / p.W : 0.f;
+  float ss = 0.f;
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    const float a = x[i].x - mean, b = x[i].y - mean, c = x[i].z - mean, d = x[i].w - mean;
+    ss = fmaf(a, a, fmaf(b, b, fmaf(c, c, fmaf(d, d, ss))));
+  }
+  const float rstd = 1.f / sqrtf(warp_sum(ss) / p.W + 1e-6f);
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    float4 y = make_float4((x[i].x - mean) * rstd, (x[i].y - mean) * rstd, (x[i].z - mean) * rstd,
+                           (x[i].w - mean) * rstd);
+    if (mod) {
+      y.x = fmaf(y.x, 1.f + sc[i].x, sh[i].x);
+      y.y = fmaf(y.y, 1.f + sc[i].y, sh[i].y);
+      y.z = fmaf(y.z, 1.f + sc[i].z, sh[i].z);
+      y.w = fmaf(y.w, 1.f + sc[i].w, sh[i].w);
+    }
+    const long long off = (long long)row * p.ldo + (i * 32 + lane) * 4;
+    if (p.out_dtype == BF16) {
+      __nv_bfloat162 lo = __floats2bfloat162_rn(y.x, y.y), hi = __floats2bfloat162_rn(y.z, y.w);
+      uint2 pk;
+      pk.x = *reinterpret_cast<uint32_t*>(&lo);
+      pk.y = *reinterpret_cast<uint32_t*>(&hi);
+      *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(p.out) + off) = pk;
+    } else {
+      *reinterpret_cast<float4*>(static_cast<float*>(p.out) + off) = y;
+    }
+  }
+}
+
 void launch_norm(const NormArgs& a, cudaStream_t s) {
   if (a.part) {
+    const bool aligned = a.ldh % 4 == 0 && a.ldo % 4 == 0 && a.scale_off % 4 == 0 && a.shift_off % 4 == 0 &&
+                         a.rgate_off % 4 == 0 && a.stride % 4 == 0 && a.W % 128 == 0;
+    const int blocks = (a.M + 7) / 8;
+    // a warp per row pays with enough rows to fill the SMs; with fewer, one CTA per row
+    switch (aligned && a.M >= 512 ? a.W / 128 : 0) {
+      case 2: launch_k(resid_norm_reg_kernel<2>, dim3(blocks), dim3(256), 0, s, a); return;
+      case 4: launch_k(resid_norm_reg_kernel<4>, dim3(blocks), dim3(256), 0, s, a); return;
+      case 8: launch_k(resid_norm_reg_kernel<8>, dim3(blocks), dim3(256), 0, s, a); return;
+      default: break;
+    }
     // the caller guarantees 16-byte rows: W, ldh, ldo, stride and the offsets multiples of 4
     const int threads = ((a.W / 4 + 31) / 32) * 32;
     launch_k(resid_norm_kernel, dim3(a.M), dim3(threads), 0, s, a);

@@ -391,7 +391,10 @@ double gemm_bytes(const GemmArgs& g, int wes) {
 void gemm(uad_ctx* c, const Lin& w, GemmArgs g, cudaStream_t s) {
   g.W = w.w;
   if (!w.tiled) {
-    if (gemv_rows_ok(g)) launch_gemv_rows(g, s);
+    // row-at-a-time kernel for a long K (action out) or few rows; a short K over many rows (the
+    // action-in projection of a batch) goes to the tiled kernel, which reuses each weight tile
+    // over 64 rows
+    if (gemv_rows_ok(g) && (g.K > 64 || g.M <= 64)) launch_gemv_rows(g, s);
     else launch_gemm_simt(g, s);
     return;
   }
