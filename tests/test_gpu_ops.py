@@ -42,6 +42,24 @@ def test_linear_matches_reference(M, N, K):
     assert np.abs(out - ref).max() <= 1e-5 * np.abs(ref).max()
 
 
+# Shapes whose tile selection on a 152-SM GB300 takes each wide form (128 x 256- or 128 x 128-token
+# tiles, one or two CTAs per SM), with ragged last token tiles; numbers of the selection rule:
+#   (2560, 2048): 160 tiles of 256 tokens >= 152 SMs -> 256 tokens, two CTAs per SM
+#   (3000, 1024): 96 tiles of 256 >= 60% of the SMs -> 256 tokens, one CTA per SM
+#   (2400, 1024): 80 tiles of 256, 152 of 128 -> 128 tokens, two CTAs per SM
+#   (800, 2560): 80 tiles of 256, 140 of 128 -> 128 tokens, one CTA per SM
+@pytest.mark.parametrize("M,N,K", [(2560, 2048, 64), (3000, 1024, 128), (2400, 1024, 128), (800, 2560, 192)])
+def test_linear_wide_tiles_match_reference(M, N, K):
+    rng = np.random.default_rng(M + N + K)
+    x = rng.normal(size=(M, K)).astype(np.float32)
+    w = (rng.normal(size=(K, N)) * 0.02).astype(np.float32)
+    bias = rng.normal(size=N).astype(np.float32)
+    rc, out = run_linear(x, w, bias)
+    assert rc == 0
+    ref = reference(x, w, bias)
+    assert np.abs(out - ref).max() <= 1e-5 * np.abs(ref).max()
+
+
 def test_linear_rejects_bad_shapes():
     assert uad.uad_linear(1, 1, None, 1, 50, 100, 64, None) == uad.UAD_EINVAL
     assert uad.uad_linear(1, 1, None, 1, 0, 128, 64, None) == uad.UAD_EINVAL
