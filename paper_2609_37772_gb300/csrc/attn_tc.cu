@@ -110,6 +110,18 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
 #pragma unroll
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
+// 32 columns of this warp's 32 TMEM lanes (one row per thread) from registers.
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const float* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};\n"
+      "tcgen05.wait::st.sync.aligned;"
+      ::"r"(taddr), "f"(v[0]), "f"(v[1]), "f"(v[2]), "f"(v[3]), "f"(v[4]), "f"(v[5]), "f"(v[6]), "f"(v[7]), "f"(v[8]),
+        "f"(v[9]), "f"(v[10]), "f"(v[11]), "f"(v[12]), "f"(v[13]), "f"(v[14]), "f"(v[15]), "f"(v[16]), "f"(v[17]),
+        "f"(v[18]), "f"(v[19]), "f"(v[20]), "f"(v[21]), "f"(v[22]), "f"(v[23]), "f"(v[24]), "f"(v[25]), "f"(v[26]),
+        "f"(v[27]), "f"(v[28]), "f"(v[29]), "f"(v[30]), "f"(v[31])
+      : "memory");
+}
 
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
   __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
@@ -274,16 +286,17 @@ __global__ void __launch_bounds__(128, 1) attn_tc_kernel(const __grid_constant__
   if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols));
 }
 
-// ---- two-pass attention for many query tiles: no partials, no combine --------------------
-// One CTA per (128-row query tile, robot-group). Keys in chunks of 128 (S = Q K^T with MMA N = 128,
-// twice the tensor rate of 64-key chunks). Shared memory: Q, two 64 KB regions, P.
-// Pass 1: S = Q K_c^T on tcgen05 (double-buffered in TMEM), row maxima in registers; K chunks
-// alternate between the two regions.
-// Pass 2: S again, P = exp(S - max) in bf16 into shared memory, O += P V_c on tcgen05 (no
-// rescaling: the maxima are final), row sums of the rounded P; K in region 0, Vt in region 1.
-// O / l is written in bf16.
+// ---- one-pass attention for many query tiles: no partials, no combine ---------------------
+// One CTA per (128-row query tile, robot-group), keys in chunks of 128 (S = Q K^T with MMA
+// N = 128). Shared memory: Q, a K region, a Vt region, P. Per chunk: S on tcgen05 (double-buffered
+// in TMEM), then each softmax thread (one query row) forms P = exp(S - M) in bf16 against its
+// running maximum M and O += P V accumulates in TMEM. M is raised only when the chunk's maximum
+// exceeds it by more than 2^8 in the exponent; the O row and the row sum are then rescaled in place
+// (after the previous P V has completed). Otherwise the stale M stays: every P is at most 2^8, and
+// O and the row sum share the same reference, so O / sum is unchanged. O / l is written in bf16.
 constexpr int kKC2 = 128;                       // keys per chunk
 constexpr uint32_t kTmem2 = 512;                // S buffers at columns [0,128) and [128,256), O at [256, 256+dh)
+constexpr float kRescaleLog2 = 8.f;             // raise M only past this many powers of two
 
 // Warps 0-3: softmax and output (they own the four TMEM lane quadrants); warp 4: TMA producer;
 // warp 5: MMA issuer. The producer and issuer wait on the softmax warps' progress, so they must
@@ -301,16 +314,17 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
   constexpr uint32_t PB = kQT * kKC2 * 2;        // P: 2 blocks of 128 rows x 64 keys
   constexpr uint32_t VBLK = DH * 128;            // one Vt block: dh rows x 64 keys
   uint8_t* sQ = smem;
-  uint8_t* sR = sQ + QB;                         // regions 0 and 1
-  uint8_t* sP = sR + 2 * RB;
+  uint8_t* sK = sQ + QB;
+  uint8_t* sV = sK + RB;
+  uint8_t* sP = sV + RB;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sP + PB);
   uint64_t* q_full = bars;          // Q landed
-  uint64_t* full = bars + 1;        // [2] region loaded
-  uint64_t* empty = bars + 3;       // [2] region free (the MMAs that read it are done)
+  uint64_t* full = bars + 1;        // [2] K / Vt region loaded
+  uint64_t* empty = bars + 3;       // [2] K / Vt region free (the MMAs that read it are done)
   uint64_t* s_full = bars + 5;      // [2] S buffer written
   uint64_t* s_empty = bars + 7;     // [2] S buffer read by the 4 warps
-  uint64_t* p_full = bars + 9;      // P written by the 4 warps
-  uint64_t* p_empty = bars + 10;    // PV MMA done reading P
+  uint64_t* p_full = bars + 9;      // P written (and O rescaled) by the 4 warps
+  uint64_t* p_empty = bars + 10;    // P V done: P free, O complete up to this chunk
   uint64_t* o_done = bars + 11;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
 
@@ -345,48 +359,35 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
   pdl_trigger();
   pdl_wait();
 
-  // load sequence: pass 1 K chunk n into region n & 1 (n < nck); pass 2 K chunk c into region 0,
-  // then Vt chunk c into region 1. Producer and issuer count the uses of each region alike.
   if (threadIdx.x == 128) {
+    // producer: chunk c's K into the K region (once S of chunk c - 1 is done), then its Vt into
+    // the Vt region (once P V of chunk c - 1 is done)
     const uint64_t pol = policy_evict_last();
     mbar_expect_tx(q_full, QB);
 #pragma unroll
     for (int c = 0; c < NC; ++c) tma_3d(sQ + c * (kQT * 128), &tq, c * 64, qt * kQT, bg, q_full, pol);
-    int use0 = 0, use1 = 0;   // loads into regions 0 and 1
     bool ok = true;
-    for (int n = 0; n < 2 * nck && ok; ++n) {
-      const bool pass2 = n >= nck;
-      const int ch = pass2 ? n - nck : n;
-      for (int part = 0; part < (pass2 ? 2 : 1) && ok; ++part) {
-        const int r = pass2 ? part : (n & 1);
-        const int u = r ? use1++ : use0++;
-        if (u > 0) ok = mbar_wait(empty + r, (u - 1) & 1, p.err, 41);
-        if (!ok) break;
-        uint8_t* dst = sR + r * RB;
-        mbar_expect_tx(full + r, RB);
-        if (part == 0) {
+    for (int ch = 0; ch < nck && ok; ++ch) {
+      if (ch > 0) ok = mbar_wait(empty + 0, (ch - 1) & 1, p.err, 41);
+      if (!ok) break;
+      mbar_expect_tx(full + 0, RB);
 #pragma unroll
-          for (int c = 0; c < NC; ++c) tma_3d(dst + c * (kKC2 * 128), &tk, c * 64, ch * kKC2, kvz, full + r, pol);
-        } else {
+      for (int c = 0; c < NC; ++c) tma_3d(sK + c * (kKC2 * 128), &tk, c * 64, ch * kKC2, kvz, full + 0, pol);
+      if (ch > 0) ok = mbar_wait(empty + 1, (ch - 1) & 1, p.err, 41);
+      if (!ok) break;
+      mbar_expect_tx(full + 1, RB);
 #pragma unroll
-          for (int kb = 0; kb < 2; ++kb) tma_3d(dst + kb * VBLK, &tv, ch * kKC2 + kb * 64, 0, kvz, full + r, pol);
-        }
-      }
+      for (int kb = 0; kb < 2; ++kb) tma_3d(sV + kb * VBLK, &tv, ch * kKC2 + kb * 64, 0, kvz, full + 1, pol);
     }
   } else if (threadIdx.x == 160) {
     bool ok = mbar_wait(q_full, 0, p.err, 42);
-    const uint32_t q0 = su32(sQ);
-    int use0 = 0, use1 = 0;   // waits on regions 0 and 1, in the producer's order
-    for (int n = 0; n < 2 * nck && ok; ++n) {
-      const int sb = n & 1;
-      const bool pass2 = n >= nck;
-      const int rk = pass2 ? 0 : (n & 1);
-      const int u = rk ? use1++ : use0++;
-      ok = mbar_wait(full + rk, u & 1, p.err, 43);
-      if (ok && n >= 2) ok = mbar_wait(s_empty + sb, ((n >> 1) - 1) & 1, p.err, 44);
+    const uint32_t q0 = su32(sQ), k0 = su32(sK), pp = su32(sP), v0 = su32(sV);
+    for (int ch = 0; ch < nck && ok; ++ch) {
+      const int sb = ch & 1;
+      ok = mbar_wait(full + 0, ch & 1, p.err, 43);
+      if (ok && ch >= 2) ok = mbar_wait(s_empty + sb, ((ch >> 1) - 1) & 1, p.err, 44);
       if (!ok) break;
       tc_fence_after();
-      const uint32_t k0 = su32(sR + rk * RB);
 #pragma unroll
       for (int c = 0; c < NC; ++c)
 #pragma unroll
@@ -394,21 +395,16 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
           mma_bf16(tmem + sb * kKC2, sw128_desc(q0 + c * (kQT * 128) + 32 * k),
                    sw128_desc(k0 + c * (kKC2 * 128) + 32 * k), idesc_m128(kKC2), (c | k) ? 1u : 0u);
       mma_commit(s_full + sb);
-      mma_commit(empty + rk);
-      if (pass2) {
-        const int c2 = n - nck;
-        ok = mbar_wait(p_full, c2 & 1, p.err, 45) && mbar_wait(full + 1, use1 & 1, p.err, 46);
-        ++use1;
-        if (!ok) break;
-        tc_fence_after();
-        const uint32_t pp = su32(sP), v0 = su32(sR + RB);
+      mma_commit(empty + 0);
+      ok = mbar_wait(p_full, ch & 1, p.err, 45) && mbar_wait(full + 1, ch & 1, p.err, 46);
+      if (!ok) break;
+      tc_fence_after();
 #pragma unroll
-        for (int k = 0; k < kKC2 / 16; ++k)
-          mma_bf16(tO, sw128_desc(pp + (k >> 2) * (kQT * 128) + 32 * (k & 3)), sw128_desc(v0 + (k >> 2) * VBLK + 32 * (k & 3)),
-                   idesc_m128(DH), (c2 | k) ? 1u : 0u);
-        mma_commit(empty + 1);
-        mma_commit(p_empty);
-      }
+      for (int k = 0; k < kKC2 / 16; ++k)
+        mma_bf16(tO, sw128_desc(pp + (k >> 2) * (kQT * 128) + 32 * (k & 3)), sw128_desc(v0 + (k >> 2) * VBLK + 32 * (k & 3)),
+                 idesc_m128(DH), (ch | k) ? 1u : 0u);
+      mma_commit(empty + 1);
+      mma_commit(p_empty);
     }
     mma_commit(o_done);
   }
@@ -423,58 +419,72 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
   const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
   const float c2s = p.scale_log2;
   float sv[32];
-  float mx = -INFINITY, l = 0.f;
+  float mref = -INFINITY, l = 0.f;   // the row's reference maximum and sum of P
   bool ok = true;
   const int r8 = row & 7;
-  for (int n = 0; n < 2 * nck; ++n) {
-    const int sb = n & 1;
-    const bool pass2 = n >= nck;
-    const int key0 = (pass2 ? n - nck : n) * kKC2;
-    ok = ok && mbar_wait(s_full + sb, (n >> 1) & 1, p.err, 47);
+  for (int ch = 0; ch < nck; ++ch) {
+    const int sb = ch & 1;
+    const int key0 = ch * kKC2;
+    ok = ok && mbar_wait(s_full + sb, (ch >> 1) & 1, p.err, 47);
     tc_fence_after();
     __syncwarp();
-    if (!pass2) {
+    float mc = -INFINITY;
 #pragma unroll 1
-      for (int cc = 0; cc < kKC2 / 32; ++cc) {
-        tmem_ld32(tmem + sb * kKC2 + lane_base + cc * 32, sv);
+    for (int cc = 0; cc < kKC2 / 32; ++cc) {
+      tmem_ld32(tmem + sb * kKC2 + lane_base + cc * 32, sv);
 #pragma unroll
-        for (int i = 0; i < 32; ++i)
-          if (key0 + cc * 32 + i < p.n_keys) mx = fmaxf(mx, sv[i]);
-      }
-    } else {
-      const int c2 = n - nck;
-      if (c2 > 0) ok = ok && mbar_wait(p_empty, (c2 - 1) & 1, p.err, 48);
-      const float mxs = mx * c2s;
-#pragma unroll 1
-      for (int cc = 0; cc < kKC2 / 32; ++cc) {
-        tmem_ld32(tmem + sb * kKC2 + lane_base + cc * 32, sv);
-        uint32_t pk[16];
-#pragma unroll
-        for (int i = 0; i < 32; i += 2) {
-          const bool v0 = key0 + cc * 32 + i < p.n_keys, v1 = key0 + cc * 32 + i + 1 < p.n_keys;
-          const float e0 = v0 ? exp2f(fmaf(sv[i], c2s, -mxs)) : 0.f;
-          const float e1 = v1 ? exp2f(fmaf(sv[i + 1], c2s, -mxs)) : 0.f;
-          const __nv_bfloat162 h = __floats2bfloat162_rn(e0, e1);
-          l += __low2float(h) + __high2float(h);
-          pk[i / 2] = *reinterpret_cast<const uint32_t*>(&h);
-        }
-        // keys 32 cc .. 32 cc + 31: P block cc / 2, 16-byte groups 4 (cc % 2) .. + 3
-        uint8_t* prow = sP + (cc >> 1) * (kQT * 128) + row * 128;
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int gidx = (cc & 1) * 4 + q;
-          *reinterpret_cast<uint4*>(prow + ((gidx ^ r8) * 16)) =
-              make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
-        }
-      }
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(p_full)) : "memory");
+      for (int i = 0; i < 32; ++i)
+        if (key0 + cc * 32 + i < p.n_keys) mc = fmaxf(mc, sv[i]);
     }
+    // raise the reference past 2^8 (and at the first chunk); the previous P V must have completed
+    // before O is touched, and before P is overwritten in any case
+    const bool raise = ch == 0 ? true : (mc - mref) * c2s > kRescaleLog2;
+    const float factor = ch == 0 ? 1.f : (raise ? exp2f((mref - mc) * c2s) : 1.f);
+    if (ch > 0) ok = ok && mbar_wait(p_empty, (ch - 1) & 1, p.err, 48);
+    tc_fence_after();
+    if (__any_sync(0xffffffffu, ch > 0 && raise)) {
+#pragma unroll 1
+      for (int cc = 0; cc < DH / 32; ++cc) {
+        tmem_ld32(tO + lane_base + cc * 32, sv);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) sv[i] *= factor;
+        tmem_st32(tO + lane_base + cc * 32, sv);
+      }
+    }
+    if (raise) {
+      l *= factor;
+      mref = mc;
+    }
+    const float ms = mref * c2s;
+#pragma unroll 1
+    for (int cc = 0; cc < kKC2 / 32; ++cc) {
+      tmem_ld32(tmem + sb * kKC2 + lane_base + cc * 32, sv);
+      uint32_t pk[16];
+#pragma unroll
+      for (int i = 0; i < 32; i += 2) {
+        const bool v0 = key0 + cc * 32 + i < p.n_keys, v1 = key0 + cc * 32 + i + 1 < p.n_keys;
+        const float e0 = v0 ? exp2f(fmaf(sv[i], c2s, -ms)) : 0.f;
+        const float e1 = v1 ? exp2f(fmaf(sv[i + 1], c2s, -ms)) : 0.f;
+        const __nv_bfloat162 h = __floats2bfloat162_rn(e0, e1);
+        l += __low2float(h) + __high2float(h);
+        pk[i / 2] = *reinterpret_cast<const uint32_t*>(&h);
+      }
+      // keys 32 cc .. 32 cc + 31: P block cc / 2, 16-byte groups 4 (cc % 2) .. + 3
+      uint8_t* prow = sP + (cc >> 1) * (kQT * 128) + row * 128;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int gidx = (cc & 1) * 4 + q;
+        *reinterpret_cast<uint4*>(prow + ((gidx ^ r8) * 16)) =
+            make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+      }
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     tc_fence_before();
     __syncwarp();
-    if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(s_empty + sb)) : "memory");
+    if (lane == 0) {
+      asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(p_full)) : "memory");
+      asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(s_empty + sb)) : "memory");
+    }
   }
   ok = ok && mbar_wait(o_done, 0, p.err, 49);
   tc_fence_after();
