@@ -110,6 +110,31 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
 #pragma unroll
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
+// 128 columns (four loads of 32, one wait) of this warp's 32 TMEM lanes, one row per thread.
+__device__ __forceinline__ void tmem_ld128(uint32_t taddr, float* v) {
+  uint32_t* r = reinterpret_cast<uint32_t*>(v);
+#pragma unroll
+  for (int q = 0; q < 4; ++q)
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[32 * q + 0]), "=r"(r[32 * q + 1]), "=r"(r[32 * q + 2]), "=r"(r[32 * q + 3]), "=r"(r[32 * q + 4]),
+          "=r"(r[32 * q + 5]), "=r"(r[32 * q + 6]), "=r"(r[32 * q + 7]), "=r"(r[32 * q + 8]), "=r"(r[32 * q + 9]),
+          "=r"(r[32 * q + 10]), "=r"(r[32 * q + 11]), "=r"(r[32 * q + 12]), "=r"(r[32 * q + 13]), "=r"(r[32 * q + 14]),
+          "=r"(r[32 * q + 15]), "=r"(r[32 * q + 16]), "=r"(r[32 * q + 17]), "=r"(r[32 * q + 18]), "=r"(r[32 * q + 19]),
+          "=r"(r[32 * q + 20]), "=r"(r[32 * q + 21]), "=r"(r[32 * q + 22]), "=r"(r[32 * q + 23]), "=r"(r[32 * q + 24]),
+          "=r"(r[32 * q + 25]), "=r"(r[32 * q + 26]), "=r"(r[32 * q + 27]), "=r"(r[32 * q + 28]), "=r"(r[32 * q + 29]),
+          "=r"(r[32 * q + 30]), "=r"(r[32 * q + 31])
+        : "r"(taddr + 32 * q)
+        : "memory");
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+// 2^x by the hardware approximation (MUFU); P is rounded to bf16 next, far coarser than its error.
+__device__ __forceinline__ float ex2_fast(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 // 32 columns of this warp's 32 TMEM lanes (one row per thread) from registers.
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const float* v) {
   asm volatile(
@@ -418,24 +443,26 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
   const int row = warp * 32 + lane;
   const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
   const float c2s = p.scale_log2;
-  float sv[32];
+  float sv[kKC2];                    // the chunk's scores of this row
   float mref = -INFINITY, l = 0.f;   // the row's reference maximum and sum of P
   bool ok = true;
   const int r8 = row & 7;
   for (int ch = 0; ch < nck; ++ch) {
     const int sb = ch & 1;
     const int key0 = ch * kKC2;
+    const int nv = p.n_keys - key0;   // valid keys of the chunk (all of them but in the last)
     ok = ok && mbar_wait(s_full + sb, (ch >> 1) & 1, p.err, 47);
     tc_fence_after();
     __syncwarp();
-    float mc = -INFINITY;
-#pragma unroll 1
-    for (int cc = 0; cc < kKC2 / 32; ++cc) {
-      tmem_ld32(tmem + sb * kKC2 + lane_base + cc * 32, sv);
+    tmem_ld128(tmem + sb * kKC2 + lane_base, sv);
+    if (nv < kKC2) {   // keys past the end (last chunk): excluded from the maximum, P = 2^-inf = 0
 #pragma unroll
-      for (int i = 0; i < 32; ++i)
-        if (key0 + cc * 32 + i < p.n_keys) mc = fmaxf(mc, sv[i]);
+      for (int i = 0; i < kKC2; ++i)
+        if (i >= nv) sv[i] = -INFINITY;
     }
+    float mc = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < kKC2; ++i) mc = fmaxf(mc, sv[i]);
     // raise the reference past 2^8 (and at the first chunk); the previous P V must have completed
     // before O is touched, and before P is overwritten in any case
     const bool raise = ch == 0 ? true : (mc - mref) * c2s > kRescaleLog2;
@@ -443,12 +470,13 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
     if (ch > 0) ok = ok && mbar_wait(p_empty, (ch - 1) & 1, p.err, 48);
     tc_fence_after();
     if (__any_sync(0xffffffffu, ch > 0 && raise)) {
+      float ov[32];
 #pragma unroll 1
       for (int cc = 0; cc < DH / 32; ++cc) {
-        tmem_ld32(tO + lane_base + cc * 32, sv);
+        tmem_ld32(tO + lane_base + cc * 32, ov);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) sv[i] *= factor;
-        tmem_st32(tO + lane_base + cc * 32, sv);
+        for (int i = 0; i < 32; ++i) ov[i] *= factor;
+        tmem_st32(tO + lane_base + cc * 32, ov);
       }
     }
     if (raise) {
@@ -456,17 +484,16 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
       mref = mc;
     }
     const float ms = mref * c2s;
-#pragma unroll 1
+#pragma unroll
     for (int cc = 0; cc < kKC2 / 32; ++cc) {
-      tmem_ld32(tmem + sb * kKC2 + lane_base + cc * 32, sv);
       uint32_t pk[16];
 #pragma unroll
       for (int i = 0; i < 32; i += 2) {
-        const bool v0 = key0 + cc * 32 + i < p.n_keys, v1 = key0 + cc * 32 + i + 1 < p.n_keys;
-        const float e0 = v0 ? exp2f(fmaf(sv[i], c2s, -ms)) : 0.f;
-        const float e1 = v1 ? exp2f(fmaf(sv[i + 1], c2s, -ms)) : 0.f;
+        const int k = cc * 32 + i;
+        const float e0 = ex2_fast(fmaf(sv[k], c2s, -ms)), e1 = ex2_fast(fmaf(sv[k + 1], c2s, -ms));
         const __nv_bfloat162 h = __floats2bfloat162_rn(e0, e1);
-        l += __low2float(h) + __high2float(h);
+        const float2 hf = __bfloat1622float2(h);
+        l += hf.x + hf.y;   // normalise by what the MMA sums
         pk[i / 2] = *reinterpret_cast<const uint32_t*>(&h);
       }
       // keys 32 cc .. 32 cc + 31: P block cc / 2, 16-byte groups 4 (cc % 2) .. + 3
@@ -486,6 +513,7 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
       asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(s_empty + sb)) : "memory");
     }
   }
+  float sv32[32];
   ok = ok && mbar_wait(o_done, 0, p.err, 49);
   tc_fence_after();
   __syncwarp();
@@ -497,15 +525,15 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
   __nv_bfloat16* orow = p.out + ((size_t)b * p.H + ii) * p.out_ld + (size_t)(g * p.group + jj) * DH;
 #pragma unroll
   for (int cc = 0; cc < DH / 32; ++cc) {
-    tmem_ld32(tO + lane_base + cc * 32, sv);
+    tmem_ld32(tO + lane_base + cc * 32, sv32);
     if (ok && qrow < p.rows) {
 #pragma unroll
       for (int i = 0; i < 32; i += 8) {
         uint4 w;
-        w.x = pack_bf16(sv[i] * inv, sv[i + 1] * inv);
-        w.y = pack_bf16(sv[i + 2] * inv, sv[i + 3] * inv);
-        w.z = pack_bf16(sv[i + 4] * inv, sv[i + 5] * inv);
-        w.w = pack_bf16(sv[i + 6] * inv, sv[i + 7] * inv);
+        w.x = pack_bf16(sv32[i] * inv, sv32[i + 1] * inv);
+        w.y = pack_bf16(sv32[i + 2] * inv, sv32[i + 3] * inv);
+        w.z = pack_bf16(sv32[i + 4] * inv, sv32[i + 5] * inv);
+        w.w = pack_bf16(sv32[i + 6] * inv, sv32[i + 7] * inv);
         *reinterpret_cast<uint4*>(orow + cc * 32 + i) = w;
       }
     }
