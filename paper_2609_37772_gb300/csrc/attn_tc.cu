@@ -229,29 +229,31 @@ __global__ void __launch_bounds__(128, 1) attn_tc_kernel(const __grid_constant__
   const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
   const float c2 = p.scale_log2;             // log2(e) / sqrt(dh)
   const int key0 = kc * kKT;
-  float mx = -INFINITY;
-  float sv[32];
+  const int nv = p.n_keys - key0;            // valid keys of the chunk (all of them but in the last)
+  float sv[kKT];                             // the chunk's scores of this row, one wait for all
   __syncwarp();
+  tmem_ld128(tS + lane_base, sv);
+  if (nv < kKT) {   // keys past the end (last chunk): excluded from the maximum, P = 2^-inf = 0
 #pragma unroll
-  for (int cc = 0; cc < kKT / 32; ++cc) {
-    tmem_ld32(tS + lane_base + cc * 32, sv);
-#pragma unroll
-    for (int i = 0; i < 32; ++i)
-      if (key0 + cc * 32 + i < p.n_keys) mx = fmaxf(mx, sv[i]);
+    for (int i = 0; i < kKT; ++i)
+      if (i >= nv) sv[i] = -INFINITY;
   }
+  float mx = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < kKT; ++i) mx = fmaxf(mx, sv[i]);
+  const float ms = mx * c2;
   float l = 0.f;
   const int r8 = row & 7;
 #pragma unroll
   for (int cc = 0; cc < kKT / 32; ++cc) {
-    tmem_ld32(tS + lane_base + cc * 32, sv);
     uint32_t pk[16];
 #pragma unroll
     for (int i = 0; i < 32; i += 2) {
-      const bool v0 = key0 + cc * 32 + i < p.n_keys, v1 = key0 + cc * 32 + i + 1 < p.n_keys;
-      const float e0 = v0 ? exp2f((sv[i] - mx) * c2) : 0.f;
-      const float e1 = v1 ? exp2f((sv[i + 1] - mx) * c2) : 0.f;
+      const int k = cc * 32 + i;
+      const float e0 = ex2_fast(fmaf(sv[k], c2, -ms)), e1 = ex2_fast(fmaf(sv[k + 1], c2, -ms));
       const __nv_bfloat162 h = __floats2bfloat162_rn(e0, e1);
-      l += __low2float(h) + __high2float(h);   // normalise by what the MMA actually sums
+      const float2 hf = __bfloat1622float2(h);
+      l += hf.x + hf.y;   // normalise by what the MMA actually sums
       pk[i / 2] = *reinterpret_cast<const uint32_t*>(&h);
     }
     // 32 keys = four 16-byte granules of row `row` in P block (cc / 2), granules (cc % 2) * 4 + q

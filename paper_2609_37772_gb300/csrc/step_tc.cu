@@ -190,6 +190,25 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
 // TMEM base address re-read from shared memory after a barrier wait: the tensor-memory loads
 // that follow take their address from this load, so they cannot be scheduled ahead of the
 // wait (the loads have no other dependence on it).
+// 64 columns (two loads of 32, one wait) of this warp's 32 TMEM lanes, one row per thread.
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float* v) {
+  uint32_t* r = reinterpret_cast<uint32_t*>(v);
+#pragma unroll
+  for (int q = 0; q < 2; ++q)
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[32 * q + 0]), "=r"(r[32 * q + 1]), "=r"(r[32 * q + 2]), "=r"(r[32 * q + 3]), "=r"(r[32 * q + 4]),
+          "=r"(r[32 * q + 5]), "=r"(r[32 * q + 6]), "=r"(r[32 * q + 7]), "=r"(r[32 * q + 8]), "=r"(r[32 * q + 9]),
+          "=r"(r[32 * q + 10]), "=r"(r[32 * q + 11]), "=r"(r[32 * q + 12]), "=r"(r[32 * q + 13]), "=r"(r[32 * q + 14]),
+          "=r"(r[32 * q + 15]), "=r"(r[32 * q + 16]), "=r"(r[32 * q + 17]), "=r"(r[32 * q + 18]), "=r"(r[32 * q + 19]),
+          "=r"(r[32 * q + 20]), "=r"(r[32 * q + 21]), "=r"(r[32 * q + 22]), "=r"(r[32 * q + 23]), "=r"(r[32 * q + 24]),
+          "=r"(r[32 * q + 25]), "=r"(r[32 * q + 26]), "=r"(r[32 * q + 27]), "=r"(r[32 * q + 28]), "=r"(r[32 * q + 29]),
+          "=r"(r[32 * q + 30]), "=r"(r[32 * q + 31])
+        : "r"(taddr + 32 * q)
+        : "memory");
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
 __device__ __forceinline__ uint32_t tmem_base_after_wait(const uint32_t* slot) {
   uint32_t t;
   asm volatile("ld.volatile.shared.u32 %0, [%1];" : "=r"(t) : "r"(su32(slot)) : "memory");
@@ -997,11 +1016,14 @@ __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, cons
         const int nvalid = p.n_keys - key0 < kKC ? p.n_keys - key0 : kKC;
         float sv[64];
         __syncwarp();
-        tmem_ld32(tS + lane_base, sv);
-        tmem_ld32(tS + lane_base + 32, sv + 32);
+        tmem_ld64(tS + lane_base, sv);
+        if (nvalid < 64) {   // keys past the end: excluded from the maximum, P = 2^-inf = 0
 #pragma unroll
-        for (int i = 0; i < 64; ++i)
-          if (i < nvalid) mx = fmaxf(mx, sv[i]);
+          for (int i = 0; i < 64; ++i)
+            if (i >= nvalid) sv[i] = -INFINITY;
+        }
+#pragma unroll
+        for (int i = 0; i < 64; ++i) mx = fmaxf(mx, sv[i]);
         const float mxs = mx * p.scale_log2;
         const int r8 = row & 7;
         uint8_t* prow = sP + row * 128;
@@ -1011,10 +1033,11 @@ __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, cons
 #pragma unroll
           for (int e = 0; e < 8; e += 2) {
             const int i0 = gi * 8 + e;
-            const float e0 = i0 < nvalid ? ex2_approx(fmaf(sv[i0], p.scale_log2, -mxs)) : 0.f;
-            const float e1 = i0 + 1 < nvalid ? ex2_approx(fmaf(sv[i0 + 1], p.scale_log2, -mxs)) : 0.f;
+            const float e0 = ex2_approx(fmaf(sv[i0], p.scale_log2, -mxs));
+            const float e1 = ex2_approx(fmaf(sv[i0 + 1], p.scale_log2, -mxs));
             const __nv_bfloat162 h = __floats2bfloat162_rn(e0, e1);
-            l_sum += __low2float(h) + __high2float(h);   // normalise by what the MMA sums
+            const float2 hf = __bfloat1622float2(h);
+            l_sum += hf.x + hf.y;   // normalise by what the MMA sums
             pk[e / 2] = *reinterpret_cast<const uint32_t*>(&h);
           }
           *reinterpret_cast<uint4*>(prow + ((gi ^ r8) * 16)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
