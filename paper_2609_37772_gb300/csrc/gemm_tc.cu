@@ -167,14 +167,21 @@ __device__ __forceinline__ void tile_epilogue(const TcGemmArgs& p, const float* 
       break;
     }
     case EPI_GEGLU: {
-      // rows 2i (gate) and 2i + 1 (up) of a lane pair: the even lane takes even tokens, the odd
-      // lane odd tokens, each reading both rows of the token from T
-      const float* Tg = T + (row & ~1);
+      // rows 2i (gate) and 2i + 1 (up) give output i: tokens over the warps, lane owns rows
+      // 4 lane .. 4 lane + 3 (outputs 2 lane, 2 lane + 1 of the tile), so that a warp writes one
+      // token's 64 outputs as one contiguous run
+      const int o0 = (n - row) / 2 + 2 * lane;
       const bool fast = p.out_dtype == BF16;
-#pragma unroll 4
-      for (int j = lane & 1; j < mcount; j += 2) {
-        const float g = Tg[j * kBM], u = Tg[j * kBM + 1];
-        store_out(p.out, (size_t)(m0 + j) * p.ldo + n / 2, (fast ? gelu_tanh_fast(g) : gelu_tanh_f(g)) * u, p.out_dtype);
+      for (int j = row >> 5; j < mcount; j += kBM / 32) {
+        const float4 v = *reinterpret_cast<const float4*>(T + j * kBM + 4 * lane);
+        const size_t off = (size_t)(m0 + j) * p.ldo + o0;
+        if (fast) {
+          *reinterpret_cast<__nv_bfloat162*>(static_cast<__nv_bfloat16*>(p.out) + off) =
+              __floats2bfloat162_rn(gelu_tanh_fast(v.x) * v.y, gelu_tanh_fast(v.z) * v.w);
+        } else {
+          store_out(p.out, off, gelu_tanh_f(v.x) * v.y, p.out_dtype);
+          store_out(p.out, off + 1, gelu_tanh_f(v.z) * v.w, p.out_dtype);
+        }
       }
       break;
     }
