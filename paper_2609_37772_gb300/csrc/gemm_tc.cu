@@ -115,6 +115,25 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
 #pragma unroll
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
+// 64 columns (two loads of 32, one wait) of this warp's 32 TMEM lanes, one row per thread.
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float* v) {
+  uint32_t* r = reinterpret_cast<uint32_t*>(v);
+#pragma unroll
+  for (int q = 0; q < 2; ++q)
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[32 * q + 0]), "=r"(r[32 * q + 1]), "=r"(r[32 * q + 2]), "=r"(r[32 * q + 3]), "=r"(r[32 * q + 4]),
+          "=r"(r[32 * q + 5]), "=r"(r[32 * q + 6]), "=r"(r[32 * q + 7]), "=r"(r[32 * q + 8]), "=r"(r[32 * q + 9]),
+          "=r"(r[32 * q + 10]), "=r"(r[32 * q + 11]), "=r"(r[32 * q + 12]), "=r"(r[32 * q + 13]), "=r"(r[32 * q + 14]),
+          "=r"(r[32 * q + 15]), "=r"(r[32 * q + 16]), "=r"(r[32 * q + 17]), "=r"(r[32 * q + 18]), "=r"(r[32 * q + 19]),
+          "=r"(r[32 * q + 20]), "=r"(r[32 * q + 21]), "=r"(r[32 * q + 22]), "=r"(r[32 * q + 23]), "=r"(r[32 * q + 24]),
+          "=r"(r[32 * q + 25]), "=r"(r[32 * q + 26]), "=r"(r[32 * q + 27]), "=r"(r[32 * q + 28]), "=r"(r[32 * q + 29]),
+          "=r"(r[32 * q + 30]), "=r"(r[32 * q + 31])
+        : "r"(taddr + 32 * q)
+        : "memory");
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
 
 __device__ __forceinline__ float gelu_tanh_f(float x) {
   const float k0 = 0.7978845608028654f;
@@ -349,8 +368,7 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   const int n = t * kBM + row;
   float v[kBN];
   __syncwarp();
-#pragma unroll
-  for (int c = 0; c < kBN; c += 16) tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + c, v + c);
+  tmem_ld64(tmem + ((uint32_t)(warp * 32) << 16), v);
   bool have = ok && nch > 0;
   // Stage the accumulator tile in shared memory, T[token j][row]: the epilogues below are
   // compact loops over it (neighbouring rows -- GeGLU and RoPE partners -- are one column
@@ -525,8 +543,7 @@ __global__ void __launch_bounds__(128, MINB) gemm_tc_wide_kernel(const __grid_co
     const int mcount = p.M - m0 < kBN ? p.M - m0 : kBN;
     float v[kBN];
     __syncwarp();
-#pragma unroll
-    for (int c = 0; c < kBN; c += 16) tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + q * kBN + c, v + c);
+    tmem_ld64(tmem + ((uint32_t)(warp * 32) << 16) + q * kBN, v);
 #pragma unroll
     for (int j = 0; j < kBN; ++j) T[j * kBM + row] = v[j];
     __syncthreads();
