@@ -52,8 +52,8 @@ for _b in (4, 16, 64):
 # file and its sha1 at measurement time (reported as null once that source changes); figures from
 # profiles/ncu_full_pi0_b1_step_kernel.md (one step-kernel launch = one evaluation).
 TRAFFIC = {
-    "step_kernel@pi0-b1": (641591552.0 + 3624704.0, "paper_2609_37772_gb300/csrc/step_tc.cu",
-                           "7baef7b2c9010f8b06277762b0886545b01836ab"),
+    "step_kernel@pi0-b1": (641496832.0 + 3673344.0, "paper_2609_37772_gb300/csrc/step_tc.cu",
+                           "a3c65088f590ddc54a039ad59e490e775620904e"),
 }
 
 
