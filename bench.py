@@ -229,6 +229,9 @@ def max_over_ranks(x, world, device="cpu"):
 
 
 # -------------------------------------------------------------------------------------------
+REF_SECONDS = 150.0   # bound on the reference arm's oracle time
+
+
 def oracle_chunks(wl, seconds, max_chunks=None):
     """Time the CPU oracle, as it stands, on whole chunks of robot 0 of this workload."""
     from oracle.model import build_model
@@ -253,8 +256,11 @@ def oracle_chunks(wl, seconds, max_chunks=None):
 def run_reference(args, wl, world, rank):
     if rank != 0:
         return 0
-    a, times = oracle_chunks(wl, float("inf"), max_chunks=args.warmup + args.steps)
-    timed = times[args.warmup:] if len(times) > args.warmup else times
+    # whole chunks of the oracle, W warm-up then up to K timed, within REF_SECONDS of CPU time so
+    # that the run ends within a few minutes whatever K is
+    a, times = oracle_chunks(wl, REF_SECONDS, max_chunks=args.warmup + args.steps)
+    warm = min(args.warmup, len(times) - 1)
+    timed = times[warm:]
     per = statistics.mean(timed)
     value = a.chunk_len / per
     cores = os.cpu_count()
@@ -265,7 +271,8 @@ def run_reference(args, wl, world, rank):
         "data": "synthetic (seeded random-init weights, N(0,1) prefix and noise)",
         "config": {"workload": wl["desc"], "global_batch": 1, "seq_len": a.chunk_len, "parallelism": "none"},
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
-                         "sample": "one full chunk of robot 0 per step (fp64 numpy oracle)"},
+                         "sample": f"{len(timed)} full chunk(s) of robot 0 timed after {warm} warm-up "
+                                   f"(fp64 numpy oracle; at most {REF_SECONDS:.0f} s of oracle time)"},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -551,7 +558,7 @@ def run_diagnostic(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="pi0-b1", choices=sorted(WORKLOADS))
