@@ -5,12 +5,14 @@
 //   Q  [B][Hkv][G][H][dh]       queries of one KV group are the R = G*H rows of one matrix
 //   K  [B][L][Hkv][NK][dh]      keys: P prefix rows then H chunk rows (NK = P + H)
 //   Vt [B][L][Hkv][dh][NKp]     values transposed (keys contiguous), NKp = NK rounded up to 8
-// One CTA = one 128-row query tile x one 128-key chunk of one (robot, group):
-//   TMA loads Q, K, Vt tiles (128-byte swizzle); S = Q K^T on tcgen05 into TMEM; four warps
-//   read S rows, apply the 1/sqrt(dh) scale and key mask, write P = exp(S - rowmax) in bf16 into
-//   shared memory in the K-major swizzled layout; O = P Vt^T on tcgen05; O rows (unnormalised)
-//   and per-row (max, sum) go to a workspace. attn_combine merges the key chunks (the usual
-//   log-sum-exp rescaling) and writes o [B*H][Hq*dh] in bf16 for the O projection.
+// Few query tiles (split-KV): one CTA = one 128-row query tile x one 128-key chunk of one
+//   (robot, group): TMA loads Q, K, Vt tiles (128-byte swizzle); S = Q K^T on tcgen05 into TMEM;
+//   four warps read S rows, apply the 1/sqrt(dh) scale and key mask, write P = exp(S - rowmax) in
+//   bf16 into shared memory in the K-major swizzled layout; O = P Vt^T on tcgen05; O rows
+//   (unnormalised) and per-row (max, sum) go to a workspace. attn_combine merges the key chunks
+//   (the usual log-sum-exp rescaling) and writes o [B*H][Hq*dh] in bf16 for the O projection.
+// Many query tiles (attn_tc2_kernel): one CTA per query tile walks all key chunks in one pass,
+//   O accumulating in TMEM, and writes o itself.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -648,7 +650,7 @@ int attn_tc_prepare(AttnTcMaps* maps, const AttnTcArgs& a, int batch_max) {
             NK * dh * 2, 64, kKT)) return -1;
   if (tmap3(&maps->vt, a.vtcache, NK, dh, (uint64_t)batch_max * a.n_layers * a.n_kv_heads, NKp * 2,
             (uint64_t)dh * NKp * 2, 64, (uint32_t)dh)) return -1;
-  // 64-key K boxes for the persistent step kernel's attention items; the two-pass kernel loads
+  // 64-key K boxes for the persistent step kernel's attention items; the one-pass kernel loads
   // 128-key K chunks through `k` and Vt in 64-key boxes
   if (tmap3(&maps->k2, a.kcache, dh, NK, (uint64_t)batch_max * a.n_layers * a.n_kv_heads, (uint64_t)dh * 2,
             NK * dh * 2, 64, 64)) return -1;

@@ -433,9 +433,10 @@ def test_pi0_full_batched_16_robots_sampled():
         ex.close()
 
 
-def test_two_pass_attention_many_tiles():
-    """32 robots x 2 query tiles on the small bf16 expert: the attention takes its two-pass path
-    (row maxima, then P V accumulated without rescaling); sampled robots vs the oracle."""
+def test_one_pass_attention_many_tiles():
+    """32 robots x 2 query tiles on the small bf16 expert: the attention takes its path for many
+    query tiles (one pass over 128-key chunks, O in tensor memory rescaled only when a row maximum
+    grows past 2^8); sampled robots vs the oracle."""
     a = ARCHS["pi0_small"]
     B = 32
     blob = make_weights(a, seed=12)
@@ -449,6 +450,35 @@ def test_two_pass_attention_many_tiles():
         ex.denoise(noise, bud)
         res = ex.finish(timeout_us=TIMEOUT)
         for b in (0, 13, 31):
+            ref = denoise(build_model(a, blob, pre[b]).velocity, noise[b], bud[b])
+            assert rel_err(res["final"][b], ref["final"]) <= TOL["bf16"]
+            assert rel_err(res["ghost"][b], ref["ghost"]) <= TOL["bf16"]
+    finally:
+        ex.close()
+
+
+def test_one_pass_attention_rescales_when_the_maximum_grows():
+    """The many-tile attention path with prefix keys past the first 128-key chunk scaled by 16
+    (a power of two: still exact in bf16), so that every query row's maximum score jumps far
+    past 2^8 in the exponent at the second chunk and the running O rows and sums are rescaled in
+    tensor memory; sampled robots vs the oracle on the same keys."""
+    a = ARCHS["pi0_small"]
+    B = 32
+    blob = make_weights(a, seed=14)
+    ex = uad.Expert(a, blob, max_batch=B)
+    try:
+        pre = []
+        for b in range(B):
+            k, v = make_prefix_kv(a, robot=b, seed=14)
+            k = k.copy()
+            k[:, 128:] *= 16.0
+            pre.append((k, v))
+            ex.set_prefix(b, k, v)
+        noise = make_noise(a, batch=B, seed=14)
+        bud = draw_sweep_schedules(a.chunk_len, B, seed=14)
+        ex.denoise(noise, bud)
+        res = ex.finish(timeout_us=TIMEOUT)
+        for b in (0, 17, 31):
             ref = denoise(build_model(a, blob, pre[b]).velocity, noise[b], bud[b])
             assert rel_err(res["final"][b], ref["final"]) <= TOL["bf16"]
             assert rel_err(res["ghost"][b], ref["ghost"]) <= TOL["bf16"]
