@@ -263,6 +263,23 @@ def test_bf16_small_archs(name):
         c.close()
 
 
+@pytest.mark.parametrize("B", [1, 4])
+def test_bf16_expert_without_rope(B):
+    """A bf16 joint-attention expert without rotary embedding: q and k leave the QKV projection's
+    epilogue as computed. B = 1 runs the persistent kernel, B = 4 the per-operation tensor-core
+    projection and attention."""
+    a = ARCHS["pi0_small"].replace(name="pi0_small_norope", rope=False)
+    c = Case(a, B=B, seed=21)
+    try:
+        noise = make_noise(a, batch=B, seed=21)
+        bud = draw_sweep_schedules(a.chunk_len, B, seed=21)
+        names = kernel_names(c, noise, bud)
+        assert ("step_kernel" in names) == (B == 1) and (B == 1 or "qkv_proj" in names), names
+        check(c, c.gpu(noise, bud), c.oracle(noise, bud), bud, TOL["bf16"])
+    finally:
+        c.close()
+
+
 def test_batched_robots_own_schedules():
     a = ARCHS["pi0_small"]
     B = 4
