@@ -450,6 +450,31 @@ def test_pi0_full_batched_16_robots_sampled():
         ex.close()
 
 
+def test_pi0_full_batched_64_robots_sampled():
+    """64 robots (M = 3200 tokens), the batched serving configuration: every projection on wide
+    tensor-core tiles (the o and down projections with the partial-plane epilogue), attention on
+    the many-tile path, the residual norm one warp per row; robots 0, 31 and 63 vs the oracle."""
+    a = ARCHS["pi0"]
+    B = 64
+    blob = make_weights(a, seed=5)
+    ex = uad.Expert(a, blob, max_batch=B)
+    try:
+        pre = [make_prefix_kv(a, robot=b, seed=5) for b in range(B)]
+        for b in range(B):
+            ex.set_prefix(b, *pre[b])
+        noise = make_noise(a, batch=B, seed=5)
+        bud = draw_sweep_schedules(a.chunk_len, B, seed=5)
+        ex.denoise(noise, bud)
+        res = ex.finish(timeout_us=TIMEOUT)
+        for b in (0, 31, 63):
+            ref = denoise(build_model(a, blob, pre[b]).velocity, noise[b], bud[b])
+            assert rel_err(res["final"][b], ref["final"]) <= TOL["bf16"]
+            assert rel_err(res["ghost"][b], ref["ghost"]) <= TOL["bf16"]
+        assert res["evals"] == 10
+    finally:
+        ex.close()
+
+
 def test_one_pass_attention_many_tiles():
     """32 robots x 2 query tiles on the small bf16 expert: the attention takes its path for many
     query tiles (one pass over 128-key chunks, O in tensor memory rescaled only when a row maximum
