@@ -1,5 +1,6 @@
 """CPU checks of bench.py's host logic: the replica (N > 1) timing reduction over gloo ranks,
-and its action-availability-latency arithmetic against the oracle's control clock."""
+its action-availability-latency arithmetic against the oracle's control clock, and the time
+bound of the reference arm."""
 import multiprocessing as mp
 import os
 import socket
@@ -85,3 +86,21 @@ def test_bootstrap_interval():
     se = v.std(ddof=1) / np.sqrt(v.size)
     assert lo < v.mean() < hi
     assert abs((hi - lo) - 2 * 1.96 * se) < 0.25 * (2 * 1.96 * se)   # normal-theory width within 25%
+
+
+def test_reference_arm_is_bounded_in_time(monkeypatch, capsys):
+    """The reference arm (the CPU oracle) stops once its time bound is spent, whatever K is, and
+    still reports at least one timed chunk; its line carries the fields the driver reads."""
+    import argparse
+    import json
+    sys.path.insert(0, ROOT)
+    import bench
+    monkeypatch.setattr(bench, "REF_SECONDS", 0.0)
+    args = argparse.Namespace(gpus=1, steps=1000, warmup=3)
+    assert bench.run_reference(args, bench.WORKLOADS["tiny"], 1, 0) == 0
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["value"] > 0 and line["steps"] == 1000
+    assert line["cpu_baseline"]["value"] == line["value"]
+    assert line["cpu_baseline"]["sample"].startswith("1 full chunk(s) of robot 0 timed after 0 warm-up")
+    assert line["e2e"] == {"value": line["value"], "unit": line["unit"], "h2d_bytes_per_step": 0,
+                           "d2h_bytes_per_step": 0}
