@@ -104,3 +104,26 @@ def test_reference_arm_is_bounded_in_time(monkeypatch, capsys):
     assert line["cpu_baseline"]["sample"].startswith("1 full chunk(s) of robot 0 timed after 0 warm-up")
     assert line["e2e"] == {"value": line["value"], "unit": line["unit"], "h2d_bytes_per_step": 0,
                            "d2h_bytes_per_step": 0}
+
+
+def test_roofline_bound_follows_the_ridge_point():
+    """The dominant kernel is held to HBM below the ridge point of the peaks and to the bf16
+    tensor rate above it; achieved = its work per launch over its average launch time."""
+    sys.path.insert(0, ROOT)
+    import bench
+    pk = (6000.0, 2000.0, 1500.0, "measured")   # GB/s, burst TFLOP/s, sustained TFLOP/s
+    # latency-bound evaluation kernel: 600 MB and 36 GFLOP per launch (60 flop/B < 250 ridge)
+    prof = [{"name": "step", "launches": 10, "total_ms": 8.0, "bytes": 6.0e9, "flops": 3.6e11},
+            {"name": "euler", "launches": 10, "total_ms": 0.1, "bytes": 1.0e6, "flops": 1.0e6}]
+    r = bench.roofline_object(prof, 10, 0.81, pk, None)
+    assert r["bound"] == "hbm" and r["unit"] == "GB/s" and r["kernel"] == "step"
+    assert abs(r["achieved"] - 6.0e9 / 8e-3 / 1e9) < 1e-6 and abs(r["frac"] - 750.0 / 6000.0) < 1e-9
+    assert r["peak_source"].startswith("measured hbm_gbs")
+    # a large-batch GEMM: 50 MB and 54 GFLOP per launch (1080 flop/B > ridge), 180 launches
+    prof = [{"name": "gate_up", "launches": 180, "total_ms": 13.5, "bytes": 9.0e9, "flops": 9.72e12},
+            {"name": "attention", "launches": 180, "total_ms": 9.0, "bytes": 3.6e9, "flops": 6.1e12}]
+    r = bench.roofline_object(prof, 10, 3.9, pk, None)
+    assert r["bound"] == "tensor" and r["unit"] == "TFLOP/s" and r["peak"] == 1500.0
+    assert abs(r["achieved"] - 9.72e12 / 13.5e-3 / 1e12) < 1e-6
+    assert abs(r["flops_per_launch"] - 5.4e10) < 1.0 and r["peak_source"].startswith("measured bf16_tflops_sustained")
+    assert abs(r["step"]["tensor_frac"] - (15.82e12 / 10) / 3.9e-3 / 1e12 / 1500.0) < 1e-9
