@@ -99,10 +99,35 @@ def _ptr(a):
     if a is None:
         return None
     if isinstance(a, np.ndarray):
-        assert a.flags["C_CONTIGUOUS"]
+        if not a.flags["C_CONTIGUOUS"]:
+            raise ValueError("buffer must be C-contiguous")
         return a.ctypes.data
-    assert a.is_contiguous()
+    if not a.is_contiguous():
+        raise ValueError("buffer must be contiguous")
     return a.data_ptr()
+
+
+def _buf(a, n, dtype, what, host=False):
+    """Address of a buffer the library reads or writes n elements of: a C-contiguous numpy
+    array or torch tensor of `dtype` ("float32", "int32", "uint8"; "bfloat16" = np.uint16 bit
+    patterns or a torch bfloat16 tensor) holding exactly n elements (host memory only when
+    `host`). The C ABI takes bare pointers and cannot check sizes, so a short buffer is
+    refused here, before the call, with ValueError; None passes through."""
+    if a is None:
+        return None
+    if isinstance(a, np.ndarray):
+        ok = a.dtype == (np.dtype(np.uint16) if dtype == "bfloat16" else np.dtype(dtype))
+        size, on_host = a.size, True
+    else:
+        ok = str(a.dtype) == "torch." + dtype
+        size, on_host = a.numel(), a.device.type == "cpu"
+    if not ok:
+        raise ValueError(f"{what}: expected {dtype} elements, got {a.dtype}")
+    if size != n:
+        raise ValueError(f"{what}: expected {n} elements, got {size}")
+    if host and not on_host:
+        raise ValueError(f"{what}: must be host memory")
+    return _ptr(a)
 
 
 def _stream_handle(stream):
@@ -142,7 +167,7 @@ class Expert:
         h = _P()
         w = weights if not isinstance(weights, np.ndarray) else np.ascontiguousarray(weights, np.float32)
         n = w.size if isinstance(w, np.ndarray) else w.numel()
-        rc = uad_init(C.byref(self.arch), _ptr(w), n, C.byref(h))
+        rc = uad_init(C.byref(self.arch), _buf(w, n, "float32", "weights"), n, C.byref(h))
         if rc != UAD_OK:
             raise UADError(rc, "uad_init failed (see stderr)")
         self.h = h
@@ -155,11 +180,23 @@ class Expert:
         return rc
 
     def set_prefix(self, robot, k, v=None, dtype="f32"):
+        """Attention-prefix experts: k, v [L][P][Hkv][dh]; DiT: k = prefix tokens
+        [P][prefix_width], v = None. dtype "f32" (float32) or "bf16" (bfloat16 tensors or
+        np.uint16 bit patterns); host or device."""
+        code = DTYPE.get(dtype, dtype)
+        el = "bfloat16" if code == DTYPE["bf16"] else "float32"
+        a = self.arch
+        if a.kind == KIND["dit"]:
+            n = a.prefix_len * a.prefix_width
+        else:
+            n = a.n_layers * a.prefix_len * a.n_kv_heads * a.head_dim
         if isinstance(k, np.ndarray):
-            k = np.ascontiguousarray(k)
-            v = None if v is None else np.ascontiguousarray(v)
-        return self._check(uad_set_prefix_kv(self.h, robot, _ptr(k), _ptr(v), self.arch.prefix_len,
-                                             DTYPE.get(dtype, dtype)), "set_prefix")
+            k = np.ascontiguousarray(k, np.float32 if el == "float32" else None)
+        if isinstance(v, np.ndarray):
+            v = np.ascontiguousarray(v, np.float32 if el == "float32" else None)
+        return self._check(uad_set_prefix_kv(self.h, robot, _buf(k, n, el, "prefix k"),
+                                             _buf(v, n, el, "prefix v"), a.prefix_len, code),
+                           "set_prefix")
 
     def prepare_times(self, max_budget):
         return self._check(uad_prepare_times(self.h, max_budget), "prepare_times")
@@ -167,6 +204,8 @@ class Expert:
     def _schedule(self, budgets, n_exec, tr, gac, chunk_relative, gac_mask, rot_dim=None):
         b = np.ascontiguousarray(budgets, dtype=np.int32).reshape(-1, self.H)
         m = None if gac_mask is None else np.ascontiguousarray(gac_mask, dtype=np.uint8)
+        if m is not None and m.size != self.D:
+            raise ValueError(f"gac_mask: expected {self.D} entries, got {m.size}")
         sc = uad_schedule(budgets=b.ctypes.data_as(C.POINTER(_I32)), batch=b.shape[0], n_exec=n_exec,
                           tr=int(tr), gac=int(gac), chunk_relative=int(chunk_relative),
                           gac_mask=None if m is None else m.ctypes.data_as(C.POINTER(C.c_uint8)),
@@ -179,10 +218,11 @@ class Expert:
         sc, keep = self._schedule(budgets, n_exec, tr, gac, chunk_relative, gac_mask, rot_dim)
         if isinstance(noise, np.ndarray):
             noise = np.ascontiguousarray(noise, dtype=np.float32)
+        B = keep[0].shape[0]
+        p = _buf(noise, B * self.H * self.D, "float32", "noise")
         self._keep = noise
-        self._B = keep[0].shape[0]
-        return self._check(uad_denoise(self.h, _ptr(noise), C.byref(sc), n_star, _stream_handle(stream)),
-                           "denoise")
+        self._B = B
+        return self._check(uad_denoise(self.h, p, C.byref(sc), n_star, _stream_handle(stream)), "denoise")
 
     def profile(self, noise, budgets, n_exec=0, tr=True, gac=True, chunk_relative=False, gac_mask=None,
                 timeout_us=120_000_000):
@@ -190,9 +230,11 @@ class Expert:
         sc, keep = self._schedule(budgets, n_exec, tr, gac, chunk_relative, gac_mask)
         if isinstance(noise, np.ndarray):
             noise = np.ascontiguousarray(noise, dtype=np.float32)
-        self._B = keep[0].shape[0]
+        B = keep[0].shape[0]
+        p = _buf(noise, B * self.H * self.D, "float32", "noise")
+        self._B = B
         stats = (uad_kernel_stat * 64)()
-        n = self._check(uad_profile_chunk(self.h, _ptr(noise), C.byref(sc), stats, 64, int(timeout_us)), "profile")
+        n = self._check(uad_profile_chunk(self.h, p, C.byref(sc), stats, 64, int(timeout_us)), "profile")
         return [dict(name=st.name.decode(), launches=st.launches, total_ms=st.total_ms, bytes=st.bytes,
                      flops=st.flops) for st in stats[:n]]
 
@@ -200,7 +242,8 @@ class Expert:
         out = np.zeros((self.H, self.D), np.float32) if out is None else out
         ready = np.zeros(self.H, np.int32)
         step = np.zeros(self.H, np.int32)
-        rc = uad_poll_released(self.h, robot, min_ready, int(timeout_us), _ptr(out), _ptr(ready), _ptr(step))
+        p = _buf(out, self.H * self.D, "float32", "out", host=True)
+        rc = uad_poll_released(self.h, robot, min_ready, int(timeout_us), p, _ptr(ready), _ptr(step))
         if rc < 0 and rc != UAD_ETIMEDOUT:
             self._check(rc, "poll")
         return rc, out, ready, step
@@ -211,7 +254,10 @@ class Expert:
         ghost = np.zeros((B, self.H, self.D), np.float32) if ghost is None else ghost
         gac_error = np.zeros((B, self.D), np.float32) if gac_error is None else gac_error
         st = uad_stats()
-        rc = uad_finish(self.h, _ptr(final), _ptr(ghost), _ptr(gac_error), C.byref(st), int(timeout_us))
+        n = B * self.H * self.D
+        pf, pg = _buf(final, n, "float32", "final"), _buf(ghost, n, "float32", "ghost")
+        pe = _buf(gac_error, B * self.D, "float32", "gac_error")
+        rc = uad_finish(self.h, pf, pg, pe, C.byref(st), int(timeout_us))
         if check and rc < 0:
             self._check(rc, "finish")
         return dict(rc=rc, final=final, ghost=ghost, E=gac_error, evals=st.evals, n_star=st.n_star,
