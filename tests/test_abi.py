@@ -43,6 +43,8 @@ SCHEDULES = [
     [3, 1, 4, 1, 5, 9, 2, 6],
     [2] * 16,
     [8, 16, 16, 16],
+    [1] * 5,                       # N* = 1: one step, nothing released early
+    [64, 1, 33, 64, 2],            # the largest budget the library accepts
 ]
 
 
