@@ -12,7 +12,7 @@ import paper_2609_37772_gb300 as uad
 from oracle.model import build_model
 from oracle.uad import denoise
 from uad_inputs import (ARCHS, draw_sweep_schedules, group_budgets, make_noise, make_prefix_kv,
-                        make_prefix_tokens, make_weights)
+                        make_prefix_tokens, make_weights, round_to_bf16)
 
 pytestmark = pytest.mark.gpu
 TOL = {"f32": 1e-4, "bf16": 2e-2}
@@ -575,3 +575,33 @@ def test_rot_dim_is_validated(tiny):
     bud = group_budgets(a.chunk_len, [(0, 3, 2), (4, a.chunk_len - 1, 4)])
     with pytest.raises(uad.UADError):
         tiny.ex.denoise(make_noise(a, seed=1), bud[None], rot_dim=a.action_dim - 2)
+
+
+@pytest.mark.parametrize("name", ["tiny", "pi0_small", "dit_small"])
+def test_prefix_given_in_bf16(name):
+    """uad_set_prefix_kv takes the prefix in fp32 or bf16, from host or device memory: the same
+    bf16-exact prefix given as fp32, as bf16 bit patterns on the host and as a bf16 device tensor
+    gives a chunk within tolerance of the oracle every time."""
+    a = ARCHS[name]
+    blob = make_weights(a, seed=21)
+    pre = prefixes(a, 1, seed=21)[0]
+    exact = [round_to_bf16(p) for p in ((pre,) if a.kind == "dit" else pre)]
+    model = build_model(a, blob, exact[0] if a.kind == "dit" else tuple(exact))
+    noise = make_noise(a, seed=21)
+    bud = group_budgets(a.chunk_len, [(0, 3, 2), (4, a.chunk_len - 1, 5)])
+    ref = denoise(model.velocity, noise[0], bud)
+    tol = TOL[a.dtype]
+    forms = [(exact, "f32"),
+             ([(e.view(np.uint32) >> 16).astype(np.uint16) for e in exact], "bf16"),
+             ([torch.from_numpy(e).to(torch.bfloat16).cuda() for e in exact], "bf16")]
+    ex = uad.Expert(a, blob)
+    try:
+        for p, dt in forms:
+            ex.set_prefix(0, *p, dtype=dt)
+            ex.denoise(noise, bud[None])
+            res = ex.finish(timeout_us=TIMEOUT)
+            assert rel_err(res["final"][0], ref["final"]) <= tol, (dt, rel_err(res["final"][0], ref["final"]))
+            assert rel_err(res["ghost"][0], ref["ghost"]) <= tol
+            assert res["evals"] == ref["evals"]
+    finally:
+        ex.close()
