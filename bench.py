@@ -266,6 +266,20 @@ def max_over_ranks(x, world, device="cpu"):
 REF_SECONDS = 150.0   # bound on the reference arm's oracle time
 
 
+def oracle_threads():
+    """Threads the oracle's numpy arithmetic runs on: the BLAS pool's size where threadpoolctl
+    can read it, else the CPUs this process may run on."""
+    try:
+        from threadpoolctl import threadpool_info
+        n = max((int(p.get("num_threads") or 0) for p in threadpool_info() if p.get("user_api") == "blas"),
+                default=0)
+        if n > 0:
+            return n
+    except ImportError:
+        pass
+    return len(os.sched_getaffinity(0))
+
+
 def oracle_chunks(wl, seconds, max_chunks=None):
     """Time the CPU oracle, as it stands, on whole chunks of robot 0 of this workload."""
     from oracle.model import build_model
@@ -297,7 +311,7 @@ def run_reference(args, wl, world, rank):
     timed = times[warm:]
     per = statistics.mean(timed)
     value = a.chunk_len / per
-    cores = os.cpu_count()
+    cores = oracle_threads()
     line = {
         "impl": "reference", "metric": "action-tokens/s", "value": value, "unit": "tokens/s",
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": per * 1e3,
@@ -429,7 +443,7 @@ def run_ours(args, wl, world, rank, local):
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         _, times = oracle_chunks(wl, args.cpu_seconds)
-        cpu = {"value": H / statistics.mean(times), "unit": "tokens/s", "cores": os.cpu_count(),
+        cpu = {"value": H / statistics.mean(times), "unit": "tokens/s", "cores": oracle_threads(),
                "kind": "oracle", "sample": f"{len(times)} full chunk(s) of robot 0 (fp64 numpy oracle), "
                                            f"{sum(times):.1f} s"}
 

@@ -127,3 +127,9 @@ def test_roofline_bound_follows_the_ridge_point():
     assert abs(r["achieved"] - 9.72e12 / 13.5e-3 / 1e12) < 1e-6
     assert abs(r["flops_per_launch"] - 5.4e10) < 1.0 and r["peak_source"].startswith("measured bf16_tflops_sustained")
     assert abs(r["step"]["tensor_frac"] - (15.82e12 / 10) / 3.9e-3 / 1e12 / 1500.0) < 1e-9
+
+
+def test_oracle_thread_count_is_what_the_process_may_use():
+    import bench
+    n = bench.oracle_threads()
+    assert 1 <= n <= (os.cpu_count() or n)
