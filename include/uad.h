@@ -51,7 +51,7 @@ extern "C" {
 
 /* Shape of the action expert F_theta (Sec. 3, Eq. 1). */
 typedef struct uad_arch {
-  int32_t kind;          /* UAD_KIND_ADARMS or UAD_KIND_DIT */
+  int32_t kind;          /* UAD_KIND_ADARMS, UAD_KIND_DIT or UAD_KIND_CONCAT */
   int32_t dtype;         /* UAD_DTYPE_F32: fp32 everywhere; UAD_DTYPE_BF16: bf16 weights and
                             GEMM/attention operands, fp32 accumulation, state and velocities */
   int32_t n_layers;
