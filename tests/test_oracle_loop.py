@@ -250,3 +250,77 @@ def test_plan_times_and_sets():
     assert times == expect
     with pytest.raises(ValueError):
         P.step_plan([0, 3], 1)
+
+
+def _random_schedules(rng, n):
+    for _ in range(n):
+        H = int(rng.integers(3, 13))
+        groups = int(rng.integers(1, 4))
+        levels = sorted(set(int(x) for x in rng.integers(1, 9, size=groups)))
+        b = np.array(levels, dtype=int)[rng.integers(0, len(levels), size=H)]
+        yield H, [int(x) for x in b]
+
+
+@pytest.mark.parametrize("tr", [True, False])
+def test_inputs_times_and_outputs_follow_eqs_5_to_9_on_random_schedules(tr):
+    """Record every call of a coupled nonlinear field and rebuild, from the recorded velocities
+    alone, what Eqs. 5-9 say the loop must have fed and returned: each action's flow time and
+    input at every step (own step 1/N_i while active; after release the reconciled state
+    x_0 + (1/N*) sum_j v_j with TR, the frozen released value at flow time 1 without), the
+    released, ghost and tail states, and E with its uniform spread over the executable tail."""
+    rng = np.random.default_rng(11 + tr)
+    for H, budgets in _random_schedules(rng, 40):
+        D = 3
+        ns = max(budgets)
+        S = int(rng.integers(1, H + 1))
+        x0 = rng.normal(size=(H, D))
+        A = rng.normal(scale=0.4, size=(H * D, H * D))
+        c = rng.normal(size=D)
+        tape = []
+
+        def vel(u, tau):
+            v = np.tanh((A @ u.reshape(-1)).reshape(H, D)) + np.asarray(tau)[:, None] * c
+            tape.append((u.copy(), np.asarray(tau, float).copy(), v.copy()))
+            return v
+
+        out = denoise(vel, x0, budgets, n_exec=S, tr=tr, gac=tr)
+        assert len(tape) == ns == out["evals"]
+        V = np.stack([t[2] for t in tape])                        # [N*, H, D]
+        for i, n_i in enumerate(budgets):
+            own = x0[i] + np.cumsum(V[:n_i, i] / n_i, axis=0)      # x_k under Eq. 5, k = 1..N_i
+            canon = x0[i] + np.cumsum(V[:, i] / ns, axis=0)       # Eqs. 6-7: step 1/N* from x_0
+            for k in range(1, ns + 1):
+                u, tau, _ = tape[k - 1]
+                if k <= n_i:
+                    want_u = x0[i] if k == 1 else own[k - 2]
+                    assert tau[i] == float(Fraction(k - 1, n_i))
+                elif tr:
+                    want_u = canon[k - 2]
+                    assert tau[i] == float(Fraction(k - 1, ns))
+                else:
+                    want_u = own[-1]
+                    assert tau[i] == 1
+                np.testing.assert_allclose(u[i], want_u, rtol=0, atol=1e-12)
+            assert out["release_step"][i] == n_i
+            if n_i < ns:
+                np.testing.assert_allclose(out["released"][i], own[-1], rtol=0, atol=1e-12)
+                np.testing.assert_array_equal(out["final"][i], out["released"][i])
+                if tr:
+                    np.testing.assert_allclose(out["ghost"][i], canon[-1], rtol=0, atol=1e-12)
+                else:                                             # no reconciled state without TR
+                    np.testing.assert_array_equal(out["ghost"][i], out["released"][i])
+        early = [i for i, n in enumerate(budgets) if n < ns]
+        tail = [i for i, n in enumerate(budgets) if n == ns and i < S]
+        assert out["tail"] == (tail if tr and early else [])        # the actions GAC corrected
+        x_end = {i: x0[i] + np.cumsum(V[:, i] / ns, axis=0)[-1] for i in range(H) if budgets[i] == ns}
+        if tr and early and tail:
+            E = sum(out["ghost"][i] - out["released"][i] for i in early)
+            np.testing.assert_allclose(out["E"], E, rtol=0, atol=1e-12)
+            for i in tail:
+                np.testing.assert_allclose(out["final"][i], x_end[i] + E / len(tail), rtol=0, atol=1e-12)
+        else:
+            for i in tail:
+                np.testing.assert_allclose(out["final"][i], x_end[i], rtol=0, atol=1e-12)
+        for i, n in enumerate(budgets):
+            if n == ns and i >= S:
+                np.testing.assert_allclose(out["final"][i], x_end[i], rtol=0, atol=1e-12)
