@@ -5,7 +5,10 @@ project's stated design and parity for it is unpinned beyond what is checked her
 building block against an independent library routine (torch fp64), and structural
 invariants of the whole network (grouped-query heads equal expanded multi-head attention,
 token-permutation equivariance without position information, RoPE scores depending only
-on relative position, per-action time conditioning being per token).
+on relative position, per-action time conditioning being per token), and special cases in
+which a block collapses to a closed form (a zero gate makes a layer the identity; a scale of
+-1 replaces the normalised stream by the shift), which pin the order of the modulation
+vectors and of the weights in the blob.
 """
 import numpy as np
 import pytest
@@ -228,3 +231,180 @@ def test_k1_exact_recovery_with_the_concat_network():
     van = denoise(m.velocity, x0, [10] * a.chunk_len)
     uad = denoise(m.velocity, x0, [1] * 4 + [10] * (a.chunk_len - 4), gac=False)
     assert np.array_equal(uad["ghost"], van["final"]) and np.array_equal(uad["final"][4:], van["final"][4:])
+
+
+def _with_prefix(a, blob, seed):
+    m = Model(a, blob)
+    if a.n_layers:
+        if a.kind == "dit":
+            m.set_prefix_tokens(make_prefix_tokens(a, seed=seed))
+        else:
+            m.set_prefix_kv(*make_prefix_kv(a, seed=seed))
+    return m
+
+
+def _gates_zeroed(a, w):
+    """Copy of the weights with every gate of every layer zero: for adaRMS the third W-slice of
+    both modulations (scale, shift, gate); for DiT gate1 and gate2 of (shift1, scale1, gate1,
+    shift2, scale2, gate2), and the ungated cross-attention's output projection."""
+    W = a.width
+    w = {k: v.copy() for k, v in w.items()}
+    for l in range(a.n_layers):
+        p = f"l{l}."
+        if a.kind == "adarms":
+            for mod in ("mod1", "mod2"):
+                w[p + mod + "_w"][:, 2 * W:] = 0
+                w[p + mod + "_b"][2 * W:] = 0
+        else:
+            for g in (2, 5):
+                w[p + "mod_w"][:, g * W:(g + 1) * W] = 0
+                w[p + "mod_b"][g * W:(g + 1) * W] = 0
+            w[p + "woc"][:] = 0
+    return w
+
+
+@pytest.mark.parametrize("name", ["tiny", "dit_small"])
+def test_layers_with_zero_gates_are_the_identity(name):
+    """Every residual branch is scaled by its gate (DiT's cross-attention, ungated, by its output
+    projection), so with those zero the network equals the same network without layers: pins
+    where the gates sit in the modulation vectors."""
+    from uad_inputs import weight_specs
+    a = ARCHS[name]
+    w = _gates_zeroed(a, split_blob(a, make_weights(a, seed=30)))
+    m = _with_prefix(a, blob_from_weights(a, w), 30)
+    a0 = a.replace(n_layers=0)
+    m0 = Model(a0, blob_from_weights(a0, {n: w[n] for n, _ in weight_specs(a0)}))
+    u = make_noise(a, seed=30)[0]
+    tau = np.linspace(0.0, 0.9, a.chunk_len)
+    np.testing.assert_allclose(m.velocity(u, tau), m0.velocity(u, tau), rtol=1e-12, atol=1e-12)
+    full = _with_prefix(a, make_weights(a, seed=30), 30)
+    assert not np.allclose(full.velocity(u, tau), m0.velocity(u, tau))
+
+
+@pytest.mark.parametrize("name", ["tiny", "dit_small"])
+def test_final_modulation_order(name):
+    """The final norm's modulation is (scale, shift) for adaRMS and (shift, scale) for DiT: with
+    scale = -1 the normalised stream drops out and v = shift W_out + b_out for every token."""
+    a = ARCHS[name]
+    W = a.width
+    w = {k: v.copy() for k, v in split_blob(a, make_weights(a, seed=31)).items()}
+    s = np.random.default_rng(31).normal(size=W).astype(np.float32)
+    minus = -np.ones(W, np.float32)
+    w["modf_w"][:] = 0
+    w["modf_b"][:] = np.concatenate([minus, s] if a.kind == "adarms" else [s, minus])
+    m = _with_prefix(a, blob_from_weights(a, w), 31)
+    v = m.velocity(make_noise(a, seed=31)[0], np.linspace(0.0, 0.9, a.chunk_len))
+    want = s.astype(np.float64) @ w["out_w"].astype(np.float64) + w["out_b"]
+    np.testing.assert_allclose(v, np.tile(want, (a.chunk_len, 1)), rtol=1e-12, atol=1e-12)
+
+
+def test_dit_tokens_are_told_apart_by_position():
+    """The DiT head adds a sinusoidal code of the token index to its input (its attention has no
+    other position information): tokens with equal states and flow times get different
+    velocities, where the attention-prefix expert without RoPE gives them equal ones."""
+    a = ARCHS["dit_small"]
+    m = _with_prefix(a, make_weights(a, seed=32), 32)
+    u = np.tile(make_noise(a, seed=32)[0][:1], (a.chunk_len, 1))
+    tau = np.full(a.chunk_len, 0.3)
+    v = m.velocity(u, tau)
+    d = np.abs(v[:, None, :] - v[None, :, :]).max(axis=-1) + np.eye(a.chunk_len)
+    assert d.min() > 1e-4
+    b = _tiny(rope=False)
+    mb = _with_prefix(b, make_weights(b, seed=32), 32)
+    ub = np.tile(make_noise(b, seed=32)[0][:1], (b.chunk_len, 1))
+    vb = mb.velocity(ub, np.full(b.chunk_len, 0.3))
+    np.testing.assert_allclose(vb, np.tile(vb[:1], (b.chunk_len, 1)), rtol=1e-12, atol=1e-12)
+
+
+def test_dit_cross_attention_reads_the_stream_through_its_norm():
+    """The DiT cross-attention's queries come from the unmodulated LayerNorm of the stream, so with
+    the gated branches off a layer's update is unchanged when every row of the stream is scaled
+    and shifted (up to the norm's epsilon)."""
+    a = ARCHS["dit_small"].replace(n_layers=1)
+    W = a.width
+    w = {k: v.copy() for k, v in split_blob(a, make_weights(a, seed=33)).items()}
+    for g in (2, 5):
+        w["l0.mod_w"][:, g * W:(g + 1) * W] = 0
+        w["l0.mod_b"][g * W:(g + 1) * W] = 0
+    m = _with_prefix(a, blob_from_weights(a, w), 33)
+    c = m.time_cond(np.linspace(0.0, 0.9, a.chunk_len))
+    h = np.random.default_rng(33).normal(size=(a.chunk_len, W))
+    h2 = 3.0 * h + 0.5
+    d1 = m._layer(0, h, c) - h
+    d2 = m._layer(0, h2, c) - h2
+    assert np.abs(d1).max() > 1e-3
+    np.testing.assert_allclose(d2, d1, rtol=0, atol=1e-5 * np.abs(d1).max())
+
+
+def _dit_layer_with_constant_modulation(seed, mod_b, woc_zero=True):
+    a = ARCHS["dit_small"].replace(n_layers=1)
+    w = {k: v.copy() for k, v in split_blob(a, make_weights(a, seed=seed)).items()}
+    w["l0.mod_w"][:] = 0
+    w["l0.mod_b"][:] = np.concatenate(mod_b).astype(np.float32)
+    if woc_zero:
+        w["l0.woc"][:] = 0
+    m = _with_prefix(a, blob_from_weights(a, w), seed)
+    h = np.random.default_rng(seed).normal(size=(a.chunk_len, a.width)) * 2 + 0.3
+    c = m.time_cond(np.linspace(0.0, 0.9, a.chunk_len))
+    return a, {k: v.astype(np.float64) for k, v in w.items()}, m._layer(0, h, c) - h
+
+
+def test_dit_self_attention_modulation_order():
+    """DiT layer modulation (shift1, scale1, gate1, ...): with scale1 = -1 every token enters the
+    self-attention as shift1, whose uniform attention returns its own value row, so the update is
+    gate1 * (shift1 Wv Wo) whatever the stream (MLP gate and cross-attention output off)."""
+    W = ARCHS["dit_small"].width
+    rng = np.random.default_rng(34)
+    sh1, g1, sh2, sc2 = (rng.normal(size=W) for _ in range(4))
+    a, w, d = _dit_layer_with_constant_modulation(34, [sh1, -np.ones(W), g1, sh2, sc2, np.zeros(W)])
+    sh1, g1 = (x.astype(np.float32).astype(np.float64) for x in (sh1, g1))
+    want = g1 * ((sh1 @ w["l0.wv"]) @ w["l0.wo"])
+    np.testing.assert_allclose(d, np.tile(want, (a.chunk_len, 1)), rtol=1e-11, atol=1e-12)
+
+
+def test_dit_mlp_modulation_order():
+    """With scale2 = -1 the MLP sees shift2 on every token: the update is
+    gate2 * (gelu_tanh(shift2 W1 + b1) W2 + b2) (self-attention gate and cross-attention output
+    off); the activation here is torch's."""
+    W = ARCHS["dit_small"].width
+    rng = np.random.default_rng(35)
+    sh1, sc1, sh2, g2 = (rng.normal(size=W) for _ in range(4))
+    a, w, d = _dit_layer_with_constant_modulation(35, [sh1, sc1, np.zeros(W), sh2, -np.ones(W), g2])
+    sh2, g2 = (x.astype(np.float32).astype(np.float64) for x in (sh2, g2))
+    act = Fnn.gelu(T(sh2 @ w["l0.w1"] + w["l0.b1"]), approximate="tanh").numpy()
+    want = g2 * (act @ w["l0.w2"] + w["l0.b2"])
+    np.testing.assert_allclose(d, np.tile(want, (a.chunk_len, 1)), rtol=1e-11, atol=1e-12)
+
+
+def test_time_mlp_has_two_silus():
+    """c = SiLU(SiLU(e W1 + b1) W2 + b2): with W2 = 0, c = SiLU(b2) for every flow time; with
+    W1 = 0, c = SiLU(SiLU(b1) W2 + b2) (torch's SiLU)."""
+    a = _tiny(rope=False)
+    m = Model(a, make_weights(a, seed=36))
+    tau = np.array([0.0, 0.25, 0.5, 0.9])
+    w2 = m.w["t_w2"].copy()
+    m.w["t_w2"][:] = 0
+    np.testing.assert_allclose(m.time_cond(tau), np.tile(Fnn.silu(T(m.w["t_b2"])).numpy(), (4, 1)), rtol=1e-13)
+    m.w["t_w2"][:] = w2
+    m.w["t_w1"][:] = 0
+    inner = Fnn.silu(T(m.w["t_b1"])).numpy()
+    want = Fnn.silu(T(inner @ w2 + m.w["t_b2"])).numpy()
+    np.testing.assert_allclose(m.time_cond(tau), np.tile(want, (4, 1)), rtol=1e-12, atol=1e-14)
+
+
+def test_concat_input_mlp_weights_read_what_they_are_named_for():
+    """SmolVLA-style input MLP: ti_wa multiplies the action embedding and ti_wt the time
+    embedding. With ti_wt = 0 the network no longer sees the flow time (its layers are
+    unmodulated); with ti_wa = 0 it no longer sees the action state."""
+    a = ARCHS["tiny_concat"]
+    u1, u2 = make_noise(a, seed=37)[0], make_noise(a, seed=38)[0]
+    t1, t2 = np.linspace(0.0, 0.9, a.chunk_len), np.linspace(0.9, 0.0, a.chunk_len)
+    m = _with_prefix(a, make_weights(a, seed=37), 37)
+    assert not np.allclose(m.velocity(u1, t1), m.velocity(u1, t2))
+    assert not np.allclose(m.velocity(u1, t1), m.velocity(u2, t1))
+    wt = m.w["ti_wt"].copy()
+    m.w["ti_wt"][:] = 0
+    np.testing.assert_allclose(m.velocity(u1, t1), m.velocity(u1, t2), rtol=1e-12, atol=1e-13)
+    m.w["ti_wt"][:] = wt
+    m.w["ti_wa"][:] = 0
+    np.testing.assert_allclose(m.velocity(u1, t1), m.velocity(u2, t1), rtol=1e-12, atol=1e-13)
