@@ -13,7 +13,8 @@ Modules
             (Eqs. 8-9); takes the velocity field as a callable
   model.py  the synthetic action expert F_theta (Eq. 1) with per-action time conditioning
             (App. C.1); its composition is this project's stated architecture, not the
-            paper's (the paper fixes none) -- parity unpinned beyond its components
+            paper's (the paper fixes none) -- parity unpinned beyond its components,
+            structural invariants and closed-form special cases
   so3.py    rotation vectors and Ghost Action Correction by composition on SO(3) (App. C.1)
   clock.py  action availability latency under the control-time alignment clock
             (Sec. 5.1 Metrics, App. C.3) and the latency model (App. B, Eqs. 11-12)
