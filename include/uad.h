@@ -81,8 +81,10 @@ typedef struct uad_schedule {
                               0 = left unchanged (rotation / gripper); NULL = all additive */
   int32_t rot_dim;         /* first of three dimensions holding a rotation vector (axis times
                               angle, radians) that GAC corrects by composition on SO(3)
-                              (App. C.1): E_R = product over early actions, in token order, of
-                              R(ghost) R(released)^T; every tail action R <- exp(log(E_R)/|tail|) R.
+                              (App. C.1): E_R = F_U ... F_2 F_1 with F_i = R(ghost_i)
+                              R(released_i)^T over the early actions in token order (each applied
+                              after the previous ones); every tail action
+                              R <- exp(log(E_R)/|tail|) R.
                               These dimensions are never additive; -1 = no rotation dimensions.
                               Must be -1 or in 0..action_dim-3 (else UAD_EINVAL). */
 } uad_schedule;

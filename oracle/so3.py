@@ -74,7 +74,8 @@ def nearest_rep(w, ref):
 def gac_rotation(released, ghost, tail_rows):
     """Eqs. 8-9 on SO(3) for one chunk. released, ghost: [U, 3] rotation vectors of the early
     actions in token order; tail_rows: [T, 3] rotation vectors of the executable tail.
-    Returns (e_R, corrected tail rows [T, 3])."""
+    The discrepancies F_i = R(ghost_i) R(released_i)^T are applied in token order, each after the
+    previous ones: E_R = F_U ... F_2 F_1. Returns (e_R, corrected tail rows [T, 3])."""
     E = np.eye(3)
     for a, g in zip(released, ghost):
         E = exp_so3(g) @ exp_so3(a).T @ E

@@ -64,6 +64,18 @@ def test_corrections_compose_to_the_accumulated_error():
     assert np.allclose(np.linalg.matrix_power(C, 6), so3.exp_so3(e), atol=1e-12)
 
 
+def test_discrepancies_compose_in_token_order():
+    """Reading of App. C.1 (rotations compose; the order is not stated): the early actions'
+    discrepancies F_i = R(ghost_i) R(released_i)^T are applied one after another in token order,
+    E_R = F_U ... F_2 F_1. Hand-worked case: a quarter turn about x (first early action) then a
+    quarter turn about y (second) is a third of a turn about (1, 1, -1)/sqrt(3); the other order
+    would give the axis (1, 1, 1)/sqrt(3)."""
+    rel = np.zeros((2, 3))
+    gho = np.array([[np.pi / 2, 0.0, 0.0], [0.0, np.pi / 2, 0.0]])
+    e, _ = so3.gac_rotation(rel, gho, np.zeros((1, 3)))
+    np.testing.assert_allclose(e, (2 * np.pi / 3) * np.array([1.0, 1.0, -1.0]) / np.sqrt(3), atol=1e-12)
+
+
 def test_no_discrepancy_changes_nothing():
     g = rng(3)
     rel = g.normal(0, 0.7, (3, 3))
