@@ -193,6 +193,15 @@ typedef struct uad_kernel_stat {
 int uad_profile_chunk(uad_ctx* ctx, const float* noise, const uad_schedule* sched,
                       uad_kernel_stat* out, int32_t max_stats, int64_t timeout_us);
 
+/* Testing aid for the bounded waits (not part of the method). Every wait inside the persistent
+ * evaluation kernel gives up after wait_ns nanoseconds (> 0; the default is 2 s), records an
+ * error code on the device and lets the launch wind down; the next uad_finish then returns
+ * UAD_ECUDA, and the context stays usable. unreachable > 0 makes the first completion count of
+ * every evaluation wait for that many arrivals more than the kernel ever makes, so that the
+ * wait is sure to run out (0 restores normal operation). Applies to chunks started afterwards
+ * (cached graphs are rebuilt). Returns UAD_OK, UAD_EINVAL or UAD_ESTATE (chunk in flight). */
+int uad_set_wait_limit(uad_ctx* ctx, int64_t wait_ns, int32_t unreachable);
+
 void uad_destroy(uad_ctx* ctx);
 const char* uad_last_error(const uad_ctx* ctx);
 
@@ -244,8 +253,10 @@ int uad_linear(const void* x, const void* w_tiled, const float* bias, float* out
  *   - Limits: M * N <= UAD_LINEAR_STATIC_MAX_ELEMS and (N / 128) * ceil(M / 64) <=
  *     UAD_LINEAR_STATIC_MAX_TILES; larger calls return UAD_ETOOBIG and launch nothing.
  *   - The first call on a device looks up the array's device address (cudaGetSymbolAddress,
- *     which may load the library's device code); make that first call before any stream
- *     capture begins.
+ *     which may load the library's device code: with lazy module loading, the CUDA default,
+ *     the driver reserves the array only then). Make one warm-up call per device during
+ *     start-up, before any stream capture begins and before the control loop runs, so that
+ *     the device code and its array are resident when "allocates nothing" matters.
  *   - Every call on a device shares the one array and it keeps the previous call's contents:
  *     each call clears the part it uses (asynchronously, on `stream`) before its kernel.
  *     Calls whose work overlaps on the GPU (different streams, or threads racing) corrupt

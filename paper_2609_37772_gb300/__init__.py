@@ -69,12 +69,13 @@ uad_profile_chunk = _fn("uad_profile_chunk", C.c_int, _P, _P, C.POINTER(uad_sche
 uad_tile_weight = _fn("uad_tile_weight", C.c_int, _P, _I32, _I32, _P)
 uad_linear = _fn("uad_linear", C.c_int, _P, _P, _P, _P, _I32, _I32, _I32, _P)
 uad_linear_static_scratch = _fn("uad_linear_static_scratch", C.c_int, _P, _P, _P, _P, _I32, _I32, _I32, _P)
+uad_set_wait_limit = _fn("uad_set_wait_limit", C.c_int, _P, C.c_int64, _I32)
 UAD_ETOOBIG = -7
 
 EXPORTS = ["uad_version", "uad_last_error", "uad_init", "uad_set_prefix_kv", "uad_prepare_times",
            "uad_denoise", "uad_poll_released", "uad_finish", "uad_step_times",
            "uad_launches_per_chunk", "uad_destroy", "uad_plan_step", "uad_profile_chunk",
-           "uad_tile_weight", "uad_linear", "uad_linear_static_scratch"]
+           "uad_tile_weight", "uad_linear", "uad_linear_static_scratch", "uad_set_wait_limit"]
 
 
 def tile_weight(w):
@@ -267,6 +268,12 @@ class Expert:
         out = np.zeros(n, np.float64)
         k = self._check(uad_step_times(self.h, _ptr(out), n), "step_times")
         return out[:k]
+
+    def set_wait_limit(self, wait_ns=2_000_000_000, unreachable=0):
+        """Testing aid: bound of every wait in the persistent kernel, and extra arrivals its
+        first completion count waits for (> 0: the wait runs out and the chunk reports an
+        error)."""
+        return self._check(uad_set_wait_limit(self.h, int(wait_ns), int(unreachable)), "set_wait_limit")
 
     def launches_per_chunk(self, batch, n_star):
         return self._check(uad_launches_per_chunk(self.h, batch, n_star), "launches")

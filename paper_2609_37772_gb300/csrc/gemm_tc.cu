@@ -18,8 +18,11 @@
 #include <cudaTypedefs.h>
 
 #include "uad_internal.cuh"
+#include "ptx.cuh"
 
 namespace uad {
+
+using namespace ptx;
 
 namespace {
 
@@ -28,95 +31,15 @@ constexpr int kStageA = kBM * kBK * 2;  // 16 KB
 constexpr int kStageB = kBN * kBK * 2;  // 8 KB
 constexpr unsigned long long kWaitNs = 2000000000ull;  // 2 s bound on any wait
 
-__device__ __forceinline__ uint32_t su32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ unsigned long long gtime() {
-  unsigned long long t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-__device__ __forceinline__ void mbar_init(uint64_t* b, uint32_t n) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(b)), "r"(n));
-}
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* b, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(b)), "r"(bytes) : "memory");
-}
-// Wait for the phase with the given parity to complete; false (and *err set) after kWaitNs.
 __device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity, int* err, int code) {
-  unsigned long long t0 = 0;
-  for (uint32_t it = 0;; ++it) {
-    uint32_t ok;
-    asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
-        : "=r"(ok) : "r"(su32(b)), "r"(parity) : "memory");
-    if (ok) return true;
-    if ((it & 255) == 0) {
-      // give up at once if another wait already failed, so that one failure cannot chain
-      // into a long sequence of timeouts
-      if (*reinterpret_cast<volatile int*>(err) != 0) return false;
-      const unsigned long long t = gtime();
-      if (t0 == 0) t0 = t;
-      else if (t - t0 > kWaitNs) {
-        atomicCAS(err, 0, code);
-        return false;
-      }
-    }
-  }
+  return ptx::mbar_wait(b, parity, err, code, kWaitNs);
 }
-__device__ __forceinline__ uint64_t policy_evict_first() {
-  uint64_t p;
-  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
-  return p;
-}
-__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar, uint64_t pol) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;"
-      ::"r"(su32(dst)), "l"(src), "r"(bytes), "r"(su32(bar)), "l"(pol) : "memory");
-}
-__device__ __forceinline__ void tma_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
-      ::"r"(su32(dst)), "l"(map), "r"(x), "r"(y), "r"(su32(bar)) : "memory");
-}
-// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row core groups 1024 B apart.
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
-  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
-         ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
-}
+
 // Instruction descriptor, kind::f16: bf16 x bf16 -> fp32, both K-major, M = 128, N = 64.
 constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kBN >> 3) << 17) |
                             ((uint32_t)(kBM >> 4) << 24);
-
 __device__ __forceinline__ void mma_bf16(uint32_t d, uint64_t a, uint64_t b, uint32_t accum) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n"
-      ::"r"(d), "l"(a), "l"(b), "r"(kIdesc), "r"(accum));
-}
-__device__ __forceinline__ void mma_commit(uint64_t* bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(su32(bar)) : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-
-// 64 columns (two loads of 32, one wait) of this warp's 32 TMEM lanes, one row per thread.
-__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float* v) {
-  uint32_t* r = reinterpret_cast<uint32_t*>(v);
-#pragma unroll
-  for (int q = 0; q < 2; ++q)
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-        : "=r"(r[32 * q + 0]), "=r"(r[32 * q + 1]), "=r"(r[32 * q + 2]), "=r"(r[32 * q + 3]), "=r"(r[32 * q + 4]),
-          "=r"(r[32 * q + 5]), "=r"(r[32 * q + 6]), "=r"(r[32 * q + 7]), "=r"(r[32 * q + 8]), "=r"(r[32 * q + 9]),
-          "=r"(r[32 * q + 10]), "=r"(r[32 * q + 11]), "=r"(r[32 * q + 12]), "=r"(r[32 * q + 13]), "=r"(r[32 * q + 14]),
-          "=r"(r[32 * q + 15]), "=r"(r[32 * q + 16]), "=r"(r[32 * q + 17]), "=r"(r[32 * q + 18]), "=r"(r[32 * q + 19]),
-          "=r"(r[32 * q + 20]), "=r"(r[32 * q + 21]), "=r"(r[32 * q + 22]), "=r"(r[32 * q + 23]), "=r"(r[32 * q + 24]),
-          "=r"(r[32 * q + 25]), "=r"(r[32 * q + 26]), "=r"(r[32 * q + 27]), "=r"(r[32 * q + 28]), "=r"(r[32 * q + 29]),
-          "=r"(r[32 * q + 30]), "=r"(r[32 * q + 31])
-        : "r"(taddr + 32 * q)
-        : "memory");
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+  ptx::mma_bf16(d, a, b, kIdesc, accum);
 }
 
 __device__ __forceinline__ float gelu_tanh_f(float x) {
@@ -137,10 +60,6 @@ __device__ __forceinline__ void store_out(void* out, long long i, float v, int d
   else static_cast<float*>(out)[i] = v;
 }
 
-__device__ __forceinline__ void red_add_v4(float* dst, float4 v) {
-  asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(dst), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
-               : "memory");
-}
 
 // Shared-memory plan: [pipeline stages, at least 32 KB (reused as the split-K staging tile)]
 // [mbarriers, TMEM slot, flag].
@@ -424,12 +343,6 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kBN));
 }
 
-// ---- wide tiles for many tokens: 128 weight rows x TN tokens per CTA, no K split ------------
-__device__ __forceinline__ void mma_bf16_idesc(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accum) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n"
-      ::"r"(d), "l"(a), "l"(b), "r"(idesc), "r"(accum));
-}
 
 // TN tokens per tile (MMA N = 128 or 256); STAGES pipeline stages of 16 KB + TN x 128 B; MINB CTAs
 // per SM (more than one: one CTA's epilogue overlaps another's main loop, which pays when there
@@ -509,7 +422,7 @@ __global__ void __launch_bounds__(128, MINB) gemm_tc_wide_kernel(const __grid_co
       const uint32_t a0 = su32(sA + (size_t)st * kStageA), b0 = su32(sB + (size_t)st * kWStageB);
 #pragma unroll
       for (int k = 0; k < kBK / 16; ++k)
-        mma_bf16_idesc(tmem, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), kIdescWide, (i > 0 || k > 0) ? 1u : 0u);
+        ptx::mma_bf16(tmem, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), kIdescWide, (i > 0 || k > 0) ? 1u : 0u);
       mma_commit(empty + st);
     }
     mma_commit(done);

@@ -74,9 +74,14 @@ extern "C" int uad_linear_static_scratch(const void* x, const void* w_tiled, con
   int* err = counters + kCounters;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   // The array keeps whatever the previous call left; the kernel needs a zero accumulator,
-  // zero counters and a clear error word, so clear the part this call uses.
-  if (cudaMemsetAsync(acc, 0, (size_t)M * N * 4, s) != cudaSuccess ||
-      cudaMemsetAsync(counters, 0, (size_t)tiles * 4, s) != cudaSuccess ||
+  // zero counters and a clear error word, so clear the part this call uses. Wide tiles (many
+  // rows) have no K split and never touch the accumulator or the counters.
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return UAD_ECUDA;
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const bool split_scratch = uad::gemm_tc_use_wide(M, N, sms) == 0;
+  if ((split_scratch && (cudaMemsetAsync(acc, 0, (size_t)M * N * 4, s) != cudaSuccess ||
+                         cudaMemsetAsync(counters, 0, (size_t)tiles * 4, s) != cudaSuccess)) ||
       cudaMemsetAsync(err, 0, 4, s) != cudaSuccess)
     return UAD_ECUDA;
   return uad::launch_linear(x, w_tiled, bias, out, M, N, K, acc, counters, err, s);

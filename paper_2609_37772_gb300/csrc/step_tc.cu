@@ -40,8 +40,12 @@
 #include <cudaTypedefs.h>
 
 #include "uad_internal.cuh"
+#include "ptx.cuh"
+#include "euler.cuh"
 
 namespace uad {
+
+using namespace ptx;
 
 namespace {
 
@@ -58,108 +62,8 @@ constexpr int kMaxRows = kStepMaxRows;   // tokens per evaluation (the N side of
 constexpr int kMaxATiles = kStepMaxATiles;
 constexpr int kMaxRing = kStepMaxRing;
 constexpr uint32_t kTmemCols = 512;  // projection segments at 64-column steps; attention S at 0, O at 256
-constexpr unsigned long long kWaitNs = 2000000000ull;   // any single wait
 constexpr unsigned long long kDrainNs = 200000000ull;   // waiting for own copies before exit
 
-__device__ __forceinline__ uint32_t su32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
-__device__ __forceinline__ unsigned long long gtime() {
-  unsigned long long t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-__device__ __forceinline__ void mbar_init(uint64_t* b, uint32_t n) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(b)), "r"(n));
-}
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* b, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(b)), "r"(bytes) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint64_t* b) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(b)) : "memory");
-}
-__device__ __forceinline__ bool mbar_test(uint64_t* b, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
-      : "=r"(ok) : "r"(su32(b)), "r"(parity) : "memory");
-  return ok != 0;
-}
-// Non-blocking test of the phase with the given parity (returns at once).
-__device__ __forceinline__ bool mbar_peek(uint64_t* b, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
-      : "=r"(ok) : "r"(su32(b)), "r"(parity) : "memory");
-  return ok != 0;
-}
-// Wait for the phase with the given parity; false at once if an error is already recorded,
-// false with *err = code after kWaitNs.
-__device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity, int* err, int code) {
-  unsigned long long t0 = 0;
-  for (uint32_t it = 0;; ++it) {
-    if (mbar_test(b, parity)) return true;
-    if ((it & 255) == 0) {
-      if (*reinterpret_cast<volatile int*>(err) != 0) return false;
-      const unsigned long long t = gtime();
-      if (t0 == 0) t0 = t;
-      else if (t - t0 > kWaitNs) {
-        atomicCAS(err, 0, code);
-        return false;
-      }
-    }
-  }
-}
-// Wait for own asynchronous work before the CTA exits: bounded by time only.
-__device__ __forceinline__ void mbar_drain(uint64_t* b, uint32_t parity) {
-  const unsigned long long t0 = gtime();
-  while (!mbar_test(b, parity))
-    if (gtime() - t0 > kDrainNs) return;
-}
-__device__ __forceinline__ uint64_t policy_evict_first() {
-  uint64_t p;
-  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
-  return p;
-}
-__device__ __forceinline__ uint64_t policy_evict_last() {
-  uint64_t p;
-  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
-  return p;
-}
-__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar, uint64_t pol) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;"
-      ::"r"(su32(dst)), "l"(src), "r"(bytes), "r"(su32(bar)), "l"(pol) : "memory");
-}
-__device__ __forceinline__ void tma_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
-      ::"r"(su32(dst)), "l"(map), "r"(x), "r"(y), "r"(su32(bar)) : "memory");
-}
-__device__ __forceinline__ void tma_3d(void* dst, const CUtensorMap* map, int x, int y, int z, uint64_t* bar,
-                                       uint64_t pol) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
-      " [%0], [%1, {%2, %3, %4}], [%5], %6;"
-      ::"r"(su32(dst)), "l"(map), "r"(x), "r"(y), "r"(z), "r"(su32(bar)), "l"(pol) : "memory");
-}
-// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row core groups 1024 B apart.
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
-  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
-         ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
-}
-// kind::f16 instruction descriptor: bf16 x bf16 -> fp32, K-major A and B, M = 128, N = n.
-__device__ __forceinline__ uint32_t idesc_m128(int n) {
-  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
-}
-__device__ __forceinline__ void mma_bf16(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accum) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n"
-      ::"r"(d), "l"(a), "l"(b), "r"(idesc), "r"(accum));
-}
-__device__ __forceinline__ void mma_commit(uint64_t* bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(su32(bar)) : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
   uint32_t r[16];
   asm volatile(
@@ -172,102 +76,11 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
 #pragma unroll
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
-  uint32_t r[32];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
-      "tcgen05.wait::ld.sync.aligned;"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr)
-      : "memory");
-#pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-}
-// TMEM base address re-read from shared memory after a barrier wait: the tensor-memory loads
-// that follow take their address from this load, so they cannot be scheduled ahead of the
-// wait (the loads have no other dependence on it).
-// 64 columns (two loads of 32, one wait) of this warp's 32 TMEM lanes, one row per thread.
-__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float* v) {
-  uint32_t* r = reinterpret_cast<uint32_t*>(v);
-#pragma unroll
-  for (int q = 0; q < 2; ++q)
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-        : "=r"(r[32 * q + 0]), "=r"(r[32 * q + 1]), "=r"(r[32 * q + 2]), "=r"(r[32 * q + 3]), "=r"(r[32 * q + 4]),
-          "=r"(r[32 * q + 5]), "=r"(r[32 * q + 6]), "=r"(r[32 * q + 7]), "=r"(r[32 * q + 8]), "=r"(r[32 * q + 9]),
-          "=r"(r[32 * q + 10]), "=r"(r[32 * q + 11]), "=r"(r[32 * q + 12]), "=r"(r[32 * q + 13]), "=r"(r[32 * q + 14]),
-          "=r"(r[32 * q + 15]), "=r"(r[32 * q + 16]), "=r"(r[32 * q + 17]), "=r"(r[32 * q + 18]), "=r"(r[32 * q + 19]),
-          "=r"(r[32 * q + 20]), "=r"(r[32 * q + 21]), "=r"(r[32 * q + 22]), "=r"(r[32 * q + 23]), "=r"(r[32 * q + 24]),
-          "=r"(r[32 * q + 25]), "=r"(r[32 * q + 26]), "=r"(r[32 * q + 27]), "=r"(r[32 * q + 28]), "=r"(r[32 * q + 29]),
-          "=r"(r[32 * q + 30]), "=r"(r[32 * q + 31])
-        : "r"(taddr + 32 * q)
-        : "memory");
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
-__device__ __forceinline__ uint32_t tmem_base_after_wait(const uint32_t* slot) {
-  uint32_t t;
-  asm volatile("ld.volatile.shared.u32 %0, [%1];" : "=r"(t) : "r"(su32(slot)) : "memory");
-  return t;
-}
-__device__ __forceinline__ void red_add_v4(float* dst, float4 v) {
-  asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(dst), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
-               : "memory");
-}
-// Named barrier among `count` threads (whole warps).
-__device__ __forceinline__ void named_sync(int id, int count) {
-  asm volatile("barrier.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
-}
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
-}
-__device__ __forceinline__ float warp_max(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-  return v;
-}
-__device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
-  unsigned v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
-}
-// Hardware approximations (MUFU): 2^x and tanh. Both feed values that are rounded to bf16
-// next (P for the P V product, the MLP activation), far coarser than their error.
-__device__ __forceinline__ float ex2_approx(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-__device__ __forceinline__ float tanh_approx(float x) {
-  float y;
-  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
 __device__ __forceinline__ float gelu_tanh(float x) {
   const float k0 = 0.7978845608028654f;
   return 0.5f * x * (1.f + tanh_approx(k0 * (x + 0.044715f * x * x * x)));
 }
-__device__ __forceinline__ void bulk_s2g(void* gdst, const void* ssrc, uint32_t bytes) {
-  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(gdst), "r"(su32(ssrc)), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
-  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
-  return *reinterpret_cast<uint32_t*>(&h);
-}
 
-__device__ __forceinline__ void cp16(void* s, const void* g) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(su32(s)), "l"(g) : "memory");
-}
-__device__ __forceinline__ void cp_wait_all() {
-  asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;" ::: "memory");
-}
 __device__ __forceinline__ void st_bf16x4(__nv_bfloat16* dst, float a, float b, float c, float d) {
   uint2 pk;
   pk.x = pack_bf16(a, b);
@@ -393,10 +206,20 @@ struct StepShared {
   unsigned shares[4];                // epilogue shares of qkv, o, gate/up; [3] = merging CTAs
 };
 
+// A function's working copy of the caller's Role, written back when the function returns (kept in
+// registers instead of being read and written through a reference in local memory).
+struct RoleCopy {
+  Role& ref;
+  Role v;
+  __device__ __forceinline__ explicit RoleCopy(Role& r) : ref(r), v(r) {}
+  __device__ __forceinline__ ~RoleCopy() { ref = v; }
+};
+
 // Grid barrier among the consumer warps and the issuer's warp of every CTA: every CTA arrives (also
 // after an error, so that no CTA waits for it), then the issuer thread spins on the counter. Returns false once any error is
 // recorded, so that the remaining steps are skipped.
-__device__ __noinline__ bool grid_sync(unsigned* ctr, bool ok, int* err, const Smem& S) {
+__device__ __noinline__ bool grid_sync(unsigned* ctr, bool ok, int* err, const Smem& S, unsigned long long lim,
+                                       unsigned extra = 0) {
   tc_fence_before();
   __syncwarp();
   named_sync(1, kSyncThreads);
@@ -406,7 +229,7 @@ __device__ __noinline__ bool grid_sync(unsigned* ctr, bool ok, int* err, const S
     // are visible at GPU scope to whoever observes the count
     asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ctr) : "memory");
     if (good) {
-      const unsigned target = gridDim.x;
+      const unsigned target = gridDim.x + extra;
       unsigned long long t0 = 0;
       for (uint32_t it = 0;; ++it) {
         if (ld_acquire(ctr) >= target) break;
@@ -414,7 +237,7 @@ __device__ __noinline__ bool grid_sync(unsigned* ctr, bool ok, int* err, const S
           if (*reinterpret_cast<volatile int*>(err) != 0) { good = false; break; }
           const unsigned long long t = gtime();
           if (t0 == 0) t0 = t;
-          else if (t - t0 > kWaitNs) {
+          else if (t - t0 > lim) {
             atomicCAS(err, 0, 51);
             good = false;
             break;
@@ -432,35 +255,24 @@ __device__ __noinline__ bool grid_sync(unsigned* ctr, bool ok, int* err, const S
   return *reinterpret_cast<volatile int*>(S.flag) != 0;
 }
 
-// Bounded wait until *ctr >= target (acquire); false (error recorded) on timeout or once any error
-// is recorded.
-__device__ __noinline__ int count_wait(const unsigned* ctr, unsigned target, int* err) {
-  unsigned long long t0 = 0;
-  for (uint32_t it = 0;; ++it) {
-    if (ld_acquire(ctr) >= target) return 1;
-    if ((it & 63) == 63) {
-      if (*reinterpret_cast<volatile int*>(err) != 0) return 0;
-      const unsigned long long t = gtime();
-      if (t0 == 0) t0 = t;
-      else if (t - t0 > kWaitNs) {
-        atomicCAS(err, 0, 52);
-        return 0;
-      }
-    }
-  }
+// Bounded wait until *ctr >= target (acquire); false (error 52 recorded) on timeout or once any
+// error is recorded.
+__device__ __noinline__ int count_wait(const unsigned* ctr, unsigned target, int* err, unsigned long long lim) {
+  return ptx::count_wait(ctr, target, err, 52, lim);
 }
 
 // Phase boundary inside a layer when the phases wait on counts: the CTA's consumers and issuer
 // meet (tensor memory and the work area are free again), the issuer waits until *ctr reaches
 // `target` (acquire: the outputs this phase reads), then they meet again, so that every thread's
 // loads come after the acquire. Returns false once any error is recorded.
-__device__ __noinline__ bool phase_wait(const unsigned* ctr, unsigned target, bool ok, int* err, const Smem& S) {
+__device__ __noinline__ bool phase_wait(const unsigned* ctr, unsigned target, bool ok, int* err, const Smem& S,
+                                        unsigned long long lim) {
   tc_fence_before();
   __syncwarp();
   named_sync(1, kSyncThreads);
   if (threadIdx.x == kMmaThread) {
     bool good = ok && *reinterpret_cast<volatile int*>(err) == 0;
-    if (good) good = count_wait(ctr, target, err) != 0;
+    if (good) good = count_wait(ctr, target, err, lim) != 0;
     // outputs written by other CTAs are read next by this thread's tensor-map loads
     asm volatile("fence.proxy.async.global;" ::: "memory");
     *S.flag = good ? 1 : 0;
@@ -737,6 +549,7 @@ __device__ __forceinline__ void combine_rows_warp(const StepArgs& __restrict__ p
   const float* __restrict__ part_ml = p.part_ml;
   __nv_bfloat16* __restrict__ o_out = p.o;
   int* err = p.err;
+  const unsigned long long wait_ns = p.wait_ns;
   constexpr int kRows = 2;                  // rows staged at once (two when n_chunks <= 16)
   const int batch = nck * kRows <= kStepMaxChunks ? kRows : 1;
 #pragma unroll 1
@@ -774,7 +587,7 @@ __device__ __forceinline__ void combine_rows_warp(const StepArgs& __restrict__ p
       wgt[k] = lane < nck && k < nr ? exp2f((mc[k] - M) * scale_log2) : 0.f;
       invL[k] = 1.f / warp_sum(wgt[k] * lc[k]);
     }
-    const bool ok = mbar_wait(bar, st.cpar, err, 53);
+    const bool ok = mbar_wait(bar, st.cpar, err, 53, wait_ns);
     st.cpar ^= 1u;
 #pragma unroll 1
     for (int k = 0; k < nr && ok; ++k) {
@@ -826,6 +639,10 @@ __device__ __noinline__ void combine_rows(const StepArgs& __restrict__ p, uint8_
   for (int idx = gw; idx < total; idx += nw) combine_rows_warp<DH>(p, idx / p.rows, idx % p.rows, idx % p.rows + 1, 1, buf, bar, st);
 }
 
+struct ConsSync {
+  __device__ void operator()() const { named_sync(2, kCons); }
+};
+
 }  // namespace
 
 // ---- projection step: acc[m][n] += sum over this CTA's weight tiles of A[m][k] W[n][k] -----
@@ -835,7 +652,9 @@ __device__ __noinline__ void combine_rows(const StepArgs& __restrict__ p, uint8_
 // block's epilogue for its share of the rows.
 template <int DH>
 __device__ __noinline__ void projection_step(const StepShared& __restrict__ sh, const CUtensorMap* amap, int l, int j,
-                                             uint32_t tmem, size_t xbytes, Role& st) {
+                                             uint32_t tmem, size_t xbytes, Role& st_) {
+  RoleCopy rc_(st_);
+  Role& st = rc_.v;
   const StepArgs& p = sh.p;
   const Smem S = smem_plan(p.ring, xbytes);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -853,10 +672,10 @@ __device__ __noinline__ void projection_step(const StepShared& __restrict__ sh, 
     // the next weight tile's barrier is tested (without blocking) before the current tile's MMAs
     // are issued, so that the test's latency overlaps the issue
     bool ready = mbar_peek(S.full + st.slot, st.par);
-    bool good = mbar_wait(S.a_full, st.apar, p.err, 42);
+    bool good = mbar_wait(S.a_full, st.apar, p.err, 42, p.wait_ns);
     for (int i = 0; i < nt && good; ++i) {
       if (!ready) {
-        good = mbar_wait(S.full + st.slot, st.par, p.err, 43);
+        good = mbar_wait(S.full + st.slot, st.par, p.err, 43, p.wait_ns);
         if (!good) break;
       }
       tc_fence_after();
@@ -873,7 +692,7 @@ __device__ __noinline__ void projection_step(const StepShared& __restrict__ sh, 
   }
   st.apar ^= 1u;
   if (cons) {
-    const bool good = mbar_wait(S.g_done, st.gpar, p.err, 44);
+    const bool good = mbar_wait(S.g_done, st.gpar, p.err, 44, p.wait_ns);
     tc_fence_after();
     const uint32_t tm = tmem_base_after_wait(S.tmem_slot);
     const int quad = warp & 3, row = quad * 32 + lane;
@@ -906,7 +725,7 @@ __device__ __noinline__ void projection_step(const StepShared& __restrict__ sh, 
       if (good) {
         unsigned* ctr = p.sync + (1 + kStepBarriersPerLayer * p.L) + (size_t)(4 * l + j) * kStepMaxNB + tl.b;
         asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ctr) : "memory");
-        go = count_wait(ctr, (unsigned)tl.contrib, p.err);
+        go = count_wait(ctr, (unsigned)tl.contrib, p.err, p.wait_ns);
       }
       *S.last = go;
     }
@@ -933,7 +752,9 @@ __device__ __noinline__ void projection_step(const StepShared& __restrict__ sh, 
 // ---- attention step: items (robot-group bg, 128-row query tile qt, 64-key chunk kc) ---------
 template <int DH>
 __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, const CUtensorMap* t_q, const CUtensorMap* t_k,
-                                            const CUtensorMap* t_vt, int l, uint32_t tmem, Role& st, bool fused) {
+                                            const CUtensorMap* t_vt, int l, uint32_t tmem, Role& st_, bool fused) {
+  RoleCopy rc_(st_);
+  Role& st = rc_.v;
   constexpr int NC = DH / 64;
   constexpr uint32_t QB = DH * kQT * 2, KB = DH * kKC * 2, VB = DH * kKC * 2;
   const Smem S = smem_plan(p.ring, step_x_bytes(DH));
@@ -953,7 +774,7 @@ __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, cons
       const int t = ci * QT / ncomb, first = (t * ncomb + QT - 1) / QT, next = ((t + 1) * ncomb + QT - 1) / QT;
       const int bg = t / nqt, qt = t % nqt, rows = min(kQT, p.rows - qt * kQT);
       const int r0 = qt * kQT + (ci - first) * rows / (next - first), r1 = qt * kQT + (ci - first + 1) * rows / (next - first);
-      if (threadIdx.x == 0) *S.last = count_wait(qtile_ctr(p, l, t), (unsigned)nck, p.err);
+      if (threadIdx.x == 0) *S.last = count_wait(qtile_ctr(p, l, t), (unsigned)nck, p.err, p.wait_ns);
       named_sync(2, kCons);
       if (*reinterpret_cast<volatile int*>(S.last)) {
         __nv_bfloat16* buf = reinterpret_cast<__nv_bfloat16*>(S.X) + (size_t)warp * kStepMaxChunks * DH;
@@ -979,7 +800,7 @@ __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, cons
       mbar_expect_tx(S.v_full, VB);
       tma_3d(sV, t_vt, kc * kKC, 0, kvz, S.v_full, pol);
       ++st.i_uses;
-      bool good = mbar_wait(S.q_full, st.ipar, p.err, 45);
+      bool good = mbar_wait(S.q_full, st.ipar, p.err, 45, p.wait_ns);
       if (good) {
         tc_fence_after();
         const uint32_t q0 = su32(sQ), k0 = su32(sK);
@@ -991,7 +812,7 @@ __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, cons
                      idesc_m128(kKC), (cc | k) ? 1u : 0u);
       }
       mma_commit(S.s_full);
-      good = good && mbar_wait(S.p_full, st.ipar, p.err, 46) && mbar_wait(S.v_full, st.ipar, p.err, 47);
+      good = good && mbar_wait(S.p_full, st.ipar, p.err, 46, p.wait_ns) && mbar_wait(S.v_full, st.ipar, p.err, 47, p.wait_ns);
       if (good) {
         tc_fence_after();
         const uint32_t p0 = su32(sP), v0 = su32(sV);
@@ -1009,7 +830,7 @@ __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, cons
       bool ok_s = true;
       float mx = -INFINITY, l_sum = 0.f;
       if (half == 0) {
-        ok_s = mbar_wait(S.s_full, st.ipar, p.err, 48);
+        ok_s = mbar_wait(S.s_full, st.ipar, p.err, 48, p.wait_ns);
         tc_fence_after();
         const uint32_t tS = tmem_base_after_wait(S.tmem_slot);
         const int key0 = kc * kKC;
@@ -1047,7 +868,7 @@ __device__ __noinline__ void attention_step(const StepArgs& __restrict__ p, cons
         __syncwarp();
         if (lane == 0) mbar_arrive(S.p_full);
       }
-      const bool ok_o = mbar_wait(S.o_done, st.ipar, p.err, 49);
+      const bool ok_o = mbar_wait(S.o_done, st.ipar, p.err, 49, p.wait_ns);
       tc_fence_after();
       const uint32_t tO = tmem_base_after_wait(S.tmem_slot) + 256;
       // unnormalised O row in bf16: staged in shared memory (the operand tiles are free once O
@@ -1197,7 +1018,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const Tiles tl = sh.tiles[j];
           const uint8_t* w = static_cast<const uint8_t*>(p.wl[4 * l + j]) + ((size_t)tl.b * (K / 64) + tl.k0) * kSlot;
           for (int t = 0; t < tl.k1 - tl.k0; ++t) {
-            if (!mbar_wait(S.empty + slot, par ^ 1u, p.err, 41)) { ok = false; break; }
+            if (!mbar_wait(S.empty + slot, par ^ 1u, p.err, 41, p.wait_ns)) { ok = false; break; }
             mbar_expect_tx(S.full + slot, kSlot);
             bulk_g2s(S.ring + (size_t)slot * kSlot, w + (size_t)t * kSlot, kSlot, S.full + slot, pol);
             ++issued;
@@ -1205,7 +1026,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       // copies still in flight land before the CTA exits
-      for (int i = issued - R > 0 ? issued - R : 0; i < issued; ++i) mbar_drain(S.full + i % R, (uint32_t)(i / R) & 1u);
+      for (int i = issued - R > 0 ? issued - R : 0; i < issued; ++i) mbar_drain(S.full + i % R, (uint32_t)(i / R) & 1u, kDrainNs);
     }
     __syncwarp();
   } else {
@@ -1215,41 +1036,58 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool ok = true;
     unsigned* bar = p.sync;
     if (cons) in_rows(sh, S.red);
-    ok = grid_sync(bar++, ok, p.err, S);
+    ok = grid_sync(bar++, ok, p.err, S, p.wait_ns, p.unreachable);
     for (int l = 0; l < p.L; ++l) {
       const bool df = sh.fused_combine != 0;   // phases inside the layer wait on counts
       if (ok) projection_step<DH>(sh, &t_z, l, 0, tmem, XB, st);
-      ok = df ? phase_wait(done_ctr(p, l, 0), sh.shares[0], ok, p.err, S) : grid_sync(bar++, ok, p.err, S);
+      ok = df ? phase_wait(done_ctr(p, l, 0), sh.shares[0], ok, p.err, S, p.wait_ns) : grid_sync(bar++, ok, p.err, S, p.wait_ns);
       if (ok) attention_step<DH>(p, &t_q, &t_k, &t_vt, l, tmem, st, df);
       if (df) {
-        ok = phase_wait(done_ctr(p, l, 3), sh.shares[3], ok, p.err, S);
+        ok = phase_wait(done_ctr(p, l, 3), sh.shares[3], ok, p.err, S, p.wait_ns);
       } else {
-        ok = grid_sync(bar++, ok, p.err, S);
+        ok = grid_sync(bar++, ok, p.err, S, p.wait_ns);
         if (ok && cons) combine_rows<DH>(p, S.X, S.cbar + warp, st);
-        ok = grid_sync(bar++, ok, p.err, S);
+        ok = grid_sync(bar++, ok, p.err, S, p.wait_ns);
       }
       if (ok) projection_step<DH>(sh, &t_o, l, 1, tmem, XB, st);
-      ok = df ? phase_wait(done_ctr(p, l, 1), sh.shares[1], ok, p.err, S) : grid_sync(bar++, ok, p.err, S);
+      ok = df ? phase_wait(done_ctr(p, l, 1), sh.shares[1], ok, p.err, S, p.wait_ns) : grid_sync(bar++, ok, p.err, S, p.wait_ns);
       if (ok) projection_step<DH>(sh, &t_z, l, 2, tmem, XB, st);
-      ok = df ? phase_wait(done_ctr(p, l, 2), sh.shares[2], ok, p.err, S) : grid_sync(bar++, ok, p.err, S);
+      ok = df ? phase_wait(done_ctr(p, l, 2), sh.shares[2], ok, p.err, S, p.wait_ns) : grid_sync(bar++, ok, p.err, S, p.wait_ns);
       // the shift rows of this layer's qkv and gate/up sums have been read by now
       if (ok && cons) clear_shift_rows(sh, true, true);
       if (ok) projection_step<DH>(sh, &t_act, l, 3, tmem, XB, st);
-      ok = grid_sync(bar++, ok, p.err, S);
+      ok = grid_sync(bar++, ok, p.err, S, p.wait_ns);
     }
-    if (ok && cons && (int)blockIdx.x < p.M) final_row(p, blockIdx.x, reinterpret_cast<float*>(S.X));
+    if (cons) {
+      if (ok && (int)blockIdx.x < p.M) final_row(p, blockIdx.x, reinterpret_cast<float*>(S.X));
+      // the step epilogue (Sec. 4.2-4.4) runs on the last CTA to finish: the count's acquire makes
+      // every CTA's velocity rows visible to it
+      named_sync(2, kCons);
+      if (threadIdx.x == 0) {
+        unsigned prev;
+        asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;"
+                     : "=r"(prev) : "l"(p.sync + step_sync_words(p.L) - 1) : "memory");
+        *S.last = ok && prev == gridDim.x - 1u && *reinterpret_cast<volatile int*>(p.err) == 0;
+      }
+      named_sync(2, kCons);
+      if (*reinterpret_cast<volatile int*>(S.last)) {
+        float* base = reinterpret_cast<float*>(S.X);
+        const EulerSmem es{base + 96, base, base + 64, reinterpret_cast<int*>(S.tmem_slot + 3)};
+        for (int b = 0; b < p.eu.B; ++b) euler_robot(p.eu, b, threadIdx.x, kCons, es, ConsSync());
+      }
+    }
     // a consumer warp exits only after its last combine copies have landed
-    if (cons && st.c_uses) mbar_drain(S.cbar + warp, (uint32_t)(st.c_uses - 1) & 1u);
+    if (cons && st.c_uses) mbar_drain(S.cbar + warp, (uint32_t)(st.c_uses - 1) & 1u, kDrainNs);
     if (mma) {
       // tensor memory is freed only after every MMA of this thread has completed, and the CTA
       // exits only after its last operand loads have landed (they are waited for on the normal
       // path; this matters only after an error)
       mma_commit(S.fin);
-      mbar_drain(S.fin, 0);
-      if (st.a_uses) mbar_drain(S.a_full, (uint32_t)(st.a_uses - 1) & 1u);
+      mbar_drain(S.fin, 0, kDrainNs);
+      if (st.a_uses) mbar_drain(S.a_full, (uint32_t)(st.a_uses - 1) & 1u, kDrainNs);
       if (st.i_uses) {
-        mbar_drain(S.q_full, (uint32_t)(st.i_uses - 1) & 1u);
-        mbar_drain(S.v_full, (uint32_t)(st.i_uses - 1) & 1u);
+        mbar_drain(S.q_full, (uint32_t)(st.i_uses - 1) & 1u, kDrainNs);
+        mbar_drain(S.v_full, (uint32_t)(st.i_uses - 1) & 1u, kDrainNs);
       }
     }
     __syncwarp();

@@ -76,6 +76,8 @@ struct uad_ctx {
   // persistent evaluation kernel (adaRMS, bf16, B * H <= 64): one launch per step
   bool step_ok = false;
   bool step_off = false;          // UAD_STEP=0: per-operation kernels only
+  unsigned long long wait_ns = 2000000000ull;   // bound on any wait inside the persistent kernel
+  int test_unreachable = 0;       // testing aid: extra arrivals the first phase count waits for
   int step_bmax = 0;              // robots per launch
   StepArgs st0;                   // shapes and buffers; M, B, tau_row set per launch
   StepMaps smaps;
@@ -585,9 +587,27 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, bool step, cudaStream_t s) {
   PendingResid pend;
   for (int k = 1; k <= n_steps; ++k) {
     const int* tr = tau + (size_t)(k - 1) * M;
+    // step epilogue (Euler, TR, release, GAC): its own kernel, or the persistent kernel's end
+    EulerArgs ea;
+    ea.B = B; ea.H = H; ea.D = D; ea.k = k;
+    ea.plan = plan + (size_t)(k - 1) * M;
+    ea.gstep = reinterpret_cast<const float*>(c->plan_dev + PL.gstep);
+    ea.last_step = reinterpret_cast<const int*>(c->plan_dev + PL.last);
+    ea.tail_count = reinterpret_cast<const int*>(c->plan_dev + PL.tailc);
+    ea.tail_flag = reinterpret_cast<const int*>(c->plan_dev + PL.tailf);
+    ea.gac_mask = c->plan_dev + PL.mask;
+    ea.epoch = reinterpret_cast<const int*>(c->plan_dev + PL.epoch);
+    ea.rot_dim = reinterpret_cast<const int*>(c->plan_dev + PL.rot);
+    ea.v = c->v; ea.x = c->x; ea.g = c->g; ea.u = c->u; ea.rel = c->rel;
+    ea.final_out = c->fin; ea.ghost_out = c->ghost; ea.E_out = c->E;
+    ea.host_rel = c->host_rel_dev; ea.host_flags = c->host_flags_dev;
+    ea.nonfinite = c->nonfinite; ea.evals = c->evals; ea.stamps = c->stamps;
     if (step) {
       StepArgs p = c->st0;
       p.M = M; p.B = B; p.tau_row = tr;
+      p.eu = ea;
+      p.wait_ns = c->wait_ns;
+      p.unreachable = (unsigned)c->test_unreachable;
       p.sidx = reinterpret_cast<const int*>(c->plan_dev + PL.sidx) + (size_t)(k - 1) * M;
       p.sinfo = reinterpret_cast<const int*>(c->plan_dev + PL.sinfo) + (size_t)(k - 1) * (1 + kStepMaxShift);
       cudaMemsetAsync(p.sync, 0, step_sync_words(a.n_layers) * 4, s);
@@ -719,27 +739,13 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, bool step, cudaStream_t s) {
       go.M = M; go.N = D; go.K = W; go.out = c->v; go.ldo = D; go.bias = c->b_out;
       { Mark mk(c, s, "out_proj", gemm_bytes(go, c->es), 2.0 * M * W * D); gemm(c, c->w_out, go, s); }
     }
-    EulerArgs ea;
-    ea.B = B; ea.H = H; ea.D = D; ea.k = k;
-    ea.plan = plan + (size_t)(k - 1) * M;
-    ea.gstep = reinterpret_cast<const float*>(c->plan_dev + PL.gstep);
-    ea.last_step = reinterpret_cast<const int*>(c->plan_dev + PL.last);
-    ea.tail_count = reinterpret_cast<const int*>(c->plan_dev + PL.tailc);
-    ea.tail_flag = reinterpret_cast<const int*>(c->plan_dev + PL.tailf);
-    ea.gac_mask = c->plan_dev + PL.mask;
-    ea.epoch = reinterpret_cast<const int*>(c->plan_dev + PL.epoch);
-    ea.rot_dim = reinterpret_cast<const int*>(c->plan_dev + PL.rot);
-    ea.v = c->v; ea.x = c->x; ea.g = c->g; ea.u = c->u; ea.rel = c->rel;
-    ea.final_out = c->fin; ea.ghost_out = c->ghost; ea.E_out = c->E;
-    ea.host_rel = c->host_rel_dev; ea.host_flags = c->host_flags_dev;
-    ea.nonfinite = c->nonfinite; ea.evals = c->evals; ea.stamps = c->stamps;
-    { Mark mk(c, s, "euler_tr_gac", 40.0 * M * D, 0); launch_euler(ea, s); }
+    if (!step) { Mark mk(c, s, "euler_tr_gac", 40.0 * M * D, 0); launch_euler(ea, s); }
   }
 }
 
 int launches_per_step(const uad_ctx* c, int B) {
   const uad_arch& a = c->a;
-  if (step_path(c, B)) return 2;   // persistent evaluation kernel + Euler step
+  if (step_path(c, B)) return 1;   // persistent evaluation kernel with the step epilogue at its end
   return a.kind == UAD_KIND_DIT ? 11 * a.n_layers + 4
                                  : (c->attn_tc ? 8 : 7) * a.n_layers + 4 + (a.kind == UAD_KIND_CONCAT ? 4 : 0);
 }
@@ -1411,6 +1417,17 @@ int uad_step_times(const uad_ctx* c, double* ms, int32_t max_entries) {
 int uad_launches_per_chunk(const uad_ctx* c, int32_t batch, int32_t n_star) {
   if (!c || batch < 1 || n_star < 1) return UAD_EINVAL;
   return 1 + n_star * launches_per_step(c, batch);
+}
+
+int uad_set_wait_limit(uad_ctx* c, int64_t wait_ns, int32_t unreachable) {
+  if (!c || wait_ns <= 0 || unreachable < 0) return UAD_EINVAL;
+  if (c->in_flight) return fail(c, UAD_ESTATE, "chunk in flight");
+  c->wait_ns = (unsigned long long)wait_ns;
+  c->test_unreachable = unreachable;
+  // the launch arguments are baked into the cached graphs
+  for (auto& kv : c->graphs) cudaGraphExecDestroy(kv.second);
+  c->graphs.clear();
+  return UAD_OK;
 }
 
 void uad_destroy(uad_ctx* c) {

@@ -214,10 +214,10 @@ constexpr int kStepMaxWidth = 2048;   // model width, a multiple of 512
 // Per-launch synchronisation block (zeroed before every launch): grid-barrier counters,
 // per-output-block arrival counters, row sums of squares of the residual stream, per-query-tile
 // counts of finished attention chunks, per-layer counts of finished epilogue shares (qkv, o,
-// gate/up) and chunk merges.
+// gate/up) and chunk merges, and the count of CTAs that finished the final phase.
 __host__ __device__ constexpr size_t step_sync_words(int L) {
   return (size_t)(1 + kStepBarriersPerLayer * L) + (size_t)L * 4 * kStepMaxNB + (size_t)(L + 1) * 2 * kStepMaxRows +
-         (size_t)L * kStepMaxQTiles + (size_t)L * 4;
+         (size_t)L * kStepMaxQTiles + (size_t)L * 4 + 1;
 }
 struct StepArgs {
   int M = 0, B = 0, H = 0, W = 0, F = 0, D = 0, L = 0;
@@ -246,6 +246,9 @@ struct StepArgs {
   const float* rope_cs = nullptr;      // [H][dh/2][cos, sin]
   unsigned* sync = nullptr;            // step_sync_words(L) words, zeroed per launch
   int* err = nullptr;
+  unsigned long long wait_ns = 2000000000ull;   // bound on any single wait
+  unsigned unreachable = 0;            // testing aid: arrivals the first grid barrier waits for in excess
+  EulerArgs eu;                        // the step epilogue, run by the last CTA to finish
 };
 struct StepMaps { CUtensorMap z, o, act, q, k, vt; };   // k: 64-key boxes
 size_t step_smem_bytes(int dh, int ring);

@@ -133,3 +133,30 @@ def test_oracle_thread_count_is_what_the_process_may_use():
     import bench
     n = bench.oracle_threads()
     assert 1 <= n <= (os.cpu_count() or n)
+
+
+def test_gpus_flag_starts_the_ranks_itself():
+    """`bench.py --gpus 2` without an outside launcher re-runs itself as two ranks under
+    torch.distributed.run (gloo here, no GPU); rank 0 alone prints the reference arm's line."""
+    import subprocess
+    env = dict(os.environ, UAD_BENCH_BACKEND="gloo")
+    for k in ("WORLD_SIZE", "RANK", "LOCAL_RANK", "MASTER_ADDR", "MASTER_PORT"):
+        env.pop(k, None)
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--gpus", "2",
+                        "--workload", "tiny", "--steps", "1", "--warmup", "0"],
+                       capture_output=True, text=True, timeout=600, env=env, cwd=ROOT)
+    assert r.returncode == 0, r.stderr[-2000:]
+    import json
+    lines = [json.loads(x) for x in r.stdout.splitlines() if x.startswith("{")]
+    assert len(lines) == 1 and lines[0]["impl"] == "reference", r.stdout
+    assert lines[0]["n_gpus"] == 2
+
+
+def test_rank_count_must_match_gpus_flag():
+    import subprocess
+    env = dict(os.environ, WORLD_SIZE="3", RANK="0", LOCAL_RANK="0")
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--gpus", "2",
+                        "--workload", "tiny", "--steps", "1", "--warmup", "0"],
+                       capture_output=True, text=True, timeout=120, env=env, cwd=ROOT)
+    assert r.returncode == 2 and "refusing" in r.stderr
+    assert not [x for x in r.stdout.splitlines() if x.startswith("{")]
