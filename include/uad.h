@@ -152,7 +152,8 @@ int uad_denoise(uad_ctx* ctx, const float* noise, const uad_schedule* sched, int
  * ready [H] (host, may be NULL): 1 if available; release_step [H] (may be NULL): the step
  * after which the action became available (N_i for early actions, N* for the tail, whose
  * rows already include GAC). Released actions never change afterwards (Sec. 4.4).
- * Returns the number of ready actions (>= min_ready), UAD_ETIMEDOUT, or an error. */
+ * Returns the number of ready actions (>= min_ready), UAD_ETIMEDOUT, or an error (UAD_EINVAL
+ * for min_ready > H). */
 int uad_poll_released(uad_ctx* ctx, int32_t robot, int32_t min_ready, int64_t timeout_us,
                       float* out, int32_t* ready, int32_t* release_step);
 

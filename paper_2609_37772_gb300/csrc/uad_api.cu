@@ -1339,6 +1339,7 @@ int uad_poll_released(uad_ctx* c, int32_t robot, int32_t min_ready, int64_t time
   if (c->cur_B == 0) return fail(c, UAD_ESTATE, "no chunk started");
   if (robot < 0 || robot >= c->cur_B) return fail(c, UAD_EINVAL, "robot %d not in this chunk", robot);
   const int H = c->a.chunk_len, D = c->a.action_dim;
+  if (min_ready > H) return fail(c, UAD_EINVAL, "min_ready %d exceeds the chunk's %d actions", min_ready, H);
   const int ns = c->cur_nstar[robot];
   const int* bud = &c->cur_budgets[(size_t)robot * H];
   const int* flags = c->host_flags + (size_t)robot * kFlagStride;
@@ -1360,6 +1361,7 @@ int uad_poll_released(uad_ctx* c, int32_t robot, int32_t min_ready, int64_t time
     if (count >= min_ready || count == H) break;
     const auto el = std::chrono::duration_cast<std::chrono::microseconds>(std::chrono::steady_clock::now() - t0).count();
     if (el >= timeout_us) break;
+    std::this_thread::yield();
   }
   if (ready)
     for (int i = 0; i < H; ++i) if (!done[i]) ready[i] = 0;

@@ -72,12 +72,23 @@ class Case:
 
 
 def check(case, res, refs, budgets, tol):
+    """Final and ghost actions within `tol` of the action scale (reading C13). E of Eq. 8 sums
+    (ghost - released) over the U early actions, so its error is bounded by the sum of those
+    actions' errors: |dE| <= U * tol * (max|ghost| + max|final|) of the oracle. Prints the errors
+    reached (shown with pytest -s)."""
     budgets = np.asarray(budgets).reshape(case.B, -1)
+    worst = {"final": 0.0, "ghost": 0.0, "E/bound": 0.0}
     for b, ref in enumerate(refs):
-        assert rel_err(res["final"][b], ref["final"]) <= tol, ("final", b, rel_err(res["final"][b], ref["final"]))
-        assert rel_err(res["ghost"][b], ref["ghost"]) <= tol, ("ghost", b, rel_err(res["ghost"][b], ref["ghost"]))
+        ef, eg = rel_err(res["final"][b], ref["final"]), rel_err(res["ghost"][b], ref["ghost"])
+        worst["final"], worst["ghost"] = max(worst["final"], ef), max(worst["ghost"], eg)
+        assert ef <= tol, ("final", b, ef)
+        assert eg <= tol, ("ghost", b, eg)
         if np.abs(ref["E"]).max() > 0:
-            assert np.abs(res["E"][b] - ref["E"]).max() <= tol * max(1e-6, np.abs(ref["final"]).max()) * 4
+            U = int((budgets[b] < budgets[b].max()).sum())
+            bound = U * tol * (np.abs(ref["ghost"]).max() + np.abs(ref["final"]).max())
+            dE = float(np.abs(res["E"][b] - ref["E"]).max())
+            worst["E/bound"] = max(worst["E/bound"], dE / bound)
+            assert dE <= bound, ("E", b, dE, bound)
         else:
             assert np.all(res["E"][b] == 0)
         if res["polled"]:
@@ -86,6 +97,8 @@ def check(case, res, refs, budgets, tol):
             # what the controller received is exactly what finish reports
             assert np.array_equal(out, res["final"][b])
     assert res["evals"] == max(r["evals"] for r in refs) and res["tr_extra_evals"] == 0
+    print(f"[{case.a.name} B={case.B}] max rel err final {worst['final']:.2e} ghost {worst['ghost']:.2e} "
+          f"(tolerance {tol:g}); E error / bound {worst['E/bound']:.2e}")
 
 
 # ---------------------------------------------------------------------------------------------
@@ -441,11 +454,14 @@ def test_pi0_full_batched_16_robots_sampled():
         bud = draw_sweep_schedules(a.chunk_len, B, seed=3)
         ex.denoise(noise, bud)
         res = ex.finish(timeout_us=TIMEOUT)
+        worst = 0.0
         for b in (0, 7, 15):
             ref = denoise(build_model(a, blob, pre[b]).velocity, noise[b], bud[b])
-            assert rel_err(res["final"][b], ref["final"]) <= TOL["bf16"]
-            assert rel_err(res["ghost"][b], ref["ghost"]) <= TOL["bf16"]
+            ef, eg = rel_err(res["final"][b], ref["final"]), rel_err(res["ghost"][b], ref["ghost"])
+            worst = max(worst, ef, eg)
+            assert ef <= TOL["bf16"] and eg <= TOL["bf16"], (b, ef, eg)
         assert res["evals"] == 10
+        print(f"[pi0 B={B}, robots (0, 7, 15)] max rel err {worst:.2e} (tolerance {TOL['bf16']:g})")
     finally:
         ex.close()
 
@@ -466,11 +482,14 @@ def test_pi0_full_batched_64_robots_sampled():
         bud = draw_sweep_schedules(a.chunk_len, B, seed=5)
         ex.denoise(noise, bud)
         res = ex.finish(timeout_us=TIMEOUT)
+        worst = 0.0
         for b in (0, 31, 63):
             ref = denoise(build_model(a, blob, pre[b]).velocity, noise[b], bud[b])
-            assert rel_err(res["final"][b], ref["final"]) <= TOL["bf16"]
-            assert rel_err(res["ghost"][b], ref["ghost"]) <= TOL["bf16"]
+            ef, eg = rel_err(res["final"][b], ref["final"]), rel_err(res["ghost"][b], ref["ghost"])
+            worst = max(worst, ef, eg)
+            assert ef <= TOL["bf16"] and eg <= TOL["bf16"], (b, ef, eg)
         assert res["evals"] == 10
+        print(f"[pi0 B={B}, robots (0, 31, 63)] max rel err {worst:.2e} (tolerance {TOL['bf16']:g})")
     finally:
         ex.close()
 
