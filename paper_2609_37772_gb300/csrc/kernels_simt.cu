@@ -565,16 +565,18 @@ __global__ void __launch_bounds__(128) attn_kernel(AttnArgs p) {
 }
 
 // ------------------------------------------------------------------------------------------
-// Attention for few queries over few keys (bf16 operands, head dim 64, at most kFewKeys keys):
-// CTA = (16 queries, one query head, one robot), 256 threads. Every key and value of the head is
-// loaded into shared memory at once (16-byte loads), the whole score block S = Q K^T is formed
-// (thread = key), each query row takes an exact softmax (warp = two rows), and O = P V is one
-// pass (thread = (query, 4 dims)). Used for the DiT head's chunk self-attention and its
-// cross-attention to the observation prefix, where a key-by-key online softmax is bound by
-// the latency of its serial key blocks.
-// ------------------------------------------------------------------------------------------
-constexpr int kFewKeys = 512, kFewDh = 64, kFewQ = 16;
+// Attention for few queries (bf16 operands, head dim 64), split over 64-key chunks (split-KV):
+// CTA (query block of 16, key chunk, head, robot) computes the chunk's scores with 256 threads over
+// (query, 4 keys) pairs, its softmax partials (max, sum) and P V with threads over (query, 4 dims).
+// With one chunk the rows are written at once; otherwise each CTA leaves its partial rows in the
+// workspace and the last CTA of the (robot, head, query block) merges them by log-sum-exp and
+// resets the arrival count for the next launch. Used by the DiT head: self-attention over the
+// chunk's tokens and cross-attention over the projected prefix.
+constexpr int kFewDh = 64, kFewQ = 16, kFewKC = 64;
+constexpr int kFewPart = kFewDh + 4;     // partial row: O, max, sum, padding (16-byte rows)
 constexpr int kFewKPitch = kFewDh + 2;   // bf16 per key row: rows 33 words apart, no bank conflicts
+
+__host__ __device__ inline int few_chunks(int n_keys) { return (n_keys + kFewKC - 1) / kFewKC; }
 
 __device__ __forceinline__ uint32_t pack_bf16_pair(float a, float b) {
   __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
@@ -582,22 +584,24 @@ __device__ __forceinline__ uint32_t pack_bf16_pair(float a, float b) {
 }
 
 __global__ void __launch_bounds__(256) attn_few_kernel(AttnArgs p) {
-  extern __shared__ float sm[];
+  __shared__ float qs[kFewQ][kFewDh];
+  __shared__ float ps[kFewQ][kFewKC];
+  __shared__ __align__(16) __nv_bfloat16 ks[kFewKC * kFewKPitch];
+  __shared__ __align__(16) __nv_bfloat16 vs[kFewKC * kFewDh];
+  __shared__ float ml[kFewQ][2];
+  __shared__ int last;
   pdl_trigger();
   pdl_wait();
   constexpr int dh = kFewDh, half = dh / 2;
   const int n_keys = p.P + (p.kc ? p.H : 0);
-  float* qs = sm;                                       // [16][dh]
-  float* ss = qs + kFewQ * dh;                          // [16][n_keys] scores, then probabilities
-  __nv_bfloat16* ks = reinterpret_cast<__nv_bfloat16*>(ss + kFewQ * kFewKeys);   // [n_keys][kFewKPitch]
-  __nv_bfloat16* vs = ks + (size_t)kFewKeys * kFewKPitch;                          // [n_keys][dh]
-  const int b = blockIdx.z, hq = blockIdx.y, i0 = blockIdx.x * kFewQ;
+  const int C = few_chunks(n_keys), qb = blockIdx.x / C, kc = blockIdx.x % C, key0 = kc * kFewKC;
+  const int nk = min(kFewKC, n_keys - key0);
+  const int b = blockIdx.z, hq = blockIdx.y, i0 = qb * kFewQ;
   const int g = hq / (p.n_heads / p.n_kv_heads);
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  // keys and values: 8 bf16 per 16-byte load, every load issued before any use
-#pragma unroll 4
-  for (int e = tid; e < n_keys * (dh / 8); e += 256) {
-    const int j = e / (dh / 8), c8 = e % (dh / 8);
+  const int tid = threadIdx.x;
+  // the chunk's keys and values: 16-byte loads, all issued before any use
+  for (int e = tid; e < nk * (dh / 8); e += 256) {
+    const int j = key0 + e / (dh / 8), c8 = e % (dh / 8);
     uint4 kv, vv;
     if (j < p.P) {
       const long long off = b * p.kp_bstride + (long long)j * p.kp_ld + g * dh + c8 * 8;
@@ -608,12 +612,12 @@ __global__ void __launch_bounds__(256) attn_few_kernel(AttnArgs p) {
       kv = *reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(p.kc) + off);
       vv = *reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(p.vc) + off);
     }
-    uint32_t* kd = reinterpret_cast<uint32_t*>(ks + (size_t)j * kFewKPitch + c8 * 8);
+    uint32_t* kd = reinterpret_cast<uint32_t*>(ks + (size_t)(j - key0) * kFewKPitch + c8 * 8);
     kd[0] = kv.x;
     kd[1] = kv.y;
     kd[2] = kv.z;
     kd[3] = kv.w;
-    *reinterpret_cast<uint4*>(vs + (size_t)j * dh + c8 * 8) = vv;
+    *reinterpret_cast<uint4*>(vs + (size_t)(j - key0) * dh + c8 * 8) = vv;
   }
   for (int e = tid; e < kFewQ * dh; e += 256) {
     const int qi = e / dh, d = e % dh, i = i0 + qi;
@@ -623,98 +627,137 @@ __global__ void __launch_bounds__(256) attn_few_kernel(AttnArgs p) {
       val = p.rope_cs ? rope_elem(p.q, off, d, half, p.rope_cs + (long long)i * dh, BF16)
                       : ldf_rt(p.q, off + d, BF16);
     }
-    qs[qi * dh + d] = val * p.scale;
+    qs[qi][d] = val * p.scale;
   }
   __syncthreads();
   // chunk keys carry RoPE like the queries (prefix keys come rotated)
   if (p.rope_cs && p.kc) {
-    for (int e = tid; e < p.H * half; e += 256) {
-      const int jj = e / half, d = e % half;
-      __nv_bfloat16* kr = ks + (size_t)(p.P + jj) * kFewKPitch;
-      const float* cs = p.rope_cs + (long long)jj * dh;
+    for (int e = tid; e < nk * half; e += 256) {
+      const int jj = e / half, d = e % half, j = key0 + jj;
+      if (j < p.P) continue;
+      __nv_bfloat16* kr = ks + (size_t)jj * kFewKPitch;
+      const float* cs = p.rope_cs + (long long)(j - p.P) * dh;
       const float x0 = __bfloat162float(kr[d]), x1 = __bfloat162float(kr[d + half]);
       kr[d] = __float2bfloat16_rn(x0 * cs[2 * d] - x1 * cs[2 * d + 1]);
       kr[d + half] = __float2bfloat16_rn(x1 * cs[2 * d] + x0 * cs[2 * d + 1]);
     }
     __syncthreads();
   }
-  // scores: thread = key, all 16 queries
-  for (int j = tid; j < n_keys; j += 256) {
-    float kf[dh];
-    const __nv_bfloat162* kr = reinterpret_cast<const __nv_bfloat162*>(ks + (size_t)j * kFewKPitch);
+  // scores: thread (query q, keys 4 kg .. 4 kg + 3); a 16-lane group shares q
+  const int q = tid >> 4, kg = tid & 15;
+  float sc[4];
 #pragma unroll
-    for (int d2 = 0; d2 < dh / 2; ++d2) {
-      const float2 f = __bfloat1622float2(kr[d2]);
-      kf[2 * d2] = f.x;
-      kf[2 * d2 + 1] = f.y;
-    }
+  for (int e = 0; e < 4; ++e) sc[e] = 0.f;
 #pragma unroll 4
-    for (int q = 0; q < kFewQ; ++q) {
-      const float4* q4 = reinterpret_cast<const float4*>(qs + q * dh);
-      float a0 = 0.f, a1 = 0.f;
+  for (int d2 = 0; d2 < dh / 2; ++d2) {
+    const float q0 = qs[q][2 * d2], q1 = qs[q][2 * d2 + 1];
 #pragma unroll
-      for (int d4 = 0; d4 < dh / 4; d4 += 2) {
-        const float4 x = q4[d4], y = q4[d4 + 1];
-        a0 = fmaf(x.x, kf[4 * d4], fmaf(x.y, kf[4 * d4 + 1], fmaf(x.z, kf[4 * d4 + 2], fmaf(x.w, kf[4 * d4 + 3], a0))));
-        a1 = fmaf(y.x, kf[4 * d4 + 4], fmaf(y.y, kf[4 * d4 + 5], fmaf(y.z, kf[4 * d4 + 6], fmaf(y.w, kf[4 * d4 + 7], a1))));
-      }
-      ss[q * kFewKeys + j] = a0 + a1;
+    for (int e = 0; e < 4; ++e) {
+      const float2 kf = __bfloat1622float2(reinterpret_cast<const __nv_bfloat162*>(ks + (size_t)(4 * kg + e) * kFewKPitch)[d2]);
+      sc[e] = fmaf(q0, kf.x, fmaf(q1, kf.y, sc[e]));
     }
   }
-  __syncthreads();
-  // softmax per query row (warp w: rows 2w, 2w + 1); 1 / sum kept in qs[q * dh]
-  for (int q = 2 * warp; q < 2 * warp + 2; ++q) {
-    float* row = ss + q * kFewKeys;
-    float mx = -INFINITY;
-    for (int j = lane; j < n_keys; j += 32) mx = fmaxf(mx, row[j]);
-    mx = warp_max(mx);
-    float sum = 0.f;
-    for (int j = lane; j < n_keys; j += 32) {
-      const float e = expf(row[j] - mx);
-      row[j] = e;
-      sum += e;
-    }
-    sum = warp_sum(sum);
-    __syncwarp();
-    if (lane == 0) qs[q * dh] = 1.f / sum;
+  float mx = -INFINITY;
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    if (4 * kg + e >= nk) sc[e] = -INFINITY;   // keys past the end
+    mx = fmaxf(mx, sc[e]);
+  }
+#pragma unroll
+  for (int o = 8; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  float sum = 0.f;
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float pe = expf(sc[e] - mx);
+    ps[q][4 * kg + e] = pe;
+    sum += pe;
+  }
+#pragma unroll
+  for (int o = 8; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+  if (kg == 0) {
+    ml[q][0] = mx;
+    ml[q][1] = sum;
   }
   __syncthreads();
-  // O = P V: thread = (query q, dims 4 c .. 4 c + 3)
-  {
-    const int q = tid / (dh / 4), c = tid % (dh / 4);
-    const float* row = ss + q * kFewKeys;
-    float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+  // O = P V: thread (query q, dims 4 c .. 4 c + 3)
+  const int c = tid & 15;
+  float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll 4
-    for (int j = 0; j < n_keys; ++j) {
-      const float pj = row[j];
-      const __nv_bfloat162* v2 = reinterpret_cast<const __nv_bfloat162*>(vs + (size_t)j * dh + 4 * c);
-      const float2 v0 = __bfloat1622float2(v2[0]), v1 = __bfloat1622float2(v2[1]);
-      o.x = fmaf(pj, v0.x, o.x);
-      o.y = fmaf(pj, v0.y, o.y);
-      o.z = fmaf(pj, v1.x, o.z);
-      o.w = fmaf(pj, v1.y, o.w);
-    }
-    const int i = i0 + q;
+  for (int j = 0; j < nk; ++j) {
+    const float pj = ps[q][j];
+    const __nv_bfloat162* v2 = reinterpret_cast<const __nv_bfloat162*>(vs + (size_t)j * dh + 4 * c);
+    const float2 v0 = __bfloat1622float2(v2[0]), v1 = __bfloat1622float2(v2[1]);
+    o.x = fmaf(pj, v0.x, o.x);
+    o.y = fmaf(pj, v0.y, o.y);
+    o.z = fmaf(pj, v1.x, o.z);
+    o.w = fmaf(pj, v1.y, o.w);
+  }
+  const int i = i0 + q;
+  __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(p.out) + (long long)(b * p.H + i) * p.out_ld + hq * dh + 4 * c;
+  if (C == 1) {
     if (i < p.H) {
-      const float inv = qs[q * dh];
-      __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(p.out) + (long long)(b * p.H + i) * p.out_ld + hq * dh + 4 * c;
+      const float inv = 1.f / ml[q][1];
       uint2 pk;
       pk.x = pack_bf16_pair(o.x * inv, o.y * inv);
       pk.y = pack_bf16_pair(o.z * inv, o.w * inv);
       *reinterpret_cast<uint2*>(dst) = pk;
     }
+    return;
+  }
+  // partial rows of this chunk: [group][chunk][q][kFewPart] (O, then max and sum)
+  const int QB = gridDim.x / C;
+  const size_t grp = ((size_t)b * p.n_heads + hq) * QB + qb;
+  float* part = p.split_ws + ((grp * C + kc) * kFewQ + q) * kFewPart;
+  *reinterpret_cast<float4*>(part + 4 * c) = o;
+  if (c == 0) {
+    part[dh] = ml[q][0];
+    part[dh + 1] = ml[q][1];
+  }
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) {
+    const unsigned prev = atomicAdd(p.split_ctr + grp, 1u);
+    last = prev == (unsigned)C - 1u;
+    if (last) p.split_ctr[grp] = 0u;   // every chunk has arrived: reset for the next launch
+  }
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  // merge the chunks by log-sum-exp
+  const float* base = p.split_ws + (grp * C * kFewQ + q) * kFewPart;
+  float M = -INFINITY;
+  for (int k = 0; k < C; ++k) M = fmaxf(M, __ldcg(base + (size_t)k * kFewQ * kFewPart + dh));
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  float L = 0.f;
+  for (int k = 0; k < C; ++k) {
+    const float* r = base + (size_t)k * kFewQ * kFewPart;
+    const float w = expf(__ldcg(r + dh) - M);
+    L = fmaf(w, __ldcg(r + dh + 1), L);
+    const float4 v = __ldcg(reinterpret_cast<const float4*>(r + 4 * c));
+    acc.x = fmaf(w, v.x, acc.x);
+    acc.y = fmaf(w, v.y, acc.y);
+    acc.z = fmaf(w, v.z, acc.z);
+    acc.w = fmaf(w, v.w, acc.w);
+  }
+  if (i < p.H) {
+    const float inv = 1.f / L;
+    uint2 pk;
+    pk.x = pack_bf16_pair(acc.x * inv, acc.y * inv);
+    pk.y = pack_bf16_pair(acc.z * inv, acc.w * inv);
+    *reinterpret_cast<uint2*>(dst) = pk;
   }
 }
 
-size_t attn_few_smem_bytes() {
-  return sizeof(float) * (kFewQ * kFewDh + kFewQ * kFewKeys) + 2 * (size_t)kFewKeys * (kFewKPitch + kFewDh);
+size_t attn_few_ws_floats(int B, int n_heads, int H, int n_keys) {
+  return (size_t)B * n_heads * ((H + kFewQ - 1) / kFewQ) * few_chunks(n_keys) * kFewQ * kFewPart;
 }
+size_t attn_few_ctr_count(int B, int n_heads, int H) { return (size_t)B * n_heads * ((H + kFewQ - 1) / kFewQ); }
 
 bool attn_few_ok(const AttnArgs& a) {
   const int n_keys = a.P + (a.kc ? a.H : 0);
   const bool aligned = a.kp_ld % 8 == 0 && a.kc_ld % 8 == 0 && a.q_ld % 8 == 0 && a.out_ld % 4 == 0;
-  return a.dtype == BF16 && a.head_dim == kFewDh && n_keys <= kFewKeys && n_keys >= 1 && aligned &&
-         (a.kp_bstride % 8) == 0 && (a.n_heads * a.head_dim) % 8 == 0;
+  return a.dtype == BF16 && a.head_dim == kFewDh && n_keys >= 1 && aligned && (a.kp_bstride % 8) == 0 &&
+         (a.n_heads * a.head_dim) % 8 == 0 && (few_chunks(n_keys) == 1 || (a.split_ws && a.split_ctr));
 }
 
 __global__ void add_tau_silu_kernel(const float* __restrict__ x, const float* __restrict__ tab, int stride, int off,
@@ -749,7 +792,6 @@ size_t attention_smem_bytes(int dh) {
 void launch_attention_prepare(int dh) {
   const int smem = (int)attention_smem_bytes(dh);
   const cudaFuncAttribute at = cudaFuncAttributeMaxDynamicSharedMemorySize;
-  cudaFuncSetAttribute(attn_few_kernel, at, (int)attn_few_smem_bytes());
   if (dh == 64) cudaFuncSetAttribute(attn_kernel<2>, at, smem);
   if (dh == 128) cudaFuncSetAttribute(attn_kernel<4>, at, smem);
   if (dh == 256) cudaFuncSetAttribute(attn_kernel<8>, at, smem);
@@ -758,7 +800,8 @@ void launch_attention_prepare(int dh) {
 void launch_attention(const AttnArgs& a, cudaStream_t s) {
   const int dh = a.head_dim;
   if (attn_few_ok(a)) {
-    launch_k(attn_few_kernel, dim3((a.H + kFewQ - 1) / kFewQ, a.n_heads, a.B), dim3(256), attn_few_smem_bytes(), s, a);
+    const int n_keys = a.P + (a.kc ? a.H : 0);
+    launch_k(attn_few_kernel, dim3(((a.H + kFewQ - 1) / kFewQ) * few_chunks(n_keys), a.n_heads, a.B), dim3(256), 0, s, a);
     return;
   }
   const size_t smem = attention_smem_bytes(dh);

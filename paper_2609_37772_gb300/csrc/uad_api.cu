@@ -105,6 +105,8 @@ struct uad_ctx {
 
   // prefix
   void *kpre = nullptr, *vpre = nullptr;  // ADARMS [B][L][P][Hkv dh]; DiT [B][L][P][Hq dh]
+  float* few_ws = nullptr;                // few-query attention: partial rows of the key chunks
+  unsigned* few_ctr = nullptr;            // and their arrival counts (zero between launches)
   std::vector<int> has_prefix;
 
   // activations / state
@@ -665,6 +667,7 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, bool step, cudaStream_t s) {
         at.vc = static_cast<const char*>(c->qkv) + (size_t)(c->qd + c->kvd) * c->es;
         at.kc_ld = c->qkvd;
         at.out = c->o; at.out_ld = c->qd; at.dtype = dt; at.scale = 1.f / std::sqrt((float)a.head_dim);
+        at.split_ws = c->few_ws; at.split_ctr = c->few_ctr;
         if (!dit) {
           at.kp = static_cast<const char*>(c->kpre) + (size_t)l * a.prefix_len * c->kvd * c->es;
           at.vp = static_cast<const char*>(c->vpre) + (size_t)l * a.prefix_len * c->kvd * c->es;
@@ -703,6 +706,7 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, bool step, cudaStream_t s) {
           ac.vp = static_cast<const char*>(c->vpre) + (size_t)l * a.prefix_len * c->qd * c->es;
           ac.P = a.prefix_len; ac.kp_bstride = (long long)a.n_layers * a.prefix_len * c->qd; ac.kp_ld = c->qd;
           ac.out = c->o; ac.out_ld = c->qd; ac.dtype = dt; ac.scale = at.scale;
+          ac.split_ws = c->few_ws; ac.split_ctr = c->few_ctr;
           {
             const double by = c->es * ((double)B * ac.P * c->qd * 2 + 2.0 * M * c->qd);
             Mark mk(c, s, "cross_attn", by, 4.0 * M * a.n_heads * (double)ac.P * a.head_dim);
@@ -978,6 +982,15 @@ int uad_init(const uad_arch* arch, const float* weights, size_t n_floats, uad_ct
   TRY(dalloc(c, &c->kpre, a.max_batch * per_robot_kv * es));
   TRY(dalloc(c, &c->vpre, a.max_batch * per_robot_kv * es));
   c->has_prefix.assign(a.max_batch, 0);
+  if (a.dtype == UAD_DTYPE_BF16 && a.head_dim == 64) {
+    // few-query attention split over key chunks (self-attention over the chunk, cross-attention
+    // over the prefix): partial rows and zeroed arrival counts
+    const int keys = std::max(a.chunk_len + (a.kind == UAD_KIND_DIT ? 0 : a.prefix_len), a.prefix_len);
+    TRY(dalloc_t(c, &c->few_ws, std::max<size_t>(1, attn_few_ws_floats(a.max_batch, a.n_heads, a.chunk_len, keys))));
+    const size_t nctr = std::max<size_t>(1, attn_few_ctr_count(a.max_batch, a.n_heads, a.chunk_len));
+    TRY(dalloc_t(c, &c->few_ctr, nctr));
+    CK(cudaMemset(c->few_ctr, 0, nctr * sizeof(unsigned)));
+  }
   const size_t M = c->mmax;
   TRY(dalloc_t(c, &c->h, M * W));
   TRY(dalloc(c, &c->y, M * W * es));

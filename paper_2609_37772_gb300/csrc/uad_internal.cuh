@@ -95,7 +95,14 @@ struct AttnArgs {
   void* out = nullptr; int out_ld = 0;                   // out[(b*H + i) * out_ld + hq*dh + d]
   int dtype = F32;
   float scale = 1.f;
+  // few-query attention split over key chunks: partial rows and per-(robot, head, query block)
+  // arrival counts (zero between launches: the last CTA of a group resets its count)
+  float* split_ws = nullptr;
+  unsigned* split_ctr = nullptr;
 };
+// Workspace of the few-query attention split over key chunks, in floats and counters.
+size_t attn_few_ws_floats(int B, int n_heads, int H, int n_keys);
+size_t attn_few_ctr_count(int B, int n_heads, int H);
 
 // Per-step, per-token plan entry (built on the host).
 enum PlanFlag { PF_ACTIVE = 1, PF_GHOST = 2, PF_RELEASE = 4, PF_EARLY = 8, PF_FROZEN = 16,
