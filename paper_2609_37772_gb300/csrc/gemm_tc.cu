@@ -13,9 +13,16 @@
 // applies the epilogue, then clears the accumulator and counter for the next launch. The
 // residual projections instead write each split's tile to a plane of its own (EPI_PARTIAL):
 // the norm that follows sums the planes in a fixed order as part of the residual update.
+// Many tokens (a batch of robots) take the persistent wide form instead: one CTA per SM walks
+// units of up to 256 tokens x 128 weight rows with two tensor-memory accumulators, so that the
+// epilogue of one unit overlaps the main loop of the next.
 // Every wait is bounded: on timeout the kernel records an error code and winds down.
 #include <cuda.h>
 #include <cudaTypedefs.h>
+
+#include <array>
+#include <cstdlib>
+#include <map>
 
 #include "uad_internal.cuh"
 #include "ptx.cuh"
@@ -30,6 +37,10 @@ constexpr int kBM = 128, kBN = 64, kBK = 64;
 constexpr int kStageA = kBM * kBK * 2;  // 16 KB
 constexpr int kStageB = kBN * kBK * 2;  // 8 KB
 constexpr unsigned long long kWaitNs = 2000000000ull;  // 2 s bound on any wait
+// persistent form: tokens per epilogue slice, epilogue groups (four warps each), staging pitch
+// in floats (132: a float4 column read across 8 tokens touches all 32 banks once), threads
+constexpr int kPersSlice = 16, kPersGroups = 4, kPersPitch = kBM + 4;
+constexpr int kPersThreads = 64 + kPersGroups * 128;
 
 __device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity, int* err, int code) {
   return ptx::mbar_wait(b, parity, err, code, kWaitNs);
@@ -73,11 +84,12 @@ __host__ __device__ __forceinline__ size_t tc_pipe_bytes(int stages) {
 }
 
 
-// Epilogue of one tile slice: T[j][row] holds the fp32 accumulator of token m0 + j (j < mcount)
-// for output row n = this thread's row; `plane` is the K split (partial epilogue). Small rolled
-// loops keep the code compact.
-__device__ __forceinline__ void tile_epilogue(const TcGemmArgs& p, const float* T, int plane, int m0, int mcount,
-                                              int n, int row, int lane) {
+// Epilogue of one tile slice: T[j * pitch + row] holds the fp32 accumulator of token m0 + j
+// (j < mcount) for output row n = this thread's row (row = 32 w + lane over the four warps w of
+// the slice's group); `plane` is the K split (partial epilogue). Small rolled loops keep the code
+// compact.
+__device__ __forceinline__ void tile_epilogue(const TcGemmArgs& p, const float* T, int pitch, int plane, int m0,
+                                              int mcount, int n, int row, int lane) {
   const float b = p.bias ? p.bias[n] : 0.f;
   const float* Tr = T + row;
   switch (p.epi) {
@@ -85,7 +97,7 @@ __device__ __forceinline__ void tile_epilogue(const TcGemmArgs& p, const float* 
       // this split's fp32 partial tile into its own plane [split][M][N]; the consumer sums
       float* dst = static_cast<float*>(p.out) + (size_t)plane * p.M * p.N;
 #pragma unroll 4
-      for (int j = 0; j < mcount; ++j) dst[(size_t)(m0 + j) * p.N + n] = Tr[j * kBM];
+      for (int j = 0; j < mcount; ++j) dst[(size_t)(m0 + j) * p.N + n] = Tr[j * pitch];
       break;
     }
     case EPI_GEGLU: {
@@ -95,7 +107,7 @@ __device__ __forceinline__ void tile_epilogue(const TcGemmArgs& p, const float* 
       const int o0 = (n - row) / 2 + 2 * lane;
       const bool fast = p.out_dtype == BF16;
       for (int j = row >> 5; j < mcount; j += kBM / 32) {
-        const float4 v = *reinterpret_cast<const float4*>(T + j * kBM + 4 * lane);
+        const float4 v = *reinterpret_cast<const float4*>(T + j * pitch + 4 * lane);
         const size_t off = (size_t)(m0 + j) * p.ldo + o0;
         if (fast) {
           *reinterpret_cast<__nv_bfloat162*>(static_cast<__nv_bfloat16*>(p.out) + off) =
@@ -110,7 +122,7 @@ __device__ __forceinline__ void tile_epilogue(const TcGemmArgs& p, const float* 
     case EPI_BIAS_GELU:
 #pragma unroll 4
       for (int j = 0; j < mcount; ++j)
-        store_out(p.out, (size_t)(m0 + j) * p.ldo + n, gelu_tanh_f(Tr[j * kBM] + b), p.out_dtype);
+        store_out(p.out, (size_t)(m0 + j) * p.ldo + n, gelu_tanh_f(Tr[j * pitch] + b), p.out_dtype);
       break;
     case EPI_QKV_TC: {
       const QkvTcOut& o = p.qkv;
@@ -127,7 +139,7 @@ __device__ __forceinline__ void tile_epilogue(const TcGemmArgs& p, const float* 
         const size_t sb = isq ? (size_t)o.Hkv * o.G * o.H * o.dh : (size_t)o.L * o.Hkv * o.NK * o.dh;
         for (int j = row >> 5; j < mcount; j += kBM / 32) {
           const int m = m0 + j, bi = m / o.H, ii = m - bi * o.H;
-          const float4 v = *reinterpret_cast<const float4*>(T + j * kBM + 4 * lane);
+          const float4 v = *reinterpret_cast<const float4*>(T + j * pitch + 4 * lane);
           __nv_bfloat16* dst = base + bi * sb + (size_t)ii * o.dh;
           if (o.rope) {
             const float4 cs = *reinterpret_cast<const float4*>(o.rope + (size_t)ii * o.dh + r);
@@ -142,15 +154,15 @@ __device__ __forceinline__ void tile_epilogue(const TcGemmArgs& p, const float* 
           }
         }
       } else {
-        // v rows: lane owns a token and reads 4 head dims of it at once; each store instruction
-        // then writes 32 consecutive keys of one head dim of Vt (keys contiguous)
+        // v rows: item (row quad rq, token j), tokens fastest: a thread reads 4 head dims of one
+        // token at once and each store instruction writes consecutive keys of one head dim of Vt
+        // (keys contiguous)
         const int sv0 = n0 - o.qd - o.kvd;   // the tile's first v feature
         const size_t sb = (size_t)o.L * o.Hkv * o.dh * o.NKp;
-        for (int it = row >> 5; it < (kBM / 4) * 2; it += kBM / 32) {
-          const int r4 = 4 * (it >> 1), j = 32 * (it & 1) + lane;
-          if (j >= mcount) continue;
+        for (int it = row; it < (kBM / 4) * mcount; it += kBM) {
+          const int r4 = 4 * (it / mcount), j = it - (it / mcount) * mcount;
           const int m = m0 + j, bi = m / o.H, ii = m - bi * o.H;
-          const float4 v = *reinterpret_cast<const float4*>(T + j * kBM + r4);
+          const float4 v = *reinterpret_cast<const float4*>(T + j * pitch + r4);
           const int sn = sv0 + r4, g = sn / o.dh, d = sn % o.dh;   // 4 dims of one head
           __nv_bfloat16* dst = o.vtcache + bi * sb + (((size_t)o.layer * o.Hkv + g) * o.dh + d) * o.NKp + o.P + ii;
           dst[0] = __float2bfloat16_rn(v.x);
@@ -164,7 +176,7 @@ __device__ __forceinline__ void tile_epilogue(const TcGemmArgs& p, const float* 
     default:
 #pragma unroll 4
       for (int j = 0; j < mcount; ++j)
-        store_out(p.out, (size_t)(m0 + j) * p.ldo + n, Tr[j * kBM] + b, p.out_dtype);
+        store_out(p.out, (size_t)(m0 + j) * p.ldo + n, Tr[j * pitch] + b, p.out_dtype);
       break;
   }
 }
@@ -335,7 +347,7 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
       }
     }
   } else if (have) {
-    tile_epilogue(p, T, s, m0, mcount, n, row, lane);
+    tile_epilogue(p, T, kBM, s, m0, mcount, n, row, lane);
   }
   tc_fence_before();
   __syncthreads();
@@ -444,12 +456,179 @@ __global__ void __launch_bounds__(128, MINB) gemm_tc_wide_kernel(const __grid_co
 #pragma unroll
     for (int j = 0; j < kBN; ++j) T[j * kBM + row] = v[j];
     __syncthreads();
-    if (ok) tile_epilogue(p, T, 0, m0, mcount, n, row, lane);
+    if (ok) tile_epilogue(p, T, kBM, 0, m0, mcount, n, row, lane);
     __syncthreads();
   }
   tc_fence_before();
   __syncthreads();
   if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kWN));
+}
+
+// Persistent form for many tokens: one CTA per SM walks the work units u = blockIdx.x,
+// blockIdx.x + gridDim.x, ... Unit u is (token tile mt of p.tn <= TN tokens, weight tile nt, K
+// split sp) with mt fastest, so the CTAs running side by side share a weight tile in L2. Warp 0
+// feeds the ring of STAGES (weights 16 KB + up to TN x 128 B of tokens) without stopping at unit
+// boundaries; warp 1 issues the MMAs into one of two TMEM accumulators (2 x TN columns) while
+// four groups of four warps (2-5, 6-9, 10-13, 14-17) drain the other one in 16-token slices,
+// slice q to group q % 4, each group through a staging slice of its own, so a unit's epilogue
+// overlaps the next unit's main loop. A ragged last token tile loads and multiplies only its
+// 64-token boxes. K splits (residual projections only) write planes of their own, summed by the
+// norm that follows.
+template <int TN, int STAGES>
+__global__ void __launch_bounds__(kPersThreads, 1) gemm_tc_pers_kernel(const __grid_constant__ CUtensorMap tmx,
+                                                                       TcGemmArgs p) {
+  constexpr int kStageBw = TN * kBK * 2;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  uint8_t* sA = smem;                                        // STAGES x 16 KB weights
+  uint8_t* sB = smem + (size_t)STAGES * kStageA;             // STAGES x TN x 128 B tokens
+  float* T = reinterpret_cast<float*>(smem + (size_t)STAGES * (kStageA + kStageBw));  // groups x 16 x pitch
+  uint64_t* full = reinterpret_cast<uint64_t*>(T + kPersGroups * kPersSlice * kPersPitch);
+  uint64_t* empty = full + STAGES;
+  uint64_t* tfull = empty + STAGES;    // accumulator b complete
+  uint64_t* tempty = tfull + 2;        // accumulator b drained (one arrival per epilogue thread)
+  uint64_t* done = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int tn = p.tn;
+  const int n_nt = p.N / kBM, n_mt = (p.M + tn - 1) / tn, S = p.splits, KC = p.K / kBK;
+  const int per = (KC + S - 1) / S;
+  const int units = n_nt * n_mt * S;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < STAGES; ++i) {
+      mbar_init(full + i, 1);
+      mbar_init(empty + i, 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(tfull + b, 1);
+      mbar_init(tempty + b, kPersGroups * 128);
+    }
+    mbar_init(done, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(tmem_slot)), "r"(2 * TN));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  pdl_trigger();
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---- producer ----
+      pdl_wait();
+      int it = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+        const int mt = u % n_mt, r = u / n_mt, nt = r % n_nt, sp = r / n_nt;
+        const int k0 = sp * per, k1 = k0 + per < KC ? k0 + per : KC;
+        const int left = p.M - mt * tn;
+        const int nb = ((left < tn ? left : tn) + kBN - 1) / kBN;
+        const uint8_t* wt = static_cast<const uint8_t*>(p.w_tiled) + (size_t)nt * KC * kStageA;
+        for (int kb = k0; kb < k1; ++kb, ++it) {
+          const int st = it % STAGES, round = it / STAGES;
+          if (round > 0 && !mbar_wait(empty + st, (round - 1) & 1, p.err, 61)) { ok = false; break; }
+          mbar_expect_tx(full + st, kStageA + nb * kStageB);
+          bulk_g2s_nohint(sA + (size_t)st * kStageA, wt + (size_t)kb * kStageA, kStageA, full + st);
+          for (int q = 0; q < nb; ++q)
+            tma_2d(sB + (size_t)st * kStageBw + q * kStageB, &tmx, kb * kBK, mt * tn + q * kBN, full + st);
+        }
+      }
+      // do not leave copies in flight into shared memory of an exiting CTA
+      for (int i = it - STAGES > 0 ? it - STAGES : 0; i < it; ++i)
+        mbar_wait(full + i % STAGES, (i / STAGES) & 1, p.err, 62);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---- MMA issuer ----
+      const uint32_t tmem = *tmem_slot;
+      int it = 0, j = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++j) {
+        const int mt = u % n_mt, sp = u / n_mt / n_nt;
+        const int k0 = sp * per, k1 = k0 + per < KC ? k0 + per : KC;
+        const int left = p.M - mt * tn;
+        const int nb = ((left < tn ? left : tn) + kBN - 1) / kBN;
+        const uint32_t idesc = idesc_m128(nb * kBN);
+        const int b = j & 1;
+        if (j >= 2 && !mbar_wait(tempty + b, ((j >> 1) - 1) & 1, p.err, 63)) break;
+        tc_fence_after();
+        const uint32_t d = tmem + (uint32_t)(b * TN);
+        for (int kb = k0; kb < k1; ++kb, ++it) {
+          const int st = it % STAGES, round = it / STAGES;
+          if (!mbar_wait(full + st, round & 1, p.err, 64)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t a0 = su32(sA + (size_t)st * kStageA), b0 = su32(sB + (size_t)st * kStageBw);
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k)
+            ptx::mma_bf16(d, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), idesc, (kb > k0 || k > 0) ? 1u : 0u);
+          mma_commit(empty + st);
+        }
+        if (ok) mma_commit(tfull + b);
+      }
+      mma_commit(done);
+      mbar_wait(done, 0, p.err, 65);
+    }
+  } else {
+    // ---- epilogue: group g = warps 2 + 4g .. 5 + 4g takes slices g, g + 4, ...; warp w reads
+    //      tensor-memory lanes 32 (w % 4) .. + 31 ----
+    const int g = (warp - 2) >> 2;
+    const int q4 = warp & 3, row = q4 * 32 + lane;
+    float* Tg = T + g * kPersSlice * kPersPitch;
+    pdl_wait();
+    int j = 0;
+    for (int u = blockIdx.x; u < units; u += gridDim.x, ++j) {
+      const int mt = u % n_mt, r = u / n_mt, nt = r % n_nt, sp = r / n_nt;
+      const int left = p.M - mt * tn;
+      const int nsl = ((left < tn ? left : tn) + kPersSlice - 1) / kPersSlice;
+      const int mylast = g < nsl ? g + kPersGroups * ((nsl - 1 - g) / kPersGroups) : -1;  // this group's last slice
+      const int b = j & 1;
+      // one decision for the group, so that none of its warps is left alone at a named barrier
+      if (!named_and(1 + g, 128, mbar_wait(tfull + b, (j >> 1) & 1, p.err, 66))) break;
+      tc_fence_after();
+      if (mylast < 0) {
+        tc_fence_before();
+        mbar_arrive(tempty + b);
+      }
+      const uint32_t tb = tmem_base_after_wait(tmem_slot) + (uint32_t)(b * TN) + ((uint32_t)(q4 * 32) << 16);
+      const int n = nt * kBM + row;
+      for (int q = g; q < nsl; q += kPersGroups) {
+        const int m0 = mt * tn + q * kPersSlice;
+        const int mcount = p.M - m0 < kPersSlice ? p.M - m0 : kPersSlice;
+        float v[kPersSlice];
+        tmem_ld16(tb + q * kPersSlice, v);
+        if (q == mylast) {
+          // the group's share of the accumulator is in registers: hand it back
+          tc_fence_before();
+          mbar_arrive(tempty + b);
+        }
+        named_sync(1 + g, 128);   // the previous slice's readers are done with Tg
+#pragma unroll
+        for (int jj = 0; jj < kPersSlice; ++jj) Tg[jj * kPersPitch + row] = v[jj];
+        named_sync(1 + g, 128);
+        if (p.epi == EPI_PARTIAL) {
+          // plane sp of [splits][M][N]: whole rows of the slice as 16-byte stores
+          float* dst = static_cast<float*>(p.out) + (size_t)sp * p.M * p.N + (size_t)m0 * p.N + nt * kBM;
+          for (int idx = row; idx < mcount * (kBM / 4); idx += 128) {
+            const int jr = idx / (kBM / 4), c4 = idx % (kBM / 4);
+            *reinterpret_cast<float4*>(dst + (size_t)jr * p.N + c4 * 4) =
+                *reinterpret_cast<const float4*>(Tg + jr * kPersPitch + c4 * 4);
+          }
+        } else {
+          tile_epilogue(p, Tg, kPersPitch, sp, m0, mcount, n, row, lane);
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(*tmem_slot), "r"(2 * TN));
+  }
 }
 
 // ---- weight re-layout into 128 x 64 swizzled blocks --------------------------------------
@@ -512,37 +691,77 @@ size_t gemm_tc_smem_bytes(int stages, int epi, int M) {
   return 1024 + tc_pipe_bytes(stages) + (2 * kTcMaxStages + 1) * 8 + 16;
 }
 
-static size_t gemm_tc_wide_smem_bytes(int tn, int stages) {
-  return 1024 + (size_t)stages * (kStageA + (size_t)tn * kBK * 2) + (2 * stages + 2) * 8 + 16;
+constexpr int kPersStages256 = 4, kPersStages128 = 6;   // 192 KB of ring either way
+// tn: the instantiation's tile capacity (256 or 128)
+static size_t gemm_tc_pers_smem_bytes(int tn) {
+  const int st = tn == 256 ? kPersStages256 : kPersStages128;
+  return 1024 + (size_t)st * (kStageA + (size_t)tn * kBK * 2) + (size_t)kPersGroups * kPersSlice * kPersPitch * 4 +
+         (2 * st + 5) * 8 + 16;
 }
 
 void gemm_tc_prepare() {
-  const size_t a = gemm_tc_smem_bytes(kTcMaxStages, EPI_STORE, kBN);
-  cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)a);
-  cudaFuncSetAttribute(gemm_tc_wide_kernel<256, 4, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)gemm_tc_wide_smem_bytes(256, 4));
-  cudaFuncSetAttribute(gemm_tc_wide_kernel<256, 2, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)gemm_tc_wide_smem_bytes(256, 2));
-  cudaFuncSetAttribute(gemm_tc_wide_kernel<128, 4, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)gemm_tc_wide_smem_bytes(128, 4));
-  cudaFuncSetAttribute(gemm_tc_wide_kernel<128, 3, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)gemm_tc_wide_smem_bytes(128, 3));
+  static bool done = false;
+  if (done) return;
+  done = true;
+  cudaFuncSetAttribute(gemm_tc_pers_kernel<256, kPersStages256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       (int)gemm_tc_pers_smem_bytes(256));
+  cudaFuncSetAttribute(gemm_tc_pers_kernel<128, kPersStages128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       (int)gemm_tc_pers_smem_bytes(128));
+  cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       (int)gemm_tc_smem_bytes(kTcMaxStages, EPI_STORE, kBN));
 }
 
-// Wide tiles (MMA N = 256 or 128 tokens) run the tensor cores near their rate (N = 64 runs at a
-// third of it) and cut L2 re-reads of the weights. Returns 0 (narrow 128 x 64 tiles with K
-// splits), or the wide form: 1 = 256 tokens, four stages, one CTA per SM; 2 = 256 tokens, two
-// stages, two CTAs per SM (with at least as many tiles as SMs, one CTA's epilogue overlaps the
-// other's main loop); 3 = 128 tokens, four stages, one CTA per SM; 4 = 128 tokens, three stages,
-// two CTAs per SM. 256-token tiles while they fill 60% of the SMs, else 128-token tiles while
-// those fill half of them (measured on the pi0-like projections from 200 to 3200 tokens: with
+// Wide tiles (MMA N up to 256 tokens) run the tensor cores near their rate (N = 64 runs at a
+// third of it) and cut L2 re-reads of the weights: 1 = the persistent wide form, 0 = narrow
+// 128 x 64 tiles with K splits. Wide while 256-token tiles fill 60% of the SMs or 128-token
+// tiles fill half of them (measured on the pi0-like projections from 200 to 3200 tokens: with
 // fewer than 256 tokens the narrow tiles win).
 int gemm_tc_use_wide(int M, int N, int sms) {
   if (M < 256 || N > 8192) return 0;
   const int t256 = (N / kBM) * ((M + 255) / 256), t128 = (N / kBM) * ((M + 127) / 128);
-  if (t256 >= sms) return 2;
-  if (t256 * 5 >= sms * 3) return 1;
-  if (t128 >= sms) return 4;
-  if (t128 * 2 >= sms) return 3;
-  return 0;
+  return t256 * 5 >= sms * 3 || t128 * 2 >= sms ? 1 : 0;
 }
-int gemm_tc_wide_tokens(int wide) { return wide >= 3 ? 128 : 256; }
+
+// The persistent form's plan: tokens per tile (256, 192 or 128) and, for partial-plane
+// epilogues, K splits. Units go to the CTAs round robin; the plan minimises the busiest CTA's
+// work, counted in k-blocks of a 256-token tile: a k-block of nb 64-token boxes costs half by
+// its MMA time (nb / 4) and half by its bytes ((2 + nb) / 6, weights 16 KB + 8 KB a box), plus
+// half a k-block per unit and, per extra plane, the cost of writing and reading it once more.
+void gemm_tc_pers_plan(int M, int N, int K, int sms, int epi, int* tn, int* splits) {
+  const int KC = K / kBK, n_nt = N / kBM;
+  double best = 1e30;
+  *tn = 256;
+  *splits = 1;
+  for (int t = 256; t >= 128; t -= 64) {
+    const int n_mt = (M + t - 1) / t;
+    const int smax = epi == EPI_PARTIAL ? 8 : 1;
+    for (int sp = 1; sp <= smax && sp <= KC; ++sp) {
+      const int per = (KC + sp - 1) / sp;
+      if ((sp - 1) * per >= KC) continue;
+      const int units = n_nt * n_mt * sp;
+      const int ctas = units < sms ? units : sms;
+      double worst = 0;
+      for (int c = 0; c < ctas; ++c) {
+        double w = 0;
+        for (int u = c; u < units; u += ctas) {
+          const int mt = u % n_mt, s = u / n_mt / n_nt;
+          const int kb = (s + 1) * per < KC ? per : KC - s * per;
+          const int left = M - mt * t;
+          const int nb = ((left < t ? left : t) + kBN - 1) / kBN;
+          w += kb * (0.5 * nb / 4.0 + 0.5 * (2 + nb) / 6.0) + 0.5;
+        }
+        worst = w > worst ? w : worst;
+      }
+      const double plane = 8.0 * M * N / 6.5e12 / 0.3e-6;   // extra plane written and read, in k-blocks
+      const double cost = worst + (sp - 1) * plane;
+      if (cost < best - 1e-9) {
+        best = cost;
+        *tn = t;
+        *splits = sp;
+      }
+    }
+  }
+}
 
 // K splits per output tile: one CTA per SM. Partial-plane epilogues (the consumer sums the
 // planes) take more splits, up to two CTAs per SM, so that every CTA holds its whole K range in
@@ -563,16 +782,40 @@ int gemm_tc_splits(int M, int N, int K, int sms, int epi) {
   return s;
 }
 
+void gemm_tc_plan(int M, int N, int K, int sms, int epi, TcGemmArgs* a) {
+  a->wide = gemm_tc_use_wide(M, N, sms);
+  a->tn = 0;
+  a->splits = 1;
+  if (a->wide) {
+    // the plan search walks every unit: remember its answers
+    thread_local std::map<std::array<int, 5>, std::pair<int, int>> memo;
+    const std::array<int, 5> key{M, N, K, sms, epi == EPI_PARTIAL};
+    auto it = memo.find(key);
+    if (it == memo.end()) {
+      std::pair<int, int> v;
+      gemm_tc_pers_plan(M, N, K, sms, epi, &v.first, &v.second);
+      it = memo.emplace(key, v).first;
+    }
+    a->tn = it->second.first;
+    a->splits = it->second.second;
+  } else {
+    a->splits = gemm_tc_splits(M, N, K, sms, epi);
+  }
+}
+
 void launch_gemm_tc(const CUtensorMap* tmx, const TcGemmArgs& a, cudaStream_t s) {
   if (a.wide) {
-    const int tn = gemm_tc_wide_tokens(a.wide);
-    const dim3 grid(a.N / kBM, (a.M + tn - 1) / tn);
-    switch (a.wide) {
-      case 1: launch_k(gemm_tc_wide_kernel<256, 4, 1>, grid, dim3(128), gemm_tc_wide_smem_bytes(256, 4), s, *tmx, a); break;
-      case 2: launch_k(gemm_tc_wide_kernel<256, 2, 2>, grid, dim3(128), gemm_tc_wide_smem_bytes(256, 2), s, *tmx, a); break;
-      case 3: launch_k(gemm_tc_wide_kernel<128, 4, 1>, grid, dim3(128), gemm_tc_wide_smem_bytes(128, 4), s, *tmx, a); break;
-      default: launch_k(gemm_tc_wide_kernel<128, 3, 2>, grid, dim3(128), gemm_tc_wide_smem_bytes(128, 3), s, *tmx, a); break;
-    }
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int units = (a.N / kBM) * ((a.M + a.tn - 1) / a.tn) * a.splits;
+    const dim3 grid(units < sms ? units : sms);
+    if (a.tn > 128)
+      launch_k(gemm_tc_pers_kernel<256, kPersStages256>, grid, dim3(kPersThreads), gemm_tc_pers_smem_bytes(256), s,
+               *tmx, a);
+    else
+      launch_k(gemm_tc_pers_kernel<128, kPersStages128>, grid, dim3(kPersThreads), gemm_tc_pers_smem_bytes(128), s,
+               *tmx, a);
     return;
   }
   const int KC = a.K / kBK;

@@ -54,8 +54,7 @@ int launch_linear(const void* x, const void* w_tiled, const float* bias, float* 
   if (encode_act_tmap(&tm, x, K, M)) return UAD_ECUDA;
   TcGemmArgs a;
   a.w_tiled = w_tiled; a.M = M; a.N = N; a.K = K;
-  a.wide = gemm_tc_use_wide(M, N, sms);   // the tile selection of the velocity network's projections
-  a.splits = a.wide ? 1 : gemm_tc_splits(M, N, K, sms, EPI_STORE);
+  gemm_tc_plan(M, N, K, sms, EPI_STORE, &a);   // the tile selection of the velocity network's projections
   a.epi = EPI_STORE; a.out = out; a.ldo = N; a.out_dtype = F32; a.bias = bias;
   a.acc = acc; a.counters = counters; a.err = err;
   gemm_tc_prepare();

@@ -376,8 +376,9 @@ struct Mark {
 
 // Partial planes a residual projection [M][W] x [W][K]^T writes on the tensor cores.
 size_t residual_planes(const uad_ctx* c, int M, int K) {
-  const int W = c->a.width;
-  return gemm_tc_use_wide(M, W, c->sms) ? 1 : (size_t)gemm_tc_splits(M, W, K, c->sms, EPI_PARTIAL);
+  TcGemmArgs t;
+  gemm_tc_plan(M, c->a.width, K, c->sms, EPI_PARTIAL, &t);
+  return (size_t)t.splits;
 }
 
 // Algorithmic HBM bytes of one projection: weights + activations in + output (+ residual r/w).
@@ -404,8 +405,7 @@ void gemm(uad_ctx* c, const Lin& w, GemmArgs g, cudaStream_t s) {
   }
   TcGemmArgs t;
   t.w_tiled = w.w; t.M = g.M; t.N = g.N; t.K = g.K;
-  t.wide = gemm_tc_use_wide(g.M, g.N, c->sms);
-  t.splits = t.wide ? 1 : gemm_tc_splits(g.M, g.N, g.K, c->sms, g.epi);
+  gemm_tc_plan(g.M, g.N, g.K, c->sms, g.epi, &t);
   t.epi = g.epi; t.out = g.out; t.ldo = g.ldo; t.out_dtype = g.out_dtype; t.bias = g.bias;
   t.qkv = g.qkv; t.acc = c->tc_acc; t.counters = c->tc_counters; t.err = c->dev_err;
   launch_gemm_tc(&c->tmaps.at(g.A), t, s);

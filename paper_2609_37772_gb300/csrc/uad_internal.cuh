@@ -167,10 +167,9 @@ struct TcGemmArgs {
   float* acc = nullptr;            // split-K accumulator [M][N] fp32, zero between launches
   int* counters = nullptr;         // split-K arrival counters per output tile, zero between launches
   int* err = nullptr;              // set to a nonzero code if a bounded wait gave up
-  int wide = 0;                    // wide tiles without K split (many tokens): 0 no; 1 256 tokens,
-                                   // four stages, one CTA per SM; 2 256 tokens, two stages, two
-                                   // CTAs per SM; 3 128 tokens, four stages, one CTA per SM;
-                                   // 4 128 tokens, three stages, two CTAs per SM
+  int wide = 0;                    // 1: the persistent wide form (one CTA per SM walking units of
+                                   // tn tokens x 128 weight rows x a K range), 0: narrow split-K tiles
+  int tn = 0;                      // persistent form: tokens per tile (256, 192 or 128)
   unsigned long long* trace = nullptr;  // optional: 16 global-timer stamps per CTA (phase times)
 };
 size_t gemm_tc_smem_bytes(int stages, int epi, int M);
@@ -179,7 +178,9 @@ size_t gemm_tc_smem_bytes(int stages, int epi, int M);
 int encode_act_tmap(CUtensorMap* m, const void* base, int K, int rows);
 void gemm_tc_prepare();
 int gemm_tc_splits(int M, int N, int K, int sms, int epi);
-int gemm_tc_use_wide(int M, int N, int sms);    // the `wide` form for this projection (0-4)
+int gemm_tc_use_wide(int M, int N, int sms);    // 1: the persistent wide form serves this projection
+// The tile plan of one projection (wide form, tokens per tile, K splits) into a.
+void gemm_tc_plan(int M, int N, int K, int sms, int epi, TcGemmArgs* a);
 void launch_gemm_tc(const CUtensorMap* tmx, const TcGemmArgs& a, cudaStream_t s);
 // element (k, n) of src [K][N] -> row n' * mult + off, column k of the tiled bf16 layout (K cols),
 // where n' = n, or with rope_dh > 0 the head-local pair interleave (d, d + dh/2) -> (2d, 2d + 1)

@@ -42,12 +42,12 @@ def test_linear_matches_reference(M, N, K):
     assert np.abs(out - ref).max() <= 1e-5 * np.abs(ref).max()
 
 
-# Shapes whose tile selection on a 152-SM GB300 takes each wide form (128 x 256- or 128 x 128-token
-# tiles, one or two CTAs per SM), with ragged last token tiles; numbers of the selection rule:
-#   (2560, 2048): 160 tiles of 256 tokens >= 152 SMs -> 256 tokens, two CTAs per SM
-#   (3000, 1024): 96 tiles of 256 >= 60% of the SMs -> 256 tokens, one CTA per SM
-#   (2400, 1024): 80 tiles of 256, 152 of 128 -> 128 tokens, two CTAs per SM
-#   (800, 2560): 80 tiles of 256, 140 of 128 -> 128 tokens, one CTA per SM
+# Shapes that take the persistent wide form on a 152-SM GB300, with each of its tile widths and
+# ragged last token tiles (plan of the busiest CTA's work):
+#   (2560, 2048, 64): 16 weight tiles x 14 tiles of 192 tokens (the last 64)
+#   (3000, 1024, 128): 8 x 16 tiles of 192 tokens (the last 120)
+#   (2400, 1024, 128): 8 x 19 tiles of 128 tokens (the last 96)
+#   (800, 2560, 192): 20 x 7 tiles of 128 tokens (the last 32)
 @pytest.mark.parametrize("M,N,K", [(2560, 2048, 64), (3000, 1024, 128), (2400, 1024, 128), (800, 2560, 192)])
 def test_linear_wide_tiles_match_reference(M, N, K):
     rng = np.random.default_rng(M + N + K)
