@@ -750,8 +750,16 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, bool step, cudaStream_t s) {
 int launches_per_step(const uad_ctx* c, int B) {
   const uad_arch& a = c->a;
   if (step_path(c, B)) return 1;   // persistent evaluation kernel with the step epilogue at its end
-  return a.kind == UAD_KIND_DIT ? 11 * a.n_layers + 4
-                                 : (c->attn_tc ? 8 : 7) * a.n_layers + 4 + (a.kind == UAD_KIND_CONCAT ? 4 : 0);
+  if (a.kind == UAD_KIND_DIT) return 11 * a.n_layers + 4;
+  // per layer: norm, qkv, attention (split-KV + combine, or the one-pass kernel), o, norm,
+  // gate/up, down
+  int attn = 1;
+  if (c->attn_tc) {
+    AttnTcArgs t = c->at0;
+    t.batch = B;
+    attn = attn_tc_use_two_pass(t) ? 1 : 2;
+  }
+  return (6 + attn) * a.n_layers + 4 + (a.kind == UAD_KIND_CONCAT ? 4 : 0);
 }
 
 }  // namespace

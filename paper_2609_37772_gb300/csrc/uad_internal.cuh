@@ -206,7 +206,10 @@ int attn_tc_prepare(AttnTcMaps* maps, const AttnTcArgs& a, int batch_max);  // 0
 int attn_tc_chunks(int n_keys);
 int attn_tc_max_keys();
 int attn_tc_rpad(int rows);
-void launch_attn_tc(const AttnTcMaps& maps, const AttnTcArgs& a, cudaStream_t s);   // 2 kernels
+// two kernels (split-KV attention, combine), or the one-pass kernel alone when
+// attn_tc_use_two_pass (many query tiles)
+void launch_attn_tc(const AttnTcMaps& maps, const AttnTcArgs& a, cudaStream_t s);
+bool attn_tc_use_two_pass(const AttnTcArgs& a);
 void launch_kv_prefix(const void* k, const void* v, int src_dtype, const AttnTcArgs& a, int robot, cudaStream_t s);
 
 // ---- persistent evaluation kernel (adaRMS experts, bf16, few tokens) ----------------------
