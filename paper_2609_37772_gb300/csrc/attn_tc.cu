@@ -198,9 +198,10 @@ __global__ void __launch_bounds__(128, 1) attn_tc_kernel(const __grid_constant__
 
 // ---- one-pass attention for many query tiles: no partials, no combine ---------------------
 // One CTA per (128-row query tile, robot-group), keys in chunks of 128 (S = Q K^T with MMA
-// N = 128). Shared memory: Q, a K region, a Vt region, P. Per chunk: S on tcgen05 (double-buffered
-// in TMEM), then each softmax thread (one query row) forms P = exp(S - M) in bf16 against its
-// running maximum M and O += P V accumulates in TMEM. M is raised only when the chunk's maximum
+// N = 128). Shared memory: Q, a K region, a Vt region. Per chunk: S on tcgen05 (double-buffered in
+// TMEM), then each softmax thread (one query row) forms P = exp(S - M) in bf16 against its running
+// maximum M and writes it into tensor memory over the S it came from, and O += P V accumulates in
+// TMEM with P as the MMA's A operand from tensor memory (P is double-buffered with S). M is raised only when the chunk's maximum
 // exceeds it by more than 2^8 in the exponent; the O row and the row sum are then rescaled in place
 // (after the previous P V has completed). Otherwise the stale M stays: every P is at most 2^8, and
 // O and the row sum share the same reference, so O / sum is unchanged. O / l is written in bf16.
@@ -221,20 +222,18 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
   constexpr uint32_t QB = DH * kQT * 2;          // Q: NC blocks of 128 rows x 64
   constexpr uint32_t RB = DH * kKC2 * 2;         // a K chunk (NC blocks of 128 keys x 64) or a Vt
                                                  // chunk (2 blocks of dh x 64 keys)
-  constexpr uint32_t PB = kQT * kKC2 * 2;        // P: 2 blocks of 128 rows x 64 keys
   constexpr uint32_t VBLK = DH * 128;            // one Vt block: dh rows x 64 keys
   uint8_t* sQ = smem;
   uint8_t* sK = sQ + QB;
   uint8_t* sV = sK + RB;
-  uint8_t* sP = sV + RB;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + PB);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sV + RB);
   uint64_t* q_full = bars;          // Q landed
   uint64_t* full = bars + 1;        // [2] K / Vt region loaded
   uint64_t* empty = bars + 3;       // [2] K / Vt region free (the MMAs that read it are done)
   uint64_t* s_full = bars + 5;      // [2] S buffer written
-  uint64_t* s_empty = bars + 7;     // [2] S buffer read by the 4 warps
+  uint64_t* s_empty = bars + 7;     // [2] S / P buffer free (the P V that read its P is done)
   uint64_t* p_full = bars + 9;      // P written (and O rescaled) by the 4 warps
-  uint64_t* p_empty = bars + 10;    // P V done: P free, O complete up to this chunk
+  uint64_t* p_empty = bars + 10;    // P V done: O complete up to this chunk
   uint64_t* o_done = bars + 11;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
 
@@ -250,7 +249,7 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
       mbar_init(full + i, 1);
       mbar_init(empty + i, 1);
       mbar_init(s_full + i, 1);
-      mbar_init(s_empty + i, 4);
+      mbar_init(s_empty + i, 1);
     }
     mbar_init(p_full, 4);
     mbar_init(p_empty, 1);
@@ -291,7 +290,7 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
     }
   } else if (threadIdx.x == 160) {
     bool ok = mbar_wait(q_full, 0, p.err, 42);
-    const uint32_t q0 = su32(sQ), k0 = su32(sK), pp = su32(sP), v0 = su32(sV);
+    const uint32_t q0 = su32(sQ), k0 = su32(sK), v0 = su32(sV);
     for (int ch = 0; ch < nck && ok; ++ch) {
       const int sb = ch & 1;
       ok = mbar_wait(full + 0, ch & 1, p.err, 43);
@@ -311,9 +310,10 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
       tc_fence_after();
 #pragma unroll
       for (int k = 0; k < kKC2 / 16; ++k)
-        mma_bf16(tO, sw128_desc(pp + (k >> 2) * (kQT * 128) + 32 * (k & 3)), sw128_desc(v0 + (k >> 2) * VBLK + 32 * (k & 3)),
-                 idesc_m128(DH), (ch | k) ? 1u : 0u);
+        mma_bf16_ts(tO, tmem + sb * kKC2 + 8 * k, sw128_desc(v0 + (k >> 2) * VBLK + 32 * (k & 3)), idesc_m128(DH),
+                    (ch | k) ? 1u : 0u);
       mma_commit(empty + 1);
+      mma_commit(s_empty + sb);
       mma_commit(p_empty);
     }
     mma_commit(o_done);
@@ -331,7 +331,6 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
   float sv[kKC2];                    // the chunk's scores of this row
   float mref = -INFINITY, l = 0.f;   // the row's reference maximum and sum of P
   bool ok = true;
-  const int r8 = row & 7;
   for (int ch = 0; ch < nck; ++ch) {
     const int sb = ch & 1;
     const int key0 = ch * kKC2;
@@ -345,16 +344,19 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
       for (int i = 0; i < kKC2; ++i)
         if (i >= nv) sv[i] = -INFINITY;
     }
-    float mc = -INFINITY;
+    float mx[8];
 #pragma unroll
-    for (int i = 0; i < kKC2; ++i) mc = fmaxf(mc, sv[i]);
+    for (int j = 0; j < 8; ++j) mx[j] = sv[j];
+#pragma unroll
+    for (int i = 8; i < kKC2; ++i) mx[i & 7] = fmaxf(mx[i & 7], sv[i]);
+    const float mc = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])), fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
     // raise the reference past 2^8 (and at the first chunk); the previous P V must have completed
-    // before O is touched, and before P is overwritten in any case
+    // before O is touched (P goes to this chunk's own buffer, free since S landed in it)
     const bool raise = ch == 0 ? true : (mc - mref) * c2s > kRescaleLog2;
     const float factor = ch == 0 ? 1.f : (raise ? exp2f((mref - mc) * c2s) : 1.f);
-    if (ch > 0) ok = ok && mbar_wait(p_empty, (ch - 1) & 1, p.err, 48);
-    tc_fence_after();
     if (__any_sync(0xffffffffu, ch > 0 && raise)) {
+      ok = ok && mbar_wait(p_empty, (ch - 1) & 1, p.err, 48);
+      tc_fence_after();
       float ov[32];
 #pragma unroll 1
       for (int cc = 0; cc < DH / 32; ++cc) {
@@ -369,6 +371,7 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
       mref = mc;
     }
     const float ms = mref * c2s;
+    float la = 0.f, lb = 0.f;
 #pragma unroll
     for (int cc = 0; cc < kKC2 / 32; ++cc) {
       uint32_t pk[16];
@@ -378,25 +381,21 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
         const float e0 = ex2_fast(fmaf(sv[k], c2s, -ms)), e1 = ex2_fast(fmaf(sv[k + 1], c2s, -ms));
         const __nv_bfloat162 h = __floats2bfloat162_rn(e0, e1);
         const float2 hf = __bfloat1622float2(h);
-        l += hf.x + hf.y;   // normalise by what the MMA sums
+        la += hf.x;   // normalise by what the MMA sums
+        lb += hf.y;
         pk[i / 2] = *reinterpret_cast<const uint32_t*>(&h);
       }
-      // keys 32 cc .. 32 cc + 31: P block cc / 2, 16-byte groups 4 (cc % 2) .. + 3
-      uint8_t* prow = sP + (cc >> 1) * (kQT * 128) + row * 128;
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int gidx = (cc & 1) * 4 + q;
-        *reinterpret_cast<uint4*>(prow + ((gidx ^ r8) * 16)) =
-            make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
-      }
+      // keys 32 cc .. 32 cc + 31 -> columns 16 cc .. + 15 of the chunk's S buffer (its scores are
+      // in registers)
+      tmem_st16_nowait(tmem + sb * kKC2 + lane_base + 16 * cc, pk);
     }
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    l += la + lb;
+    tmem_wait_st();
+    // (the issuer waits for this announcement before it issues S of the next chunk, so no phase of
+    // p_full completes ahead of its wait)
     tc_fence_before();
     __syncwarp();
-    if (lane == 0) {
-      asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(p_full)) : "memory");
-      asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(s_empty + sb)) : "memory");
-    }
+    if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(p_full)) : "memory");
   }
   float sv32[32];
   ok = ok && mbar_wait(o_done, 0, p.err, 49);
@@ -509,7 +508,7 @@ int tmap3(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d
 }  // namespace
 
 size_t attn_tc2_smem_bytes(int dh) {
-  return 1024 + (size_t)dh * kQT * 2 + 2 * (size_t)dh * kKC2 * 2 + (size_t)kQT * kKC2 * 2 + 16 * 8;
+  return 1024 + (size_t)dh * kQT * 2 + 2 * (size_t)dh * kKC2 * 2 + 16 * 8;
 }
 
 bool attn_tc_use_two_pass(const AttnTcArgs& a) {
