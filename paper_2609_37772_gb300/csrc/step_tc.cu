@@ -1142,10 +1142,9 @@ int step_prepare(int dh, int ring, int* blocks_per_sm) {
 // One CTA per SM. The grid barriers need every CTA resident at once: the shared-memory plan
 // admits one CTA per SM (checked at set-up with the occupancy calculator) and the kernel is
 // launched after the previous kernel has drained, so all `grid` CTAs start together. The
-// launch is not marked cooperative: under a cooperative launch, warps other than the MMA
-// issuer read stale tensor memory for a short time after the commit-driven barrier completes.
-// Should the CTAs ever not all be resident, the bounded barrier wait reports an error
-// instead of hanging.
+// launch is not marked cooperative because the kernel needs none of its semantics (the same
+// kernel launched cooperatively gives the same results). Should the CTAs ever not all be
+// resident, the bounded barrier wait reports an error instead of hanging.
 int launch_step(const StepMaps& m, const StepArgs& a, int grid, cudaStream_t s) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
