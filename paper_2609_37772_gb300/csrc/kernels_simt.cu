@@ -347,11 +347,12 @@ __global__ void __launch_bounds__(1024) resid_norm_kernel(NormArgs p) {
 }
 
 // The same with one warp per token row and the whole row in registers (W = 128 * NV): the row's
-// h, planes, gate and modulation vectors are all loaded before the arithmetic that needs them,
-// and its sums are warp reductions (no CTA barrier), so a row costs two memory round trips (the
-// modulation-row index, then the data). The planes are summed in plane order as above.
+// h, planes and gate are loaded before the arithmetic that needs them, and its sums are warp
+// reductions (no CTA barrier); the scale and shift vectors are loaded after the reduction, so
+// that a thread holds three row-sized arrays at most and four-warp CTAs fit three or four to an
+// SM (more rows in flight). The planes are summed in plane order as above.
 template <int NV>
-__global__ void __launch_bounds__(256) resid_norm_reg_kernel(NormArgs p) {
+__global__ void __launch_bounds__(128) resid_norm_reg_kernel(NormArgs p) {
   pdl_trigger();
   pdl_wait();
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
@@ -361,7 +362,7 @@ __global__ void __launch_bounds__(256) resid_norm_reg_kernel(NormArgs p) {
   const float4* pp = reinterpret_cast<const float4*>(p.part + (long long)row * p.W);
   const long long plane4 = (long long)p.M * p.W / 4;
   const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f), one = make_float4(1.f, 1.f, 1.f, 1.f);
-  float4 x[NV], acc[NV], gt[NV], sc[NV], sh[NV];
+  float4 x[NV], acc[NV], gt[NV];
 #pragma unroll
   for (int i = 0; i < NV; ++i) {
     x[i] = h4[i * 32 + lane];
@@ -370,11 +371,7 @@ __global__ void __launch_bounds__(256) resid_norm_reg_kernel(NormArgs p) {
   const float* mod = p.tab ? p.tab + (long long)tr * p.stride : nullptr;
   const float4* g4 = p.rgate_tab ? reinterpret_cast<const float4*>(p.rgate_tab + (long long)tr * p.stride + p.rgate_off) : nullptr;
 #pragma unroll
-  for (int i = 0; i < NV; ++i) {
-    gt[i] = g4 ? __ldg(g4 + i * 32 + lane) : one;
-    sc[i] = mod ? __ldg(reinterpret_cast<const float4*>(mod + p.scale_off) + i * 32 + lane) : zero;
-    sh[i] = mod ? __ldg(reinterpret_cast<const float4*>(mod + p.shift_off) + i * 32 + lane) : zero;
-  }
+  for (int i = 0; i < NV; ++i) gt[i] = g4 ? __ldg(g4 + i * 32 + lane) : one;
   for (int sp = 1; sp < p.n_part; ++sp) {
 #pragma unroll
     for (int i = 0; i < NV; ++i) {
@@ -404,6 +401,12 @@ __global__ void __launch_bounds__(256) resid_norm_reg_kernel(NormArgs p) {
     ss = fmaf(a, a, fmaf(b, b, fmaf(c, c, fmaf(d, d, ss))));
   }
   const float rstd = 1.f / sqrtf(warp_sum(ss) / p.W + 1e-6f);
+  float4 sc[NV], sh[NV];
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    sc[i] = mod ? __ldg(reinterpret_cast<const float4*>(mod + p.scale_off) + i * 32 + lane) : zero;
+    sh[i] = mod ? __ldg(reinterpret_cast<const float4*>(mod + p.shift_off) + i * 32 + lane) : zero;
+  }
 #pragma unroll
   for (int i = 0; i < NV; ++i) {
     float4 y = make_float4((x[i].x - mean) * rstd, (x[i].y - mean) * rstd, (x[i].z - mean) * rstd,
@@ -431,12 +434,12 @@ void launch_norm(const NormArgs& a, cudaStream_t s) {
   if (a.part) {
     const bool aligned = a.ldh % 4 == 0 && a.ldo % 4 == 0 && a.scale_off % 4 == 0 && a.shift_off % 4 == 0 &&
                          a.rgate_off % 4 == 0 && a.stride % 4 == 0 && a.W % 128 == 0;
-    const int blocks = (a.M + 7) / 8;
+    const int blocks = (a.M + 3) / 4;
     // a warp per row pays with enough rows to fill the SMs; with fewer, one CTA per row
     switch (aligned && a.M >= 512 ? a.W / 128 : 0) {
-      case 2: launch_k(resid_norm_reg_kernel<2>, dim3(blocks), dim3(256), 0, s, a); return;
-      case 4: launch_k(resid_norm_reg_kernel<4>, dim3(blocks), dim3(256), 0, s, a); return;
-      case 8: launch_k(resid_norm_reg_kernel<8>, dim3(blocks), dim3(256), 0, s, a); return;
+      case 2: launch_k(resid_norm_reg_kernel<2>, dim3(blocks), dim3(128), 0, s, a); return;
+      case 4: launch_k(resid_norm_reg_kernel<4>, dim3(blocks), dim3(128), 0, s, a); return;
+      case 8: launch_k(resid_norm_reg_kernel<8>, dim3(blocks), dim3(128), 0, s, a); return;
       default: break;
     }
     // the caller guarantees 16-byte rows: W, ldh, ldo, stride and the offsets multiples of 4
