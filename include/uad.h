@@ -165,7 +165,11 @@ int uad_poll_released(uad_ctx* ctx, int32_t robot, int32_t min_ready, int64_t ti
  * gac_error [batch][D]: E of Eq. 8 (zeros where GAC did not run).
  * Any output may be NULL; each may be host or device memory.
  * Returns UAD_OK, UAD_ENONFINITE (outputs written), UAD_ETIMEDOUT (the chunk stays in
- * flight; call again), UAD_ESTATE, UAD_ECUDA. */
+ * flight; call again), UAD_ESTATE, UAD_ECUDA. UAD_ECUDA after a bounded device-side wait ran
+ * out: if the chunk ran on the persistent evaluation kernel (whose grid barriers need all of
+ * its CTAs resident at once, which a shared or partitioned GPU may not grant), the context runs
+ * every later chunk on the per-operation kernels (uad_set_wait_limit tries the persistent
+ * kernel again). */
 int uad_finish(uad_ctx* ctx, float* final_actions, float* ghost, float* gac_error,
                uad_stats* stats, int64_t timeout_us);
 
@@ -200,7 +204,8 @@ int uad_profile_chunk(uad_ctx* ctx, const float* noise, const uad_schedule* sche
  * UAD_ECUDA, and the context stays usable. unreachable > 0 makes the first completion count of
  * every evaluation wait for that many arrivals more than the kernel ever makes, so that the
  * wait is sure to run out (0 restores normal operation). Applies to chunks started afterwards
- * (cached graphs are rebuilt). Returns UAD_OK, UAD_EINVAL or UAD_ESTATE (chunk in flight). */
+ * (cached graphs are rebuilt), and re-enables the persistent kernel after a fall-back (see
+ * uad_finish). Returns UAD_OK, UAD_EINVAL or UAD_ESTATE (chunk in flight). */
 int uad_set_wait_limit(uad_ctx* ctx, int64_t wait_ns, int32_t unreachable);
 
 void uad_destroy(uad_ctx* ctx);

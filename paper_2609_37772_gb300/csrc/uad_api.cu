@@ -79,6 +79,8 @@ struct uad_ctx {
   unsigned long long wait_ns = 2000000000ull;   // bound on any wait inside the persistent kernel
   int test_unreachable = 0;       // testing aid: extra arrivals the first phase count waits for
   int step_bmax = 0;              // robots per launch
+  bool step_failed = false;       // a wait of the persistent kernel ran out: per-operation kernels
+  bool cur_step = false;          // the chunk in flight runs on the persistent kernel
   StepArgs st0;                   // shapes and buffers; M, B, tau_row set per launch
   StepMaps smaps;
   double step_bytes_w = 0, step_flops_w = 0;   // weight bytes / 2 x params per evaluation
@@ -556,7 +558,7 @@ int step_setup(uad_ctx* c) {
   return UAD_OK;
 }
 
-bool step_path(const uad_ctx* c, int B) { return c->step_ok && B <= c->step_bmax; }
+bool step_path(const uad_ctx* c, int B) { return c->step_ok && !c->step_failed && B <= c->step_bmax; }
 
 // Whether a chunk runs on the persistent kernel: it serves the batch and every step has room
 // for its distinct flow times next to the tokens (set by the host plan).
@@ -1313,6 +1315,7 @@ static int denoise_impl(uad_ctx* c, const float* noise, const uad_schedule* sc, 
   CK(cudaEventRecord(c->ev_done, s));
   CK(cudaStreamWaitEvent(user, c->ev_done, 0));
   c->in_flight = true;
+  c->cur_step = use_step;
   c->cur_B = B;
   c->cur_steps = steps;
   c->cur_budgets.assign(sc->budgets, sc->budgets + (size_t)B * H);
@@ -1414,6 +1417,14 @@ int uad_finish(uad_ctx* c, float* final_actions, float* ghost, float* gac_error,
   CK(cudaMemcpy(&derr, c->dev_err, 4, cudaMemcpyDeviceToHost));
   if (derr) {
     cudaMemset(c->dev_err, 0, 4);
+    if (c->cur_step) {
+      // the persistent kernel's grid barriers need all of its CTAs resident at once, which a
+      // shared GPU (or one partitioned among processes) may not grant: later chunks run on the
+      // per-operation kernels
+      c->step_failed = true;
+      return fail(c, UAD_ECUDA, "a wait of the persistent kernel timed out (code %d); outputs are not valid; "
+                  "later chunks run on the per-operation kernels", derr);
+    }
     return fail(c, UAD_ECUDA, "a kernel wait timed out (code %d); outputs are not valid", derr);
   }
   CK(cudaMemcpy(&nonfinite, c->nonfinite, 4, cudaMemcpyDeviceToHost));
@@ -1447,6 +1458,7 @@ int uad_set_wait_limit(uad_ctx* c, int64_t wait_ns, int32_t unreachable) {
   if (c->in_flight) return fail(c, UAD_ESTATE, "chunk in flight");
   c->wait_ns = (unsigned long long)wait_ns;
   c->test_unreachable = unreachable;
+  c->step_failed = false;   // the persistent kernel is tried again
   // the launch arguments are baked into the cached graphs
   for (auto& kv : c->graphs) cudaGraphExecDestroy(kv.second);
   c->graphs.clear();

@@ -44,3 +44,36 @@ def test_expired_wait_is_reported_and_the_context_recovers():
         assert ok["rc"] == 0 and err <= 2e-2 and ok["evals"] == 6
     finally:
         ex.close()
+
+
+def test_expired_wait_falls_back_to_per_operation_kernels():
+    """After a wait of the persistent kernel ran out (as it would if its CTAs were not all
+    resident), the context runs later chunks on the per-operation kernels, correctly, until the
+    wait limit is set again."""
+    a = ARCHS["pi0_small"]
+    blob = make_weights(a, seed=22)
+    kv = make_prefix_kv(a, seed=22)
+    noise = make_noise(a, seed=22)
+    bud = group_budgets(a.chunk_len, [(0, 9, 3), (10, a.chunk_len - 1, 6)])
+    ex = uad.Expert(a, blob)
+    try:
+        ex.set_prefix(0, *kv)
+        ex.set_wait_limit(wait_ns=1_000_000, unreachable=1)
+        ex.denoise(noise, bud[None])
+        r = ex.finish(timeout_us=60_000_000, check=False)
+        assert r["rc"] == uad.UAD_ECUDA, r["rc"]
+        msg = uad.uad_last_error(ex.h).decode()
+        assert "per-operation kernels" in msg, msg
+        names = {r["name"] for r in ex.profile(noise, bud[None])}
+        assert "step_kernel" not in names and "qkv_proj" in names, names
+        ex.denoise(noise, bud[None])
+        ok = ex.finish(timeout_us=60_000_000)
+        ref = denoise(build_model(a, blob, kv).velocity, noise[0], bud)
+        err = np.abs(ok["final"][0] - ref["final"]).max() / np.abs(ref["final"]).max()
+        print(f"per-operation fall-back: max rel err {err:.2e}")
+        assert ok["rc"] == 0 and err <= 2e-2 and ok["evals"] == 6
+        ex.set_wait_limit()
+        names = {r["name"] for r in ex.profile(noise, bud[None])}
+        assert names == {"begin", "step_kernel"}, names
+    finally:
+        ex.close()
