@@ -208,6 +208,14 @@ int uad_profile_chunk(uad_ctx* ctx, const float* noise, const uad_schedule* sche
  * uad_finish). Returns UAD_OK, UAD_EINVAL or UAD_ESTATE (chunk in flight). */
 int uad_set_wait_limit(uad_ctx* ctx, int64_t wait_ns, int32_t unreachable);
 
+/* Testing aid (not part of the method): the fp32 rotations that Ghost Action Correction applies
+ * on SO(3) (App. C.1; Sec. 4.4, Eqs. 8-9), run on the GPU for n rotation vectors w[n][3] (host
+ * memory, axis times angle in radians): log_exp[i] = log(exp(w_i)) and
+ * log_comp[i] = log(exp(w_i) exp(w_{(i+1) mod n})^T), log giving the principal vector (angle in
+ * [0, pi]). Synchronous; allocates its own device memory. Returns UAD_OK, UAD_EINVAL (null
+ * pointer, n < 1 or n > 2^20) or UAD_ECUDA. */
+int uad_so3_check(const float* w, int32_t n, float* log_exp, float* log_comp);
+
 void uad_destroy(uad_ctx* ctx);
 const char* uad_last_error(const uad_ctx* ctx);
 

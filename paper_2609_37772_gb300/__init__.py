@@ -70,12 +70,14 @@ uad_tile_weight = _fn("uad_tile_weight", C.c_int, _P, _I32, _I32, _P)
 uad_linear = _fn("uad_linear", C.c_int, _P, _P, _P, _P, _I32, _I32, _I32, _P)
 uad_linear_static_scratch = _fn("uad_linear_static_scratch", C.c_int, _P, _P, _P, _P, _I32, _I32, _I32, _P)
 uad_set_wait_limit = _fn("uad_set_wait_limit", C.c_int, _P, C.c_int64, _I32)
+uad_so3_check = _fn("uad_so3_check", C.c_int, _P, _I32, _P, _P)
 UAD_ETOOBIG = -7
 
 EXPORTS = ["uad_version", "uad_last_error", "uad_init", "uad_set_prefix_kv", "uad_prepare_times",
            "uad_denoise", "uad_poll_released", "uad_finish", "uad_step_times",
            "uad_launches_per_chunk", "uad_destroy", "uad_plan_step", "uad_profile_chunk",
-           "uad_tile_weight", "uad_linear", "uad_linear_static_scratch", "uad_set_wait_limit"]
+           "uad_tile_weight", "uad_linear", "uad_linear_static_scratch", "uad_set_wait_limit",
+           "uad_so3_check"]
 
 
 def tile_weight(w):

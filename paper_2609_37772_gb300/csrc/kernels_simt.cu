@@ -894,6 +894,27 @@ __global__ void convert_kernel(const void* src, int sdt, void* dst, int ddt, lon
     stf(dst, i, ldf_rt(src, i, sdt), ddt);
 }
 
+// The rotations of Ghost Action Correction on SO(3) on given rotation vectors (testing aid):
+// log_exp[i] = log(exp(w_i)), log_comp[i] = log(exp(w_i) exp(w_{i+1 mod n})^T).
+__global__ void so3_check_kernel(const float* w, int n, float* log_exp, float* log_comp) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  float A[9], B[9], Bt[9], C[9];
+  so3_exp(w + 3 * i, A);
+  so3_log(A, log_exp + 3 * i);
+  so3_exp(w + 3 * ((i + 1) % n), B);
+#pragma unroll
+  for (int r = 0; r < 3; ++r)
+#pragma unroll
+    for (int c = 0; c < 3; ++c) Bt[r * 3 + c] = B[c * 3 + r];
+  mat3_mul(A, Bt, C);
+  so3_log(C, log_comp + 3 * i);
+}
+
+void launch_so3_check(const float* w, int n, float* log_exp, float* log_comp, cudaStream_t s) {
+  so3_check_kernel<<<(n + 127) / 128, 128, 0, s>>>(w, n, log_exp, log_comp);
+}
+
 void launch_convert(const void* src, int src_dtype, void* dst, int dst_dtype, long long n, cudaStream_t s) {
   const int blocks = (int)((n + 255) / 256 < 4096 ? (n + 255) / 256 : 4096);
   convert_kernel<<<blocks > 0 ? blocks : 1, 256, 0, s>>>(src, src_dtype, dst, dst_dtype, n);

@@ -1453,6 +1453,24 @@ int uad_launches_per_chunk(const uad_ctx* c, int32_t batch, int32_t n_star) {
   return 1 + n_star * launches_per_step(c, batch);
 }
 
+int uad_so3_check(const float* w, int32_t n, float* log_exp, float* log_comp) {
+  if (!w || !log_exp || !log_comp || n < 1 || n > (1 << 20)) return UAD_EINVAL;
+  const size_t bytes = (size_t)n * 3 * 4;
+  float* d = nullptr;
+  if (cudaMalloc(&d, 3 * bytes) != cudaSuccess) return UAD_ECUDA;
+  int rc = UAD_OK;
+  if (cudaMemcpy(d, w, bytes, cudaMemcpyHostToDevice) != cudaSuccess) rc = UAD_ECUDA;
+  if (!rc) {
+    launch_so3_check(d, n, d + 3 * (size_t)n, d + 6 * (size_t)n, nullptr);
+    if (cudaGetLastError() != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess ||
+        cudaMemcpy(log_exp, d + 3 * (size_t)n, bytes, cudaMemcpyDeviceToHost) != cudaSuccess ||
+        cudaMemcpy(log_comp, d + 6 * (size_t)n, bytes, cudaMemcpyDeviceToHost) != cudaSuccess)
+      rc = UAD_ECUDA;
+  }
+  cudaFree(d);
+  return rc;
+}
+
 int uad_set_wait_limit(uad_ctx* c, int64_t wait_ns, int32_t unreachable) {
   if (!c || wait_ns <= 0 || unreachable < 0) return UAD_EINVAL;
   if (c->in_flight) return fail(c, UAD_ESTATE, "chunk in flight");

@@ -150,6 +150,7 @@ void launch_relayout(const float* src, int K, int N, void* dst, int dtype, int m
 size_t attention_smem_bytes(int dh);
 void launch_attention_prepare(int dh);  // opt in to > 48 KB dynamic shared memory (call once)
 void launch_convert(const void* src, int src_dtype, void* dst, int dst_dtype, long long n, cudaStream_t s);
+void launch_so3_check(const float* w, int n, float* log_exp, float* log_comp, cudaStream_t s);
 // y[m][n] = SiLU(x[m][n] + tab[tau_row[m] * stride + off + n]) in dtype dt (the input MLP of the
 // time-concatenating expert: the table holds e(tau) W_it + b_it per flow time)
 void launch_add_tau_silu(const float* x, const float* tab, int stride, int off, const int* tau_row, int M, int N,
