@@ -100,3 +100,21 @@ def test_u_selection_matches_the_oracle_clock(pi0):
         print(f"T_act {t_act} ms: selected U = {sel_bench}")
     # with a 0.5 ms action the tail cannot keep up for small U: blocking at U = 1 is positive
     assert latency_model_uaer(0.0, statistics.mean(t_evals), N_STAR, 1, 1, 0.5, S) > 0
+
+
+def test_chunk_time_linear_in_uniform_n(pi0):
+    """App. B: with every action at the same budget N, a chunk is N evaluations, so its time is
+    linear in N (a small constant for the chunk's start-up and the time table aside)."""
+    a, ex, noise = pi0
+    ns = [1, 2, 4, 6, 8, 10]
+    t = []
+    for n in ns:
+        bud = group_budgets(a.chunk_len, [(0, a.chunk_len - 1, n)])[None]
+        rows, evals, _ = run(ex, noise, bud, reps=3, warm=1)
+        assert evals == {n}
+        t.append(statistics.median(max(r) for r in rows))
+    slope, icpt = np.polyfit(ns, t, 1)
+    resid = max(abs(ti - (slope * n + icpt)) for n, ti in zip(ns, t))
+    print(f"chunk ms = {icpt:.3f} + {slope:.4f} N (largest residual {resid:.4f} ms)")
+    assert resid <= 0.02 * max(t)
+    assert abs(icpt) <= 0.25 * slope
