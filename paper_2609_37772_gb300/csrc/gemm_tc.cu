@@ -86,20 +86,13 @@ __host__ __device__ __forceinline__ size_t tc_pipe_bytes(int stages) {
 
 // Epilogue of one tile slice: T[j * pitch + row] holds the fp32 accumulator of token m0 + j
 // (j < mcount) for output row n = this thread's row (row = 32 w + lane over the four warps w of
-// the slice's group); `plane` is the K split (partial epilogue). Small rolled loops keep the code
-// compact.
-__device__ __forceinline__ void tile_epilogue(const TcGemmArgs& p, const float* T, int pitch, int plane, int m0,
+// the slice's group). Partial-plane epilogues (EPI_PARTIAL) are written by the kernels themselves
+// as whole-row 16-byte stores. Small rolled loops keep the code compact.
+__device__ __forceinline__ void tile_epilogue(const TcGemmArgs& p, const float* T, int pitch, int m0,
                                               int mcount, int n, int row, int lane) {
   const float b = p.bias ? p.bias[n] : 0.f;
   const float* Tr = T + row;
   switch (p.epi) {
-    case EPI_PARTIAL: {
-      // this split's fp32 partial tile into its own plane [split][M][N]; the consumer sums
-      float* dst = static_cast<float*>(p.out) + (size_t)plane * p.M * p.N;
-#pragma unroll 4
-      for (int j = 0; j < mcount; ++j) dst[(size_t)(m0 + j) * p.N + n] = Tr[j * pitch];
-      break;
-    }
     case EPI_GEGLU: {
       // rows 2i (gate) and 2i + 1 (up) give output i: tokens over the warps, lane owns rows
       // 4 lane .. 4 lane + 3 (outputs 2 lane, 2 lane + 1 of the tile), so that a warp writes one
@@ -347,7 +340,7 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
       }
     }
   } else if (have) {
-    tile_epilogue(p, T, kBM, s, m0, mcount, n, row, lane);
+    tile_epilogue(p, T, kBM, m0, mcount, n, row, lane);
   }
   tc_fence_before();
   __syncthreads();
@@ -355,114 +348,6 @@ __global__ void __launch_bounds__(128, 1) gemm_tc_kernel(const __grid_constant__
   if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kBN));
 }
 
-
-// TN tokens per tile (MMA N = 128 or 256); STAGES pipeline stages of 16 KB + TN x 128 B; MINB CTAs
-// per SM (more than one: one CTA's epilogue overlaps another's main loop, which pays when there
-// are at least as many tiles as SMs).
-template <int TN, int STAGES, int MINB>
-__global__ void __launch_bounds__(128, MINB) gemm_tc_wide_kernel(const __grid_constant__ CUtensorMap tmx, TcGemmArgs p) {
-  constexpr int kWN = TN;
-  constexpr int kWStages = STAGES;
-  constexpr int kWStageB = kWN * kBK * 2;
-  constexpr uint32_t kIdescWide = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kWN >> 3) << 17) |
-                                  ((uint32_t)(kBM >> 4) << 24);
-  static_assert(STAGES * (kStageA + kWStageB) >= kBM * kBN * 4, "the stage area holds the epilogue slice");
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-  const int t = blockIdx.x, mt = blockIdx.y;
-  const int KC = p.K / kBK;
-  const int stages = KC < kWStages ? KC : kWStages;
-  uint8_t* sA = smem;                                        // stages x 16 KB weights
-  uint8_t* sB = smem + (size_t)kWStages * kStageA;           // stages x 32 KB activations
-  // after the main loop the stage area holds the epilogue slice T (32 KB)
-  float* T = reinterpret_cast<float*>(smem);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)kWStages * (kStageA + kWStageB));
-  uint64_t* empty = full + kWStages;
-  uint64_t* done = empty + kWStages;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
-  if (threadIdx.x == 0) {
-    for (int i = 0; i < kWStages; ++i) {
-      mbar_init(full + i, 1);
-      mbar_init(empty + i, 1);
-    }
-    mbar_init(done, 1);
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  }
-  if (warp == 0) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(tmem_slot)), "r"(kWN));
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
-  }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
-  pdl_trigger();
-
-  if (threadIdx.x == 0) {
-    const uint64_t pol = policy_evict_first();
-    const uint8_t* wt = static_cast<const uint8_t*>(p.w_tiled) + (size_t)t * KC * kStageA;
-    const int first = stages;
-    for (int i = 0; i < first; ++i) {
-      mbar_expect_tx(full + i, kStageA + kWStageB);
-      bulk_g2s(sA + (size_t)i * kStageA, wt + (size_t)i * kStageA, kStageA, full + i, pol);
-    }
-    pdl_wait();
-    for (int i = 0; i < first; ++i)
-      for (int q = 0; q < kWN / kBN; ++q)
-        tma_2d(sB + (size_t)i * kWStageB + q * kStageB, &tmx, i * kBK, mt * kWN + q * kBN, full + i);
-    int issued = first;
-    for (int i = first; i < KC; ++i) {
-      const int st = i % stages, round = i / stages;
-      if (!mbar_wait(empty + st, (round - 1) & 1, p.err, 31)) break;
-      mbar_expect_tx(full + st, kStageA + kWStageB);
-      bulk_g2s(sA + (size_t)st * kStageA, wt + (size_t)i * kStageA, kStageA, full + st, pol);
-      for (int q = 0; q < kWN / kBN; ++q)
-        tma_2d(sB + (size_t)st * kWStageB + q * kStageB, &tmx, i * kBK, mt * kWN + q * kBN, full + st);
-      ++issued;
-    }
-    for (int i = issued - stages > 0 ? issued - stages : 0; i < issued; ++i)
-      mbar_wait(full + i % stages, (i / stages) & 1, p.err, 32);
-  } else if (threadIdx.x == 32) {
-    bool ok = true;
-    for (int i = 0; i < KC && ok; ++i) {
-      const int st = i % stages, round = i / stages;
-      ok = mbar_wait(full + st, round & 1, p.err, 33);
-      if (!ok) break;
-      tc_fence_after();
-      const uint32_t a0 = su32(sA + (size_t)st * kStageA), b0 = su32(sB + (size_t)st * kWStageB);
-#pragma unroll
-      for (int k = 0; k < kBK / 16; ++k)
-        ptx::mma_bf16(tmem, sw128_desc(a0 + 32 * k), sw128_desc(b0 + 32 * k), kIdescWide, (i > 0 || k > 0) ? 1u : 0u);
-      mma_commit(empty + st);
-    }
-    mma_commit(done);
-  }
-  __syncwarp();
-  pdl_wait();
-  const bool ok = mbar_wait(done, 0, p.err, 34);
-  tc_fence_after();
-  const int row = warp * 32 + lane;
-  const int n = t * kBM + row;
-  // epilogue in four slices of 64 tokens (TMEM columns [64 q, 64 q + 64))
-  for (int q = 0; q < kWN / kBN; ++q) {
-    const int m0 = mt * kWN + q * kBN;
-    if (m0 >= p.M) break;
-    const int mcount = p.M - m0 < kBN ? p.M - m0 : kBN;
-    float v[kBN];
-    __syncwarp();
-    tmem_ld64(tmem + ((uint32_t)(warp * 32) << 16) + q * kBN, v);
-#pragma unroll
-    for (int j = 0; j < kBN; ++j) T[j * kBM + row] = v[j];
-    __syncthreads();
-    if (ok) tile_epilogue(p, T, kBM, 0, m0, mcount, n, row, lane);
-    __syncthreads();
-  }
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kWN));
-}
 
 // Persistent form for many tokens: one CTA per SM walks the work units u = blockIdx.x,
 // blockIdx.x + gridDim.x, ... Unit u is (token tile mt of p.tn <= TN tokens, weight tile nt, K
@@ -618,7 +503,7 @@ __global__ void __launch_bounds__(kPersThreads, 1) gemm_tc_pers_kernel(const __g
                 *reinterpret_cast<const float4*>(Tg + jr * kPersPitch + c4 * 4);
           }
         } else {
-          tile_epilogue(p, Tg, kPersPitch, sp, m0, mcount, n, row, lane);
+          tile_epilogue(p, Tg, kPersPitch, m0, mcount, n, row, lane);
         }
       }
     }
