@@ -90,7 +90,7 @@ __host__ __device__ __forceinline__ size_t tc_pipe_bytes(int stages) {
 // as whole-row 16-byte stores. Small rolled loops keep the code compact.
 __device__ __forceinline__ void tile_epilogue(const TcGemmArgs& p, const float* T, int pitch, int m0,
                                               int mcount, int n, int row, int lane) {
-  const float b = p.bias ? p.bias[n] : 0.f;
+  const float b = p.bias && (p.n_store <= 0 || n < p.n_store) ? p.bias[n] : 0.f;
   const float* Tr = T + row;
   switch (p.epi) {
     case EPI_GEGLU: {
@@ -167,6 +167,7 @@ __device__ __forceinline__ void tile_epilogue(const TcGemmArgs& p, const float* 
       break;
     }
     default:
+      if (p.n_store > 0 && n >= p.n_store) break;   // padding rows of a narrow projection
 #pragma unroll 4
       for (int j = 0; j < mcount; ++j)
         store_out(p.out, (size_t)(m0 + j) * p.ldo + n, Tr[j * pitch] + b, p.out_dtype);

@@ -89,6 +89,7 @@ struct uad_ctx {
   float *t_w1 = nullptr, *t_b1 = nullptr, *t_w2 = nullptr, *t_b2 = nullptr;  // t_w* are dtype
   void* w_in = nullptr; float* b_in = nullptr;   // [W][D]
   void* w_out = nullptr; float* b_out = nullptr; // [D][W]
+  Lin w_out_tc;                                  // the same padded to 128 rows, tiled (tensor cores)
   void* w_mod = nullptr; float* b_mod = nullptr; // [rowlen][W], all layers' modulation + final
   // time-concatenating expert (UAD_KIND_CONCAT): input MLP; e(tau) W_it + b_it sits in the table
   void* w_it = nullptr; float* b_it = nullptr;   // [W][W] (table fill)
@@ -409,7 +410,7 @@ void gemm(uad_ctx* c, const Lin& w, GemmArgs g, cudaStream_t s) {
   t.w_tiled = w.w; t.M = g.M; t.N = g.N; t.K = g.K;
   gemm_tc_plan(g.M, g.N, g.K, c->sms, g.epi, &t);
   t.epi = g.epi; t.out = g.out; t.ldo = g.ldo; t.out_dtype = g.out_dtype; t.bias = g.bias;
-  t.qkv = g.qkv; t.acc = c->tc_acc; t.counters = c->tc_counters; t.err = c->dev_err;
+  t.qkv = g.qkv; t.n_store = g.n_store; t.acc = c->tc_acc; t.counters = c->tc_counters; t.err = c->dev_err;
   launch_gemm_tc(&c->tmaps.at(g.A), t, s);
 }
 
@@ -743,7 +744,17 @@ void enqueue_chunk(uad_ctx* c, int B, int n_steps, bool step, cudaStream_t s) {
       GemmArgs go;
       go.A = c->y; go.lda = W; go.a_dtype = dt; go.w_dtype = dt;
       go.M = M; go.N = D; go.K = W; go.out = c->v; go.ldo = D; go.bias = c->b_out;
-      { Mark mk(c, s, "out_proj", gemm_bytes(go, c->es), 2.0 * M * W * D); gemm(c, c->w_out, go, s); }
+      {
+        Mark mk(c, s, "out_proj", gemm_bytes(go, c->es), 2.0 * M * W * D);
+        if (c->w_out_tc.tiled) {
+          // on the tensor cores: the weight padded to 128 rows, only the first D stored
+          go.N = 128;
+          go.n_store = D;
+          gemm(c, c->w_out_tc, go, s);
+        } else {
+          gemm(c, c->w_out, go, s);
+        }
+      }
     }
     if (!step) { Mark mk(c, s, "euler_tr_gac", 40.0 * M * D, 0); launch_euler(ea, s); }
   }
@@ -928,6 +939,11 @@ int uad_init(const uad_arch* arch, const float* weights, size_t n_floats, uad_ct
   c->attn_tc = a.kind != UAD_KIND_DIT && dt == BF16 && !c->force_simt && c->qd % 128 == 0 && c->kvd % 128 == 0 &&
               W % 64 == 0 && a.prefix_len + H <= attn_tc_max_keys();
   const int qk_perm = c->attn_tc && a.rope ? a.head_dim : 0;
+  // the action-out projection on the tensor cores (D <= 128 rows padded to 128, zero)
+  if (D <= 128) {
+    TRY(mklin(&c->w_out_tc, 128, W));
+    if (c->w_out_tc.tiled) put("out_w", c->w_out_tc, 1, 0);
+  }
   for (int l = 0; l < a.n_layers; ++l) {
     const std::string p = "l" + std::to_string(l) + ".";
     LayerW& w = c->L[l];

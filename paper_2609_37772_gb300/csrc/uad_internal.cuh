@@ -69,6 +69,7 @@ struct GemmArgs {
   const float* gate_tab = nullptr; int gate_stride = 0;  // gate(m, n) = gate_tab[tau_row[m] * gate_stride + n]
   const int* tau_row = nullptr;
   QkvTcOut qkv;                                    // EPI_QKV_TC
+  int n_store = 0;                                 // > 0: outputs n >= n_store are padding, not stored
 };
 
 struct NormArgs {
@@ -165,6 +166,7 @@ struct TcGemmArgs {
   void* out = nullptr; int ldo = 0; int out_dtype = BF16;
   const float* bias = nullptr;
   QkvTcOut qkv;                    // EPI_QKV_TC
+  int n_store = 0;                 // EPI_STORE: > 0: rows n >= n_store are padding (not stored, no bias)
   float* acc = nullptr;            // split-K accumulator [M][N] fp32, zero between launches
   int* counters = nullptr;         // split-K arrival counters per output tile, zero between launches
   int* err = nullptr;              // set to a nonzero code if a bounded wait gave up
