@@ -198,7 +198,10 @@ __global__ void __launch_bounds__(128, 1) attn_tc_kernel(const __grid_constant__
 
 // ---- one-pass attention for many query tiles: no partials, no combine ---------------------
 // One CTA per (128-row query tile, robot-group), keys in chunks of 128 (S = Q K^T with MMA
-// N = 128). Shared memory: Q, a K region, a Vt region. Per chunk: S on tcgen05 (double-buffered in
+// N = 128). Shared memory: Q and a ring of five operand slots that take, in the order the MMAs
+// read them, each chunk's K in head-dim pieces and its Vt in two 64-key halves; a slot is refilled
+// as soon as the MMAs that read it are done, so the next chunk's operands load while S and P V of
+// this one run. Per chunk: S on tcgen05 (double-buffered in
 // TMEM), then each softmax thread (one query row) forms P = exp(S - M) in bf16 against its running
 // maximum M and writes it into tensor memory over the S it came from, and O += P V accumulates in
 // TMEM with P as the MMA's A operand from tensor memory (P is double-buffered with S). M is raised only when the chunk's maximum
@@ -208,6 +211,14 @@ __global__ void __launch_bounds__(128, 1) attn_tc_kernel(const __grid_constant__
 constexpr int kKC2 = 128;                       // keys per chunk
 constexpr uint32_t kTmem2 = 512;                // S buffers at columns [0,128) and [128,256), O at [256, 256+dh)
 constexpr float kRescaleLog2 = 8.f;             // raise M only past this many powers of two
+constexpr int kSlots2 = 5;                      // operand ring slots
+constexpr int kBars2 = 9 + 2 * kSlots2;         // mbarriers of the kernel
+__host__ __device__ constexpr int attn2_kpieces(int dh) { return dh >= 128 ? 2 : 1; }
+// ring slot bytes: a K piece (128 keys x dh / pieces) or a Vt half (dh x 64 keys), the larger
+__host__ __device__ constexpr uint32_t attn2_slot_bytes(int dh) {
+  return (uint32_t)(dh / attn2_kpieces(dh)) * kKC2 * 2 > (uint32_t)dh * 128 ? (uint32_t)(dh / attn2_kpieces(dh)) * kKC2 * 2
+                                                                           : (uint32_t)dh * 128;
+}
 
 // Warps 0-3: softmax and output (they own the four TMEM lane quadrants); warp 4: TMA producer;
 // warp 5: MMA issuer. The producer and issuer wait on the softmax warps' progress, so they must
@@ -219,23 +230,25 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   constexpr int NC = DH / 64;
+  constexpr int KP = attn2_kpieces(DH);          // K pieces per chunk
+  constexpr int NCP = NC / KP;                   // 64-dim blocks of 128 keys per piece
+  constexpr int PPC = KP + 2;                    // ring entries per chunk: K pieces, two Vt halves
   constexpr uint32_t QB = DH * kQT * 2;          // Q: NC blocks of 128 rows x 64
-  constexpr uint32_t RB = DH * kKC2 * 2;         // a K chunk (NC blocks of 128 keys x 64) or a Vt
-                                                 // chunk (2 blocks of dh x 64 keys)
-  constexpr uint32_t VBLK = DH * 128;            // one Vt block: dh rows x 64 keys
+  constexpr uint32_t PB = NCP * kKC2 * 128;      // one K piece
+  constexpr uint32_t VBLK = DH * 128;            // one Vt half: dh rows x 64 keys
+  constexpr uint32_t SLOT = attn2_slot_bytes(DH);
   uint8_t* sQ = smem;
-  uint8_t* sK = sQ + QB;
-  uint8_t* sV = sK + RB;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sV + RB);
+  uint8_t* sR = sQ + QB;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sR + kSlots2 * SLOT);
   uint64_t* q_full = bars;          // Q landed
-  uint64_t* full = bars + 1;        // [2] K / Vt region loaded
-  uint64_t* empty = bars + 3;       // [2] K / Vt region free (the MMAs that read it are done)
-  uint64_t* s_full = bars + 5;      // [2] S buffer written
-  uint64_t* s_empty = bars + 7;     // [2] S / P buffer free (the P V that read its P is done)
-  uint64_t* p_full = bars + 9;      // P written (and O rescaled) by the 4 warps
-  uint64_t* p_empty = bars + 10;    // P V done: O complete up to this chunk
-  uint64_t* o_done = bars + 11;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
+  uint64_t* s_full = bars + 1;      // [2] S buffer written
+  uint64_t* s_empty = bars + 3;     // [2] S / P buffer free (the P V that read its P is done)
+  uint64_t* p_full = bars + 5;      // [2] P of the S buffer written (and O rescaled) by the 4 warps
+  uint64_t* p_empty = bars + 7;     // P V done: O complete up to this chunk
+  uint64_t* o_done = bars + 8;
+  uint64_t* r_full = bars + 9;            // [kSlots2] ring slot loaded
+  uint64_t* r_empty = r_full + kSlots2;   // [kSlots2] ring slot free (the MMAs that read it are done)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + kBars2);
 
   const int qt = blockIdx.x, bg = blockIdx.y;
   const int b = bg / p.n_kv_heads, g = bg % p.n_kv_heads;
@@ -246,12 +259,14 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
     for (int i = 0; i < 2; ++i) {
-      mbar_init(full + i, 1);
-      mbar_init(empty + i, 1);
       mbar_init(s_full + i, 1);
       mbar_init(s_empty + i, 1);
+      mbar_init(p_full + i, 4);
     }
-    mbar_init(p_full, 4);
+    for (int i = 0; i < kSlots2; ++i) {
+      mbar_init(r_full + i, 1);
+      mbar_init(r_empty + i, 1);
+    }
     mbar_init(p_empty, 1);
     mbar_init(o_done, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -268,53 +283,86 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
   pdl_trigger();
   pdl_wait();
 
+  // Ring entries in the order the MMAs read them: K of chunk 0, then per chunk c the K of chunk
+  // c + 1 (S runs a chunk ahead of P V) and the Vt of chunk c.
+  const auto k_entry = [&](int c, int j) { return c == 0 ? j : KP + (c - 1) * PPC + j; };
+  const auto v_entry = [&](int c, int h) { return KP + c * PPC + (c + 1 < nck ? KP : 0) + h; };
+
   if (threadIdx.x == 128) {
-    // producer: chunk c's K into the K region (once S of chunk c - 1 is done), then its Vt into
-    // the Vt region (once P V of chunk c - 1 is done)
+    // producer: ring entry e into slot e % kSlots2 once entry e - kSlots2 has been read
     const uint64_t pol = policy_evict_last();
     mbar_expect_tx(q_full, QB);
 #pragma unroll
     for (int c = 0; c < NC; ++c) tma_3d(sQ + c * (kQT * 128), &tq, c * 64, qt * kQT, bg, q_full, pol);
+    int e = 0;
     bool ok = true;
-    for (int ch = 0; ch < nck && ok; ++ch) {
-      if (ch > 0) ok = mbar_wait(empty + 0, (ch - 1) & 1, p.err, 41);
-      if (!ok) break;
-      mbar_expect_tx(full + 0, RB);
+    const auto slot = [&](int& t) {
+      t = e % kSlots2;
+      const int u = e / kSlots2;
+      ++e;
+      return u == 0 || mbar_wait(r_empty + t, (u - 1) & 1, p.err, 41);
+    };
+    const auto load_k = [&](int c) {
+      for (int j = 0; j < KP && ok; ++j) {
+        int t;
+        if (!(ok = slot(t))) break;
+        mbar_expect_tx(r_full + t, PB);
 #pragma unroll
-      for (int c = 0; c < NC; ++c) tma_3d(sK + c * (kKC2 * 128), &tk, c * 64, ch * kKC2, kvz, full + 0, pol);
-      if (ch > 0) ok = mbar_wait(empty + 1, (ch - 1) & 1, p.err, 41);
-      if (!ok) break;
-      mbar_expect_tx(full + 1, RB);
-#pragma unroll
-      for (int kb = 0; kb < 2; ++kb) tma_3d(sV + kb * VBLK, &tv, ch * kKC2 + kb * 64, 0, kvz, full + 1, pol);
+        for (int cc = 0; cc < NCP; ++cc)
+          tma_3d(sR + t * SLOT + cc * (kKC2 * 128), &tk, (j * NCP + cc) * 64, c * kKC2, kvz, r_full + t, pol);
+      }
+    };
+    load_k(0);
+    for (int c = 0; c < nck && ok; ++c) {
+      if (c + 1 < nck) load_k(c + 1);
+      for (int h = 0; h < 2 && ok; ++h) {
+        int t;
+        if (!(ok = slot(t))) break;
+        mbar_expect_tx(r_full + t, VBLK);
+        tma_3d(sR + t * SLOT, &tv, c * kKC2 + h * 64, 0, kvz, r_full + t, pol);
+      }
     }
   } else if (threadIdx.x == 160) {
+    // issuer: S(0); per chunk c: S(c + 1), then P V(c) once the softmax warps have written P(c)
     bool ok = mbar_wait(q_full, 0, p.err, 42);
-    const uint32_t q0 = su32(sQ), k0 = su32(sK), v0 = su32(sV);
+    const uint32_t q0 = su32(sQ), r0 = su32(sR);
+    const auto issue_s = [&](int c) {
+      const int sb = c & 1;
+      if (c >= 2) ok = mbar_wait(s_empty + sb, ((c >> 1) - 1) & 1, p.err, 44);
+      for (int j = 0; j < KP && ok; ++j) {
+        const int e = k_entry(c, j), t = e % kSlots2;
+        ok = mbar_wait(r_full + t, (e / kSlots2) & 1, p.err, 43);
+        if (!ok) break;
+        tc_fence_after();
+#pragma unroll
+        for (int cc = 0; cc < NCP; ++cc)
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            mma_bf16(tmem + sb * kKC2, sw128_desc(q0 + (j * NCP + cc) * (kQT * 128) + 32 * k),
+                     sw128_desc(r0 + t * SLOT + cc * (kKC2 * 128) + 32 * k), idesc_m128(kKC2), (j | cc | k) ? 1u : 0u);
+        mma_commit(r_empty + t);
+      }
+      if (ok) mma_commit(s_full + sb);
+    };
+    if (ok) issue_s(0);
     for (int ch = 0; ch < nck && ok; ++ch) {
       const int sb = ch & 1;
-      ok = mbar_wait(full + 0, ch & 1, p.err, 43);
-      if (ok && ch >= 2) ok = mbar_wait(s_empty + sb, ((ch >> 1) - 1) & 1, p.err, 44);
-      if (!ok) break;
-      tc_fence_after();
-#pragma unroll
-      for (int c = 0; c < NC; ++c)
+      if (ch + 1 < nck) issue_s(ch + 1);
+      ok = ok && mbar_wait(p_full + sb, (ch >> 1) & 1, p.err, 45);
+      for (int h = 0; h < 2 && ok; ++h) {
+        const int e = v_entry(ch, h), t = e % kSlots2;
+        ok = mbar_wait(r_full + t, (e / kSlots2) & 1, p.err, 46);
+        if (!ok) break;
+        tc_fence_after();
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          mma_bf16(tmem + sb * kKC2, sw128_desc(q0 + c * (kQT * 128) + 32 * k),
-                   sw128_desc(k0 + c * (kKC2 * 128) + 32 * k), idesc_m128(kKC2), (c | k) ? 1u : 0u);
-      mma_commit(s_full + sb);
-      mma_commit(empty + 0);
-      ok = mbar_wait(p_full, ch & 1, p.err, 45) && mbar_wait(full + 1, ch & 1, p.err, 46);
+          mma_bf16_ts(tO, tmem + sb * kKC2 + 8 * (4 * h + k), sw128_desc(r0 + t * SLOT + 32 * k), idesc_m128(DH),
+                      (ch | h | k) ? 1u : 0u);
+        mma_commit(r_empty + t);
+      }
       if (!ok) break;
-      tc_fence_after();
-#pragma unroll
-      for (int k = 0; k < kKC2 / 16; ++k)
-        mma_bf16_ts(tO, tmem + sb * kKC2 + 8 * k, sw128_desc(v0 + (k >> 2) * VBLK + 32 * (k & 3)), idesc_m128(DH),
-                    (ch | k) ? 1u : 0u);
-      mma_commit(empty + 1);
-      mma_commit(s_empty + sb);
       mma_commit(p_empty);
+      mma_commit(s_empty + sb);
     }
     mma_commit(o_done);
   }
@@ -391,11 +439,11 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
     }
     l += la + lb;
     tmem_wait_st();
-    // (the issuer waits for this announcement before it issues S of the next chunk, so no phase of
-    // p_full completes ahead of its wait)
+    // (p_full of this S buffer completes again only after S of chunk ch + 2, which the issuer
+    // issues after its wait for this phase)
     tc_fence_before();
     __syncwarp();
-    if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(p_full)) : "memory");
+    if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(p_full + sb)) : "memory");
   }
   float sv32[32];
   ok = ok && mbar_wait(o_done, 0, p.err, 49);
@@ -508,7 +556,7 @@ int tmap3(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d
 }  // namespace
 
 size_t attn_tc2_smem_bytes(int dh) {
-  return 1024 + (size_t)dh * kQT * 2 + 2 * (size_t)dh * kKC2 * 2 + 16 * 8;
+  return 1024 + (size_t)dh * kQT * 2 + (size_t)kSlots2 * attn2_slot_bytes(dh) + (kBars2 + 1) * 8;
 }
 
 bool attn_tc_use_two_pass(const AttnTcArgs& a) {
