@@ -599,13 +599,14 @@ void gemm_tc_prepare() {
 
 // Wide tiles (MMA N up to 256 tokens) run the tensor cores near their rate (N = 64 runs at a
 // third of it) and cut L2 re-reads of the weights: 1 = the persistent wide form, 0 = narrow
-// 128 x 64 tiles with K splits. Wide while 256-token tiles fill 60% of the SMs or 128-token
-// tiles fill half of them (measured on the pi0-like projections from 200 to 3200 tokens: with
-// fewer than 256 tokens the narrow tiles win).
+// 128 x 64 tiles with K splits. Wide from 512 tokens, or while 256-token tiles fill 60% of the
+// SMs or 128-token tiles fill half of them (measured on the pi0-like projections from 200 to 3200
+// tokens: with fewer than 256 tokens the narrow tiles win; at 800 tokens the wide form with K
+// split planes wins for the 1024-row o and down projections too).
 int gemm_tc_use_wide(int M, int N, int sms) {
   if (M < 256 || N > 8192) return 0;
   const int t256 = (N / kBM) * ((M + 255) / 256), t128 = (N / kBM) * ((M + 127) / 128);
-  return t256 * 5 >= sms * 3 || t128 * 2 >= sms ? 1 : 0;
+  return M >= 512 || t256 * 5 >= sms * 3 || t128 * 2 >= sms ? 1 : 0;
 }
 
 // The persistent form's plan: tokens per tile (256, 192 or 128) and, for partial-plane
