@@ -222,8 +222,10 @@ __host__ __device__ constexpr uint32_t attn2_slot_bytes(int dh) {
 
 // Warps 0-3: softmax and output (they own the four TMEM lane quadrants); warp 4: TMA producer;
 // warp 5: MMA issuer. The producer and issuer wait on the softmax warps' progress, so they must
-// not share a warp with them.
-template <int DH>
+// not share a warp with them. DV = head dims of O per CTA: DH, or DH / 2 when the query tiles are
+// at most half as many as the SMs (two CTAs per tile, blockIdx.z = which half of the head dims;
+// each computes S and P in full, and P V and the output for its half only).
+template <int DH, int DV>
 __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant__ CUtensorMap tq,
                                                           const __grid_constant__ CUtensorMap tk,
                                                           const __grid_constant__ CUtensorMap tv, AttnTcArgs p) {
@@ -235,7 +237,7 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
   constexpr int PPC = KP + 2;                    // ring entries per chunk: K pieces, two Vt halves
   constexpr uint32_t QB = DH * kQT * 2;          // Q: NC blocks of 128 rows x 64
   constexpr uint32_t PB = NCP * kKC2 * 128;      // one K piece
-  constexpr uint32_t VBLK = DH * 128;            // one Vt half: dh rows x 64 keys
+  constexpr uint32_t VBLK = DV * 128;            // one Vt half: DV rows x 64 keys
   constexpr uint32_t SLOT = attn2_slot_bytes(DH);
   uint8_t* sQ = smem;
   uint8_t* sR = sQ + QB;
@@ -250,7 +252,7 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
   uint64_t* r_empty = r_full + kSlots2;   // [kSlots2] ring slot free (the MMAs that read it are done)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + kBars2);
 
-  const int qt = blockIdx.x, bg = blockIdx.y;
+  const int qt = blockIdx.x, bg = blockIdx.y, d0 = blockIdx.z * DV;
   const int b = bg / p.n_kv_heads, g = bg % p.n_kv_heads;
   const int kvz = (b * p.n_layers + p.layer) * p.n_kv_heads + g;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -319,7 +321,7 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
         int t;
         if (!(ok = slot(t))) break;
         mbar_expect_tx(r_full + t, VBLK);
-        tma_3d(sR + t * SLOT, &tv, c * kKC2 + h * 64, 0, kvz, r_full + t, pol);
+        tma_3d(sR + t * SLOT, &tv, c * kKC2 + h * 64, d0, kvz, r_full + t, pol);
       }
     }
   } else if (threadIdx.x == 160) {
@@ -356,7 +358,7 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
         tc_fence_after();
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          mma_bf16_ts(tO, tmem + sb * kKC2 + 8 * (4 * h + k), sw128_desc(r0 + t * SLOT + 32 * k), idesc_m128(DH),
+          mma_bf16_ts(tO, tmem + sb * kKC2 + 8 * (4 * h + k), sw128_desc(r0 + t * SLOT + 32 * k), idesc_m128(DV),
                       (ch | h | k) ? 1u : 0u);
         mma_commit(r_empty + t);
       }
@@ -407,7 +409,7 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
       tc_fence_after();
       float ov[32];
 #pragma unroll 1
-      for (int cc = 0; cc < DH / 32; ++cc) {
+      for (int cc = 0; cc < DV / 32; ++cc) {
         tmem_ld32(tO + lane_base + cc * 32, ov);
 #pragma unroll
         for (int i = 0; i < 32; ++i) ov[i] *= factor;
@@ -454,9 +456,9 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
   const int qrow = qt * kQT + row;
   const float inv = 1.f / l;
   const int jj = qrow / p.H, ii = qrow % p.H;
-  __nv_bfloat16* orow = p.out + ((size_t)b * p.H + ii) * p.out_ld + (size_t)(g * p.group + jj) * DH;
+  __nv_bfloat16* orow = p.out + ((size_t)b * p.H + ii) * p.out_ld + (size_t)(g * p.group + jj) * DH + d0;
 #pragma unroll
-  for (int cc = 0; cc < DH / 32; ++cc) {
+  for (int cc = 0; cc < DV / 32; ++cc) {
     tmem_ld32(tO + lane_base + cc * 32, sv32);
     if (ok && qrow < p.rows) {
 #pragma unroll
@@ -582,11 +584,23 @@ int attn_tc_prepare(AttnTcMaps* maps, const AttnTcArgs& a, int batch_max) {
   // 128-key K chunks through `k` and Vt in 64-key boxes
   if (tmap3(&maps->k2, a.kcache, dh, NK, (uint64_t)batch_max * a.n_layers * a.n_kv_heads, (uint64_t)dh * 2,
             NK * dh * 2, 64, 64)) return -1;
-  maps->vt2 = maps->vt;
+  // Vt boxes of half the head dims for the one-pass kernel's split form
+  if (dh >= 128) {
+    if (tmap3(&maps->vt2, a.vtcache, NK, dh, (uint64_t)batch_max * a.n_layers * a.n_kv_heads, NKp * 2,
+              (uint64_t)dh * NKp * 2, 64, (uint32_t)dh / 2)) return -1;
+  } else {
+    maps->vt2 = maps->vt;
+  }
   const int smem2 = (int)attn_tc2_smem_bytes(dh);
-  if (dh == 64) cudaFuncSetAttribute(attn_tc2_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem2);
-  if (dh == 128) cudaFuncSetAttribute(attn_tc2_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem2);
-  if (dh == 256) cudaFuncSetAttribute(attn_tc2_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem2);
+  if (dh == 64) cudaFuncSetAttribute(attn_tc2_kernel<64, 64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem2);
+  if (dh == 128) {
+    cudaFuncSetAttribute(attn_tc2_kernel<128, 128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem2);
+    cudaFuncSetAttribute(attn_tc2_kernel<128, 64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem2);
+  }
+  if (dh == 256) {
+    cudaFuncSetAttribute(attn_tc2_kernel<256, 256>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem2);
+    cudaFuncSetAttribute(attn_tc2_kernel<256, 128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem2);
+  }
   const int smem = (int)attn_tc_smem_bytes(dh);
   if (dh == 64) cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (dh == 128) cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
@@ -600,11 +614,22 @@ int attn_tc_rpad(int rows) { return (rows + kQT - 1) / kQT * kQT; }
 
 void launch_attn_tc(const AttnTcMaps& maps, const AttnTcArgs& a, cudaStream_t s) {
   if (attn_tc_use_two_pass(a)) {
-    dim3 grid2((a.rows + kQT - 1) / kQT, a.batch * a.n_kv_heads);
+    const int tiles = (a.rows + kQT - 1) / kQT * a.batch * a.n_kv_heads;
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const bool split = a.head_dim >= 128 && 2 * tiles <= sms;
+    dim3 grid2((a.rows + kQT - 1) / kQT, a.batch * a.n_kv_heads, split ? 2 : 1);
     const size_t smem2 = attn_tc2_smem_bytes(a.head_dim);
-    if (a.head_dim == 64) launch_k(attn_tc2_kernel<64>, grid2, dim3(192), smem2, s, maps.q, maps.k, maps.vt2, a);
-    if (a.head_dim == 128) launch_k(attn_tc2_kernel<128>, grid2, dim3(192), smem2, s, maps.q, maps.k, maps.vt2, a);
-    if (a.head_dim == 256) launch_k(attn_tc2_kernel<256>, grid2, dim3(192), smem2, s, maps.q, maps.k, maps.vt2, a);
+    if (a.head_dim == 64) launch_k(attn_tc2_kernel<64, 64>, grid2, dim3(192), smem2, s, maps.q, maps.k, maps.vt, a);
+    if (a.head_dim == 128) {
+      if (split) launch_k(attn_tc2_kernel<128, 64>, grid2, dim3(192), smem2, s, maps.q, maps.k, maps.vt2, a);
+      else launch_k(attn_tc2_kernel<128, 128>, grid2, dim3(192), smem2, s, maps.q, maps.k, maps.vt, a);
+    }
+    if (a.head_dim == 256) {
+      if (split) launch_k(attn_tc2_kernel<256, 128>, grid2, dim3(192), smem2, s, maps.q, maps.k, maps.vt2, a);
+      else launch_k(attn_tc2_kernel<256, 256>, grid2, dim3(192), smem2, s, maps.q, maps.k, maps.vt, a);
+    }
     return;
   }
   dim3 grid((a.rows + kQT - 1) / kQT, attn_tc_chunks(a.n_keys), a.batch * a.n_kv_heads);

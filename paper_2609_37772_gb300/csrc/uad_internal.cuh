@@ -203,7 +203,9 @@ struct AttnTcArgs {
   __nv_bfloat16* out = nullptr; int out_ld = 0;   // o [B*H][Hq*dh]
   int* err = nullptr;
 };
-struct AttnTcMaps { CUtensorMap q, k, vt, k2, vt2; };   // k: 128-key boxes; k2 / vt2: 64-key boxes (step kernel)
+// k: 128-key boxes; k2: 64-key boxes (step kernel); vt: 64-key Vt boxes of all head dims; vt2: of
+// half of them (the one-pass kernel's split form)
+struct AttnTcMaps { CUtensorMap q, k, vt, k2, vt2; };
 size_t attn_tc_smem_bytes(int dh);
 int attn_tc_prepare(AttnTcMaps* maps, const AttnTcArgs& a, int batch_max);  // 0 on success
 int attn_tc_chunks(int n_keys);
