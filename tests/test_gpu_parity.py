@@ -519,6 +519,30 @@ def test_one_pass_attention_many_tiles(B):
         ex.close()
 
 
+@pytest.mark.parametrize("prefix,B", [(78, 32), (206, 32), (206, 40)])
+def test_one_pass_attention_key_counts(prefix, B):
+    """The many-tile attention at the key-count edges: 128 keys (one chunk, no later chunk to load
+    ahead) and 256 keys (two full chunks, no masked keys), split over head-dim halves (64 tiles)
+    and not (80 tiles); sampled robots vs the oracle."""
+    a = ARCHS["pi0_small"].replace(name=f"pi0_small_p{prefix}", prefix_len=prefix)
+    blob = make_weights(a, seed=15)
+    ex = uad.Expert(a, blob, max_batch=B)
+    try:
+        pre = [make_prefix_kv(a, robot=b, seed=15) for b in range(B)]
+        for b in range(B):
+            ex.set_prefix(b, *pre[b])
+        noise = make_noise(a, batch=B, seed=15)
+        bud = draw_sweep_schedules(a.chunk_len, B, seed=15)
+        ex.denoise(noise, bud)
+        res = ex.finish(timeout_us=TIMEOUT)
+        for b in (0, B // 2, B - 1):
+            ref = denoise(build_model(a, blob, pre[b]).velocity, noise[b], bud[b])
+            assert rel_err(res["final"][b], ref["final"]) <= TOL["bf16"]
+            assert rel_err(res["ghost"][b], ref["ghost"]) <= TOL["bf16"]
+    finally:
+        ex.close()
+
+
 def test_one_pass_attention_rescales_when_the_maximum_grows():
     """The many-tile attention path with prefix keys past the first 128-key chunk scaled by 16
     (a power of two: still exact in bf16), so that every query row's maximum score jumps far
