@@ -121,6 +121,10 @@ struct uad_ctx {
   int* evals = nullptr;
   unsigned long long* stamps = nullptr;
 
+  // the finished chunk's status words, copied back in one batch of asynchronous copies (pinned)
+  struct ChunkStatus { int derr, nonfinite, evals, pad; unsigned long long stamps[kFlagStride]; };
+  ChunkStatus* status_host = nullptr;
+
   // plan block (device) + pinned staging
   unsigned char* plan_dev = nullptr;
   unsigned char* plan_host = nullptr;
@@ -1070,6 +1074,7 @@ int uad_init(const uad_arch* arch, const float* weights, size_t n_floats, uad_ct
   c->plan_bytes_cap = plan_layout(kMaxSteps, a.max_batch, H, D).total;
   TRY(dalloc(c, (void**)&c->plan_dev, c->plan_bytes_cap));
   CK(cudaHostAlloc((void**)&c->plan_host, c->plan_bytes_cap, cudaHostAllocDefault));
+  CK(cudaHostAlloc((void**)&c->status_host, sizeof(uad_ctx::ChunkStatus), cudaHostAllocDefault));
   CK(cudaHostAlloc((void**)&c->host_rel, M * D * 4, cudaHostAllocMapped));
   CK(cudaHostGetDevicePointer((void**)&c->host_rel_dev, c->host_rel, 0));
   CK(cudaHostAlloc((void**)&c->host_flags, (size_t)a.max_batch * kFlagStride * 4, cudaHostAllocMapped));
@@ -1425,12 +1430,20 @@ int uad_finish(uad_ctx* c, float* final_actions, float* ghost, float* gac_error,
     std::this_thread::yield();
   }
   c->in_flight = false;
+  // the outputs and the status words as one batch of copies on the (now idle) worker stream and a
+  // single wait, so that the GPU idles for one host round trip between chunks, not one per copy
   const size_t n = (size_t)c->cur_B * c->a.chunk_len * c->a.action_dim;
-  if (final_actions) CK(cudaMemcpy(final_actions, c->fin, n * 4, cudaMemcpyDefault));
-  if (ghost) CK(cudaMemcpy(ghost, c->ghost, n * 4, cudaMemcpyDefault));
-  if (gac_error) CK(cudaMemcpy(gac_error, c->E, (size_t)c->cur_B * c->a.action_dim * 4, cudaMemcpyDefault));
-  int nonfinite = 0, evals = 0, derr = 0;
-  CK(cudaMemcpy(&derr, c->dev_err, 4, cudaMemcpyDeviceToHost));
+  cudaStream_t s = c->worker;
+  uad_ctx::ChunkStatus* cs = c->status_host;
+  if (final_actions) CK(cudaMemcpyAsync(final_actions, c->fin, n * 4, cudaMemcpyDefault, s));
+  if (ghost) CK(cudaMemcpyAsync(ghost, c->ghost, n * 4, cudaMemcpyDefault, s));
+  if (gac_error) CK(cudaMemcpyAsync(gac_error, c->E, (size_t)c->cur_B * c->a.action_dim * 4, cudaMemcpyDefault, s));
+  CK(cudaMemcpyAsync(&cs->derr, c->dev_err, 4, cudaMemcpyDeviceToHost, s));
+  CK(cudaMemcpyAsync(&cs->nonfinite, c->nonfinite, 4, cudaMemcpyDeviceToHost, s));
+  CK(cudaMemcpyAsync(&cs->evals, c->evals, 4, cudaMemcpyDeviceToHost, s));
+  CK(cudaMemcpyAsync(cs->stamps, c->stamps, kFlagStride * 8, cudaMemcpyDeviceToHost, s));
+  CK(cudaStreamSynchronize(s));
+  const int derr = cs->derr, nonfinite = cs->nonfinite, evals = cs->evals;
   if (derr) {
     cudaMemset(c->dev_err, 0, 4);
     if (c->cur_step) {
@@ -1443,10 +1456,7 @@ int uad_finish(uad_ctx* c, float* final_actions, float* ghost, float* gac_error,
     }
     return fail(c, UAD_ECUDA, "a kernel wait timed out (code %d); outputs are not valid", derr);
   }
-  CK(cudaMemcpy(&nonfinite, c->nonfinite, 4, cudaMemcpyDeviceToHost));
-  CK(cudaMemcpy(&evals, c->evals, 4, cudaMemcpyDeviceToHost));
-  c->last_stamps.assign(kFlagStride, 0);
-  CK(cudaMemcpy(c->last_stamps.data(), c->stamps, kFlagStride * 8, cudaMemcpyDeviceToHost));
+  c->last_stamps.assign(cs->stamps, cs->stamps + kFlagStride);
   c->last_steps = c->cur_steps;
   if (st) {
     st->evals = evals;
@@ -1520,6 +1530,7 @@ void uad_destroy(uad_ctx* c) {
   if (c->ev_done) cudaEventDestroy(c->ev_done);
   for (void* p : c->allocs) cudaFree(p);
   if (c->plan_host) cudaFreeHost(c->plan_host);
+  if (c->status_host) cudaFreeHost(c->status_host);
   if (c->host_rel) cudaFreeHost(c->host_rel);
   if (c->host_flags) cudaFreeHost(c->host_flags);
   delete c;
