@@ -12,7 +12,8 @@
 //   (unnormalised) and per-row (max, sum) go to a workspace. attn_combine merges the key chunks
 //   (the usual log-sum-exp rescaling) and writes o [B*H][Hq*dh] in bf16 for the O projection.
 // Many query tiles (attn_tc2_kernel): one CTA per query tile walks all key chunks in one pass,
-//   O accumulating in TMEM, and writes o itself.
+//   O accumulating in TMEM, and writes o itself; with at most half as many tiles as SMs, two CTAs
+//   per tile, one per half of the head dims.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
