@@ -130,20 +130,36 @@ __device__ __forceinline__ void tile_epilogue(const TcGemmArgs& p, const float* 
         __nv_bfloat16* base = isq ? o.q + ((size_t)(h / o.G) * o.G + (h % o.G)) * o.H * o.dh
                                   : o.kcache + (((size_t)o.layer * o.Hkv + h) * o.NK + o.P) * o.dh;
         const size_t sb = isq ? (size_t)o.Hkv * o.G * o.H * o.dh : (size_t)o.L * o.Hkv * o.NK * o.dh;
-        for (int j = row >> 5; j < mcount; j += kBM / 32) {
-          const int m = m0 + j, bi = m / o.H, ii = m - bi * o.H;
-          const float4 v = *reinterpret_cast<const float4*>(T + j * pitch + 4 * lane);
-          __nv_bfloat16* dst = base + bi * sb + (size_t)ii * o.dh;
-          if (o.rope) {
-            const float4 cs = *reinterpret_cast<const float4*>(o.rope + (size_t)ii * o.dh + r);
-            const int d = r >> 1;
-            *reinterpret_cast<__nv_bfloat162*>(dst + d) =
-                __floats2bfloat162_rn(v.x * cs.x - v.y * cs.y, v.z * cs.z - v.w * cs.w);
-            *reinterpret_cast<__nv_bfloat162*>(dst + d + half) =
-                __floats2bfloat162_rn(v.y * cs.x + v.x * cs.y, v.w * cs.z + v.z * cs.w);
-          } else {
-            *reinterpret_cast<__nv_bfloat162*>(dst + r) = __floats2bfloat162_rn(v.x, v.y);
-            *reinterpret_cast<__nv_bfloat162*>(dst + r + 2) = __floats2bfloat162_rn(v.z, v.w);
+        // four tokens at a time (a warp's tokens j, j + 4, ...): every (cos, sin) load of the four
+        // is issued before the first use, so that the table's L2 round trips overlap
+        constexpr int kStep = kBM / 32, kU = 4;
+        for (int j0 = row >> 5; j0 < mcount; j0 += kStep * kU) {
+          float4 v[kU], cs[kU];
+          int ii[kU];
+          __nv_bfloat16* dst[kU];
+#pragma unroll
+          for (int u = 0; u < kU; ++u) {
+            const int j = j0 + kStep * u;
+            if (j >= mcount) continue;
+            const int m = m0 + j, bi = m / o.H;
+            ii[u] = m - bi * o.H;
+            dst[u] = base + bi * sb + (size_t)ii[u] * o.dh;
+            v[u] = *reinterpret_cast<const float4*>(T + j * pitch + 4 * lane);
+            if (o.rope) cs[u] = __ldg(reinterpret_cast<const float4*>(o.rope + (size_t)ii[u] * o.dh + r));
+          }
+#pragma unroll
+          for (int u = 0; u < kU; ++u) {
+            if (j0 + kStep * u >= mcount) continue;
+            if (o.rope) {
+              const int d = r >> 1;
+              *reinterpret_cast<__nv_bfloat162*>(dst[u] + d) =
+                  __floats2bfloat162_rn(v[u].x * cs[u].x - v[u].y * cs[u].y, v[u].z * cs[u].z - v[u].w * cs[u].w);
+              *reinterpret_cast<__nv_bfloat162*>(dst[u] + d + half) =
+                  __floats2bfloat162_rn(v[u].y * cs[u].x + v[u].x * cs[u].y, v[u].w * cs[u].z + v[u].z * cs[u].w);
+            } else {
+              *reinterpret_cast<__nv_bfloat162*>(dst[u] + r) = __floats2bfloat162_rn(v[u].x, v[u].y);
+              *reinterpret_cast<__nv_bfloat162*>(dst[u] + r + 2) = __floats2bfloat162_rn(v[u].z, v[u].w);
+            }
           }
         }
       } else {
