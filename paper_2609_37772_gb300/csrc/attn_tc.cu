@@ -202,15 +202,17 @@ __global__ void __launch_bounds__(128, 1) attn_tc_kernel(const __grid_constant__
 // N = 128). Shared memory: Q and a ring of five operand slots that take, in the order the MMAs
 // read them, each chunk's K in head-dim pieces and its Vt in two 64-key halves; a slot is refilled
 // as soon as the MMAs that read it are done, so the next chunk's operands load while S and P V of
-// this one run. Per chunk: S on tcgen05 (double-buffered in
-// TMEM), then each softmax thread (one query row) forms P = exp(S - M) in bf16 against its running
-// maximum M and writes it into tensor memory over the S it came from, and O += P V accumulates in
-// TMEM with P as the MMA's A operand from tensor memory (P is double-buffered with S). M is raised only when the chunk's maximum
-// exceeds it by more than 2^8 in the exponent; the O row and the row sum are then rescaled in place
-// (after the previous P V has completed). Otherwise the stale M stays: every P is at most 2^8, and
-// O and the row sum share the same reference, so O / sum is unchanged. O / l is written in bf16.
+// this one run. Per chunk: S on tcgen05 (double-buffered in TMEM), then each softmax thread (one
+// query row) forms P = exp(S - M) in bf16 against its running maximum M and writes it into tensor
+// memory over the S it came from, and O += P V accumulates in TMEM with P as the MMA's A operand
+// from tensor memory (P is double-buffered with S). The issuer issues S of chunk c + 1 before
+// P V of chunk c, so that it runs while the softmax of chunk c does. M is raised only when the
+// chunk's maximum exceeds it by more than 2^8 in the exponent; the O row and the row sum are then
+// rescaled in place (after the previous P V has completed). Otherwise the stale M stays: every P
+// is at most 2^8, and O and the row sum share the same reference, so O / sum is unchanged. O / l
+// is written in bf16.
 constexpr int kKC2 = 128;                       // keys per chunk
-constexpr uint32_t kTmem2 = 512;                // S buffers at columns [0,128) and [128,256), O at [256, 256+dh)
+constexpr uint32_t kTmem2 = 512;                // S buffers at columns [0,128) and [128,256), O at [256, 256 + DV)
 constexpr float kRescaleLog2 = 8.f;             // raise M only past this many powers of two
 constexpr int kSlots2 = 5;                      // operand ring slots
 constexpr int kBars2 = 9 + 2 * kSlots2;         // mbarriers of the kernel
