@@ -466,6 +466,36 @@ def test_pi0_full_batched_16_robots_sampled():
         ex.close()
 
 
+@pytest.mark.parametrize("B", [8, 24])
+def test_pi0_full_batched_between_sampled(B):
+    """Batch sizes between the serving configurations: 8 robots (400 tokens: the qkv and gate/up
+    projections on the persistent wide form, o and down on narrow split-K tiles with partial
+    planes, the split-KV attention) and 24 (1200 tokens: every projection wide, the many-tile
+    attention on 96 query tiles without the head-dim split); first, middle and last robot vs the
+    oracle."""
+    a = ARCHS["pi0"]
+    blob = make_weights(a, seed=9)
+    ex = uad.Expert(a, blob, max_batch=B)
+    try:
+        pre = [make_prefix_kv(a, robot=b, seed=9) for b in range(B)]
+        for b in range(B):
+            ex.set_prefix(b, *pre[b])
+        noise = make_noise(a, batch=B, seed=9)
+        bud = draw_sweep_schedules(a.chunk_len, B, seed=9)
+        ex.denoise(noise, bud)
+        res = ex.finish(timeout_us=TIMEOUT)
+        worst = 0.0
+        for b in (0, B // 2, B - 1):
+            ref = denoise(build_model(a, blob, pre[b]).velocity, noise[b], bud[b])
+            ef, eg = rel_err(res["final"][b], ref["final"]), rel_err(res["ghost"][b], ref["ghost"])
+            worst = max(worst, ef, eg)
+            assert ef <= TOL["bf16"] and eg <= TOL["bf16"], (b, ef, eg)
+        assert res["evals"] == 10
+        print(f"[pi0 B={B}, robots (0, {B // 2}, {B - 1})] max rel err {worst:.2e} (tolerance {TOL['bf16']:g})")
+    finally:
+        ex.close()
+
+
 def test_pi0_full_batched_64_robots_sampled():
     """64 robots (M = 3200 tokens), the batched serving configuration: every projection on wide
     tensor-core tiles (the o and down projections with the partial-plane epilogue), attention on
