@@ -345,6 +345,24 @@ def test_dit_full(ns):
         c.close()
 
 
+@pytest.mark.parametrize("name,B", [("dit", 4), ("dit_small", 6)])
+def test_dit_batched(name, B):
+    """The DiT head for several robots, each with its own prefix tokens and schedule: at 4 robots
+    (64 tokens, one token tile: every projection takes the extra K splits) and at 6 (96 tokens,
+    two token tiles); every robot vs the oracle."""
+    a = ARCHS[name]
+    c = Case(a, B=B, seed=4)
+    try:
+        noise = make_noise(a, batch=B, seed=4)
+        if name == "dit":   # N* = 4 keeps the fp64 oracle of the full head short
+            bud = np.stack([group_budgets(a.chunk_len, [(0, 1 + b, 2), (2 + b, a.chunk_len - 1, 4)]) for b in range(B)])
+        else:
+            bud = draw_sweep_schedules(a.chunk_len, B, seed=4)
+        check(c, c.gpu(noise, bud), c.oracle(noise, bud), bud, TOL["bf16"])
+    finally:
+        c.close()
+
+
 def test_tensor_core_gemm_matches_cuda_core_gemm(monkeypatch):
     """The tcgen05 projection path against the CUDA-core GEMM on the same bf16 operands."""
     a = ARCHS["pi0_small"]
