@@ -481,39 +481,43 @@ __global__ void __launch_bounds__(192, 1) attn_tc2_kernel(const __grid_constant_
 }
 
 // Merge the key chunks of every query row: o = sum_c w_c O_c / sum_c w_c l_c, w_c = 2^((m_c - M) c2).
-// One CTA per (query row, robot-group), one thread per head dim; every partial is loaded
-// before any arithmetic. Writes o [(b*H + i)][(g*G + j)*dh + d] in bf16.
+// One CTA per (query row, robot-group), one thread per two head dims (dh / 2 threads: the grid
+// fits the GPU in one wave, 8-byte loads); every partial is loaded before any arithmetic. Writes
+// o [(b*H + i)][(g*G + j)*dh + d] in bf16.
 __global__ void attn_combine_kernel(AttnTcArgs p, int n_chunks) {
   constexpr int MAXC = kMaxKeyChunks;
   pdl_trigger();
   pdl_wait();
-  const int r = blockIdx.x, bg = blockIdx.y, d = threadIdx.x, DH = blockDim.x;
+  const int r = blockIdx.x, bg = blockIdx.y, d = 2 * threadIdx.x, DH = 2 * blockDim.x;
   const int b = bg / p.n_kv_heads, g = bg % p.n_kv_heads;
-  float m[MAXC], l[MAXC], o[MAXC];
+  float m[MAXC], l[MAXC];
+  float2 o[MAXC];
 #pragma unroll
   for (int c = 0; c < MAXC; ++c) {
     if (c < n_chunks) {
       const size_t idx = ((size_t)bg * n_chunks + c) * p.r_pad + r;
       m[c] = p.part_ml[idx * 2];
       l[c] = p.part_ml[idx * 2 + 1];
-      o[c] = p.part_o[idx * DH + d];
+      o[c] = *reinterpret_cast<const float2*>(p.part_o + idx * DH + d);
     }
   }
   float M = -INFINITY;
 #pragma unroll
   for (int c = 0; c < MAXC; ++c)
     if (c < n_chunks) M = fmaxf(M, m[c]);
-  float L = 0.f, acc = 0.f;
+  float L = 0.f, ax = 0.f, ay = 0.f;
 #pragma unroll
   for (int c = 0; c < MAXC; ++c) {
     if (c < n_chunks) {
       const float w = exp2f((m[c] - M) * p.scale_log2);
       L = fmaf(w, l[c], L);
-      acc = fmaf(w, o[c], acc);
+      ax = fmaf(w, o[c].x, ax);
+      ay = fmaf(w, o[c].y, ay);
     }
   }
   const int j = r / p.H, i = r % p.H;
-  p.out[((size_t)b * p.H + i) * p.out_ld + (size_t)(g * p.group + j) * DH + d] = __float2bfloat16_rn(acc / L);
+  *reinterpret_cast<__nv_bfloat162*>(p.out + ((size_t)b * p.H + i) * p.out_ld + (size_t)(g * p.group + j) * DH + d) =
+      __floats2bfloat162_rn(ax / L, ay / L);
 }
 
 // Prefix K/V of one robot (fp32 or bf16 source [L][P][Hkv][dh]) into the K and Vt caches.
@@ -640,7 +644,7 @@ void launch_attn_tc(const AttnTcMaps& maps, const AttnTcArgs& a, cudaStream_t s)
   if (a.head_dim == 64) launch_k(attn_tc_kernel<64>, grid, dim3(128), smem, s, maps.q, maps.k, maps.vt, a);
   if (a.head_dim == 128) launch_k(attn_tc_kernel<128>, grid, dim3(128), smem, s, maps.q, maps.k, maps.vt, a);
   if (a.head_dim == 256) launch_k(attn_tc_kernel<256>, grid, dim3(128), smem, s, maps.q, maps.k, maps.vt, a);
-  launch_k(attn_combine_kernel, dim3(a.rows, a.batch * a.n_kv_heads), dim3(a.head_dim), 0, s, a,
+  launch_k(attn_combine_kernel, dim3(a.rows, a.batch * a.n_kv_heads), dim3(a.head_dim / 2), 0, s, a,
            attn_tc_chunks(a.n_keys));
 }
 
